@@ -1,0 +1,480 @@
+"""Throughput benchmark of the BCMT token mixer (forward + backward) on GB300.
+
+One step = bcmt_forward + bcmt_backward of one BCMT layer over one batch of
+synthetic inputs already resident in HBM (workload: B=8, T=1024, L=64,
+D=512, 8 heads of 64, bf16 storage with fp32 accumulation).  Prints one JSON
+line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (launched by torchrun, one rank per GPU) every rank runs its own
+batch (weak scaling, no data-path collective); the time is the maximum over
+ranks.  ``--impl reference`` times the float64 CPU oracle on a bounded sample
+of the same workload on the host cores.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "BCMT layer fwd+bwd tokens/s on 1 GB300 and % of tensor/HBM roofline vs oracle"
+UNIT = "tokens/s"
+L2_FLUSH_BYTES = 256 << 20  # > 129 MB L2
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-dense", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+# ----------------------------------------------------------------- CPU oracle
+ORACLE_SNIPPET = r"""
+import json, os, sys, time
+sys.path.insert(0, {root!r})
+from oracle import bcmt_oracle as O
+from paper_2608_13578_gb300.inputs import WORKLOADS, as_float64, make_inputs
+w = WORKLOADS[{name!r}].replace(B=1)
+t = {{k: as_float64(v) for k, v in make_inputs(w).items()}}
+budget, reps, t0 = {budget}, 0, time.perf_counter()
+times = []
+while True:
+    s = time.perf_counter()
+    fw = O.forward_from_inputs(t, w.L, w.H)
+    O.backward(fw, t["dy"])
+    times.append(time.perf_counter() - s)
+    reps += 1
+    if time.perf_counter() - t0 > budget or reps >= {max_reps}:
+        break
+print(json.dumps({{"tokens": w.T, "reps": reps, "seconds": sum(times), "times": times}}))
+"""
+
+
+def run_oracle_sample(name: str, budget_s: float, max_reps: int):
+    """Times the oracle's fwd+bwd on one batch element of the workload in a fresh
+    process (no CUDA context) with every BLAS thread count pinned to the host's
+    core count."""
+    cores = os.cpu_count() or 1
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(cores)
+    code = ORACLE_SNIPPET.format(root=ROOT, name=name, budget=budget_s, max_reps=max_reps)
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                       timeout=600)
+    if r.returncode != 0:
+        raise RuntimeError("oracle timing failed: " + r.stderr[-2000:])
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    d["cores"] = cores
+    return d
+
+
+# ------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------ roofline model
+def kernel_model(w):
+    """Algorithmic work per launch of each named kernel: (bound, amount) with
+    amount in flops for tensor-core GEMMs and bytes for HBM-bound kernels."""
+    n, D, H, Nb, B = w.B * w.T, w.D, w.H, w.n_blocks, w.B
+    es = 2 if w.dtype == "bf16" else 4
+    g = lambda m, nn, k: ("tensor", 2.0 * m * nn * k)
+    return {
+        "gemm_qkv": g(n, 3 * D, D),
+        "gemm_wo": g(n, D, D),
+        "gemm_gate_inject": g(n, D, D),
+        "gemm_dh": g(n, D, D),
+        "gemm_dhhat": g(n, D, D),
+        "gemm_dx": g(n, D, 3 * D),
+        "gemm_dw_g": g(D, D, n),
+        "gemm_dw_o": g(D, D, n),
+        "gemm_dw_qkv": g(D, 3 * D, n),
+        # read Q, K, V; write Concat(heads) and the log-sum-exp
+        "attn_fwd_tc": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
+        "attn_fwd_simt": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
+        # read Q, K, V, dO, O and the log-sum-exp; write dQ, dK, dV
+        "attn_bwd_tc": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
+        "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
+        # read H; write pooling weights and summaries
+        "summary_fwd": ("hbm", n * D * es + n * 4 + B * Nb * D * 4),
+        "memory_fwd": ("hbm", B * Nb * D * 4 * 3 + D * D * es),
+        # read dY, G, C; write dU and the shifted memory gradient
+        "gate_bwd": ("hbm", 3 * n * D * es + 2 * B * Nb * D * 4),
+        "memory_bwd": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
+        "summary_bwd": ("hbm", n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
+    }
+
+
+def csrc_digest():
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2608_13578_gb300", "csrc")
+    for f in sorted(os.listdir(d)):
+        with open(os.path.join(d, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"], "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+
+
+def ncu_traffic(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it
+    was taken on the current kernel sources."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        e = d.get(kernel)
+        if e and e.get("csrc_digest") == csrc_digest():
+            return e.get("dram_bytes_per_launch")
+    except (OSError, ValueError):
+        pass
+    return None
+
+
+# ------------------------------------------------------------- our arm (GPU)
+def bench_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    if local_rank == 0:
+        from paper_2608_13578_gb300 import build
+        build.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2608_13578_gb300 import bcmt as C
+    from paper_2608_13578_gb300 import layer
+    from paper_2608_13578_gb300.inputs import HEADLINE, WORKLOADS, make_inputs
+
+    name = args.workload or HEADLINE
+    w = WORKLOADS[name]
+    t_cpu = make_inputs(w, seed=w.seed + rank)
+    t = {k: v.to(dev) for k, v in t_cpu.items()}
+    p = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype)
+    pprof = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype, flags=C.BCMT_FLAG_PROFILE)
+    ws = torch.empty(C.bcmt_workspace_size(p), dtype=torch.uint8, device=dev)
+    sc = torch.empty(C.bcmt_scratch_size(p), dtype=torch.uint8, device=dev)
+    y = torch.empty_like(t["x"])
+    grads = {"dx": torch.empty_like(t["x"]), "dw_qkv": torch.empty_like(t["w_qkv"])}
+    for n in ("w_o", "w_p", "w_m", "w_g"):
+        grads["d" + n] = torch.empty_like(t[n])
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def step(pp):
+        C.bcmt_forward(pp, t["x"], None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                       t["w_g"], t["decay"], y, ws, stream)
+        C.bcmt_backward(pp, t["dy"], t["x"], None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                        t["w_g"], t["decay"], ws, sc, grads["dx"], None, None, grads["dw_qkv"],
+                        grads["dw_o"], grads["dw_p"], grads["dw_m"], grads["dw_g"], stream)
+
+    for _ in range(max(3, args.warmup)):
+        step(p)
+    C.bcmt_device_status(stream)
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    C.bcmt_profile_reset()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)            # evict L2 between timed steps
+        ev[i][0].record(stream)
+        step(pprof)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    C.bcmt_device_status(stream)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    prof = C.bcmt_profile_read()
+    launches = sum(c for c, _ in prof.values())
+
+    # plain timing of the same steps without per-kernel events (overhead check)
+    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        ev2[i][0].record(stream)
+        step(p)
+        ev2[i][1].record(stream)
+    torch.cuda.synchronize()
+    plain_ms = sum(a.elapsed_time(b) for a, b in ev2)
+
+    if world > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = tt.item()
+
+    tokens_per_step = w.B * w.T
+    value = world * tokens_per_step * args.steps / (total_ms / 1e3)
+
+    # ---- end to end through the public API: pinned host inputs in, results out
+    x_h = t_cpu["x"].pin_memory()
+    dy_h = t_cpu["dy"].pin_memory()
+    outs_h = {"y": torch.empty_like(t_cpu["x"]).pin_memory()}
+    for n, g_ in grads.items():
+        outs_h[n] = torch.empty(g_.shape, dtype=g_.dtype).pin_memory()
+    x_d, dy_d = torch.empty_like(t["x"]), torch.empty_like(t["dy"])
+    h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
+    d2h = sum(v.numel() * v.element_size() for v in outs_h.values())
+
+    def e2e_step():
+        x_d.copy_(x_h, non_blocking=True)
+        dy_d.copy_(dy_h, non_blocking=True)
+        C.bcmt_forward(p, x_d, None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                       t["w_g"], t["decay"], y, ws, stream)
+        C.bcmt_backward(p, dy_d, x_d, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                        t["w_g"], t["decay"], ws, sc, grads["dx"], None, None, grads["dw_qkv"],
+                        grads["dw_o"], grads["dw_p"], grads["dw_m"], grads["dw_g"], stream)
+        outs_h["y"].copy_(y, non_blocking=True)
+        for n, g_ in grads.items():
+            outs_h[n].copy_(g_, non_blocking=True)
+
+    for _ in range(3):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = tt.item()
+    e2e_value = world * tokens_per_step * args.steps / (e2e_ms / 1e3)
+
+    # ---- roofline of the dominant kernel
+    model = kernel_model(w)
+    peaks = load_peaks()
+    dom = max(prof.items(), key=lambda kv: kv[1][1])
+    dname, (dcount, dms) = dom
+    bound, amount = model.get(dname, ("hbm", None))
+    roof = None
+    if amount is not None:
+        per_launch_s = dms / dcount / 1e3
+        if bound == "tensor":
+            ach = amount / per_launch_s / 1e12
+            peak = peaks["bf16_tflops"]
+            unit = "TFLOP/s"
+        else:
+            ach = amount / per_launch_s / 1e9
+            peak = peaks["hbm_gbs"]
+            unit = "GB/s"
+        roof = {"kernel": dname, "bound": bound, "achieved": round(ach, 2), "peak": peak,
+                "unit": unit, "frac": round(ach / peak, 4), "traffic": ncu_traffic(dname),
+                "algorithmic_per_launch": amount, "avg_launch_us": round(per_launch_s * 1e6, 3),
+                "peak_source": peaks["source"] + " (burst)"}
+    kernels = {k: {"launches": c, "avg_us": round(ms / c * 1e3, 3),
+                   "share": round(ms / sum(v[1] for v in prof.values()), 4)}
+               for k, (c, ms) in sorted(prof.items(), key=lambda kv: -kv[1][1])}
+
+    # ---- dense causal attention of the same shape (library SDPA), context only
+    dense = None
+    if not args.no_dense and rank == 0:
+        dense = bench_dense(w, t, stream, flush, args)
+
+    out = None
+    if rank == 0:
+        cpu = None
+        if not args.no_cpu_baseline:
+            d = run_oracle_sample(name, budget_s=15.0, max_reps=50)
+            cpu = {"value": round(d["tokens"] * d["reps"] / d["seconds"], 2), "unit": UNIT,
+                   "cores": d["cores"], "kind": "oracle",
+                   "sample": f"float64 oracle fwd+bwd on batch element 0 of the workload "
+                             f"({d['tokens']} tokens), {d['reps']} repetitions, "
+                             f"{d['seconds']:.1f} s"}
+        out = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup),
+            "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic (seeded N(0,1) tokens, N(0,1/D) weights, decay 0.8)",
+            "config": {"workload": name, "B": w.B, "T": w.T, "L": w.L, "D": w.D, "H": w.H,
+                       "per_rank_batch": w.B, "parallelism": f"batch-sharded x{world}",
+                       "l2": "flushed between timed steps (256 MiB write)"},
+            "clocks": clk,
+            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches,
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "kernels": kernels,
+            "timing_overhead": {"ms_per_step_without_kernel_events": round(plain_ms / args.steps, 4)},
+            "dense_causal_baseline": dense,
+        }
+        print(json.dumps(out))
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return out
+
+
+def bench_dense(w, t, stream, flush, args):
+    """Same projections with torch's dense causal SDPA (flash backend) instead of
+    the blockwise mixer: fwd+bwd tokens/s.  A library baseline for context."""
+    import torch
+    import torch.nn.functional as F
+    B, T, D, H = w.B, w.T, w.D, w.H
+    params = [t[n].detach().clone().requires_grad_(True) for n in ("w_qkv", "w_o")]
+    x = t["x"].detach().clone().requires_grad_(True)
+    dy = t["dy"]
+
+    def step():
+        qkv = x @ params[0]
+        q, k, v = qkv.view(B, T, 3, H, D // H).permute(2, 0, 3, 1, 4)
+        o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+        y = o.transpose(1, 2).reshape(B, T, D) @ params[1]
+        y.backward(dy)
+
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    tot = 0.0
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        tot += a.elapsed_time(b)
+    return {"value": round(B * T * args.steps / (tot / 1e3), 1), "unit": UNIT,
+            "what": "x W_qkv -> torch SDPA(is_causal) over the full sequence -> W_O, fwd+bwd, bf16"}
+
+
+# ------------------------------------------------------ reference arm (oracle)
+def bench_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    from paper_2608_13578_gb300.inputs import HEADLINE, WORKLOADS
+    name = args.workload or HEADLINE
+    w = WORKLOADS[name]
+    # each step: the oracle's fwd+bwd on one batch element of the workload
+    budget = max(5.0, 150.0 / max(1, args.steps + args.warmup))
+    d = run_oracle_sample(name, budget_s=0.0, max_reps=args.warmup + args.steps)
+    times = d["times"][args.warmup:] or d["times"]
+    secs = sum(times)
+    value = d["tokens"] * len(times) / secs
+    cpu = {"value": round(value, 2), "unit": UNIT, "cores": d["cores"], "kind": "oracle",
+           "sample": f"float64 oracle fwd+bwd on batch element 0 of {name} ({d['tokens']} tokens) "
+                     f"per step"}
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": UNIT,
+           "n_gpus": world, "steps": len(times), "warmup": args.warmup,
+           "ms_per_step": round(secs / len(times) * 1e3, 2), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic (seeded), one batch element per step",
+           "config": {"workload": name, "B": w.B, "T": w.T, "L": w.L, "D": w.D, "H": w.H},
+           "cpu_baseline": cpu,
+           "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    del budget
+    print(json.dumps(out))
+    return out
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        bench_reference(args)
+    else:
+        bench_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,51 @@
+/*
+ * bcmt_testing.h -- entry points of the BCMT library meant for its tests.
+ *
+ * They expose single kernels of the layer (the GEMM and the intra-block
+ * attention of Sec. 3.3) so each can be checked alone against the float64
+ * oracle, and let a test run the layer with the tensor-core kernels switched
+ * off.  Same conventions as bcmt.h: device pointers, caller-owned memory,
+ * asynchronous on `stream`, nothing allocated.
+ */
+#ifndef BCMT_TESTING_H
+#define BCMT_TESTING_H
+
+#include "bcmt.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Selects the kernels bcmt_forward / bcmt_backward use from now on in this
+ * process: gemm_on / attn_on = 1 for the tcgen05 tensor-core kernels (the
+ * default), 0 for the SIMT kernels.  Returns a bit mask of what this GPU and
+ * build support: bit 0 the tcgen05 GEMM, bit 1 the tcgen05 attention. */
+int bcmt_test_set_tensor_cores(int gemm_on, int attn_on);
+
+/* C[M,N] = A[M,K] B[K,N] with fp32 accumulation, element (m,k) of A at
+ * A[m*sam + k*sak] and (k,n) of B at B[k*sbk + n*sbn] (elements, not bytes);
+ * C row-major with leading dimension ldc, of type dtype_out.  impl: 0 SIMT,
+ * 1 tcgen05 (bf16 inputs; A and B each K-major or MN-major).  With
+ * splits > 1, K is cut into ranges whose fp32 partial products go to
+ * C + z*M*ldc (C must then be fp32 and hold every split).  N % 64 == 0.
+ * Returns the number of K-splits written, or -1 on error. */
+int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, const void* A,
+                   long sam, long sak, const void* B, long sbk, long sbn, void* C, long ldc,
+                   int splits, void* stream);
+
+/* The intra-block causal attention of Sec. 3.3 alone, forward (backward = 0)
+ * or backward (backward = 1), for the shape in *p (B, T, D, H, L, dtype).
+ * q, k, v: rows of token (b,t) start at q + (b*T+t)*ld, head h at column
+ * h*D/H.  o [B*T, D] Concat(heads), lse [B,H,T] fp32 (written by the forward,
+ * read by the backward).  Backward: dO [B*T, D]; drow [B,H,T] fp32 scratch;
+ * dq, dk, dv with row stride ld_d.  impl: 0 SIMT, 1 tcgen05.  Returns 0, or
+ * -1 on error (bcmt_last_error()). */
+int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, const void* k,
+                   const void* v, long ld, void* o, float* lse, const void* dO, float* drow,
+                   void* dq, void* dk, void* dv, long ld_d, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BCMT_TESTING_H */

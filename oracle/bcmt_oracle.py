@@ -104,15 +104,20 @@ def forward(x: Optional[np.ndarray], w_qkv: Optional[np.ndarray], w_o, w_p, w_m,
     G = np.zeros((B, T, D))
     Y = np.zeros((B, T, D))
 
+    if input_is_x:
+        W_Q = np.ascontiguousarray(w_qkv[:, 0:D])
+        W_K = np.ascontiguousarray(w_qkv[:, D:2 * D])
+        W_V = np.ascontiguousarray(w_qkv[:, 2 * D:3 * D])
+
     for b in range(B):
         # Sec. 3.3: local multi-head causal attention, block by block.
         for i, (t0, t1) in enumerate(blocks):
             Li = t1 - t0
             if input_is_x:
                 Xb = x[b, t0:t1]
-                Qb = Xb @ w_qkv[:, 0:D]
-                Kb = Xb @ w_qkv[:, D:2 * D]
-                Vb = Xb @ w_qkv[:, 2 * D:3 * D]
+                Qb = Xb @ W_Q
+                Kb = Xb @ W_K
+                Vb = Xb @ W_V
             else:
                 Qb, Kb, Vb = q[b, t0:t1], k[b, t0:t1], v[b, t0:t1]
             Q[b, t0:t1], K[b, t0:t1], V[b, t0:t1] = Qb, Kb, Vb
@@ -157,8 +162,8 @@ def forward(x: Optional[np.ndarray], w_qkv: Optional[np.ndarray], w_o, w_p, w_m,
         # Sec. 3.7-3.8: broadcast to the block's tokens, gate, inject.
         G[b] = _sigmoid(Hloc[b] @ w_g)
         for i, (t0, t1) in enumerate(blocks):
-            for t in range(t0, t1):
-                Y[b, t] = Hloc[b, t] + G[b, t] * C[b, i]
+            # every token of block i receives the same memory row C_i
+            Y[b, t0:t1] = Hloc[b, t0:t1] + G[b, t0:t1] * C[b, i][None, :]
 
     return dict(Y=Y, Q=Q, K=K, V=V, A=A, Hhat=Hhat, H=Hloc, s=s, alpha=alpha,
                 S=S, M=M, Z=Z, P=P, C=C, G=G,
@@ -197,10 +202,9 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
             dC = np.zeros((n_b, D))
             dU = np.zeros((T, D))
             for i, (t0, t1) in enumerate(blocks):
-                for t in range(t0, t1):
-                    dG = dY[b, t] * C[b, i]
-                    dU[t] = dG * G[b, t] * (1.0 - G[b, t])
-                    dC[i] += dY[b, t] * G[b, t]
+                dG = dY[b, t0:t1] * C[b, i][None, :]
+                dU[t0:t1] = dG * G[b, t0:t1] * (1.0 - G[b, t0:t1])
+                dC[i] = np.sum(dY[b, t0:t1] * G[b, t0:t1], axis=0)
             dw_g += Hloc[b].T @ dU
             dH[b] += dU @ w_g.T
 
@@ -247,7 +251,7 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
         x = inp["x"]
         dQKV = np.concatenate([dQ, dK, dV], axis=2)       # [B,T,3D]
         out["dx"] = dQKV @ w_qkv.T
-        out["dw_qkv"] = np.einsum("btd,bte->de", x, dQKV)
+        out["dw_qkv"] = x.reshape(B * T, D).T @ dQKV.reshape(B * T, 3 * D)
     else:
         out["dq"], out["dk"], out["dv"] = dQ, dK, dV
     return out

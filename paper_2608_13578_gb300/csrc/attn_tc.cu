@@ -1,0 +1,431 @@
+// Intra-block causal attention on the tcgen05 tensor cores (Sec. 3.3), bf16
+// operands, head width 64, block size L in {16, 32, 64, 128}.
+//
+// One CTA per (128-token tile, head, batch); 128 % L == 0, so a tile holds
+// 128 / L whole blocks and its keys are its own 128 tokens.  The attention
+// pattern inside the tile is block-diagonal causal: query r sees keys
+// [blockstart(r), r].  TMA brings the Q, K, V head slices of the tile into
+// shared memory (128-byte swizzle; a 3-D tensor map per operand zero-fills
+// tokens past the end of the sequence), tcgen05.mma computes the scores into
+// TMEM, each thread owns one query row for the masked softmax (the whole row
+// fits in TMEM, so there is no online rescaling), writes P in bf16 back to
+// shared memory as the A operand of P V, and the normalised output leaves
+// through a TMA store.  The backward recomputes P from the saved log-sum-exp
+// and runs the five products S = Q K^T, dP = dO V^T, dV = P^T dO,
+// dQ = dS K, dK = dS^T Q on the tensor cores, reading the same shared tiles
+// K-major or MN-major as each product needs.
+#include "common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+#include "tmap.h"
+
+namespace bcmt {
+
+namespace {
+constexpr int kTile = 128;
+constexpr int kDh = 64;
+constexpr uint32_t kTB = kTile * kDh * 2;  // one 128 x 64 bf16 tile: 16 KB
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Writes 16-byte unit `u` (keys 8u .. 8u+7) of row r of a 128 x 128 bf16
+// K-major operand stored as two 128-row swizzle-128 atoms (keys 0-63, 64-127).
+__device__ __forceinline__ void put_unit(uint8_t* base, int r, int u, uint4 val) {
+  *reinterpret_cast<uint4*>(base + (u >> 3) * 16384 + tc::sw128_offset(r, u & 7)) = val;
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+
+// Stores one 64-wide fp32 row (two 32-column halves) as bf16 into a
+// 128-row x 128-byte swizzled staging tile (the TMA store layout).
+__device__ __forceinline__ void stage_half(uint8_t* tile, int r, int half, const float* v, float mul) {
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    uint4 q;
+    q.x = pack2(v[8 * u + 0] * mul, v[8 * u + 1] * mul);
+    q.y = pack2(v[8 * u + 2] * mul, v[8 * u + 3] * mul);
+    q.z = pack2(v[8 * u + 4] * mul, v[8 * u + 5] * mul);
+    q.w = pack2(v[8 * u + 6] * mul, v[8 * u + 7] * mul);
+    *reinterpret_cast<uint4*>(tile + tc::sw128_offset(r, half * 4 + u)) = q;
+  }
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+}  // namespace
+
+// ====================================================================== forward
+__global__ void __launch_bounds__(128)
+    attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
+                       const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mO,
+                       float* __restrict__ lse, int Tlen, int H, int L, float scale,
+                       unsigned* status) {
+  if (tc::status_failed(status)) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sQ = smem;             // Q; then P keys 0-63; then the output staging tile
+  uint8_t* sK = smem + kTB;       // K; then P keys 64-127
+  uint8_t* sV = smem + 2 * kTB;   // V
+  uint8_t* sP = sQ;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 3 * kTB);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, 128);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 3 * kTB);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
+    const bool ok = tc::mbar_wait(&bar[0], 0, status);
+    tc::fence_after_sync();
+    if (ok) {
+      constexpr uint32_t idS = tc::idesc_bf16(128, 128, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < kDh / 16; ++kk)
+        tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sQ) + kk * 32, 16, 1024),
+                     tc::sdesc(tc::smem_u32(sK) + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar[1]);
+  }
+  __syncwarp();
+
+  bool ok = tc::mbar_wait(&bar[1], 0, status);
+  tc::fence_after_sync();
+
+  // ---- masked softmax, thread = query row r of the tile
+  const int r = warp * 32 + lane;
+  const int nc = L < 32 ? 32 : L;                           // columns this warp reads
+  const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;  // first of them
+  const int rbs = (r / L) * L;                              // first key row r may see
+  const float sl2 = scale * kLog2e;
+  float mx = -INFINITY;
+  for (int c = 0; c < nc; c += 32) {
+    float v[32];
+    tc::tmem_ld32(trow + (uint32_t)(wbs + c), v);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int kk = wbs + c + j;
+      if (kk >= rbs && kk <= r) mx = fmaxf(mx, v[j]);
+    }
+  }
+  float sum = 0.f;
+  for (int c = 0; c < nc; c += 32) {
+    float v[32];
+    tc::tmem_ld32(trow + (uint32_t)(wbs + c), v);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int kk = wbs + c + j;
+      const float p = (kk >= rbs && kk <= r) ? exp2f((v[j] - mx) * sl2) : 0.f;
+      v[j] = p;
+      sum += p;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      uint4 q;
+      q.x = pack2(v[8 * u + 0], v[8 * u + 1]);
+      q.y = pack2(v[8 * u + 2], v[8 * u + 3]);
+      q.z = pack2(v[8 * u + 4], v[8 * u + 5]);
+      q.w = pack2(v[8 * u + 6], v[8 * u + 7]);
+      put_unit(sP, r, (wbs + c) / 8 + u, q);
+    }
+  }
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  for (int u = 0; u < 16; ++u)
+    if (u * 8 < wbs || u * 8 >= wbs + nc) put_unit(sP, r, u, zero);
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+
+  if (tid == 0) {
+    tc::fence_after_sync();
+    constexpr uint32_t idO = tc::idesc_bf16(128, kDh, 0, 1);
+#pragma unroll
+    for (int kk = 0; kk < kTile / 16; ++kk)
+      tc::mma_bf16(tmem,
+                   tc::sdesc(tc::smem_u32(sP) + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                   tc::sdesc(tc::smem_u32(sV) + kk * 2048, 8192, 1024), idO, kk > 0 ? 1u : 0u);
+    tc::mma_commit(&bar[2]);
+  }
+  __syncwarp();
+  ok = tc::mbar_wait(&bar[2], 0, status) && ok;
+  tc::fence_after_sync();
+
+  // ---- epilogue: O = (P V) / sum, staged in the (now free) Q/P tile
+  const float inv = 1.0f / sum;
+  for (int half = 0; half < 2; ++half) {
+    float v[32];
+    tc::tmem_ld32(trow + (uint32_t)(half * 32), v);
+    stage_half(sQ, r, half, v, inv);
+  }
+  if (ok && t0 + r < Tlen) lse[((long)b * H + h) * Tlen + t0 + r] = mx * scale + logf(sum);
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+  if (tid == 0 && ok) {
+    tc::tma_store_3d(&mO, sQ, h * kDh, t0, b);
+    tc::tma_store_commit();
+    tc::tma_store_wait_all();
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 128);
+}
+
+// ===================================================================== backward
+__global__ void __launch_bounds__(128)
+    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
+                       const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
+                       const __grid_constant__ CUtensorMap mdQ, const __grid_constant__ CUtensorMap mdK,
+                       const __grid_constant__ CUtensorMap mdV, const bf16* __restrict__ O, long ld_o,
+                       const float* __restrict__ lse, int Tlen, int H, int L, float scale,
+                       unsigned* status) {
+  if (tc::status_failed(status)) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sQ = smem;              // Q; then dQ staging
+  uint8_t* sK = smem + kTB;        // K; then dK staging
+  uint8_t* sdO = smem + 2 * kTB;   // dO; then dV staging
+  uint8_t* sV = smem + 3 * kTB;    // V, then (with the next 16 KB) P
+  uint8_t* sP = sV;                // 32 KB: P, two key atoms
+  uint8_t* sdS = smem + 5 * kTB;   // 32 KB: scale * dS, two key atoms
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 7 * kTB);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, 256);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * kTB);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
+    const bool ok = tc::mbar_wait(&bar[0], 0, status);
+    tc::fence_after_sync();
+    if (ok) {
+      constexpr uint32_t id128 = tc::idesc_bf16(128, 128, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < kDh / 16; ++kk)  // S = Q K^T -> TMEM columns 0..127
+        tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sQ) + kk * 32, 16, 1024),
+                     tc::sdesc(tc::smem_u32(sK) + kk * 32, 16, 1024), id128, kk > 0 ? 1u : 0u);
+#pragma unroll
+      for (int kk = 0; kk < kDh / 16; ++kk)  // dP = dO V^T -> TMEM columns 128..255
+        tc::mma_bf16(tmem + 128, tc::sdesc(tc::smem_u32(sdO) + kk * 32, 16, 1024),
+                     tc::sdesc(tc::smem_u32(sV) + kk * 32, 16, 1024), id128, kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar[1]);
+  }
+  __syncwarp();
+
+  const int r = warp * 32 + lane;
+  const bool row_ok = (t0 + r) < Tlen;
+  // Drow = dO_r . O_r, dO from the swizzled tile once it has landed, O from global
+  bool ok = tc::mbar_wait(&bar[0], 0, status);
+  float drow = 0.f, lr = 0.f;
+  if (row_ok) {
+    const bf16* orow = O + ((long)b * Tlen + t0 + r) * ld_o + h * kDh;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const uint4 gv = *reinterpret_cast<const uint4*>(sdO + tc::sw128_offset(r, u));
+      const uint4 ov = *reinterpret_cast<const uint4*>(orow + 8 * u);
+      const bf16* gp = reinterpret_cast<const bf16*>(&gv);
+      const bf16* op = reinterpret_cast<const bf16*>(&ov);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) drow = fmaf(__bfloat162float(gp[e]), __bfloat162float(op[e]), drow);
+    }
+    lr = lse[((long)b * H + h) * Tlen + t0 + r];
+  }
+  ok = tc::mbar_wait(&bar[1], 0, status) && ok;
+  tc::fence_after_sync();
+
+  // ---- P = exp(S*scale - lse), dS = scale * P * (dP - Drow), both to shared memory
+  const int nc = L < 32 ? 32 : L;
+  const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;
+  const int rbs = (r / L) * L;
+  const float sl2 = scale * kLog2e, ll2 = lr * kLog2e;
+  for (int c = 0; c < nc; c += 32) {
+    float s[32], dp[32];
+    tc::tmem_ld32(trow + (uint32_t)(wbs + c), s);
+    tc::tmem_ld32(trow + 128u + (uint32_t)(wbs + c), dp);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int kk = wbs + c + j;
+      const float p = (row_ok && kk >= rbs && kk <= r) ? exp2f(s[j] * sl2 - ll2) : 0.f;
+      s[j] = p;
+      dp[j] = p * (dp[j] - drow) * scale;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      uint4 q, d;
+      q.x = pack2(s[8 * u + 0], s[8 * u + 1]);
+      q.y = pack2(s[8 * u + 2], s[8 * u + 3]);
+      q.z = pack2(s[8 * u + 4], s[8 * u + 5]);
+      q.w = pack2(s[8 * u + 6], s[8 * u + 7]);
+      d.x = pack2(dp[8 * u + 0], dp[8 * u + 1]);
+      d.y = pack2(dp[8 * u + 2], dp[8 * u + 3]);
+      d.z = pack2(dp[8 * u + 4], dp[8 * u + 5]);
+      d.w = pack2(dp[8 * u + 6], dp[8 * u + 7]);
+      put_unit(sP, r, (wbs + c) / 8 + u, q);
+      put_unit(sdS, r, (wbs + c) / 8 + u, d);
+    }
+  }
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  for (int u = 0; u < 16; ++u)
+    if (u * 8 < wbs || u * 8 >= wbs + nc) {
+      put_unit(sP, r, u, zero);
+      put_unit(sdS, r, u, zero);
+    }
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+
+  if (tid == 0) {
+    tc::fence_after_sync();
+    const uint32_t aP = tc::smem_u32(sP), adS = tc::smem_u32(sdS);
+    // dV = P^T dO -> columns 0..63 (A = P read MN-major: M = keys, K = queries)
+    constexpr uint32_t idMN = tc::idesc_bf16(128, kDh, 1, 1);
+#pragma unroll
+    for (int kk = 0; kk < kTile / 16; ++kk)
+      tc::mma_bf16(tmem, tc::sdesc(aP + kk * 2048, 16384, 1024),
+                   tc::sdesc(tc::smem_u32(sdO) + kk * 2048, 8192, 1024), idMN, kk > 0 ? 1u : 0u);
+    // dK = dS^T Q -> columns 64..127
+#pragma unroll
+    for (int kk = 0; kk < kTile / 16; ++kk)
+      tc::mma_bf16(tmem + 64, tc::sdesc(adS + kk * 2048, 16384, 1024),
+                   tc::sdesc(tc::smem_u32(sQ) + kk * 2048, 8192, 1024), idMN, kk > 0 ? 1u : 0u);
+    // dQ = dS K -> columns 128..191 (A = dS K-major, B = K read MN-major)
+    constexpr uint32_t idKM = tc::idesc_bf16(128, kDh, 0, 1);
+#pragma unroll
+    for (int kk = 0; kk < kTile / 16; ++kk)
+      tc::mma_bf16(tmem + 128, tc::sdesc(adS + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
+                   tc::sdesc(tc::smem_u32(sK) + kk * 2048, 8192, 1024), idKM, kk > 0 ? 1u : 0u);
+    tc::mma_commit(&bar[2]);
+  }
+  __syncwarp();
+  ok = tc::mbar_wait(&bar[2], 0, status) && ok;
+  tc::fence_after_sync();
+
+  // ---- epilogue: rows of dV, dK (key r) and dQ (query r) through staging tiles
+  {
+    float v[32];
+    tc::tmem_ld32(trow + 0u, v);
+    stage_half(sdO, r, 0, v, 1.0f);
+    tc::tmem_ld32(trow + 32u, v);
+    stage_half(sdO, r, 1, v, 1.0f);
+    tc::tmem_ld32(trow + 64u, v);
+    stage_half(sK, r, 0, v, 1.0f);
+    tc::tmem_ld32(trow + 96u, v);
+    stage_half(sK, r, 1, v, 1.0f);
+    tc::tmem_ld32(trow + 128u, v);
+    stage_half(sQ, r, 0, v, 1.0f);
+    tc::tmem_ld32(trow + 160u, v);
+    stage_half(sQ, r, 1, v, 1.0f);
+  }
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+  if (tid == 0 && ok) {
+    tc::tma_store_3d(&mdQ, sQ, h * kDh, t0, b);
+    tc::tma_store_3d(&mdK, sK, h * kDh, t0, b);
+    tc::tma_store_3d(&mdV, sdO, h * kDh, t0, b);
+    tc::tma_store_commit();
+    tc::tma_store_wait_all();
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+}
+
+// ========================================================================= host
+bool attn_tc_supported(int dtype, int dh, int L) {
+  return dtype == 1 && dh == kDh && (L == 16 || L == 32 || L == 64 || L == 128) &&
+         tmap_encoder() != nullptr;
+}
+
+static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, int B) {
+  const uint64_t dims[3] = {(uint64_t)D, (uint64_t)T, (uint64_t)B};
+  const uint64_t st[2] = {(uint64_t)ld * 2, (uint64_t)ld * 2 * (uint64_t)T};
+  const uint32_t box[3] = {kDh, kTile, 1};
+  return make_tmap_bf16(m, base, 3, dims, st, box);
+}
+
+static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
+static constexpr int kBwdSmem = 7 * kTB + 1024 + 64;
+
+cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
+  if (!attn_tc_supported(1, a.dh, a.L)) return cudaErrorNotSupported;
+  const int D = a.H * kDh;
+  CUtensorMap mQ, mK, mV, mO;
+  if (!head_map(&mQ, a.Q, a.ld_qkv, D, a.T, a.B) || !head_map(&mK, a.K, a.ld_qkv, D, a.T, a.B) ||
+      !head_map(&mV, a.V, a.ld_qkv, D, a.T, a.B) || !head_map(&mO, a.O, a.ld_o, D, a.T, a.B))
+    return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kFwdSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
+  attn_fwd_tc_kernel<<<grid, 128, kFwdSmem, lc.stream>>>(mQ, mK, mV, mO, a.lse, a.T, a.H, a.L,
+                                                         1.0f / sqrtf((float)a.dh), lc.status);
+  return cudaGetLastError();
+}
+
+cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
+  const AttnArgs& f = a.f;
+  if (!attn_tc_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
+  const int D = f.H * kDh;
+  CUtensorMap mQ, mK, mV, mdO, mdQ, mdK, mdV;
+  if (!head_map(&mQ, f.Q, f.ld_qkv, D, f.T, f.B) || !head_map(&mK, f.K, f.ld_qkv, D, f.T, f.B) ||
+      !head_map(&mV, f.V, f.ld_qkv, D, f.T, f.B) || !head_map(&mdO, a.dO, f.ld_o, D, f.T, f.B) ||
+      !head_map(&mdQ, a.dQ, a.ld_dqkv, D, f.T, f.B) ||
+      !head_map(&mdK, a.dK, a.ld_dqkv, D, f.T, f.B) ||
+      !head_map(&mdV, a.dV, a.ld_dqkv, D, f.T, f.B))
+    return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
+  attn_bwd_tc_kernel<<<grid, 128, kBwdSmem, lc.stream>>>(
+      mQ, mK, mV, mdO, mdQ, mdK, mdV, (const bf16*)f.O, f.ld_o, f.lse, f.T, f.H, f.L,
+      1.0f / sqrtf((float)f.dh), lc.status);
+  return cudaGetLastError();
+}
+
+}  // namespace bcmt

@@ -1,0 +1,656 @@
+// C ABI of the BCMT token mixer: argument validation, workspace layout, and
+// the launch sequence of the forward (Sec. 3.2-3.8) and backward passes on the
+// caller's stream.  No device memory is allocated per call.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/bcmt.h"
+#include "../../include/bcmt_testing.h"
+#include "common.cuh"
+#include "internal.h"
+
+namespace bcmt {
+
+// Device status word: kernels OR kStatus* bits into it when a bounded wait
+// expires.  Module-scope, one per device; its device address is looked up
+// once per device.
+__device__ unsigned g_status_word;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+bcmt_status fail(bcmt_status code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+unsigned* status_ptr() {
+  static std::mutex mu;
+  static std::vector<unsigned*> per_dev;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if ((int)per_dev.size() <= dev) per_dev.resize(dev + 1, nullptr);
+  if (!per_dev[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    per_dev[dev] = static_cast<unsigned*>(p);
+  }
+  return per_dev[dev];
+}
+
+// Tensor-core paths of the layer (switchable only through bcmt_testing.h).
+bool g_use_tc_gemm = true;
+bool g_use_tc_attn = true;
+
+// ------------------------------------------------------------------ profiling
+struct ProfRec {
+  const char* name;
+  cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+std::vector<ProfRec> g_prof_recs;
+std::vector<cudaEvent_t> g_prof_pool;
+size_t g_prof_pool_used = 0;
+constexpr size_t kProfMaxRecs = 1 << 16;
+
+cudaEvent_t prof_event() {
+  if (g_prof_pool_used == g_prof_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    g_prof_pool.push_back(e);
+  }
+  return g_prof_pool[g_prof_pool_used++];
+}
+
+struct Prof {
+  bool on;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  const char* name = nullptr;
+  void begin(const char* n) {
+    if (!on) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (g_prof_recs.size() >= kProfMaxRecs) return;
+    name = n;
+    a = prof_event();
+    if (a) cudaEventRecord(a, s);
+  }
+  void end(const char* n) {
+    if (!on || !a) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    cudaEvent_t b = prof_event();
+    if (!b) return;
+    cudaEventRecord(b, s);
+    g_prof_recs.push_back({n ? n : name, a, b});
+    a = nullptr;
+  }
+};
+
+// ---------------------------------------------------------------- validation
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bcmt_status check_params(const bcmt_params* p) {
+  if (!p) return fail(BCMT_ERR_ARG, "params is NULL");
+  if (p->B < 1 || p->T < 1 || p->D < 1 || p->H < 1 || p->L < 1)
+    return fail(BCMT_ERR_SHAPE, "B, T, D, H, L must be >= 1 (got %d %d %d %d %d)", p->B, p->T,
+                p->D, p->H, p->L);
+  if (p->dtype != BCMT_F32 && p->dtype != BCMT_BF16)
+    return fail(BCMT_ERR_ARG, "dtype must be BCMT_F32 or BCMT_BF16 (got %d)", p->dtype);
+  if (p->D % 64 != 0) return fail(BCMT_ERR_SHAPE, "D = %d is not a multiple of 64", p->D);
+  if (p->D % p->H != 0) return fail(BCMT_ERR_SHAPE, "D = %d is not divisible by H = %d", p->D, p->H);
+  const int dh = p->D / p->H;
+  if (dh % 32 != 0 || dh > 128)
+    return fail(BCMT_ERR_SHAPE, "head width D/H = %d must be a multiple of 32 and <= 128", dh);
+  if (p->L > 1024) return fail(BCMT_ERR_UNSUPPORTED, "block size L = %d > 1024", p->L);
+  if ((long long)p->B * p->T > (1ll << 30))
+    return fail(BCMT_ERR_SHAPE, "B*T = %lld tokens is too large", (long long)p->B * p->T);
+  if (p->flags & ~(unsigned)(BCMT_FLAG_HONLY | BCMT_FLAG_CHECK | BCMT_FLAG_PROFILE))
+    return fail(BCMT_ERR_ARG, "unknown flag bits 0x%x", p->flags);
+  return BCMT_OK;
+}
+
+bcmt_status check_ptr(const void* ptr, const char* name) {
+  if (!ptr) return fail(BCMT_ERR_ARG, "%s is NULL", name);
+  if (!aligned16(ptr)) return fail(BCMT_ERR_ALIGN, "%s is not 16-byte aligned", name);
+  return BCMT_OK;
+}
+
+#define BCMT_TRY(expr)                  \
+  do {                                  \
+    bcmt_status _s = (expr);            \
+    if (_s != BCMT_OK) return _s;       \
+  } while (0)
+
+// ----------------------------------------------------------- workspace layout
+size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct Geometry {
+  int B, T, D, H, L, Nb, dh, es;
+  long n;  // tokens B*T
+  bool honly, from_x;
+  int dtype;
+  explicit Geometry(const bcmt_params* p)
+      : B(p->B), T(p->T), D(p->D), H(p->H), L(p->L), Nb((p->T + p->L - 1) / p->L), dh(p->D / p->H),
+        es(p->dtype == BCMT_BF16 ? 2 : 4), n((long)p->B * p->T),
+        honly((p->flags & BCMT_FLAG_HONLY) != 0), from_x(p->input_is_x != 0), dtype(p->dtype) {}
+};
+
+// K-split count of a weight-gradient GEMM [M x N], K = tokens: about one
+// wave of 128 x 128 tiles on the GPU.
+int dw_splits(int M, int N, long K) {
+  const int tiles = ((M + 127) / 128) * ((N + 127) / 128);
+  int s = std::max(1, 148 / std::max(1, tiles));
+  const int nkb = (int)((K + 63) / 64);
+  return std::min(s, nkb);
+}
+
+struct FwdWs {
+  char *qkv, *hhat, *hloc, *G;
+  float *lse, *alpha, *S, *M, *Z, *C;
+  size_t bytes;
+};
+
+FwdWs fwd_layout(const Geometry& g, void* base) {
+  FwdWs w;
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    char* r = p ? p + off : nullptr;
+    off += al256(bytes);
+    return r;
+  };
+  w.qkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
+  w.lse = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
+  w.hhat = take((size_t)g.n * g.D * g.es);
+  if (!g.honly) {
+    w.hloc = take((size_t)g.n * g.D * g.es);
+    w.alpha = reinterpret_cast<float*>(take((size_t)g.n * 4));
+    w.S = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.M = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.Z = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
+    w.C = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.G = take((size_t)g.n * g.D * g.es);
+  } else {
+    w.hloc = w.G = nullptr;
+    w.alpha = w.S = w.M = w.Z = w.C = nullptr;
+  }
+  w.bytes = off;
+  return w;
+}
+
+struct BwdWs {
+  char *dU, *dH, *dHhat, *dqkv;
+  float *dP, *dS, *ds, *dwp_part, *Drow, *part;
+  size_t bytes;
+};
+
+BwdWs bwd_layout(const Geometry& g, void* base) {
+  BwdWs w;
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    char* r = p ? p + off : nullptr;
+    off += al256(bytes);
+    return r;
+  };
+  if (!g.honly) {
+    w.dU = take((size_t)g.n * g.D * g.es);
+    w.dH = take((size_t)g.n * g.D * g.es);
+    w.dP = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
+    w.dwp_part = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+  } else {
+    w.dU = w.dH = nullptr;
+    w.dP = w.dS = w.ds = w.dwp_part = nullptr;
+  }
+  w.dHhat = take((size_t)g.n * g.D * g.es);
+  w.dqkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
+  w.Drow = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
+  size_t part = (size_t)dw_splits(g.D, g.D, g.n) * g.D * g.D * 4;
+  if (g.from_x) part = std::max(part, (size_t)dw_splits(g.D, 3 * g.D, g.n) * g.D * 3 * g.D * 4);
+  w.part = reinterpret_cast<float*>(take(part));
+  w.bytes = off;
+  return w;
+}
+
+bcmt_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(BCMT_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Weight gradient dW[M,N] = A^T B over K tokens via K-split partials and an
+// ordered reduction.
+cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype, int dtype_out,
+                        int M, int N, long K,
+                        const void* A, long lda, const void* B, long ldb, float* part, void* out) {
+  const int splits = dw_splits(M, N, K);
+  EpiArgs ea;
+  ea.out = part;
+  ea.ldo = N;
+  ea.split_stride = (long)M * N;
+  pr.begin(name);
+  cudaError_t e = (dtype == 1 && g_use_tc_gemm)
+                      ? gemm_tc(lc, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits)
+                      : gemm_simt(lc, dtype, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea,
+                                  splits);
+  pr.end(nullptr);
+  if (e != cudaSuccess) return e;
+  pr.begin("reduce_splits");
+  e = reduce_splits(lc, part, effective_splits((int)K, splits), (long)M * N, dtype_out, out);
+  pr.end(nullptr);
+  return e;
+}
+
+cudaError_t run_gemm(const Launch& lc, Prof& pr, const char* name, int dtype, int dtype_out, int M,
+                     int N, int K, const void* A, long sam, long sak, const void* B, long sbk,
+                     long sbn, EpiKind epi, const EpiArgs& ea) {
+  pr.begin(name);
+  cudaError_t e = (dtype == 1 && g_use_tc_gemm)
+                      ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1)
+                      : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
+  pr.end(nullptr);
+  return e;
+}
+
+bool use_attn_tc(const Geometry& g) {
+  return g_use_tc_attn && attn_tc_supported(g.dtype, g.dh, g.L);
+}
+
+bcmt_status finish(const bcmt_params* p, cudaStream_t s) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+  if (p->flags & BCMT_FLAG_CHECK) return bcmt_device_status(s);
+  return BCMT_OK;
+}
+
+}  // namespace
+}  // namespace bcmt
+
+using namespace bcmt;
+
+extern "C" {
+
+size_t bcmt_workspace_size(const bcmt_params* p) {
+  if (check_params(p) != BCMT_OK) return 0;
+  Geometry g(p);
+  return fwd_layout(g, nullptr).bytes;
+}
+
+size_t bcmt_scratch_size(const bcmt_params* p) {
+  if (check_params(p) != BCMT_OK) return 0;
+  Geometry g(p);
+  return bwd_layout(g, nullptr).bytes;
+}
+
+const char* bcmt_last_error(void) { return g_last_error.c_str(); }
+
+bcmt_status bcmt_device_status(void* stream) {
+  unsigned* sp = status_ptr();
+  if (!sp) return fail(BCMT_ERR_CUDA, "device status word unavailable");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, sp, sizeof(v), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sp, 0, sizeof(unsigned), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "reading device status");
+  if (v & kStatusTimeout) return fail(BCMT_ERR_TIMEOUT, "a bounded device-side wait expired");
+  if (v) return fail(BCMT_ERR_CUDA, "device status 0x%x", v);
+  return BCMT_OK;
+}
+
+bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, const void* k,
+                         const void* v, const void* w_qkv, const void* w_o, const void* w_p,
+                         const void* w_m, const void* w_g, const float* decay, void* y,
+                         void* workspace, void* stream) {
+  BCMT_TRY(check_params(p));
+  Geometry g(p);
+  if (g.from_x) {
+    BCMT_TRY(check_ptr(x, "x"));
+    BCMT_TRY(check_ptr(w_qkv, "w_qkv"));
+  } else {
+    BCMT_TRY(check_ptr(q, "q"));
+    BCMT_TRY(check_ptr(k, "k"));
+    BCMT_TRY(check_ptr(v, "v"));
+  }
+  BCMT_TRY(check_ptr(w_o, "w_o"));
+  if (!g.honly) {
+    BCMT_TRY(check_ptr(w_p, "w_p"));
+    BCMT_TRY(check_ptr(w_m, "w_m"));
+    BCMT_TRY(check_ptr(w_g, "w_g"));
+    BCMT_TRY(check_ptr(decay, "decay"));
+  }
+  BCMT_TRY(check_ptr(y, "y"));
+  BCMT_TRY(check_ptr(workspace, "workspace"));
+  unsigned* sp = status_ptr();
+  if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Launch lc{s, sp};
+  Prof pr{(p->flags & BCMT_FLAG_PROFILE) != 0, s};
+  FwdWs w = fwd_layout(g, workspace);
+  const int D = g.D, n = (int)g.n;
+  cudaError_t e;
+
+  // Sec. 3.3: Q, K, V projections.
+  const void *Qp = q, *Kp = k, *Vp = v;
+  long ld = D;
+  if (g.from_x) {
+    EpiArgs ea;
+    ea.out = w.qkv;
+    ea.ldo = 3 * D;
+    e = run_gemm(lc, pr, "gemm_qkv", g.dtype, g.dtype, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1,
+                 EPI_STORE, ea);
+    if (e != cudaSuccess) return cuda_fail(e, "QKV projection");
+    Qp = w.qkv;
+    Kp = w.qkv + (size_t)D * g.es;
+    Vp = w.qkv + (size_t)2 * D * g.es;
+    ld = 3 * D;
+  }
+  // Sec. 3.3: intra-block causal attention -> Concat(heads).
+  AttnArgs aa{Qp, Kp, Vp, ld, w.hhat, D, w.lse, g.B, g.T, g.H, g.dh, g.L};
+  if (use_attn_tc(g)) {
+    pr.begin("attn_fwd_tc");
+    e = attn_fwd_tc(lc, aa);
+  } else {
+    pr.begin("attn_fwd_simt");
+    e = attn_fwd_simt(lc, g.dtype, aa);
+  }
+  pr.end(nullptr);
+  if (e != cudaSuccess) return cuda_fail(e, "block attention");
+  // Sec. 3.3: H = Concat(heads) W_O (HOnly: this is the output, Sec. 4.5).
+  {
+    EpiArgs ea;
+    ea.out = g.honly ? y : w.hloc;
+    ea.ldo = D;
+    e = run_gemm(lc, pr, "gemm_wo", g.dtype, g.dtype, n, D, D, w.hhat, D, 1, w_o, D, 1, EPI_STORE,
+                 ea);
+    if (e != cudaSuccess) return cuda_fail(e, "output projection");
+  }
+  if (!g.honly) {
+    // Sec. 3.4: adaptive block summaries.
+    pr.begin("summary_fwd");
+    e = summary_fwd(lc, g.dtype, w.hloc, w_p, w.alpha, w.S, g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "block summaries");
+    // Sec. 3.5: exponential causal memory, projection, shift.
+    pr.begin("memory_fwd");
+    e = memory_fwd(lc, g.dtype, w.S, decay, w_m, w.M, w.Z, w.C, g.B, g.Nb, D);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "causal memory");
+    // Sec. 3.7-3.8: gate and injection fused into the W_g GEMM.
+    EpiArgs ea;
+    ea.H = w.hloc;
+    ea.Cmem = w.C;
+    ea.G = w.G;
+    ea.Y = y;
+    ea.T = g.T;
+    ea.L = g.L;
+    ea.Nb = g.Nb;
+    ea.D = D;
+    e = run_gemm(lc, pr, "gemm_gate_inject", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
+                 EPI_GATE_INJECT, ea);
+    if (e != cudaSuccess) return cuda_fail(e, "gated injection");
+  }
+  return finish(p, s);
+}
+
+bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or_q, const void* k,
+                          const void* v, const void* w_qkv,
+                          const void* w_o, const void* w_p, const void* w_m, const void* w_g,
+                          const float* decay, const void* workspace, void* scratch, void* dx_or_dq,
+                          void* dk, void* dv, void* dw_qkv, void* dw_o, void* dw_p, void* dw_m,
+                          void* dw_g, void* stream) {
+  BCMT_TRY(check_params(p));
+  Geometry g(p);
+  BCMT_TRY(check_ptr(dy, "dy"));
+  BCMT_TRY(check_ptr(x_or_q, "x_or_q"));
+  if (g.from_x) {
+    BCMT_TRY(check_ptr(w_qkv, "w_qkv"));
+    BCMT_TRY(check_ptr(dw_qkv, "dw_qkv"));
+  } else {
+    BCMT_TRY(check_ptr(k, "k"));
+    BCMT_TRY(check_ptr(v, "v"));
+    BCMT_TRY(check_ptr(dk, "dk"));
+    BCMT_TRY(check_ptr(dv, "dv"));
+  }
+  BCMT_TRY(check_ptr(dx_or_dq, "dx_or_dq"));
+  BCMT_TRY(check_ptr(w_o, "w_o"));
+  BCMT_TRY(check_ptr(dw_o, "dw_o"));
+  BCMT_TRY(check_ptr(dw_p, "dw_p"));
+  BCMT_TRY(check_ptr(dw_m, "dw_m"));
+  BCMT_TRY(check_ptr(dw_g, "dw_g"));
+  if (!g.honly) {
+    BCMT_TRY(check_ptr(w_p, "w_p"));
+    BCMT_TRY(check_ptr(w_m, "w_m"));
+    BCMT_TRY(check_ptr(w_g, "w_g"));
+    BCMT_TRY(check_ptr(decay, "decay"));
+  }
+  BCMT_TRY(check_ptr(workspace, "workspace"));
+  BCMT_TRY(check_ptr(scratch, "scratch"));
+  unsigned* sp = status_ptr();
+  if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Launch lc{s, sp};
+  Prof pr{(p->flags & BCMT_FLAG_PROFILE) != 0, s};
+  FwdWs w = fwd_layout(g, const_cast<void*>(workspace));
+  BwdWs bw = bwd_layout(g, scratch);
+  const int D = g.D, n = (int)g.n;
+  cudaError_t e;
+
+  const void* dH = dy;  // HOnly: Y = H
+  if (!g.honly) {
+    // Sec. 3.8 reversed: dU and the per-block memory gradient (shifted: dP).
+    pr.begin("gate_bwd");
+    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "gate backward");
+    // Sec. 3.5 reversed: dM = dP W_m^T, reverse decayed scan -> dS; dW_m = M^T dP.
+    pr.begin("memory_bwd");
+    e = memory_bwd(lc, g.dtype, bw.dP, decay, w.Z, w_m, bw.dS, g.B, g.Nb, D);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "memory backward");
+    {
+      EpiArgs ea;
+      ea.out = dw_m;
+      ea.ldo = D;
+      e = run_gemm(lc, pr, "gemm_dwm", 0, g.dtype, D, D, g.B * g.Nb, w.M, 1, D, bw.dP, D, 1,
+                   EPI_STORE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "dW_m");
+    }
+    // Sec. 3.4 reversed: pooling scores and dW_p.
+    pr.begin("summary_bwd");
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "summary backward");
+    pr.begin("reduce_rows");
+    e = reduce_rows(lc, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_p");
+    // dW_g = H^T dU
+    e = weight_grad(lc, pr, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D, bw.part,
+                    dw_g);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_g");
+    // dH = dY + dU W_g^T + alpha dS + ds w_p
+    EpiArgs ea;
+    ea.out = bw.dH;
+    ea.dY = dy;
+    ea.alpha = w.alpha;
+    ea.dS = bw.dS;
+    ea.ds = bw.ds;
+    ea.w_p = w_p;
+    ea.T = g.T;
+    ea.L = g.L;
+    ea.Nb = g.Nb;
+    ea.D = D;
+    e = run_gemm(lc, pr, "gemm_dh", g.dtype, g.dtype, n, D, D, bw.dU, D, 1, w_g, 1, D, EPI_DH, ea);
+    if (e != cudaSuccess) return cuda_fail(e, "dH");
+    dH = bw.dH;
+  } else {
+    const size_t wb = (size_t)D * D * g.es;
+    if ((e = fill_zero(lc, dw_m, wb)) != cudaSuccess || (e = fill_zero(lc, dw_g, wb)) != cudaSuccess ||
+        (e = fill_zero(lc, dw_p, (size_t)D * g.es)) != cudaSuccess)
+      return cuda_fail(e, "zeroing HOnly gradients");
+  }
+  // Sec. 3.3 reversed: dHhat = dH W_O^T, dW_O = Hhat^T dH.
+  {
+    EpiArgs ea;
+    ea.out = bw.dHhat;
+    ea.ldo = D;
+    e = run_gemm(lc, pr, "gemm_dhhat", g.dtype, g.dtype, n, D, D, dH, D, 1, w_o, 1, D, EPI_STORE,
+                 ea);
+    if (e != cudaSuccess) return cuda_fail(e, "dHhat");
+    e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part,
+                    dw_o);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_O");
+  }
+  // Attention backward -> dQ, dK, dV.
+  {
+    const void *Qp, *Kp, *Vp;
+    long ld;
+    void *dQ, *dK, *dV;
+    long ldd;
+    if (g.from_x) {
+      Qp = w.qkv;
+      Kp = w.qkv + (size_t)D * g.es;
+      Vp = w.qkv + (size_t)2 * D * g.es;
+      ld = 3 * D;
+      dQ = bw.dqkv;
+      dK = bw.dqkv + (size_t)D * g.es;
+      dV = bw.dqkv + (size_t)2 * D * g.es;
+      ldd = 3 * D;
+    } else {
+      Qp = x_or_q;
+      Kp = k;
+      Vp = v;
+      ld = D;
+      dQ = dx_or_dq;
+      dK = dk;
+      dV = dv;
+      ldd = D;
+    }
+    AttnBwdArgs ab{{Qp, Kp, Vp, ld, w.hhat, D, w.lse, g.B, g.T, g.H, g.dh, g.L},
+                   bw.dHhat, bw.Drow, dQ, dK, dV, ldd};
+    if (use_attn_tc(g)) {
+      pr.begin("attn_bwd_tc");
+      e = attn_bwd_tc(lc, ab);
+    } else {
+      pr.begin("attn_bwd_simt");
+      e = attn_bwd_simt(lc, g.dtype, ab);
+    }
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "attention backward");
+  }
+  // Sec. 3.3 reversed: dX = dQKV W_qkv^T, dW_qkv = X^T dQKV.
+  if (g.from_x) {
+    EpiArgs ea;
+    ea.out = dx_or_dq;
+    ea.ldo = D;
+    e = run_gemm(lc, pr, "gemm_dx", g.dtype, g.dtype, n, D, 3 * D, bw.dqkv, 3 * D, 1, w_qkv, 1,
+                 3 * D, EPI_STORE, ea);
+    if (e != cudaSuccess) return cuda_fail(e, "dX");
+    e = weight_grad(lc, pr, "gemm_dw_qkv", g.dtype, g.dtype, D, 3 * D, g.n, x_or_q, D, bw.dqkv,
+                    3 * D, bw.part, dw_qkv);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_qkv");
+  }
+  return finish(p, s);
+}
+
+int bcmt_profile_read(const char** names, int* launches, double* ms, int cap) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (cudaDeviceSynchronize() != cudaSuccess) return -1;
+  std::vector<const char*> nm;
+  std::vector<int> cnt;
+  std::vector<double> tot;
+  for (auto& r : g_prof_recs) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) return -1;
+    size_t i = 0;
+    for (; i < nm.size(); ++i)
+      if (strcmp(nm[i], r.name) == 0) break;
+    if (i == nm.size()) {
+      nm.push_back(r.name);
+      cnt.push_back(0);
+      tot.push_back(0.0);
+    }
+    cnt[i] += 1;
+    tot[i] += t;
+  }
+  for (size_t i = 0; i < nm.size() && (int)i < cap; ++i) {
+    if (names) names[i] = nm[i];
+    if (launches) launches[i] = cnt[i];
+    if (ms) ms[i] = tot[i];
+  }
+  return (int)nm.size();
+}
+
+void bcmt_profile_reset(void) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof_recs.clear();
+  g_prof_pool_used = 0;
+}
+
+// ------------------------------------------------------------ test entry points
+int bcmt_test_set_tensor_cores(int gemm_on, int attn_on) {
+  g_use_tc_gemm = gemm_on != 0;
+  g_use_tc_attn = attn_on != 0;
+  return (gemm_tc_available() ? 1 : 0) | (attn_tc_supported(1, 64, 64) ? 2 : 0);
+}
+
+int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, const void* A, long sam,
+                   long sak, const void* B, long sbk, long sbn, void* C, long ldc, int splits,
+                   void* stream) {
+  unsigned* sp = status_ptr();
+  if (!sp) return -1;
+  Launch lc{static_cast<cudaStream_t>(stream), sp};
+  EpiArgs ea;
+  ea.out = C;
+  ea.ldo = ldc;
+  ea.split_stride = (long)M * ldc;
+  const EpiKind ek = splits > 1 ? EPI_PARTIAL : EPI_STORE;
+  cudaError_t e = impl == 1 ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
+                            : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek,
+                                        ea, splits);
+  if (e != cudaSuccess) {
+    fail(BCMT_ERR_CUDA, "test gemm: %s", cudaGetErrorString(e));
+    return -1;
+  }
+  return splits > 1 ? effective_splits(K, splits) : 1;
+}
+
+int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, const void* k,
+                   const void* v, long ld, void* o, float* lse, const void* dO, float* drow,
+                   void* dq, void* dk, void* dv, long ld_d, void* stream) {
+  if (check_params(p) != BCMT_OK) return -1;
+  unsigned* sp = status_ptr();
+  if (!sp) return -1;
+  Launch lc{static_cast<cudaStream_t>(stream), sp};
+  Geometry g(p);
+  AttnArgs aa{q, k, v, ld, o, g.D, lse, g.B, g.T, g.H, g.dh, g.L};
+  cudaError_t e;
+  if (!backward) {
+    e = impl == 1 ? attn_fwd_tc(lc, aa) : attn_fwd_simt(lc, g.dtype, aa);
+  } else {
+    AttnBwdArgs ab{aa, dO, drow, dq, dk, dv, ld_d};
+    e = impl == 1 ? attn_bwd_tc(lc, ab) : attn_bwd_simt(lc, g.dtype, ab);
+  }
+  if (e != cudaSuccess) {
+    fail(BCMT_ERR_CUDA, "test attention: %s", cudaGetErrorString(e));
+    return -1;
+  }
+  return 0;
+}
+
+}  // extern "C"

@@ -1,0 +1,78 @@
+// GEMM epilogues shared by the SIMT and tcgen05 GEMMs.  A GEMM hands each
+// epilogue a run of n consecutive accumulator values of one output row:
+// (row, col .. col+n-1), n a multiple of 4 and col a multiple of 4, plus the
+// K-split index z.  Row m is token (b, t) = (m / T, m % T) of block t / L.
+#pragma once
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace bcmt {
+
+template <class TO>
+struct EpiStoreF {
+  TO* out;
+  long ldo;
+  long split_stride;
+  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int z) const {
+    TO* p = out + (long)z * split_stride + (long)row * ldo + col;
+    for (int j = 0; j < n; j += 4) store4(p + j, v + j);
+  }
+};
+
+// Sec. 3.8: G = sigmoid(H W_g), Y = H + G * M_tokens, M_tokens row = Cmem[b, t/L].
+template <class T>
+struct EpiGateInjectF {
+  const T* H;
+  const float* Cmem;
+  T* G;
+  T* Y;
+  int Tlen, L, Nb, D;
+  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
+    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
+    const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
+    const long o = (long)row * D + col;
+    for (int j = 0; j < n; j += 4) {
+      float h[4], c[4], g[4], y[4];
+      load4(H + o + j, h);
+      load4(cm + j, c);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        g[e] = sigmoidf_(v[j + e]);
+        y[e] = h[e] + g[e] * c[e];
+      }
+      store4(G + o + j, g);
+      store4(Y + o + j, y);
+    }
+  }
+};
+
+// Backward into H: dH = dU W_g^T (the accumulator) + dY (identity path of
+// Y = H + ...) + alpha_t dS_blk (pooling S = H^T alpha) + ds_t w_p (scores).
+template <class T>
+struct EpiDHF {
+  const T* dY;
+  const float* alpha;
+  const float* dS;
+  const float* ds;
+  const T* w_p;
+  T* out;
+  int Tlen, L, Nb, D;
+  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
+    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
+    const float* dsb = dS + ((long)b * Nb + blk) * D + col;
+    const float at = alpha[row], st = ds[row];
+    const long o = (long)row * D + col;
+    for (int j = 0; j < n; j += 4) {
+      float dy[4], sv[4], wp[4], r[4];
+      load4(dY + o + j, dy);
+      load4(dsb + j, sv);
+      load4(w_p + col + j, wp);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) r[e] = v[j + e] + dy[e] + at * sv[e] + st * wp[e];
+      store4(out + o + j, r);
+    }
+  }
+};
+
+}  // namespace bcmt

@@ -1,0 +1,376 @@
+// Dense GEMMs of the BCMT layer: the Q/K/V, W_O, W_g and W_m projections of
+// Sec. 3.3-3.8 and their backward products.
+//
+//  * gemm_tc: bf16 inputs on the tcgen05 tensor cores.  One CTA computes a
+//    128 x BN output tile with the fp32 accumulator in TMEM.  Warp 0 (one lane)
+//    streams 64-deep K slices of A and B into a STAGES-deep shared-memory ring
+//    with TMA (128-byte swizzle); warp 1 (one lane) issues tcgen05.mma and
+//    releases each slot with tcgen05.commit; then all four warps read the
+//    accumulator back with tcgen05.ld (thread = output row) and run the fused
+//    epilogue.  Every mbarrier wait is bounded.
+//  * gemm_simt: true-fp32 FMA, used for fp32 tensors (a TF32 tensor-core
+//    product cannot meet a 1e-4 absolute error bound).
+#include <stdio.h>
+
+#include "common.cuh"
+#include "epilogues.cuh"
+#include "internal.h"
+#include "tc.cuh"
+#include "tmap.h"
+
+namespace bcmt {
+
+int effective_splits(int K, int splits) {
+  const int nkb = (K + 63) / 64;
+  if (splits < 1) splits = 1;
+  if (splits > nkb) splits = nkb;
+  const int kps = (nkb + splits - 1) / splits;
+  return (nkb + kps - 1) / kps;
+}
+
+// ======================================================================== SIMT
+template <class TI, class Epi>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, const TI* __restrict__ A,
+                                                        long sam, long sak,
+                                                        const TI* __restrict__ B, long sbk,
+                                                        long sbn, Epi epi, int kps) {
+  __shared__ float As[16][64 + 4];
+  __shared__ float Bs[16][64 + 4];
+  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64, z = blockIdx.z;
+  const int kb = z * kps, ke = min(K, kb + kps);
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+  for (int k0 = kb; k0 < ke; k0 += 16) {
+    for (int e = tid; e < 16 * 64; e += 256) {
+      int mm, ka;
+      if (sak == 1) { ka = e % 16; mm = e / 16; } else { mm = e % 64; ka = e / 64; }
+      const int m = m0 + mm, k = k0 + ka;
+      As[ka][mm] = (m < M && k < ke) ? to_f(A[(long)m * sam + (long)k * sak]) : 0.f;
+      int nn, kb2;
+      if (sbn == 1) { nn = e % 64; kb2 = e / 64; } else { kb2 = e % 16; nn = e / 16; }
+      const int n = n0 + nn, k2 = k0 + kb2;
+      Bs[kb2][nn] = (n < N && k2 < ke) ? to_f(B[(long)k2 * sbk + (long)n * sbn]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  const int col = n0 + tx * 4;
+  if (col >= N) return;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = m0 + ty * 4 + i;
+    if (row < M) epi(row, col, acc[i], 4, z);
+  }
+}
+
+template <class TI, class Epi>
+static cudaError_t simt_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                               long sak, const void* B, long sbk, long sbn, const Epi& epi,
+                               int splits) {
+  const int nkb = (K + 63) / 64;
+  const int kps = ((nkb + splits - 1) / splits) * 64;
+  dim3 grid((N + 63) / 64, (M + 63) / 64, splits);
+  gemm_simt_kernel<TI, Epi><<<grid, 256, 0, lc.stream>>>(
+      M, N, K, static_cast<const TI*>(A), sam, sak, static_cast<const TI*>(B), sbk, sbn, epi, kps);
+  return cudaGetLastError();
+}
+
+template <class TI>
+static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
+                              long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                              const EpiArgs& ea, int splits) {
+  switch (epi) {
+    case EPI_STORE:
+      if (dtype_out == 0)
+        return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                               EpiStoreF<float>{(float*)ea.out, ea.ldo, 0}, 1);
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiStoreF<bf16>{(bf16*)ea.out, ea.ldo, 0}, 1);
+    case EPI_PARTIAL:
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiStoreF<float>{(float*)ea.out, ea.ldo, ea.split_stride}, splits);
+    case EPI_GATE_INJECT:
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiGateInjectF<TI>{(const TI*)ea.H, ea.Cmem, (TI*)ea.G, (TI*)ea.Y,
+                                                ea.T, ea.L, ea.Nb, ea.D},
+                             1);
+    case EPI_DH:
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiDHF<TI>{(const TI*)ea.dY, ea.alpha, ea.dS, ea.ds,
+                                        (const TI*)ea.w_p, (TI*)ea.out, ea.T, ea.L, ea.Nb, ea.D},
+                             1);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t gemm_simt(const Launch& lc, int dtype, int dtype_out, int M, int N, int K,
+                      const void* A, long sam, long sak, const void* B, long sbk, long sbn,
+                      EpiKind epi, const EpiArgs& ea, int splits) {
+  if (N % 64 != 0) return cudaErrorInvalidValue;
+  splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
+  if (dtype == 0)
+    return simt_typed<float>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  return simt_typed<bf16>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+}
+
+// ===================================================================== tcgen05
+namespace {
+constexpr int kBM = 128, kBK = 64;
+
+template <int BN, int STAGES>
+struct TcCfg {
+  static constexpr int A_BYTES = kBM * kBK * 2;
+  static constexpr int B_BYTES = BN * kBK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+};
+}  // namespace
+
+template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
+__global__ void __launch_bounds__(128, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+                   int M, int N, int kps, int nkb, Epi epi, unsigned* status) {
+  using Cfg = TcCfg<BN, STAGES>;
+  if (tc::status_failed(status)) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* done = empty + STAGES;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(done + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * BN, z = blockIdx.z;
+  const int kb0 = z * kps;
+  const int nk = min(nkb, kb0 + kps) - kb0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&empty[s], 1);
+    }
+    tc::mbar_init(done, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, BN);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+
+  if (warp == 0 && lane == 0) {
+    // ---- TMA producer
+    int issued = 0;
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % STAGES;
+      if (i >= STAGES && !tc::mbar_wait(&empty[s], ((i / STAGES) - 1) & 1, status)) break;
+      uint8_t* sa = smem + s * Cfg::STAGE_BYTES;
+      uint8_t* sb = sa + Cfg::A_BYTES;
+      tc::mbar_arrive_expect_tx(&full[s], Cfg::STAGE_BYTES);
+      const int k0 = (kb0 + i) * kBK;
+      if (!A_MN) {
+        tc::tma_load_2d(sa, &mA, &full[s], k0, m0);
+      } else {
+        tc::tma_load_2d(sa, &mA, &full[s], m0, k0);
+        tc::tma_load_2d(sa + 8192, &mA, &full[s], m0 + 64, k0);
+      }
+      if (!B_MN) {
+        tc::tma_load_2d(sb, &mB, &full[s], k0, n0);
+      } else {
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j) tc::tma_load_2d(sb + j * 8192, &mB, &full[s], n0 + 64 * j, k0);
+      }
+      issued = i + 1;
+    }
+    // No copy may still be in flight when the CTA exits.
+    for (int i = (issued > STAGES ? issued - STAGES : 0); i < issued; ++i)
+      tc::mbar_wait(&full[i % STAGES], (i / STAGES) & 1, status);
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer
+    constexpr uint32_t idesc = tc::idesc_bf16(kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % STAGES;
+      if (!tc::mbar_wait(&full[s], (i / STAGES) & 1, status)) break;
+      tc::fence_after_sync();
+      const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE_BYTES);
+      const uint32_t sb = sa + Cfg::A_BYTES;
+#pragma unroll
+      for (int kk = 0; kk < kBK / 16; ++kk) {
+        const uint64_t ad = A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024) : tc::sdesc(sa + kk * 32, 16, 1024);
+        const uint64_t bd = B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024) : tc::sdesc(sb + kk * 32, 16, 1024);
+        tc::mma_bf16(tmem, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
+      }
+      tc::mma_commit(&empty[s]);
+    }
+    tc::mma_commit(done);
+  }
+  __syncwarp();
+
+  // ---- epilogue: thread = output row, 32 columns per TMEM load
+  const bool ok = tc::mbar_wait(done, 0, status) && nk > 0;
+  tc::fence_after_sync();
+  const int row = m0 + warp * 32 + lane;
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    float v[32];
+    tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c, v);
+    if (ok && row < M && n0 + c < N) epi(row, n0 + c, v, 32, z);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, BN);
+}
+
+namespace {
+bool g_tc_ok = true;
+}
+
+bool gemm_tc_available() { return g_tc_ok && tmap_encoder() != nullptr; }
+
+template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
+static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                             long sak, const void* B, long sbk, long sbn, const Epi& epi,
+                             int splits) {
+  using Cfg = TcCfg<BN, STAGES>;
+  CUtensorMap mA, mB;
+  if (!A_MN) {
+    uint64_t d[2] = {(uint64_t)K, (uint64_t)M}, st[1] = {(uint64_t)sam * 2};
+    uint32_t box[2] = {64, 128};
+    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+  } else {
+    uint64_t d[2] = {(uint64_t)M, (uint64_t)K}, st[1] = {(uint64_t)sak * 2};
+    uint32_t box[2] = {64, 64};
+    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+  }
+  if (!B_MN) {
+    uint64_t d[2] = {(uint64_t)K, (uint64_t)N}, st[1] = {(uint64_t)sbn * 2};
+    uint32_t box[2] = {64, (uint32_t)BN};
+    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+  } else {
+    uint64_t d[2] = {(uint64_t)N, (uint64_t)K}, st[1] = {(uint64_t)sbk * 2};
+    uint32_t box[2] = {64, 64};
+    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+  }
+  const int nkb = (K + kBK - 1) / kBK;
+  const int kps = (nkb + splits - 1) / splits;
+  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid((N + BN - 1) / BN, (M + kBM - 1) / kBM, splits);
+  kern<<<grid, 128, Cfg::SMEM, lc.stream>>>(mA, mB, M, N, kps, nkb, epi, lc.status);
+  return cudaGetLastError();
+}
+
+template <bool A_MN, bool B_MN>
+static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
+                          long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                          const EpiArgs& ea, int splits) {
+  constexpr int BN = 128, ST = 4;
+  switch (epi) {
+    case EPI_STORE:
+      if (dtype_out == 0)
+        return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                             EpiStoreF<float>{(float*)ea.out, ea.ldo, 0}, 1);
+      return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                           EpiStoreF<bf16>{(bf16*)ea.out, ea.ldo, 0}, 1);
+    case EPI_PARTIAL:
+      return tc_launch<BN, ST, A_MN, B_MN>(
+          lc, M, N, K, A, sam, sak, B, sbk, sbn,
+          EpiStoreF<float>{(float*)ea.out, ea.ldo, ea.split_stride}, splits);
+    case EPI_GATE_INJECT:
+      return tc_launch<BN, ST, A_MN, B_MN>(
+          lc, M, N, K, A, sam, sak, B, sbk, sbn,
+          EpiGateInjectF<bf16>{(const bf16*)ea.H, ea.Cmem, (bf16*)ea.G, (bf16*)ea.Y, ea.T, ea.L,
+                               ea.Nb, ea.D},
+          1);
+    case EPI_DH:
+      return tc_launch<BN, ST, A_MN, B_MN>(
+          lc, M, N, K, A, sam, sak, B, sbk, sbn,
+          EpiDHF<bf16>{(const bf16*)ea.dY, ea.alpha, ea.dS, ea.ds, (const bf16*)ea.w_p,
+                       (bf16*)ea.out, ea.T, ea.L, ea.Nb, ea.D},
+          1);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
+                    long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
+                    int splits) {
+  if (N % 64 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
+  splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
+  const bool a_k = (sak == 1), a_m = (sam == 1) && !a_k;
+  const bool b_k = (sbk == 1), b_n = (sbn == 1) && !b_k;
+  if (a_k && b_n) return tc_epi<false, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_k && b_k) return tc_epi<false, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_m && b_n) return tc_epi<true, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_m && b_k) return tc_epi<true, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  return cudaErrorNotSupported;
+}
+
+cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K, const void* A,
+                 long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                 const EpiArgs& ea, int splits, const char** kernel_name) {
+  if (dtype == 1 && gemm_tc_available()) {
+    if (kernel_name) *kernel_name = "gemm_tc";
+    cudaError_t e = gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+    if (e != cudaErrorNotSupported) return e;
+  }
+  if (kernel_name) *kernel_name = "gemm_simt";
+  return gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+}
+
+// ============================================================ split reduction
+template <class TO>
+__global__ void reduce_splits_kernel(const float* __restrict__ part, int splits, long count,
+                                     TO* __restrict__ out) {
+  const long i4 = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (i4 >= count) return;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int s = 0; s < splits; ++s) {
+    float v[4];
+    load4(part + (long)s * count + i4, v);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[e] += v[e];
+  }
+  store4(out + i4, acc);
+}
+
+cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long count,
+                          int dtype_out, void* out) {
+  if (count % 4 != 0) return cudaErrorInvalidValue;
+  const long n4 = count / 4;
+  const int threads = 256;
+  const unsigned blocks = (unsigned)((n4 + threads - 1) / threads);
+  if (dtype_out == 0)
+    reduce_splits_kernel<float><<<blocks, threads, 0, lc.stream>>>(part, splits, count, (float*)out);
+  else
+    reduce_splits_kernel<bf16><<<blocks, threads, 0, lc.stream>>>(part, splits, count, (bf16*)out);
+  return cudaGetLastError();
+}
+
+}  // namespace bcmt

@@ -1,0 +1,130 @@
+// Host-side interface between the C-ABI layer (bcmt_api.cu) and the kernel
+// translation units.  Nothing here is exported from the shared library.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+
+namespace bcmt {
+
+// Where and how a kernel is launched.
+struct Launch {
+  cudaStream_t stream;
+  unsigned* status;  // device status word (bounded waits OR bits into it)
+};
+
+// ----------------------------------------------------------------- GEMM
+// C[M,N] = A[M,K] B[K,N] with fp32 accumulation, element (m,k) of A at
+// A[m*sam + k*sak] and (k,n) of B at B[k*sbk + n*sbn].  The epilogue decides
+// what is stored.  N must be a multiple of 64.
+enum EpiKind {
+  EPI_STORE = 0,        // out[m*ldo + n] = acc                       (out dtype = dtype_out)
+  EPI_PARTIAL = 1,      // out(fp32)[z*split_stride + m*ldo + n] = acc of K-split z
+  EPI_GATE_INJECT = 2,  // G = sigmoid(acc); Y = H + G * Cmem[b, blk(t)]      (Sec. 3.8)
+  EPI_DH = 3,           // dH = acc + dY + alpha_t dS[b, blk(t)] + ds_t w_p   (backward)
+};
+
+struct EpiArgs {
+  void* out = nullptr;
+  long ldo = 0;
+  long split_stride = 0;
+  // EPI_GATE_INJECT
+  const void* H = nullptr;
+  const float* Cmem = nullptr;
+  void* G = nullptr;
+  void* Y = nullptr;
+  // EPI_DH
+  const void* dY = nullptr;
+  const float* alpha = nullptr;
+  const float* dS = nullptr;
+  const float* ds = nullptr;
+  const void* w_p = nullptr;
+  // token geometry: row m = b*T + t, block blk(t) = t / L, Nb blocks, width D
+  int T = 1, L = 1, Nb = 1, D = 0;
+};
+
+// Number of non-empty K-splits when K (in 64-deep slices) is cut into
+// `splits` equal ranges.
+int effective_splits(int K, int splits);
+
+// dtype: 0 fp32, 1 bf16 (inputs A and B); dtype_out applies to EPI_STORE.
+// splits > 1 splits K into `splits` contiguous ranges (only with EPI_PARTIAL).
+cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K, const void* A,
+                 long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                 const EpiArgs& ea, int splits, const char** kernel_name);
+
+// SIMT GEMM (true fp32 FMA); used for fp32 tensors and for small problems.
+cudaError_t gemm_simt(const Launch& lc, int dtype, int dtype_out, int M, int N, int K,
+                      const void* A, long sam, long sak, const void* B, long sbk, long sbn,
+                      EpiKind epi, const EpiArgs& ea, int splits);
+
+// tcgen05 GEMM (bf16 inputs, fp32 TMEM accumulation).  A must be either
+// K-major (sak == 1) or M-major (sam == 1), B either K-major (sbk == 1) or
+// N-major (sbn == 1).  Returns cudaErrorNotSupported for other layouts.
+cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
+                    long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
+                    int splits);
+bool gemm_tc_available();
+
+// Sum of `splits` fp32 partial buffers of `count` elements each, in split
+// order, stored in dtype_out.
+cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long count, int dtype_out,
+                          void* out);
+
+// ------------------------------------------------------------ attention
+// Intra-block causal attention (Sec. 3.3).  Q, K, V rows of token (b,t) start
+// at X + (b*T + t) * ld_qkv + head*dh.  O is [B*T, ld_o] (Concat of heads),
+// lse [B, H, T] fp32 (natural-log sum-exp of the scaled scores per row).
+struct AttnArgs {
+  const void* Q;
+  const void* K;
+  const void* V;
+  long ld_qkv;
+  void* O;
+  long ld_o;
+  float* lse;
+  int B, T, H, dh, L;
+};
+cudaError_t attn_fwd_simt(const Launch& lc, int dtype, const AttnArgs& a);
+// Backward: dO = dL/dO [B*T, ld_o]; Drow scratch [B, H, T] fp32; writes dQ,
+// dK, dV with the row stride ld_dqkv.
+struct AttnBwdArgs {
+  AttnArgs f;
+  const void* dO;
+  float* Drow;
+  void* dQ;
+  void* dK;
+  void* dV;
+  long ld_dqkv;
+};
+cudaError_t attn_bwd_simt(const Launch& lc, int dtype, const AttnBwdArgs& a);
+
+cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a);
+cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
+bool attn_tc_supported(int dtype, int dh, int L);
+
+// ------------------------------------------------ summary, memory, gate
+// Sec. 3.4: per block, s = H w_p, alpha = softmax(s), S = H^T alpha.
+cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const void* w_p, float* alpha,
+                        float* S, int B, int T, int D, int L);
+// Sec. 3.5: M = normalised decayed scan of S over blocks, Z its denominator
+// [Nb, D], C[b,0] = 0, C[b,i] = M[b,i-1] W_m.
+cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
+                       const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D);
+// Backward of the gate and injection: dU = dY*C*G*(1-G); dP[b,i-1] = sum over
+// block i of dY*G; dP[b,Nb-1] = 0.
+cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
+                     void* dU, float* dP, int B, int T, int D, int L);
+// Backward of the memory: dM = dP W_m^T, dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i.
+cudaError_t memory_bwd(const Launch& lc, int dtype, const float* dP, const float* decay,
+                       const float* Z, const void* w_m, float* dS, int B, int Nb, int D);
+// Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
+// dwp_part[b*Nb+i] = sum_t ds_t H_t.
+cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
+                        const float* dS, float* ds, float* dwp_part, int B, int T, int D, int L);
+// Column sums of an fp32 [rows, cols] matrix in row order, stored in dtype_out.
+cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, int dtype_out,
+                        void* out);
+cudaError_t fill_zero(const Launch& lc, void* p, size_t bytes);
+
+}  // namespace bcmt

@@ -1,0 +1,136 @@
+"""Parity of the whole CUDA mixer (forward and backward, through the C ABI)
+with the float64 oracle on the same seeded inputs.
+
+Bar: fp32 max abs error <= 1e-4; bf16 max|gpu - oracle| / max|oracle| <= 2e-2,
+for Y and every gradient.  Small cases span several tiles and ragged tails;
+the named workloads run at their full sizes in the launch configuration the
+benchmark times."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_13578_gb300.inputs import WORKLOADS, Workload, make_inputs
+from tests.helpers import (GRAD_NAMES_QKV, GRAD_NAMES_X, assert_close, gpu_run, oracle_run,
+                           to_device)
+
+pytestmark = pytest.mark.gpu
+
+
+def W(B, T, D, H, L, dtype, **kw):
+    return Workload(name=f"b{B}_t{T}_d{D}_h{H}_l{L}_{dtype}", B=B, T=T, D=D, H=H, L=L,
+                    dtype=dtype, decay=kw.pop("decay", (0.5, 0.99)), **kw)
+
+
+SMALL = [
+    W(2, 100, 128, 4, 16, "fp32"),
+    W(1, 256, 128, 4, 32, "fp32"),
+    W(2, 77, 64, 2, 10, "fp32"),
+    W(2, 64, 128, 2, 64, "fp32", decay=(0.0, 0.0)),
+    W(1, 50, 128, 4, 64, "fp32"),                      # one ragged block: no memory
+    W(2, 256, 128, 2, 64, "bf16"),
+    W(2, 200, 256, 4, 32, "bf16"),
+    W(1, 384, 128, 2, 128, "bf16"),
+    W(2, 130, 128, 2, 16, "bf16"),
+    W(1, 300, 128, 2, 256, "bf16"),
+    W(2, 150, 128, 2, 48, "bf16"),
+    W(1, 96, 192, 2, 32, "bf16"),                       # dh = 96 -> SIMT attention
+    W(2, 256, 128, 2, 64, "bf16", decay=(0.0, 0.0)),
+]
+VARIANTS = [
+    W(2, 100, 128, 4, 16, "fp32", input_is_x=False),
+    W(2, 200, 256, 4, 32, "bf16", input_is_x=False),
+    W(2, 100, 128, 4, 16, "fp32", honly=True),
+    W(2, 200, 256, 4, 32, "bf16", honly=True),
+]
+
+
+def _check(w: Workload, backward=True, batch=None):
+    t = make_inputs(w)
+    y, g = gpu_run(w, to_device(t), backward)
+    fw, gr = oracle_run(w, t, backward, batch=batch)
+    if batch is not None:
+        y = y[batch]
+    assert_close("Y", y, fw["Y"], w.dtype)
+    if backward:
+        names = GRAD_NAMES_X if w.input_is_x else GRAD_NAMES_QKV
+        for n in names:
+            got = g[n]
+            if batch is not None:
+                if n in ("dx", "dq", "dk", "dv"):
+                    got = got[batch]
+                else:
+                    continue
+            if w.honly and n in ("dw_p", "dw_m", "dw_g"):
+                assert torch.count_nonzero(got).item() == 0
+                continue
+            assert_close(n, got, gr[n], w.dtype)
+
+
+@pytest.mark.parametrize("w", SMALL + VARIANTS, ids=lambda w: w.name + ("_qkv" if not w.input_is_x else "") + ("_honly" if w.honly else ""))
+def test_layer_small(cuda_ok, w):
+    _check(w)
+
+
+def test_tensor_core_and_simt_paths_agree(cuda_ok):
+    """The same bf16 layer through the tcgen05 kernels and the SIMT kernels."""
+    from paper_2608_13578_gb300 import bcmt as C
+    w = W(2, 256, 128, 2, 64, "bf16")
+    t = to_device(make_inputs(w))
+    try:
+        C.bcmt_test_set_tensor_cores(False, False)
+        y0, g0 = gpu_run(w, t)
+    finally:
+        C.bcmt_test_set_tensor_cores(True, True)
+    y1, g1 = gpu_run(w, t)
+    scale = y0.float().abs().max().item()
+    assert (y0.float() - y1.float()).abs().max().item() / scale < 2e-2
+    for n in GRAD_NAMES_X:
+        s = g0[n].float().abs().max().item()
+        assert (g0[n].float() - g1[n].float()).abs().max().item() / s < 2e-2, n
+
+
+def test_deterministic(cuda_ok):
+    w = WORKLOADS["fwdbwd_bf16_b8_t1024_l64_d512_h8"].replace(B=2)
+    t = to_device(make_inputs(w))
+    y0, g0 = gpu_run(w, t)
+    y1, g1 = gpu_run(w, t)
+    assert torch.equal(y0, y1)
+    for n in GRAD_NAMES_X:
+        assert torch.equal(g0[n], g1[n]), n
+
+
+def test_causality_bitwise(cuda_ok):
+    """Sec. 3.6 on the GPU: perturbing token t leaves every output before t
+    bitwise unchanged."""
+    w = W(1, 256, 128, 2, 64, "bf16")
+    t = make_inputs(w)
+    y0, _ = gpu_run(w, to_device(t), backward=False)
+    for tok in (5, 64, 130, 255):
+        t2 = dict(t)
+        x = t["x"].clone()
+        x[0, tok] += 1.0
+        t2["x"] = x
+        y1, _ = gpu_run(w, to_device(t2), backward=False)
+        assert torch.equal(y0[0, :tok], y1[0, :tok]), tok
+        assert not torch.equal(y0[0, tok], y1[0, tok])
+
+
+# ------------------------------------------------- the named workloads, full size
+@pytest.mark.parametrize("name", ["fwd_fp32_b1_t256_l32_d128_h4", "fwdbwd_bf16_b8_t1024_l64_d512_h8"])
+def test_workload_full(cuda_ok, name):
+    w = WORKLOADS[name]
+    _check(w, backward=True)
+
+
+@pytest.mark.parametrize("L", [32, 64, 128, 256])
+def test_block_size_sweep(cuda_ok, L):
+    _check(WORKLOADS[f"sweep_bf16_b16_t1024_l{L}_d768_h12"], backward=True)
+
+
+@pytest.mark.parametrize("T", [2048, 4096, 8192, 16384])
+def test_sequence_scaling(cuda_ok, T):
+    w = WORKLOADS[f"seqscale_bf16_b4_t{T}_l128_d1024_h16"]
+    # Full comparison at the shortest length; batch element 0 of Y and dX at the
+    # longer ones (the mixer is independent across the batch).
+    _check(w, backward=True, batch=None if T == 2048 else slice(0, 1))

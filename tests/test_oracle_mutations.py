@@ -19,20 +19,20 @@ SRC = open(bcmt_oracle.__file__).read()
 
 MUTATIONS = {
     "W_O transposed": ("Hloc[b, t0:t1] = Hhat[b, t0:t1] @ w_o", "Hloc[b, t0:t1] = Hhat[b, t0:t1] @ w_o.T"),
-    "Q projected with W_K": ("Qb = Xb @ w_qkv[:, 0:D]", "Qb = Xb @ w_qkv[:, D:2 * D]"),
+    "Q projected with W_K": ("W_Q = np.ascontiguousarray(w_qkv[:, 0:D])", "W_Q = np.ascontiguousarray(w_qkv[:, D:2 * D])"),
     "no 1/sqrt(d_h)": ("/ math.sqrt(d_h) + mask", "+ mask"),
     "mask lets one future key in": ("np.full((Li, Li), -np.inf), k=1)", "np.full((Li, Li), -np.inf), k=2)"),
     "memory not shifted": ("C[b, i] = P[b, i - 1]", "C[b, i] = P[b, i]"),
     "decay exponent off by one": ("wgt = a ** (i - j)", "wgt = a ** (i - j + 1)"),
     "memory not normalised": ("M[b, i] = num / den", "M[b, i] = num"),
     "W_g transposed": ("G[b] = _sigmoid(Hloc[b] @ w_g)", "G[b] = _sigmoid(Hloc[b] @ w_g.T)"),
-    "injection sign": ("Y[b, t] = Hloc[b, t] + G[b, t] * C[b, i]", "Y[b, t] = Hloc[b, t] - G[b, t] * C[b, i]"),
+    "injection sign": ("Y[b, t0:t1] = Hloc[b, t0:t1] + G[b, t0:t1]", "Y[b, t0:t1] = Hloc[b, t0:t1] - G[b, t0:t1]"),
     "summary pools W_p-weighted tokens unnormalised": ("S[b, i] = Hb.T @ ab", "S[b, i] = Hb.T @ np.exp(sb)"),
     "bwd: softmax Jacobian term dropped": ("ds = ab * (g - np.dot(ab, g))", "ds = ab * g"),
     "bwd: reverse scan divides by Z_j": ("dS[j] += (a ** (i - j)) * dM[i] / Z[i]", "dS[j] += (a ** (i - j)) * dM[i] / Z[j]"),
     "bwd: shift not reversed": ("dP[i] = dC[i + 1]", "dP[i] = dC[i]"),
     "bwd: dK with untransposed scores": ("dK[b, t0:t1, cols] = dScore.T @ Qb", "dK[b, t0:t1, cols] = dScore @ Qb"),
-    "bwd: gate derivative": ("dU[t] = dG * G[b, t] * (1.0 - G[b, t])", "dU[t] = dG * G[b, t]"),
+    "bwd: gate derivative": ("dU[t0:t1] = dG * G[b, t0:t1] * (1.0 - G[b, t0:t1])", "dU[t0:t1] = dG * G[b, t0:t1]"),
 }
 
 PINS = [
