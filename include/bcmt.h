@@ -133,6 +133,33 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                           void* scratch, void* dx_or_dq, void* dk, void* dv, void* dw_qkv,
                           void* dw_o, void* dw_p, void* dw_m, void* dw_g, void* stream);
 
+/* Allocation-free backward of the intra-block attention alone (the SIMT
+ * kernels of the layer's backward; the paper has no counterpart -- it is an
+ * interface for callers that cannot call cudaMalloc, such as a host framework
+ * that owns all device memory and hands this library only input and output
+ * buffers, or a latency-critical path where an allocation's implicit device
+ * synchronisation is not acceptable).  It computes dq, dk, dv from the
+ * forward's q, k, v (row stride ld, head h at column h*D/H), its output o
+ * [B*T, D] and log-sum-exp lse [B,H,T] fp32, and the upstream gradient dO
+ * [B*T, D]; dq, dk, dv are written with row stride ld_d.  Shapes as in *p
+ * (B, T, D, H, L, dtype; input_is_x and flags other than BCMT_FLAG_CHECK are
+ * ignored).
+ *
+ * Its one scratch buffer (one fp32 per batch, head and token) is a device
+ * array inside the library: 4 MiB, allocated on every GPU that loads the
+ * library and held until the process exits.  B*H*T must not exceed 1048576;
+ * larger shapes are rejected with BCMT_ERR_SHAPE before anything is launched.
+ * The first call on a device looks up that array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  All calls share the array and it keeps the last call's contents:
+ * calls that overlap on the GPU (other streams, other threads) race on it, so
+ * serialise them.  Nothing is allocated: no cudaMalloc, cudaFree or
+ * allocating library routine is called. */
+bcmt_status bcmt_attention_backward_noalloc(const bcmt_params* p, const void* q, const void* k,
+                                            const void* v, long ld, const void* o,
+                                            const float* lse, const void* dO, void* dq, void* dk,
+                                            void* dv, long ld_d, void* stream);
+
 /* Reads and clears the device status word of the current device after
  * synchronising `stream`: BCMT_OK, or BCMT_ERR_TIMEOUT if any bounded
  * device-side wait has expired since the last read. */

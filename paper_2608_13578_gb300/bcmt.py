@@ -72,6 +72,9 @@ def _load():
     lib.bcmt_profile_read.restype = ctypes.c_int
     lib.bcmt_profile_reset.argtypes = []
     lib.bcmt_profile_reset.restype = None
+    lib.bcmt_attention_backward_noalloc.argtypes = [_P, _VP, _VP, _VP, ctypes.c_long, _VP, _VP,
+                                                    _VP, _VP, _VP, _VP, ctypes.c_long, _VP]
+    lib.bcmt_attention_backward_noalloc.restype = ctypes.c_int
     lib.bcmt_test_set_tensor_cores.argtypes = [ctypes.c_int, ctypes.c_int]
     lib.bcmt_test_set_tensor_cores.restype = ctypes.c_int
     lib.bcmt_test_gemm.argtypes = [ctypes.c_int] * 6 + [_VP, ctypes.c_long, ctypes.c_long, _VP,
@@ -89,6 +92,7 @@ LIB = _load()
 # Symbols include/bcmt.h and include/bcmt_testing.h declare.
 EXPORTED = ("bcmt_workspace_size", "bcmt_scratch_size", "bcmt_forward", "bcmt_backward",
             "bcmt_device_status", "bcmt_last_error", "bcmt_profile_read", "bcmt_profile_reset",
+            "bcmt_attention_backward_noalloc",
             "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_attn")
 
 
@@ -144,6 +148,15 @@ def bcmt_backward(p: bcmt_params, dy, x_or_q, k, v, w_qkv, w_o, w_p, w_m, w_g, d
 
 def bcmt_device_status(stream=None) -> None:
     _check(LIB.bcmt_device_status(_stream(stream)))
+
+
+def bcmt_attention_backward_noalloc(p: bcmt_params, q, k, v, ld, o, lse, dO, dq, dk, dv, ld_d,
+                                    stream=None) -> None:
+    """Attention backward whose scratch is a device array inside the library
+    (for callers that cannot allocate device memory); see include/bcmt.h."""
+    _check(LIB.bcmt_attention_backward_noalloc(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), ld,
+                                               _ptr(o), _ptr(lse), _ptr(dO), _ptr(dq), _ptr(dk),
+                                               _ptr(dv), ld_d, _stream(stream)))
 
 
 def bcmt_profile_reset() -> None:

@@ -3,6 +3,8 @@
 // shapes the tensor-core kernel does not cover.  One warp per query row
 // (forward, dQ) or key row (dK, dV); each lane owns keys (scores) or channels
 // (outputs).  Deterministic: every sum runs in a fixed order.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -188,6 +190,48 @@ cudaError_t attn_fwd_simt(const Launch& lc, int dtype, const AttnArgs& a) {
 cudaError_t attn_bwd_simt(const Launch& lc, int dtype, const AttnBwdArgs& a) {
   if (a.f.dh > kMaxDh || a.f.L > kMaxL) return cudaErrorInvalidValue;
   return dtype == 0 ? bwd_typed<float>(lc, a) : bwd_typed<bf16>(lc, a);
+}
+
+// ------------------------------------------- allocation-free backward variant
+// The backward above needs one fp32 scratch value per (batch, head, token):
+// Drow = dO . O, written by the dQ kernel and read by the dK/dV kernel.  For
+// callers that cannot allocate device memory, this variant keeps that scratch
+// in a file-scope device array instead of caller memory.  It is allocated when
+// the library is loaded, once on every GPU that loads it, and held until the
+// process exits.  Every call shares it, so calls that overlap on the GPU (on
+// different streams, or from different threads) race on it.  The dQ kernel
+// writes every entry the dK/dV kernel reads, so nothing needs clearing between
+// calls even though the array keeps the last call's contents.
+static __device__ __align__(256) float g_noalloc_drow[kNoAllocDrowRows];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float* g_noalloc_ptr[kMaxDevices] = {};
+}  // namespace
+
+cudaError_t attn_bwd_simt_noalloc(const Launch& lc, int dtype, const AttnBwdArgs& a) {
+  if ((long long)a.f.B * a.f.H * a.f.T > kNoAllocDrowRows) return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  float* drow = nullptr;
+  {
+    // Set-up, once per device with that device current: the array's name is
+    // only a host-side stand-in, so look up its device address.
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_drow);
+      if (e != cudaSuccess) return e;
+      g_noalloc_ptr[dev] = static_cast<float*>(p);
+    }
+    drow = g_noalloc_ptr[dev];
+  }
+  AttnBwdArgs b = a;
+  b.Drow = drow;
+  return attn_bwd_simt(lc, dtype, b);
 }
 
 }  // namespace bcmt

@@ -568,6 +568,40 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   return finish(p, s);
 }
 
+bcmt_status bcmt_attention_backward_noalloc(const bcmt_params* p, const void* q, const void* k,
+                                            const void* v, long ld, const void* o,
+                                            const float* lse, const void* dO, void* dq, void* dk,
+                                            void* dv, long ld_d, void* stream) {
+  BCMT_TRY(check_params(p));
+  Geometry g(p);
+  BCMT_TRY(check_ptr(q, "q"));
+  BCMT_TRY(check_ptr(k, "k"));
+  BCMT_TRY(check_ptr(v, "v"));
+  BCMT_TRY(check_ptr(o, "o"));
+  BCMT_TRY(check_ptr(lse, "lse"));
+  BCMT_TRY(check_ptr(dO, "dO"));
+  BCMT_TRY(check_ptr(dq, "dq"));
+  BCMT_TRY(check_ptr(dk, "dk"));
+  BCMT_TRY(check_ptr(dv, "dv"));
+  if (ld < g.D || ld_d < g.D)
+    return fail(BCMT_ERR_ARG, "row strides ld = %ld and ld_d = %ld must be >= D = %d", ld, ld_d, g.D);
+  const long long rows = (long long)g.B * g.H * g.T;
+  if (rows > kNoAllocDrowRows)
+    return fail(BCMT_ERR_SHAPE,
+                "B*H*T = %lld exceeds the %lld rows of the built-in scratch of "
+                "bcmt_attention_backward_noalloc",
+                rows, kNoAllocDrowRows);
+  unsigned* sp = status_ptr();
+  if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
+  Launch lc{static_cast<cudaStream_t>(stream), sp};
+  AttnBwdArgs ab{{q, k, v, ld, const_cast<void*>(o), g.D, const_cast<float*>(lse), g.B, g.T, g.H,
+                  g.dh, g.L},
+                 dO, nullptr, dq, dk, dv, ld_d};
+  cudaError_t e = attn_bwd_simt_noalloc(lc, g.dtype, ab);
+  if (e != cudaSuccess) return cuda_fail(e, "allocation-free attention backward");
+  return finish(p, lc.stream);
+}
+
 int bcmt_profile_read(const char** names, int* launches, double* ms, int cap) {
   std::lock_guard<std::mutex> lk(g_prof_mu);
   if (cudaDeviceSynchronize() != cudaSuccess) return -1;

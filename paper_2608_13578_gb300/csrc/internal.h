@@ -98,6 +98,10 @@ struct AttnBwdArgs {
   long ld_dqkv;
 };
 cudaError_t attn_bwd_simt(const Launch& lc, int dtype, const AttnBwdArgs& a);
+// The same backward with its Drow scratch in a static device array of
+// kNoAllocDrowRows floats instead of a.Drow; B*H*T must not exceed it.
+constexpr long long kNoAllocDrowRows = 1ll << 20;
+cudaError_t attn_bwd_simt_noalloc(const Launch& lc, int dtype, const AttnBwdArgs& a);
 
 cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a);
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
