@@ -20,6 +20,46 @@ struct EpiStoreF {
   }
 };
 
+// Sec. 3.3 + 3.4: stores H = Concat(heads) W_O and, for the pooling scores
+// s = H w_p, one partial dot product per output row and run of n columns
+// (spart[(col / n) * n_rows + row]); the summary kernel adds them up.
+template <class TO>
+struct EpiStoreScoreF {
+  TO* out;
+  long ldo;
+  const TO* w_p;
+  float* spart;
+  long n_rows;
+  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
+    TO* p = out + (long)row * ldo + col;
+    float s = 0.f;
+    for (int j = 0; j < n; j += 4) {
+      float w[4];
+      load4(w_p + col + j, w);
+      // score from the stored (rounded) H, the value the summary pools
+      float h[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) h[e] = to_f(from_f<TO>(v[j + e]));
+      s += h[0] * w[0] + h[1] * w[1] + h[2] * w[2] + h[3] * w[3];
+      store4(p + j, v + j);
+    }
+    spart[(long)(col / n) * n_rows + row] = s;
+  }
+};
+
+// Sec. 3.5 shift: row m = b*Nb + i of M W_m becomes the memory row of block
+// i+1 of the same sequence; the last block's row is dropped.
+struct EpiShiftF {
+  float* out;
+  long ldo;
+  int Nb;
+  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
+    if ((row % Nb) + 1 >= Nb) return;
+    float* p = out + (long)(row + 1) * ldo + col;
+    for (int j = 0; j < n; j += 4) store4(p + j, v + j);
+  }
+};
+
 // Sec. 3.8: G = sigmoid(H W_g), Y = H + G * M_tokens, M_tokens row = Cmem[b, t/L].
 template <class T>
 struct EpiGateInjectF {

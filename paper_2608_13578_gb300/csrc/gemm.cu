@@ -111,6 +111,19 @@ static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int
                              EpiGateInjectF<TI>{(const TI*)ea.H, ea.Cmem, (TI*)ea.G, (TI*)ea.Y,
                                                 ea.T, ea.L, ea.Nb, ea.D},
                              1);
+    case EPI_STORE_SCORE:
+      if (dtype_out == 0)
+        return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                               EpiStoreScoreF<float>{(float*)ea.out, ea.ldo,
+                                                     (const float*)ea.w_p, ea.spart, M},
+                               1);
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo, (const bf16*)ea.w_p,
+                                                  ea.spart, M},
+                             1);
+    case EPI_SHIFT:
+      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                             EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
     case EPI_DH:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                              EpiDHF<TI>{(const TI*)ea.dY, ea.alpha, ea.dS, ea.ds,
@@ -308,6 +321,14 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
           EpiGateInjectF<bf16>{(const bf16*)ea.H, ea.Cmem, (bf16*)ea.G, (bf16*)ea.Y, ea.T, ea.L,
                                ea.Nb, ea.D},
           1);
+    case EPI_STORE_SCORE:
+      return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                           EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
+                                                                (const bf16*)ea.w_p, ea.spart, M},
+                                           1);
+    case EPI_SHIFT:
+      return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                           EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
     case EPI_DH:
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,

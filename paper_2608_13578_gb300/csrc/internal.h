@@ -22,6 +22,8 @@ enum EpiKind {
   EPI_PARTIAL = 1,      // out(fp32)[z*split_stride + m*ldo + n] = acc of K-split z
   EPI_GATE_INJECT = 2,  // G = sigmoid(acc); Y = H + G * Cmem[b, blk(t)]      (Sec. 3.8)
   EPI_DH = 3,           // dH = acc + dY + alpha_t dS[b, blk(t)] + ds_t w_p   (backward)
+  EPI_SHIFT = 4,        // out(fp32)[m+1] = acc for row m = b*Nb + i with i+1 < Nb (Sec. 3.5 shift)
+  EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
 };
 
 struct EpiArgs {
@@ -33,6 +35,8 @@ struct EpiArgs {
   const float* Cmem = nullptr;
   void* G = nullptr;
   void* Y = nullptr;
+  // EPI_STORE_SCORE: partial pooling scores, [D / n, M] fp32
+  float* spart = nullptr;
   // EPI_DH
   const void* dY = nullptr;
   const float* alpha = nullptr;
@@ -108,20 +112,23 @@ cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
 bool attn_tc_supported(int dtype, int dh, int L);
 
 // ------------------------------------------------ summary, memory, gate
-// Sec. 3.4: per block, s = H w_p, alpha = softmax(s), S = H^T alpha.
-cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const void* w_p, float* alpha,
-                        float* S, int B, int T, int D, int L);
-// Sec. 3.5: M = normalised decayed scan of S over blocks, Z its denominator
-// [Nb, D], C[b,0] = 0, C[b,i] = M[b,i-1] W_m.
-cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
-                       const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D);
+// Sec. 3.4: per block, s = H w_p (summed from npart partial dot products
+// spart[j * B*T + token]), alpha = softmax(s), S = H^T alpha.
+cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
+                        float* alpha, float* S, int B, int T, int D, int L);
+// Sec. 3.5: M = normalised decayed scan of S over blocks (fp32, plus a bf16
+// copy in Mb when non-null), Z its denominator [Nb, D], C[b, 0] = 0.  The
+// projection C[b, i+1] = M_i W_m is a GEMM with the EPI_SHIFT epilogue.
+cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
+                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D);
 // Backward of the gate and injection: dU = dY*C*G*(1-G); dP[b,i-1] = sum over
-// block i of dY*G; dP[b,Nb-1] = 0.
+// block i of dY*G (also as bf16 in dPb when non-null); dP[b,Nb-1] = 0.
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, int B, int T, int D, int L);
-// Backward of the memory: dM = dP W_m^T, dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i.
-cudaError_t memory_bwd(const Launch& lc, int dtype, const float* dP, const float* decay,
-                       const float* Z, const void* w_m, float* dS, int B, int Nb, int D);
+                     void* dU, float* dP, void* dPb, int B, int T, int D, int L);
+// Backward of the memory scan: dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i, given
+// dM = dP W_m^T.
+cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
+                            float* dS, int B, int Nb, int D);
 // Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
 // dwp_part[b*Nb+i] = sum_t ds_t H_t.
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,

@@ -15,28 +15,26 @@ constexpr int kMaxL = 1024;
 }
 
 // -------------------------------------------------------------- Sec. 3.4
-// One CTA per (block i, batch b): s_t = H_t . w_p; alpha = softmax(s) over the
-// block's tokens; S_i = sum_t alpha_t H_t.
+// One CTA per (block i, batch b, 256 channels).  The pooling scores
+// s_t = H_t . w_p arrive as npart partial dot products per token (written by
+// the W_O GEMM epilogue over disjoint column ranges) and are summed here in a
+// fixed order; alpha = softmax(s) over the block's tokens; S_i = sum_t alpha_t H_t
+// for this CTA's channels.
 template <class T>
 __global__ void __launch_bounds__(256)
-    summary_fwd_kernel(const T* __restrict__ Hm, const T* __restrict__ w_p,
-                       float* __restrict__ alpha, float* __restrict__ S, int Tlen, int D, int L) {
+    summary_fwd_kernel(const T* __restrict__ Hm, const float* __restrict__ spart, int npart,
+                       long n_tok, float* __restrict__ alpha, float* __restrict__ S, int Tlen,
+                       int D, int L) {
   __shared__ float sc[kMaxL];
   __shared__ float red[2];
   const int i = blockIdx.x, b = blockIdx.y, Nb = gridDim.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t0 = i * L, n = min(L, Tlen - t0);
-  const T* Hb = Hm + ((long)b * Tlen + t0) * D;
-  for (int r = warp; r < n; r += 8) {
-    float d = 0.f;
-    for (int c = lane * 4; c < D; c += 128) {
-      float h[4], w[4];
-      load4(Hb + (long)r * D + c, h);
-      load4(w_p + c, w);
-      d += h[0] * w[0] + h[1] * w[1] + h[2] * w[2] + h[3] * w[3];
-    }
-    d = warp_sum(d);
-    if (lane == 0) sc[r] = d;
+  const long row0 = (long)b * Tlen + t0;
+  for (int r = threadIdx.x; r < n; r += blockDim.x) {
+    float s = 0.f;
+    for (int j = 0; j < npart; ++j) s += spart[(long)j * n_tok + row0 + r];
+    sc[r] = s;
   }
   __syncthreads();
   if (warp == 0) {
@@ -52,118 +50,79 @@ __global__ void __launch_bounds__(256)
   const float mx = red[0], inv = red[1];
   for (int r = threadIdx.x; r < n; r += blockDim.x) {
     const float a = expf(sc[r] - mx) * inv;
-    alpha[(long)b * Tlen + t0 + r] = a;
+    if (blockIdx.z == 0) alpha[row0 + r] = a;
     sc[r] = a;
   }
   __syncthreads();
-  for (int c = threadIdx.x * 4; c < D; c += blockDim.x * 4) {
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int r = 0; r < n; ++r) {
-      float h[4];
-      load4(Hb + (long)r * D + c, h);
-      const float a = sc[r];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[e] = fmaf(a, h[e], acc[e]);
-    }
-    store4(S + ((long)b * Nb + i) * D + c, acc);
+  const int c = blockIdx.z * blockDim.x + threadIdx.x;
+  if (c >= D) return;
+  const T* Hc = Hm + row0 * D + c;
+  float acc0 = 0.f, acc1 = 0.f;
+  int r = 0;
+  for (; r + 1 < n; r += 2) {
+    acc0 = fmaf(sc[r], to_f(Hc[(long)r * D]), acc0);
+    acc1 = fmaf(sc[r + 1], to_f(Hc[(long)(r + 1) * D]), acc1);
   }
+  if (r < n) acc0 = fmaf(sc[r], to_f(Hc[(long)r * D]), acc0);
+  S[((long)b * Nb + i) * D + c] = acc0 + acc1;
 }
 
-cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const void* w_p, float* alpha,
-                        float* S, int B, int T, int D, int L) {
+cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
+                        float* alpha, float* S, int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
-  dim3 grid(Nb, B);
+  dim3 grid(Nb, B, (D + 255) / 256);
+  const long n_tok = (long)B * T;
   if (dtype == 0)
-    summary_fwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)Hm, (const float*)w_p,
+    summary_fwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)Hm, spart, npart, n_tok,
                                                            alpha, S, T, D, L);
   else
-    summary_fwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)Hm, (const bf16*)w_p, alpha,
-                                                          S, T, D, L);
+    summary_fwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)Hm, spart, npart, n_tok,
+                                                          alpha, S, T, D, L);
   return cudaGetLastError();
 }
 
 // -------------------------------------------------------------- Sec. 3.5
-// One CTA per (64 output channels, batch b).  The decayed scan
-//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i
-// (the recurrence form of the normalised double sum) is recomputed per
-// 64-channel slice of the K dimension straight into shared memory and
-// multiplied by the matching W_m slice: C[b, i+1] = M_i W_m, C[b, 0] = 0.
-template <class T>
-__global__ void __launch_bounds__(256)
-    memory_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
-                      const T* __restrict__ w_m, float* __restrict__ M, float* __restrict__ Z,
-                      float* __restrict__ Cmem, int Nb, int D) {
-  __shared__ float Ms[64][64 + 4];
-  __shared__ float Ws[64][64 + 4];
-  const int n0 = blockIdx.x * 64, b = blockIdx.y;
-  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
-  const bool write_m = (blockIdx.x == 0), write_z = write_m && b == 0;
-  for (int ic = 0; ic < Nb; ic += 64) {
-    const int iend = min(Nb, ic + 64);
-    float acc[4][4];
+// One thread per (batch b, channel c): the decayed scan over blocks
+//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i,
+// the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j).
+// Writes M (fp32, and a bf16 copy for the tensor-core projection when Mb is
+// given), Z (batch 0 only; it does not depend on b) and the first block's
+// memory row C[b, 0] = 0.  The projection C[b, i+1] = M_i W_m follows as a GEMM.
+__global__ void __launch_bounds__(128)
+    memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
+                           float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
+                           float* __restrict__ Cmem, int Nb, int D) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
+  if (c >= D) return;
+  const float a = decay[c];
+  const long base = (long)b * Nb * D + c;
+  float Nn = 0.f, Zz = 0.f;
+  constexpr int U = 8;
+  for (int i0 = 0; i0 < Nb; i0 += U) {
+    float sv[U];
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
+    for (int u = 0; u < U; ++u) sv[u] = (i0 + u < Nb) ? S[base + (long)(i0 + u) * D] : 0.f;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
-    for (int kc = 0; kc < D; kc += 64) {
-      if (tid < 64) {
-        const int k = kc + tid;
-        const float a = decay[k];
-        float Nn = 0.f, Zz = 0.f;
-        for (int i = 0; i < iend; ++i) {
-          Nn = fmaf(a, Nn, S[((long)b * Nb + i) * D + k]);
-          Zz = fmaf(a, Zz, 1.0f);
-          if (i >= ic) {
-            const float m = Nn / Zz;
-            Ms[i - ic][tid] = m;
-            if (write_m) M[((long)b * Nb + i) * D + k] = m;
-            if (write_z) Z[(long)i * D + k] = Zz;
-          }
-        }
-        for (int i = iend; i < ic + 64; ++i) Ms[i - ic][tid] = 0.f;
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u;
+      if (i < Nb) {
+        Nn = fmaf(a, Nn, sv[u]);
+        Zz = fmaf(a, Zz, 1.0f);
+        const float m = Nn / Zz;
+        M[base + (long)i * D] = m;
+        if (Mb) Mb[base + (long)i * D] = __float2bfloat16_rn(m);
+        if (b == 0) Z[(long)i * D + c] = Zz;
       }
-      for (int e = tid; e < 64 * 64; e += 256) {
-        const int kk = e / 64, nn = e % 64;
-        Ws[kk][nn] = to_f(w_m[(long)(kc + kk) * D + n0 + nn]);
-      }
-      __syncthreads();
-#pragma unroll 8
-      for (int kk = 0; kk < 64; ++kk) {
-        float a[4], w[4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) a[r] = Ms[ty * 4 + r][kk];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) w[c] = Ws[kk][tx * 4 + c];
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(a[r], w[c], acc[r][c]);
-      }
-      __syncthreads();
-    }
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const int i = ic + ty * 4 + r;
-      if (i + 1 < Nb) store4(Cmem + ((long)b * Nb + i + 1) * D + n0 + tx * 4, acc[r]);
     }
   }
-  if (tid < 16) {
-    const float zero[4] = {0.f, 0.f, 0.f, 0.f};
-    store4(Cmem + (long)b * Nb * D + n0 + tid * 4, zero);
-  }
+  Cmem[base] = 0.f;
 }
 
-cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
-                       const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D) {
-  if (D % 64 != 0) return cudaErrorInvalidValue;
-  dim3 grid(D / 64, B);
-  if (dtype == 0)
-    memory_fwd_kernel<float><<<grid, 256, 0, lc.stream>>>(S, decay, (const float*)w_m, M, Z, Cmem,
-                                                          Nb, D);
-  else
-    memory_fwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>(S, decay, (const bf16*)w_m, M, Z, Cmem,
-                                                         Nb, D);
+cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
+                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D) {
+  dim3 grid((D + 127) / 128, B);
+  memory_scan_fwd_kernel<<<grid, 128, 0, lc.stream>>>(S, decay, M, (bf16*)Mb, Z, Cmem, Nb, D);
   return cudaGetLastError();
 }
 
@@ -176,7 +135,7 @@ template <class T>
 __global__ void __launch_bounds__(256)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
                     const float* __restrict__ Cmem, T* __restrict__ dU, float* __restrict__ dP,
-                    int Tlen, int D, int L) {
+                    bf16* __restrict__ dPb, int Tlen, int D, int L) {
   const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
   const int i = blockIdx.y, b = blockIdx.z, Nb = gridDim.y;
   if (c >= D) return;
@@ -196,96 +155,61 @@ __global__ void __launch_bounds__(256)
     }
     store4(dU + o, du);
   }
-  if (i > 0) store4(dP + ((long)b * Nb + i - 1) * D + c, acc);
-  else {
-    const float zero[4] = {0.f, 0.f, 0.f, 0.f};
-    store4(dP + ((long)b * Nb + Nb - 1) * D + c, zero);
-  }
+  const long o = (i > 0) ? ((long)b * Nb + i - 1) * D + c : ((long)b * Nb + Nb - 1) * D + c;
+  if (i == 0) acc[0] = acc[1] = acc[2] = acc[3] = 0.f;
+  store4(dP + o, acc);
+  if (dPb) store4(dPb + o, acc);
 }
 
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, int B, int T, int D, int L) {
+                     void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
   dim3 grid((D / 4 + 255) / 256, Nb, B);
   if (dtype == 0)
     gate_bwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)dY, (const float*)G, Cmem,
-                                                        (float*)dU, dP, T, D, L);
+                                                        (float*)dU, dP, (bf16*)dPb, T, D, L);
   else
     gate_bwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)dY, (const bf16*)G, Cmem,
-                                                       (bf16*)dU, dP, T, D, L);
+                                                       (bf16*)dU, dP, (bf16*)dPb, T, D, L);
   return cudaGetLastError();
 }
 
 // ----------------------------------------------------- Sec. 3.5 backward
-// One CTA per (64 channels c, batch b): dM_i[c] = sum_k dP_i[k] W_m[c][k]
-// (P = M W_m), then the reverse decayed scan of M_i = N_i / Z_i:
+// One thread per (batch b, channel c): with dM = dP W_m^T already computed,
+// the reverse decayed scan of M_i = N_i / Z_i,
 //   R_i = dM_i / Z_i + a R_{i+1},  dS_i = R_i  (= sum_{i'>=i} a^(i'-i) dM_i' / Z_i').
-template <class T>
-__global__ void __launch_bounds__(256)
-    memory_bwd_kernel(const float* __restrict__ dP, const float* __restrict__ decay,
-                      const float* __restrict__ Z, const T* __restrict__ w_m,
-                      float* __restrict__ dS, int Nb, int D) {
-  __shared__ float Ps[64][64 + 4];
-  __shared__ float Ws[64][64 + 4];
-  const int c0 = blockIdx.x * 64, b = blockIdx.y;
-  const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+__global__ void __launch_bounds__(128)
+    memory_scan_bwd_kernel(const float* __restrict__ dM, const float* __restrict__ decay,
+                           const float* __restrict__ Z, float* __restrict__ dS, int Nb, int D) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
+  if (c >= D) return;
+  const float a = decay[c];
+  const long base = (long)b * Nb * D + c;
   float R = 0.f;
-  const float a = (tid < 64) ? decay[c0 + tid] : 0.f;
-  for (int iend = Nb; iend > 0; iend -= 64) {
-    const int ic = max(0, iend - 64);
-    float acc[4][4];
+  constexpr int U = 8;
+  for (int i1 = Nb; i1 > 0; i1 -= U) {
+    float mv[U], zv[U];
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
-    for (int kc = 0; kc < D; kc += 64) {
-      for (int e = tid; e < 64 * 64; e += 256) {
-        const int ii = e / 64, kk = e % 64;
-        const int i = ic + ii;
-        Ps[ii][kk] = (i < iend) ? dP[((long)b * Nb + i) * D + kc + kk] : 0.f;
-        const int cc = e / 64, k2 = e % 64;
-        Ws[k2][cc] = to_f(w_m[(long)(c0 + cc) * D + kc + k2]);
-      }
-      __syncthreads();
-#pragma unroll 8
-      for (int kk = 0; kk < 64; ++kk) {
-        float p[4], w[4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) p[r] = Ps[ty * 4 + r][kk];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) w[c] = Ws[kk][tx * 4 + c];
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(p[r], w[c], acc[r][c]);
-      }
-      __syncthreads();
+    for (int u = 0; u < U; ++u) {
+      const int i = i1 - 1 - u;
+      mv[u] = (i >= 0) ? dM[base + (long)i * D] : 0.f;
+      zv[u] = (i >= 0) ? Z[(long)i * D + c] : 1.f;
     }
-    // stash dM for the chunk in Ps, then scan it backwards per channel
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) Ps[ty * 4 + r][tx * 4 + c] = acc[r][c];
-    __syncthreads();
-    if (tid < 64) {
-      const int c = c0 + tid;
-      for (int i = iend - 1; i >= ic; --i) {
-        R = fmaf(a, R, Ps[i - ic][tid] / Z[(long)i * D + c]);
-        dS[((long)b * Nb + i) * D + c] = R;
+    for (int u = 0; u < U; ++u) {
+      const int i = i1 - 1 - u;
+      if (i >= 0) {
+        R = fmaf(a, R, mv[u] / zv[u]);
+        dS[base + (long)i * D] = R;
       }
     }
-    __syncthreads();
   }
 }
 
-cudaError_t memory_bwd(const Launch& lc, int dtype, const float* dP, const float* decay,
-                       const float* Z, const void* w_m, float* dS, int B, int Nb, int D) {
-  if (D % 64 != 0) return cudaErrorInvalidValue;
-  dim3 grid(D / 64, B);
-  if (dtype == 0)
-    memory_bwd_kernel<float><<<grid, 256, 0, lc.stream>>>(dP, decay, Z, (const float*)w_m, dS, Nb, D);
-  else
-    memory_bwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>(dP, decay, Z, (const bf16*)w_m, dS, Nb, D);
+cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
+                            float* dS, int B, int Nb, int D) {
+  dim3 grid((D + 127) / 128, B);
+  memory_scan_bwd_kernel<<<grid, 128, 0, lc.stream>>>(dM, decay, Z, dS, Nb, D);
   return cudaGetLastError();
 }
 
