@@ -63,7 +63,6 @@ __global__ void __launch_bounds__(128)
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mO,
                        float* __restrict__ lse, int Tlen, int H, int L, float scale,
                        unsigned* status) {
-  if (tc::status_failed(status)) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sQ = smem;             // Q; then P keys 0-63; then the output staging tile
@@ -76,10 +75,16 @@ __global__ void __launch_bounds__(128)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
 
+  // Loads first, so the TMEM allocation and the block barrier overlap them.
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
+    tc::mbar_arrive_expect_tx(&bar[0], 3 * kTB);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
   }
+  __syncwarp();
   if (warp == 0) {
     tc::tmem_alloc(tslot, 128);
     tc::tmem_relinquish();
@@ -91,10 +96,6 @@ __global__ void __launch_bounds__(128)
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 3 * kTB);
-    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
     const bool ok = tc::mbar_wait(&bar[0], 0, status);
     tc::fence_after_sync();
     if (ok) {
@@ -197,7 +198,6 @@ __global__ void __launch_bounds__(128)
                        const __grid_constant__ CUtensorMap mdV, const bf16* __restrict__ O, long ld_o,
                        const float* __restrict__ lse, int Tlen, int H, int L, float scale,
                        unsigned* status) {
-  if (tc::status_failed(status)) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sQ = smem;              // Q; then dQ staging
@@ -215,7 +215,13 @@ __global__ void __launch_bounds__(128)
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * kTB);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
   }
+  __syncwarp();
   if (warp == 0) {
     tc::tmem_alloc(tslot, 256);
     tc::tmem_relinquish();
@@ -227,11 +233,6 @@ __global__ void __launch_bounds__(128)
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 4 * kTB);
-    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sdO, &mdO, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
     const bool ok = tc::mbar_wait(&bar[0], 0, status);
     tc::fence_after_sync();
     if (ok) {

@@ -60,4 +60,34 @@ __device__ __forceinline__ void store4(bf16* p, const float* v) {
   *reinterpret_cast<uint2*>(p) = t;
 }
 
+// 8 consecutive elements (16 B for bf16, 32 B for fp32); 16-byte aligned.
+__device__ __forceinline__ void load8(const float* p, float* v) {
+  load4(p, v);
+  load4(p + 4, v + 4);
+}
+__device__ __forceinline__ void load8(const bf16* p, float* v) {
+  uint4 t = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+    float2 f = __bfloat1622float2(h);
+    v[2 * i] = f.x;
+    v[2 * i + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void store8(float* p, const float* v) {
+  store4(p, v);
+  store4(p + 4, v + 4);
+}
+__device__ __forceinline__ void store8(bf16* p, const float* v) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    w[i] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 }  // namespace bcmt

@@ -16,7 +16,11 @@ struct EpiStoreF {
   long split_stride;
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int z) const {
     TO* p = out + (long)z * split_stride + (long)row * ldo + col;
-    for (int j = 0; j < n; j += 4) store4(p + j, v + j);
+    if (n % 8 == 0) {
+      for (int j = 0; j < n; j += 8) store8(p + j, v + j);
+    } else {
+      for (int j = 0; j < n; j += 4) store4(p + j, v + j);
+    }
   }
 };
 
@@ -56,7 +60,7 @@ struct EpiShiftF {
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     if ((row % Nb) + 1 >= Nb) return;
     float* p = out + (long)(row + 1) * ldo + col;
-    for (int j = 0; j < n; j += 4) store4(p + j, v + j);
+    for (int j = 0; j < n; j += 4) store4(p + j, v + j);  // fp32: 16-byte stores
   }
 };
 

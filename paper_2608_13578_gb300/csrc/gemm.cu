@@ -153,38 +153,60 @@ struct TcCfg {
   static constexpr int B_BYTES = BN * kBK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr int TMEM_COLS = 2 * BN;  // two accumulators
 };
+
+int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+      n = 1;
+  }
+  return n;
+}
 }  // namespace
 
+// Persistent, warp-specialised tcgen05 GEMM.  Tiles are 128 x BN output
+// blocks (optionally one K-split each), taken round-robin by the CTAs, m
+// fastest.  Warp 0 / lane 0 streams 64-deep K slices of A and B into a
+// STAGES-deep ring with TMA; warp 1 / lane 0 issues the MMAs into one of two
+// TMEM accumulators; warps 2-5 drain the other accumulator through the
+// epilogue at the same time, so a tile's epilogue overlaps the next tile's
+// main loop.
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   int M, int N, int kps, int nkb, Epi epi, unsigned* status) {
+                   int M, int N, int kps, int nkb, int tiles_m, int tiles_n, int n_tiles, Epi epi,
+                   unsigned* status) {
   using Cfg = TcCfg<BN, STAGES>;
-  if (tc::status_failed(status)) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
   uint64_t* empty = full + STAGES;
-  uint64_t* done = empty + STAGES;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* tfull = empty + STAGES;   // accumulator ready for the epilogue
+  uint64_t* tempty = tfull + 2;       // accumulator drained by the epilogue
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tempty + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * BN, z = blockIdx.z;
-  const int kb0 = z * kps;
-  const int nk = min(nkb, kb0 + kps) - kb0;
 
-  if (threadIdx.x == 0) {
+  if (warp == 0 && lane == 0) {
     for (int s = 0; s < STAGES; ++s) {
       tc::mbar_init(&full[s], 1);
       tc::mbar_init(&empty[s], 1);
     }
-    tc::mbar_init(done, 1);
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(&tfull[a], 1);
+      tc::mbar_init(&tempty[a], 4);
+    }
     tc::fence_mbar_init();
+    tc::prefetch_tmap(&mA);
+    tc::prefetch_tmap(&mB);
   }
-  if (warp == 0) {
-    tc::tmem_alloc(tslot, BN);
+  if (warp == 1) {
+    tc::tmem_alloc(tslot, Cfg::TMEM_COLS);
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
@@ -192,67 +214,108 @@ __global__ void __launch_bounds__(128, 1)
   tc::fence_after_sync();
   const uint32_t tmem = *tslot;
 
-  if (warp == 0 && lane == 0) {
-    // ---- TMA producer
-    int issued = 0;
-    for (int i = 0; i < nk; ++i) {
-      const int s = i % STAGES;
-      if (i >= STAGES && !tc::mbar_wait(&empty[s], ((i / STAGES) - 1) & 1, status)) break;
-      uint8_t* sa = smem + s * Cfg::STAGE_BYTES;
-      uint8_t* sb = sa + Cfg::A_BYTES;
-      tc::mbar_arrive_expect_tx(&full[s], Cfg::STAGE_BYTES);
-      const int k0 = (kb0 + i) * kBK;
-      if (!A_MN) {
-        tc::tma_load_2d(sa, &mA, &full[s], k0, m0);
-      } else {
-        tc::tma_load_2d(sa, &mA, &full[s], m0, k0);
-        tc::tma_load_2d(sa + 8192, &mA, &full[s], m0 + 64, k0);
-      }
-      if (!B_MN) {
-        tc::tma_load_2d(sb, &mB, &full[s], k0, n0);
-      } else {
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        const int m_blk = tile % tiles_m, rest = tile / tiles_m;
+        const int n_blk = rest % tiles_n, z = rest / tiles_n;
+        const int m0 = m_blk * kBM, n0 = n_blk * BN, kb0 = z * kps;
+        const int nk = min(nkb, kb0 + kps) - kb0;
+        for (int i = 0; i < nk; ++i, ++it) {
+          const int s = it % STAGES;
+          if (it >= STAGES && !tc::mbar_wait(&empty[s], ((it / STAGES) - 1) & 1, status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + s * Cfg::STAGE_BYTES;
+          uint8_t* sb = sa + Cfg::A_BYTES;
+          tc::mbar_arrive_expect_tx(&full[s], Cfg::STAGE_BYTES);
+          const int k0 = (kb0 + i) * kBK;
+          if (!A_MN) {
+            tc::tma_load_2d(sa, &mA, &full[s], k0, m0);
+          } else {
+            tc::tma_load_2d(sa, &mA, &full[s], m0, k0);
+            tc::tma_load_2d(sa + 8192, &mA, &full[s], m0 + 64, k0);
+          }
+          if (!B_MN) {
+            tc::tma_load_2d(sb, &mB, &full[s], k0, n0);
+          } else {
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tc::tma_load_2d(sb + j * 8192, &mB, &full[s], n0 + 64 * j, k0);
+            for (int j = 0; j < BN / 64; ++j)
+              tc::tma_load_2d(sb + j * 8192, &mB, &full[s], n0 + 64 * j, k0);
+          }
+        }
       }
-      issued = i + 1;
+      // No copy may still be in flight when the CTA exits.
+      for (int i = (it > STAGES ? it - STAGES : 0); i < it; ++i)
+        tc::mbar_wait(&full[i % STAGES], (i / STAGES) & 1, status);
     }
-    // No copy may still be in flight when the CTA exits.
-    for (int i = (issued > STAGES ? issued - STAGES : 0); i < issued; ++i)
-      tc::mbar_wait(&full[i % STAGES], (i / STAGES) & 1, status);
-  } else if (warp == 1 && lane == 0) {
-    // ---- MMA issuer
-    constexpr uint32_t idesc = tc::idesc_bf16(kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
-    for (int i = 0; i < nk; ++i) {
-      const int s = i % STAGES;
-      if (!tc::mbar_wait(&full[s], (i / STAGES) & 1, status)) break;
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issuer
+      constexpr uint32_t idesc = tc::idesc_bf16(kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+      int it = 0, j = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++j) {
+        const int z = (tile / tiles_m) / tiles_n;
+        const int kb0 = z * kps, nk = min(nkb, kb0 + kps) - kb0;
+        const int acc = j & 1, use = j >> 1;
+        if (use > 0 && !tc::mbar_wait(&tempty[acc], (use - 1) & 1, status)) break;
+        tc::fence_after_sync();
+        const uint32_t d = tmem + (uint32_t)(acc * BN);
+        for (int i = 0; i < nk; ++i, ++it) {
+          const int s = it % STAGES;
+          if (!tc::mbar_wait(&full[s], (it / STAGES) & 1, status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE_BYTES);
+          const uint32_t sb = sa + Cfg::A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024)
+                                     : tc::sdesc(sa + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024)
+                                     : tc::sdesc(sb + kk * 32, 16, 1024);
+            tc::mma_bf16(d, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
+          }
+          tc::mma_commit(&empty[s]);
+        }
+        tc::mma_commit(&tfull[acc]);
+      }
+    }
+  } else {
+    // ---- epilogue warps 2..5: warp w reads TMEM lanes 32*(w%4) .. +31
+    const int q = warp & 3;
+    int j = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++j) {
+      const int m_blk = tile % tiles_m, rest = tile / tiles_m;
+      const int n_blk = rest % tiles_n, z = rest / tiles_n;
+      const int acc = j & 1, use = j >> 1;
+      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
       tc::fence_after_sync();
-      const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE_BYTES);
-      const uint32_t sb = sa + Cfg::A_BYTES;
-#pragma unroll
-      for (int kk = 0; kk < kBK / 16; ++kk) {
-        const uint64_t ad = A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024) : tc::sdesc(sa + kk * 32, 16, 1024);
-        const uint64_t bd = B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024) : tc::sdesc(sb + kk * 32, 16, 1024);
-        tc::mma_bf16(tmem, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
-      }
-      tc::mma_commit(&empty[s]);
-    }
-    tc::mma_commit(done);
-  }
-  __syncwarp();
-
-  // ---- epilogue: thread = output row, 32 columns per TMEM load
-  const bool ok = tc::mbar_wait(done, 0, status) && nk > 0;
-  tc::fence_after_sync();
-  const int row = m0 + warp * 32 + lane;
+      const int row = m_blk * kBM + q * 32 + lane;
+      const int n0 = n_blk * BN;
+      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll 1
-  for (int c = 0; c < BN; c += 32) {
-    float v[32];
-    tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c, v);
-    if (ok && row < M && n0 + c < N) epi(row, n0 + c, v, 32, z);
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tc::tmem_ld32(base + (uint32_t)c, v);
+        if (ok && row < M && n0 + c < N) epi(row, n0 + c, v, 32, z);
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&tempty[acc]);
+      if (!ok) break;
+    }
   }
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, BN);
+  if (warp == 1) tc::tmem_dealloc(tmem, Cfg::TMEM_COLS);
 }
 
 namespace {
@@ -287,6 +350,8 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   }
   const int nkb = (K + kBK - 1) / kBK;
   const int kps = (nkb + splits - 1) / splits;
+  const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
+  const int n_tiles = tiles_m * tiles_n * splits;
   auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -294,8 +359,9 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  dim3 grid((N + BN - 1) / BN, (M + kBM - 1) / kBM, splits);
-  kern<<<grid, 128, Cfg::SMEM, lc.stream>>>(mA, mB, M, N, kps, nkb, epi, lc.status);
+  const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
+  kern<<<grid, 192, Cfg::SMEM, lc.stream>>>(mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
+                                            lc.status);
   return cudaGetLastError();
 }
 
@@ -303,7 +369,7 @@ template <bool A_MN, bool B_MN>
 static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                           long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                           const EpiArgs& ea, int splits) {
-  constexpr int BN = 128, ST = 4;
+  constexpr int BN = 128, ST = 6;
   switch (epi) {
     case EPI_STORE:
       if (dtype_out == 0)
@@ -372,6 +438,7 @@ __global__ void reduce_splits_kernel(const float* __restrict__ part, int splits,
   const long i4 = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
   if (i4 >= count) return;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
   for (int s = 0; s < splits; ++s) {
     float v[4];
     load4(part + (long)s * count + i4, v);

@@ -54,17 +54,32 @@ __global__ void __launch_bounds__(256)
     sc[r] = a;
   }
   __syncthreads();
-  const int c = blockIdx.z * blockDim.x + threadIdx.x;
-  if (c >= D) return;
-  const T* Hc = Hm + row0 * D + c;
-  float acc0 = 0.f, acc1 = 0.f;
-  int r = 0;
-  for (; r + 1 < n; r += 2) {
-    acc0 = fmaf(sc[r], to_f(Hc[(long)r * D]), acc0);
-    acc1 = fmaf(sc[r + 1], to_f(Hc[(long)(r + 1) * D]), acc1);
+  // S_i[c] = sum_t alpha_t H_t[c]: 8 row groups x 32 threads of 8 channels each,
+  // then a fixed-order sum over the row groups.
+  __shared__ float part[8][256 + 4];
+  const int rg = threadIdx.x >> 5, co = threadIdx.x & 31;
+  const int c = blockIdx.z * 256 + co * 8;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (c < D) {
+    const T* Hc = Hm + row0 * D + c;
+    for (int r = rg; r < n; r += 8) {
+      float h[8];
+      load8(Hc + (long)r * D, h);
+      const float a = sc[r];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[e], acc[e]);
+    }
   }
-  if (r < n) acc0 = fmaf(sc[r], to_f(Hc[(long)r * D]), acc0);
-  S[((long)b * Nb + i) * D + c] = acc0 + acc1;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) part[rg][co * 8 + e] = acc[e];
+  __syncthreads();
+  const int cc = blockIdx.z * 256 + threadIdx.x;
+  if (cc < D) {
+    float t = 0.f;
+#pragma unroll
+    for (int g = 0; g < 8; ++g) t += part[g][threadIdx.x];
+    S[((long)b * Nb + i) * D + cc] = t;
+  }
 }
 
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
@@ -136,35 +151,51 @@ __global__ void __launch_bounds__(256)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
                     const float* __restrict__ Cmem, T* __restrict__ dU, float* __restrict__ dP,
                     bf16* __restrict__ dPb, int Tlen, int D, int L) {
-  const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  // 8 row groups x 32 threads of 4 channels: 128 channels per CTA.
+  __shared__ float part[8][128 + 4];
   const int i = blockIdx.y, b = blockIdx.z, Nb = gridDim.y;
-  if (c >= D) return;
+  const int rg = threadIdx.x >> 5, cq = threadIdx.x & 31;
+  const int c = blockIdx.x * 128 + cq * 4;
   const int t0 = i * L, n = min(L, Tlen - t0);
-  float cm[4];
-  load4(Cmem + ((long)b * Nb + i) * D + c, cm);
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int r = 0; r < n; ++r) {
-    const long o = ((long)b * Tlen + t0 + r) * D + c;
-    float dy[4], g[4], du[4];
-    load4(dY + o, dy);
-    load4(G + o, g);
+  if (c < D) {
+    float cm[4];
+    load4(Cmem + ((long)b * Nb + i) * D + c, cm);
+    for (int r = rg; r < n; r += 8) {
+      const long o = ((long)b * Tlen + t0 + r) * D + c;
+      float dy[4], g[4], du[4];
+      load4(dY + o, dy);
+      load4(G + o, g);
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      du[e] = dy[e] * cm[e] * g[e] * (1.0f - g[e]);
-      acc[e] = fmaf(dy[e], g[e], acc[e]);
+      for (int e = 0; e < 4; ++e) {
+        du[e] = dy[e] * cm[e] * g[e] * (1.0f - g[e]);
+        acc[e] = fmaf(dy[e], g[e], acc[e]);
+      }
+      store4(dU + o, du);
     }
-    store4(dU + o, du);
   }
-  const long o = (i > 0) ? ((long)b * Nb + i - 1) * D + c : ((long)b * Nb + Nb - 1) * D + c;
-  if (i == 0) acc[0] = acc[1] = acc[2] = acc[3] = 0.f;
-  store4(dP + o, acc);
-  if (dPb) store4(dPb + o, acc);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) part[rg][cq * 4 + e] = acc[e];
+  __syncthreads();
+  if (threadIdx.x < 128) {
+    const int cc = blockIdx.x * 128 + threadIdx.x;
+    if (cc < D) {
+      float t = 0.f;
+#pragma unroll
+      for (int g = 0; g < 8; ++g) t += part[g][threadIdx.x];
+      // dC_i becomes dP[b, i-1] (C_i = P_{i-1}); block 0 writes the zero row dP[b, Nb-1]
+      const long o = (i > 0) ? ((long)b * Nb + i - 1) * D + cc : ((long)b * Nb + Nb - 1) * D + cc;
+      if (i == 0) t = 0.f;
+      dP[o] = t;
+      if (dPb) dPb[o] = __float2bfloat16_rn(t);
+    }
+  }
 }
 
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
                      void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
-  dim3 grid((D / 4 + 255) / 256, Nb, B);
+  dim3 grid((D + 127) / 128, Nb, B);
   if (dtype == 0)
     gate_bwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)dY, (const float*)G, Cmem,
                                                         (float*)dU, dP, (bf16*)dPb, T, D, L);
@@ -224,19 +255,22 @@ __global__ void __launch_bounds__(256)
                        float* __restrict__ dwp_part, int Tlen, int D, int L) {
   __shared__ float g[kMaxL];
   __shared__ float cdot;
+  __shared__ float part[8][256 + 4];
   const int i = blockIdx.x, b = blockIdx.y, Nb = gridDim.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t0 = i * L, n = min(L, Tlen - t0);
   const T* Hb = Hm + ((long)b * Tlen + t0) * D;
   const float* dSi = dS + ((long)b * Nb + i) * D;
   const float* ab = alpha + (long)b * Tlen + t0;
+  // g_t = H_t . dS_i, one warp per row, 8 channels per lane
   for (int r = warp; r < n; r += 8) {
     float d = 0.f;
-    for (int c = lane * 4; c < D; c += 128) {
-      float h[4], s[4];
-      load4(Hb + (long)r * D + c, h);
-      load4(dSi + c, s);
-      d += h[0] * s[0] + h[1] * s[1] + h[2] * s[2] + h[3] * s[3];
+    for (int c = lane * 8; c < D; c += 256) {
+      float h[8], sv[8];
+      load8(Hb + (long)r * D + c, h);
+      load8(dSi + c, sv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) d = fmaf(h[e], sv[e], d);
     }
     d = warp_sum(d);
     if (lane == 0) g[r] = d;
@@ -250,22 +284,37 @@ __global__ void __launch_bounds__(256)
   }
   __syncthreads();
   const float cd = cdot;
-  __syncthreads();
   for (int r = threadIdx.x; r < n; r += blockDim.x) {
     const float v = ab[r] * (g[r] - cd);
     ds_out[(long)b * Tlen + t0 + r] = v;
     g[r] = v;
   }
   __syncthreads();
-  for (int c = threadIdx.x * 4; c < D; c += blockDim.x * 4) {
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int r = 0; r < n; ++r) {
-      float h[4];
-      load4(Hb + (long)r * D + c, h);
+  // the block's share of dW_p = sum_t ds_t H_t: 8 row groups x 32 lanes x 8 channels
+  const int rg = warp, co = lane;
+  for (int c0 = 0; c0 < D; c0 += 256) {
+    const int c = c0 + co * 8;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (c < D) {
+      for (int r = rg; r < n; r += 8) {
+        float h[8];
+        load8(Hb + (long)r * D + c, h);
+        const float w = g[r];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) acc[e] = fmaf(g[r], h[e], acc[e]);
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(w, h[e], acc[e]);
+      }
     }
-    store4(dwp_part + ((long)b * Nb + i) * D + c, acc);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part[rg][co * 8 + e] = acc[e];
+    __syncthreads();
+    const int cc = c0 + threadIdx.x;
+    if (cc < D) {
+      float t = 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) t += part[q][threadIdx.x];
+      dwp_part[((long)b * Nb + i) * D + cc] = t;
+    }
+    __syncthreads();
   }
 }
 
@@ -283,20 +332,30 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
   return cudaGetLastError();
 }
 
-// Column sums in row order.
+// Column sums in a fixed order: 8 row groups of 32 columns per CTA, then the
+// group sums added in group order.
 template <class TO>
-__global__ void reduce_rows_kernel(const float* __restrict__ in, int rows, int cols,
-                                   TO* __restrict__ out) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= cols) return;
+__global__ void __launch_bounds__(256)
+    reduce_rows_kernel(const float* __restrict__ in, int rows, int cols, TO* __restrict__ out) {
+  __shared__ float part[8][33];
+  const int rg = threadIdx.x >> 5, cl = threadIdx.x & 31;
+  const int c = blockIdx.x * 32 + cl;
   float acc = 0.f;
-  for (int r = 0; r < rows; ++r) acc += in[(long)r * cols + c];
-  out[c] = from_f<TO>(acc);
+  if (c < cols)
+    for (int r = rg; r < rows; r += 8) acc += in[(long)r * cols + c];
+  part[rg][cl] = acc;
+  __syncthreads();
+  if (threadIdx.x < 32 && c < cols) {
+    float t = 0.f;
+#pragma unroll
+    for (int g = 0; g < 8; ++g) t += part[g][threadIdx.x];
+    out[c] = from_f<TO>(t);
+  }
 }
 
 cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, int dtype_out,
                         void* out) {
-  const int blocks = (cols + 255) / 256;
+  const int blocks = (cols + 31) / 32;
   if (dtype_out == 0)
     reduce_rows_kernel<float><<<blocks, 256, 0, lc.stream>>>(in, rows, cols, (float*)out);
   else
