@@ -249,18 +249,27 @@ def bench_ours(args):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
 
     def step(pp):
+        # launches on the current stream (the capture stream while a graph is recorded)
         C.bcmt_forward(pp, t["x"], None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
-                       t["w_g"], t["decay"], y, ws, stream)
+                       t["w_g"], t["decay"], y, ws, None)
         C.bcmt_backward(pp, t["dy"], t["x"], None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
                         t["w_g"], t["decay"], ws, sc, grads["dx"], None, None, grads["dw_qkv"],
-                        grads["dw_o"], grads["dw_p"], grads["dw_m"], grads["dw_g"], stream)
+                        grads["dw_o"], grads["dw_p"], grads["dw_m"], grads["dw_g"], None)
 
     for _ in range(max(3, args.warmup)):
         step(p)
     C.bcmt_device_status(stream)
     torch.cuda.synchronize()
+    # One step recorded as a CUDA graph: the same launches, replayed without
+    # per-launch host work.
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step(p)
+    graph.replay()
+    torch.cuda.synchronize()
+    C.bcmt_device_status(stream)
 
-    def timed(pp):
+    def timed(run):
         """K steps, each bracketed by CUDA events on the launching stream, with
         L2 evicted before each step; returns the summed device time in ms."""
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -271,24 +280,25 @@ def bench_ours(args):
         for i in range(args.steps):
             flush.fill_(i & 0xFF)            # evict L2 between timed steps
             ev[i][0].record(stream)
-            step(pp)
+            run()
             ev[i][1].record(stream)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         return sum(a.elapsed_time(b) for a, b in ev)
 
-    # the measured region: no per-kernel events
+    # the measured region: graph replays of the step, no per-kernel events
     clocks = ClockSampler(local_rank)
     clocks.start()
     time.sleep(0.3)
-    total_ms = timed(p)
+    total_ms = timed(graph.replay)
+    eager_ms = timed(lambda: step(p))
     clk = clocks.stop()
     C.bcmt_device_status(stream)
     # the same K steps again with CUDA events around every kernel, for the
     # per-kernel breakdown and the roofline of the dominant kernel
     C.bcmt_profile_reset()
-    prof_ms = timed(pprof)
+    prof_ms = timed(lambda: step(pprof))
     C.bcmt_device_status(stream)
     prof = C.bcmt_profile_read()
     launches = sum(c for c, _ in prof.values())
@@ -387,6 +397,7 @@ def bench_ours(args):
             "data": "synthetic (seeded N(0,1) tokens, N(0,1/D) weights, decay 0.8)",
             "config": {"workload": name, "B": w.B, "T": w.T, "L": w.L, "D": w.D, "H": w.H,
                        "per_rank_batch": w.B, "parallelism": f"batch-sharded x{world}",
+                       "launch": "CUDA graph of bcmt_forward + bcmt_backward",
                        "l2": "flushed between timed steps (256 MiB write)"},
             "clocks": clk,
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -395,6 +406,9 @@ def bench_ours(args):
             "roofline": roof,
             "cpu_baseline": cpu,
             "kernels": kernels,
+            "eager": {"ms_per_step": round(eager_ms / args.steps, 4),
+                      "value": round(world * tokens_per_step * args.steps / (eager_ms / 1e3), 1),
+                      "note": "same steps launched call by call instead of as a graph"},
             "profiled_pass": {"ms_per_step_with_kernel_events": round(prof_ms / args.steps, 4),
                               "note": "per-kernel times come from this second pass of the "
                                       "same steps; value comes from the pass without them"},

@@ -22,6 +22,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     attn_fwd_simt_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V,
                          long ld, T* __restrict__ O, long ld_o, float* __restrict__ lse, int Tlen,
                          int H, int dh, int L, float scale) {
+  pdl_enter();
   __shared__ float qs[kWarps][kMaxDh];
   __shared__ float ps[kWarps][kMaxL];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -69,6 +70,7 @@ __global__ void __launch_bounds__(kWarps * 32)
                            const T* __restrict__ dO, long ld_o, const float* __restrict__ lse,
                            float* __restrict__ Drow, T* __restrict__ dQ, long ld_d, int Tlen, int H,
                            int dh, int L, float scale) {
+  pdl_enter();
   __shared__ float qs[kWarps][kMaxDh];
   __shared__ float gs[kWarps][kMaxDh];
   __shared__ float ds[kWarps][kMaxL];
@@ -116,6 +118,7 @@ __global__ void __launch_bounds__(kWarps * 32)
                             const float* __restrict__ lse, const float* __restrict__ Drow,
                             T* __restrict__ dK, T* __restrict__ dV, long ld_d, int Tlen, int H,
                             int dh, int L, float scale) {
+  pdl_enter();
   __shared__ float ks[kWarps][kMaxDh];
   __shared__ float vs[kWarps][kMaxDh];
   __shared__ float ps[kWarps][kMaxL];
@@ -160,7 +163,8 @@ __global__ void __launch_bounds__(kWarps * 32)
 template <class T>
 static cudaError_t fwd_typed(const Launch& lc, const AttnArgs& a) {
   dim3 grid((a.T + kWarps - 1) / kWarps, a.H, a.B);
-  attn_fwd_simt_kernel<T><<<grid, kWarps * 32, 0, lc.stream>>>(
+  launch_k(attn_fwd_simt_kernel<T>, dim3(grid), dim3(kWarps * 32), 0, lc.stream,
+
       (const T*)a.Q, (const T*)a.K, (const T*)a.V, a.ld_qkv, (T*)a.O, a.ld_o, a.lse, a.T, a.H,
       a.dh, a.L, 1.0f / sqrtf((float)a.dh));
   return cudaGetLastError();
@@ -171,12 +175,14 @@ static cudaError_t bwd_typed(const Launch& lc, const AttnBwdArgs& a) {
   const AttnArgs& f = a.f;
   dim3 grid((f.T + kWarps - 1) / kWarps, f.H, f.B);
   const float scale = 1.0f / sqrtf((float)f.dh);
-  attn_bwd_q_simt_kernel<T><<<grid, kWarps * 32, 0, lc.stream>>>(
+  launch_k(attn_bwd_q_simt_kernel<T>, dim3(grid), dim3(kWarps * 32), 0, lc.stream,
+
       (const T*)f.Q, (const T*)f.K, (const T*)f.V, f.ld_qkv, (const T*)f.O, (const T*)a.dO, f.ld_o,
       f.lse, a.Drow, (T*)a.dQ, a.ld_dqkv, f.T, f.H, f.dh, f.L, scale);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  attn_bwd_kv_simt_kernel<T><<<grid, kWarps * 32, 0, lc.stream>>>(
+  launch_k(attn_bwd_kv_simt_kernel<T>, dim3(grid), dim3(kWarps * 32), 0, lc.stream,
+
       (const T*)f.Q, (const T*)f.K, (const T*)f.V, f.ld_qkv, (const T*)a.dO, f.ld_o, f.lse, a.Drow,
       (T*)a.dK, (T*)a.dV, a.ld_dqkv, f.T, f.H, f.dh, f.L, scale);
   return cudaGetLastError();

@@ -75,10 +75,17 @@ __global__ void __launch_bounds__(128)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
 
-  // Loads first, so the TMEM allocation and the block barrier overlap them.
+  // Setup overlaps the previous kernel (before pdl_wait); the loads go out
+  // first after it, so the TMEM allocation and the block barrier overlap them.
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+  }
+  pdl_enter();
+  if (tid == 0) {
     tc::mbar_arrive_expect_tx(&bar[0], 3 * kTB);
     tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
     tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
@@ -215,6 +222,13 @@ __global__ void __launch_bounds__(128)
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+    tc::prefetch_tmap(&mdO);
+  }
+  pdl_enter();
+  if (tid == 0) {
     tc::mbar_arrive_expect_tx(&bar[0], 4 * kTB);
     tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
     tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
@@ -399,7 +413,8 @@ cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
     attr = true;
   }
   dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
-  attn_fwd_tc_kernel<<<grid, 128, kFwdSmem, lc.stream>>>(mQ, mK, mV, mO, a.lse, a.T, a.H, a.L,
+  launch_k(attn_fwd_tc_kernel, dim3(grid), dim3(128), kFwdSmem, lc.stream,
+mQ, mK, mV, mO, a.lse, a.T, a.H, a.L,
                                                          1.0f / sqrtf((float)a.dh), lc.status);
   return cudaGetLastError();
 }
@@ -423,7 +438,8 @@ cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
     attr = true;
   }
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
-  attn_bwd_tc_kernel<<<grid, 128, kBwdSmem, lc.stream>>>(
+  launch_k(attn_bwd_tc_kernel, dim3(grid), dim3(128), kBwdSmem, lc.stream,
+
       mQ, mK, mV, mdO, mdQ, mdK, mdV, (const bf16*)f.O, f.ld_o, f.lse, f.T, f.H, f.L,
       1.0f / sqrtf((float)f.dh), lc.status);
   return cudaGetLastError();

@@ -6,12 +6,47 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace bcmt {
 
 typedef __nv_bfloat16 bf16;
 
 // Bits OR-ed into the device status word.
 enum : unsigned { kStatusTimeout = 1u, kStatusBadLaunch = 2u };
+
+// Programmatic dependent launch.  Every kernel of the library is launched with
+// programmatic stream serialisation (launch_k below) and starts with
+// pdl_enter(): it lets the next kernel on the stream begin launching at once,
+// then waits until the previous kernel has finished and its writes are
+// visible.  Work placed before pdl_wait() (barrier init, TMEM allocation,
+// tensor-map prefetch) overlaps the previous kernel; no global memory may be
+// touched before it.  Both are no-ops for a launch without the attribute.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_enter() {
+  pdl_trigger();
+  pdl_wait();
+}
+
+// Host: launches `kernel` on `stream` with programmatic stream serialisation.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                            cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 template <class T> __device__ __forceinline__ float to_f(T v);
 template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }

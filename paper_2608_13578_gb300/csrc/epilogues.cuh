@@ -27,6 +27,9 @@ struct EpiStoreF {
 // Sec. 3.3 + 3.4: stores H = Concat(heads) W_O and, for the pooling scores
 // s = H w_p, one partial dot product per output row and run of n columns
 // (spart[(col / n) * n_rows + row]); the summary kernel adds them up.
+// Every epilogue below reads all of its inputs before its first store: the
+// pointers may alias as far as the compiler knows, so interleaving loads and
+// stores would serialise one memory round trip per vector.
 template <class TO>
 struct EpiStoreScoreF {
   TO* out;
@@ -35,17 +38,15 @@ struct EpiStoreScoreF {
   float* spart;
   long n_rows;
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
+    float w[32];
+    for (int j = 0; j < n; j += 4) load4(w_p + col + j, w + j);
     TO* p = out + (long)row * ldo + col;
     float s = 0.f;
-    for (int j = 0; j < n; j += 4) {
-      float w[4];
-      load4(w_p + col + j, w);
-      // score from the stored (rounded) H, the value the summary pools
-      float h[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) h[e] = to_f(from_f<TO>(v[j + e]));
-      s += h[0] * w[0] + h[1] * w[1] + h[2] * w[2] + h[3] * w[3];
-      store4(p + j, v + j);
+    for (int j = 0; j < n; ++j) s = fmaf(to_f(from_f<TO>(v[j])), w[j], s);  // the stored value
+    if (n % 8 == 0) {
+      for (int j = 0; j < n; j += 8) store8(p + j, v + j);
+    } else {
+      for (int j = 0; j < n; j += 4) store4(p + j, v + j);
     }
     spart[(long)(col / n) * n_rows + row] = s;
   }
@@ -76,17 +77,26 @@ struct EpiGateInjectF {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
     const long o = (long)row * D + col;
+    float h[32], c[32];
     for (int j = 0; j < n; j += 4) {
-      float h[4], c[4], g[4], y[4];
-      load4(H + o + j, h);
-      load4(cm + j, c);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        g[e] = sigmoidf_(v[j + e]);
-        y[e] = h[e] + g[e] * c[e];
+      load4(H + o + j, h + j);
+      load4(cm + j, c + j);
+    }
+    float g[32];
+    for (int j = 0; j < n; ++j) {
+      g[j] = sigmoidf_(v[j]);
+      h[j] = fmaf(g[j], c[j], h[j]);
+    }
+    if (n % 8 == 0) {
+      for (int j = 0; j < n; j += 8) {
+        store8(G + o + j, g + j);
+        store8(Y + o + j, h + j);
       }
-      store4(G + o + j, g);
-      store4(Y + o + j, y);
+    } else {
+      for (int j = 0; j < n; j += 4) {
+        store4(G + o + j, g + j);
+        store4(Y + o + j, h + j);
+      }
     }
   }
 };
@@ -105,16 +115,19 @@ struct EpiDHF {
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* dsb = dS + ((long)b * Nb + blk) * D + col;
-    const float at = alpha[row], st = ds[row];
     const long o = (long)row * D + col;
+    const float at = alpha[row], st = ds[row];
+    float dy[32], sv[32], wp[32];
     for (int j = 0; j < n; j += 4) {
-      float dy[4], sv[4], wp[4], r[4];
-      load4(dY + o + j, dy);
-      load4(dsb + j, sv);
-      load4(w_p + col + j, wp);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) r[e] = v[j + e] + dy[e] + at * sv[e] + st * wp[e];
-      store4(out + o + j, r);
+      load4(dY + o + j, dy + j);
+      load4(dsb + j, sv + j);
+      load4(w_p + col + j, wp + j);
+    }
+    for (int j = 0; j < n; ++j) dy[j] = v[j] + dy[j] + at * sv[j] + st * wp[j];
+    if (n % 8 == 0) {
+      for (int j = 0; j < n; j += 8) store8(out + o + j, dy + j);
+    } else {
+      for (int j = 0; j < n; j += 4) store4(out + o + j, dy + j);
     }
   }
 };

@@ -34,6 +34,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
                                                         long sam, long sak,
                                                         const TI* __restrict__ B, long sbk,
                                                         long sbn, Epi epi, int kps) {
+  pdl_enter();
   __shared__ float As[16][64 + 4];
   __shared__ float Bs[16][64 + 4];
   const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
@@ -87,7 +88,8 @@ static cudaError_t simt_launch(const Launch& lc, int M, int N, int K, const void
   const int nkb = (K + 63) / 64;
   const int kps = ((nkb + splits - 1) / splits) * 64;
   dim3 grid((N + 63) / 64, (M + 63) / 64, splits);
-  gemm_simt_kernel<TI, Epi><<<grid, 256, 0, lc.stream>>>(
+  launch_k(gemm_simt_kernel<TI, Epi>, dim3(grid), dim3(256), 0, lc.stream,
+
       M, N, K, static_cast<const TI*>(A), sam, sak, static_cast<const TI*>(B), sbk, sbn, epi, kps);
   return cudaGetLastError();
 }
@@ -213,6 +215,7 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = *tslot;
+  pdl_enter();  // setup above overlapped the previous kernel
 
   if (warp == 0) {
     if (lane == 0) {
@@ -360,7 +363,8 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
     attr_set = true;
   }
   const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
-  kern<<<grid, 192, Cfg::SMEM, lc.stream>>>(mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
+  launch_k(kern, dim3(grid), dim3(192), Cfg::SMEM, lc.stream,
+mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
                                             lc.status);
   return cudaGetLastError();
 }
@@ -435,6 +439,7 @@ cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K
 template <class TO>
 __global__ void reduce_splits_kernel(const float* __restrict__ part, int splits, long count,
                                      TO* __restrict__ out) {
+  pdl_enter();
   const long i4 = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
   if (i4 >= count) return;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -455,9 +460,11 @@ cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long 
   const int threads = 256;
   const unsigned blocks = (unsigned)((n4 + threads - 1) / threads);
   if (dtype_out == 0)
-    reduce_splits_kernel<float><<<blocks, threads, 0, lc.stream>>>(part, splits, count, (float*)out);
+    launch_k(reduce_splits_kernel<float>, dim3(blocks), dim3(threads), 0, lc.stream,
+part, splits, count, (float*)out);
   else
-    reduce_splits_kernel<bf16><<<blocks, threads, 0, lc.stream>>>(part, splits, count, (bf16*)out);
+    launch_k(reduce_splits_kernel<bf16>, dim3(blocks), dim3(threads), 0, lc.stream,
+part, splits, count, (bf16*)out);
   return cudaGetLastError();
 }
 

@@ -25,6 +25,7 @@ __global__ void __launch_bounds__(256)
     summary_fwd_kernel(const T* __restrict__ Hm, const float* __restrict__ spart, int npart,
                        long n_tok, float* __restrict__ alpha, float* __restrict__ S, int Tlen,
                        int D, int L) {
+  pdl_enter();
   __shared__ float sc[kMaxL];
   __shared__ float red[2];
   const int i = blockIdx.x, b = blockIdx.y, Nb = gridDim.x;
@@ -89,10 +90,12 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
   dim3 grid(Nb, B, (D + 255) / 256);
   const long n_tok = (long)B * T;
   if (dtype == 0)
-    summary_fwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)Hm, spart, npart, n_tok,
+    launch_k(summary_fwd_kernel<float>, dim3(grid), dim3(256), 0, lc.stream,
+(const float*)Hm, spart, npart, n_tok,
                                                            alpha, S, T, D, L);
   else
-    summary_fwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)Hm, spart, npart, n_tok,
+    launch_k(summary_fwd_kernel<bf16>, dim3(grid), dim3(256), 0, lc.stream,
+(const bf16*)Hm, spart, npart, n_tok,
                                                           alpha, S, T, D, L);
   return cudaGetLastError();
 }
@@ -108,6 +111,7 @@ __global__ void __launch_bounds__(128)
     memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
                            float* __restrict__ Cmem, int Nb, int D) {
+  pdl_enter();
   const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
   if (c >= D) return;
   const float a = decay[c];
@@ -137,7 +141,8 @@ __global__ void __launch_bounds__(128)
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
                             void* Mb, float* Z, float* Cmem, int B, int Nb, int D) {
   dim3 grid((D + 127) / 128, B);
-  memory_scan_fwd_kernel<<<grid, 128, 0, lc.stream>>>(S, decay, M, (bf16*)Mb, Z, Cmem, Nb, D);
+  launch_k(memory_scan_fwd_kernel, dim3(grid), dim3(128), 0, lc.stream,
+S, decay, M, (bf16*)Mb, Z, Cmem, Nb, D);
   return cudaGetLastError();
 }
 
@@ -151,6 +156,7 @@ __global__ void __launch_bounds__(256)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
                     const float* __restrict__ Cmem, T* __restrict__ dU, float* __restrict__ dP,
                     bf16* __restrict__ dPb, int Tlen, int D, int L) {
+  pdl_enter();
   // 8 row groups x 32 threads of 4 channels: 128 channels per CTA.
   __shared__ float part[8][128 + 4];
   const int i = blockIdx.y, b = blockIdx.z, Nb = gridDim.y;
@@ -197,10 +203,12 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
   const int Nb = (T + L - 1) / L;
   dim3 grid((D + 127) / 128, Nb, B);
   if (dtype == 0)
-    gate_bwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)dY, (const float*)G, Cmem,
+    launch_k(gate_bwd_kernel<float>, dim3(grid), dim3(256), 0, lc.stream,
+(const float*)dY, (const float*)G, Cmem,
                                                         (float*)dU, dP, (bf16*)dPb, T, D, L);
   else
-    gate_bwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)dY, (const bf16*)G, Cmem,
+    launch_k(gate_bwd_kernel<bf16>, dim3(grid), dim3(256), 0, lc.stream,
+(const bf16*)dY, (const bf16*)G, Cmem,
                                                        (bf16*)dU, dP, (bf16*)dPb, T, D, L);
   return cudaGetLastError();
 }
@@ -212,6 +220,7 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 __global__ void __launch_bounds__(128)
     memory_scan_bwd_kernel(const float* __restrict__ dM, const float* __restrict__ decay,
                            const float* __restrict__ Z, float* __restrict__ dS, int Nb, int D) {
+  pdl_enter();
   const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
   if (c >= D) return;
   const float a = decay[c];
@@ -240,7 +249,8 @@ __global__ void __launch_bounds__(128)
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
                             float* dS, int B, int Nb, int D) {
   dim3 grid((D + 127) / 128, B);
-  memory_scan_bwd_kernel<<<grid, 128, 0, lc.stream>>>(dM, decay, Z, dS, Nb, D);
+  launch_k(memory_scan_bwd_kernel, dim3(grid), dim3(128), 0, lc.stream,
+dM, decay, Z, dS, Nb, D);
   return cudaGetLastError();
 }
 
@@ -253,6 +263,7 @@ __global__ void __launch_bounds__(256)
     summary_bwd_kernel(const T* __restrict__ Hm, const float* __restrict__ alpha,
                        const float* __restrict__ dS, float* __restrict__ ds_out,
                        float* __restrict__ dwp_part, int Tlen, int D, int L) {
+  pdl_enter();
   __shared__ float g[kMaxL];
   __shared__ float cdot;
   __shared__ float part[8][256 + 4];
@@ -324,10 +335,12 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
   const int Nb = (T + L - 1) / L;
   dim3 grid(Nb, B);
   if (dtype == 0)
-    summary_bwd_kernel<float><<<grid, 256, 0, lc.stream>>>((const float*)Hm, alpha, dS, ds,
+    launch_k(summary_bwd_kernel<float>, dim3(grid), dim3(256), 0, lc.stream,
+(const float*)Hm, alpha, dS, ds,
                                                            dwp_part, T, D, L);
   else
-    summary_bwd_kernel<bf16><<<grid, 256, 0, lc.stream>>>((const bf16*)Hm, alpha, dS, ds, dwp_part,
+    launch_k(summary_bwd_kernel<bf16>, dim3(grid), dim3(256), 0, lc.stream,
+(const bf16*)Hm, alpha, dS, ds, dwp_part,
                                                           T, D, L);
   return cudaGetLastError();
 }
@@ -337,6 +350,7 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
 template <class TO>
 __global__ void __launch_bounds__(256)
     reduce_rows_kernel(const float* __restrict__ in, int rows, int cols, TO* __restrict__ out) {
+  pdl_enter();
   __shared__ float part[8][33];
   const int rg = threadIdx.x >> 5, cl = threadIdx.x & 31;
   const int c = blockIdx.x * 32 + cl;
@@ -357,9 +371,11 @@ cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, i
                         void* out) {
   const int blocks = (cols + 31) / 32;
   if (dtype_out == 0)
-    reduce_rows_kernel<float><<<blocks, 256, 0, lc.stream>>>(in, rows, cols, (float*)out);
+    launch_k(reduce_rows_kernel<float>, dim3(blocks), dim3(256), 0, lc.stream,
+in, rows, cols, (float*)out);
   else
-    reduce_rows_kernel<bf16><<<blocks, 256, 0, lc.stream>>>(in, rows, cols, (bf16*)out);
+    launch_k(reduce_rows_kernel<bf16>, dim3(blocks), dim3(256), 0, lc.stream,
+in, rows, cols, (bf16*)out);
   return cudaGetLastError();
 }
 
