@@ -50,6 +50,27 @@ def dist_env():
             int(os.environ.get("WORLD_SIZE", 1)))
 
 
+def rank_seed(base_seed: int, rank: int) -> int:
+    """Every rank draws its own batch (weak scaling over independent batches)."""
+    return base_seed + rank
+
+
+def max_over_ranks(ms: float, world: int, device=None) -> float:
+    """The slowest rank's time: the job's time."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(world: int, tokens_per_rank_step: int, steps: int, max_ms: float) -> float:
+    """Whole-job throughput: the tokens all ranks processed over the slowest rank's time."""
+    return world * tokens_per_rank_step * steps / (max_ms / 1e3)
+
+
 # ----------------------------------------------------------------- CPU oracle
 ORACLE_SNIPPET = r"""
 import json, os, sys, time
@@ -235,7 +256,7 @@ def bench_ours(args):
 
     name = args.workload or HEADLINE
     w = WORKLOADS[name]
-    t_cpu = make_inputs(w, seed=w.seed + rank)
+    t_cpu = make_inputs(w, seed=rank_seed(w.seed, rank))
     t = {k: v.to(dev) for k, v in t_cpu.items()}
     p = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype)
     pprof = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype, flags=C.BCMT_FLAG_PROFILE)
@@ -303,13 +324,10 @@ def bench_ours(args):
     prof = C.bcmt_profile_read()
     launches = sum(c for c, _ in prof.values())
 
-    if world > 1:
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = tt.item()
-
+    total_ms = max_over_ranks(total_ms, world, dev)
+    eager_ms = max_over_ranks(eager_ms, world, dev)
     tokens_per_step = w.B * w.T
-    value = world * tokens_per_step * args.steps / (total_ms / 1e3)
+    value = job_tokens_per_s(world, tokens_per_step, args.steps, total_ms)
 
     # ---- end to end through the public API: pinned host inputs in, results out
     x_h = t_cpu["x"].pin_memory()
@@ -343,11 +361,8 @@ def bench_ours(args):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = tt.item()
-    e2e_value = world * tokens_per_step * args.steps / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
+    e2e_value = job_tokens_per_s(world, tokens_per_step, args.steps, e2e_ms)
 
     # ---- roofline of the dominant kernel
     model = kernel_model(w)
@@ -407,7 +422,7 @@ def bench_ours(args):
             "cpu_baseline": cpu,
             "kernels": kernels,
             "eager": {"ms_per_step": round(eager_ms / args.steps, 4),
-                      "value": round(world * tokens_per_step * args.steps / (eager_ms / 1e3), 1),
+                      "value": round(job_tokens_per_s(world, tokens_per_step, args.steps, eager_ms), 1),
                       "note": "same steps launched call by call instead of as a graph"},
             "profiled_pass": {"ms_per_step_with_kernel_events": round(prof_ms / args.steps, 4),
                               "note": "per-kernel times come from this second pass of the "
