@@ -189,13 +189,13 @@ def kernel_model(w):
         "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
         # read H; write pooling weights and summaries
         "summary_fwd": ("hbm", n * D * es + n * 4 + B * Nb * D * 4),
-        "memory_scan_fwd": ("hbm", B * Nb * D * (4 + 4 + es) + Nb * D * 4),
-        "gemm_wm": g(B * Nb, D, D),
+        # read S, W_m; write M, Z and the projected, shifted memory C
+        "memory_fwd": ("hbm", B * Nb * D * 4 * 3 + Nb * D * 4 + D * D * es),
         # read dY, G, C; write dU and the shifted memory gradient
         "gate_bwd": ("hbm", 3 * n * D * es + 2 * B * Nb * D * 4),
-        "gemm_dm": g(B * Nb, D, D),
+        "memory_dm": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
         "memory_scan_bwd": ("hbm", B * Nb * D * 8 + Nb * D * 4),
-        "gemm_dwm": g(D, D, B * Nb),
+        "memory_dwm": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
         "summary_bwd": ("hbm", n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
     }
 

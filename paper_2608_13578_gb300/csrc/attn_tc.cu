@@ -198,6 +198,9 @@ __global__ void __launch_bounds__(128)
 }
 
 // ===================================================================== backward
+// Shared memory: Q, K, dO (16 KB each) and a 32 KB region that holds V, then
+// P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in registers
+// until the dV product has consumed P.  80 KB per CTA: two CTAs per SM.
 __global__ void __launch_bounds__(128)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
@@ -210,17 +213,16 @@ __global__ void __launch_bounds__(128)
   uint8_t* sQ = smem;              // Q; then dQ staging
   uint8_t* sK = smem + kTB;        // K; then dK staging
   uint8_t* sdO = smem + 2 * kTB;   // dO; then dV staging
-  uint8_t* sV = smem + 3 * kTB;    // V, then (with the next 16 KB) P
-  uint8_t* sP = sV;                // 32 KB: P, two key atoms
-  uint8_t* sdS = smem + 5 * kTB;   // 32 KB: scale * dS, two key atoms
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 7 * kTB);
+  uint8_t* sV = smem + 3 * kTB;    // V, then (with the next 16 KB) P, then scale * dS
+  uint8_t* sP = sV;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 5 * kTB);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
 
   if (tid == 0) {
-    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    for (int i = 0; i < 4; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
     tc::prefetch_tmap(&mQ);
     tc::prefetch_tmap(&mK);
@@ -266,76 +268,105 @@ __global__ void __launch_bounds__(128)
 
   const int r = warp * 32 + lane;
   const bool row_ok = (t0 + r) < Tlen;
-  // Drow = dO_r . O_r, dO from the swizzled tile once it has landed, O from global
-  bool ok = tc::mbar_wait(&bar[0], 0, status);
-  float drow = 0.f, lr = 0.f;
+  // Drow = dO_r . O_r: the O row (global) is fetched before waiting for the tiles
+  uint4 ov[8];
+  float lr = 0.f;
   if (row_ok) {
     const bf16* orow = O + ((long)b * Tlen + t0 + r) * ld_o + h * kDh;
 #pragma unroll
+    for (int u = 0; u < 8; ++u) ov[u] = *reinterpret_cast<const uint4*>(orow + 8 * u);
+    lr = lse[((long)b * H + h) * Tlen + t0 + r];
+  }
+  bool ok = tc::mbar_wait(&bar[0], 0, status);
+  float drow = 0.f;
+  if (row_ok) {
+#pragma unroll
     for (int u = 0; u < 8; ++u) {
       const uint4 gv = *reinterpret_cast<const uint4*>(sdO + tc::sw128_offset(r, u));
-      const uint4 ov = *reinterpret_cast<const uint4*>(orow + 8 * u);
       const bf16* gp = reinterpret_cast<const bf16*>(&gv);
-      const bf16* op = reinterpret_cast<const bf16*>(&ov);
+      const bf16* op = reinterpret_cast<const bf16*>(&ov[u]);
 #pragma unroll
       for (int e = 0; e < 8; ++e) drow = fmaf(__bfloat162float(gp[e]), __bfloat162float(op[e]), drow);
     }
-    lr = lse[((long)b * H + h) * Tlen + t0 + r];
   }
   ok = tc::mbar_wait(&bar[1], 0, status) && ok;
   tc::fence_after_sync();
 
-  // ---- P = exp(S*scale - lse), dS = scale * P * (dP - Drow), both to shared memory
+  // ---- P = exp(S*scale - lse) to shared memory; scale * P * (dP - Drow) kept
+  // packed in registers (up to 128 keys: 64 words)
   const int nc = L < 32 ? 32 : L;
   const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;
   const int rbs = (r / L) * L;
   const float sl2 = scale * kLog2e, ll2 = lr * kLog2e;
-  for (int c = 0; c < nc; c += 32) {
-    float s[32], dp[32];
-    tc::tmem_ld32(trow + (uint32_t)(wbs + c), s);
-    tc::tmem_ld32(trow + 128u + (uint32_t)(wbs + c), dp);
+  uint32_t dsp[64];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      const int kk = wbs + c + j;
-      const float p = (row_ok && kk >= rbs && kk <= r) ? exp2f(s[j] * sl2 - ll2) : 0.f;
-      s[j] = p;
-      dp[j] = p * (dp[j] - drow) * scale;
-    }
+  for (int ci = 0; ci < 4; ++ci) {
+    if (ci * 32 < nc) {
+      const int c = ci * 32;
+      float s[32], dp[32];
+      tc::tmem_ld32(trow + (uint32_t)(wbs + c), s);
+      tc::tmem_ld32(trow + 128u + (uint32_t)(wbs + c), dp);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      uint4 q, d;
-      q.x = pack2(s[8 * u + 0], s[8 * u + 1]);
-      q.y = pack2(s[8 * u + 2], s[8 * u + 3]);
-      q.z = pack2(s[8 * u + 4], s[8 * u + 5]);
-      q.w = pack2(s[8 * u + 6], s[8 * u + 7]);
-      d.x = pack2(dp[8 * u + 0], dp[8 * u + 1]);
-      d.y = pack2(dp[8 * u + 2], dp[8 * u + 3]);
-      d.z = pack2(dp[8 * u + 4], dp[8 * u + 5]);
-      d.w = pack2(dp[8 * u + 6], dp[8 * u + 7]);
-      put_unit(sP, r, (wbs + c) / 8 + u, q);
-      put_unit(sdS, r, (wbs + c) / 8 + u, d);
+      for (int j = 0; j < 32; ++j) {
+        const int kk = wbs + c + j;
+        const float p = (row_ok && kk >= rbs && kk <= r) ? exp2f(s[j] * sl2 - ll2) : 0.f;
+        s[j] = p;
+        dp[j] = p * (dp[j] - drow) * scale;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        uint4 q;
+        q.x = pack2(s[8 * u + 0], s[8 * u + 1]);
+        q.y = pack2(s[8 * u + 2], s[8 * u + 3]);
+        q.z = pack2(s[8 * u + 4], s[8 * u + 5]);
+        q.w = pack2(s[8 * u + 6], s[8 * u + 7]);
+        put_unit(sP, r, (wbs + c) / 8 + u, q);
+      }
+#pragma unroll
+      for (int j = 0; j < 16; ++j) dsp[ci * 16 + j] = pack2(dp[2 * j], dp[2 * j + 1]);
     }
   }
   const uint4 zero = make_uint4(0, 0, 0, 0);
   for (int u = 0; u < 16; ++u)
-    if (u * 8 < wbs || u * 8 >= wbs + nc) {
-      put_unit(sP, r, u, zero);
-      put_unit(sdS, r, u, zero);
-    }
+    if (u * 8 < wbs || u * 8 >= wbs + nc) put_unit(sP, r, u, zero);
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
 
   if (tid == 0) {
     tc::fence_after_sync();
-    const uint32_t aP = tc::smem_u32(sP), adS = tc::smem_u32(sdS);
     // dV = P^T dO -> columns 0..63 (A = P read MN-major: M = keys, K = queries)
     constexpr uint32_t idMN = tc::idesc_bf16(128, kDh, 1, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
-      tc::mma_bf16(tmem, tc::sdesc(aP + kk * 2048, 16384, 1024),
+      tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sP) + kk * 2048, 16384, 1024),
                    tc::sdesc(tc::smem_u32(sdO) + kk * 2048, 8192, 1024), idMN, kk > 0 ? 1u : 0u);
+    tc::mma_commit(&bar[2]);
+  }
+  __syncwarp();
+  // P consumed: overwrite it with scale * dS
+  ok = tc::mbar_wait(&bar[2], 0, status) && ok;
+  tc::fence_after_sync();
+#pragma unroll
+  for (int ci = 0; ci < 4; ++ci) {
+    if (ci * 32 < nc) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint4 d = make_uint4(dsp[ci * 16 + 4 * u], dsp[ci * 16 + 4 * u + 1],
+                                   dsp[ci * 16 + 4 * u + 2], dsp[ci * 16 + 4 * u + 3]);
+        put_unit(sP, r, (wbs + ci * 32) / 8 + u, d);
+      }
+    }
+  }
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+
+  if (tid == 0) {
+    tc::fence_after_sync();
+    const uint32_t adS = tc::smem_u32(sP);
     // dK = dS^T Q -> columns 64..127
+    constexpr uint32_t idMN = tc::idesc_bf16(128, kDh, 1, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
       tc::mma_bf16(tmem + 64, tc::sdesc(adS + kk * 2048, 16384, 1024),
@@ -346,10 +377,10 @@ __global__ void __launch_bounds__(128)
     for (int kk = 0; kk < kTile / 16; ++kk)
       tc::mma_bf16(tmem + 128, tc::sdesc(adS + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
                    tc::sdesc(tc::smem_u32(sK) + kk * 2048, 8192, 1024), idKM, kk > 0 ? 1u : 0u);
-    tc::mma_commit(&bar[2]);
+    tc::mma_commit(&bar[3]);
   }
   __syncwarp();
-  ok = tc::mbar_wait(&bar[2], 0, status) && ok;
+  ok = tc::mbar_wait(&bar[3], 0, status) && ok;
   tc::fence_after_sync();
 
   // ---- epilogue: rows of dV, dK (key r) and dQ (query r) through staging tiles
@@ -396,7 +427,7 @@ static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, in
 }
 
 static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
-static constexpr int kBwdSmem = 7 * kTB + 1024 + 64;
+static constexpr int kBwdSmem = 5 * kTB + 1024 + 64;
 
 cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
   if (!attn_tc_supported(1, a.dh, a.L)) return cudaErrorNotSupported;

@@ -158,7 +158,7 @@ int dw_splits(int M, int N, long K) {
 }
 
 struct FwdWs {
-  char *qkv, *hhat, *hloc, *G, *Mb;
+  char *qkv, *hhat, *hloc, *G;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
   size_t bytes;
 };
@@ -182,13 +182,11 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     w.spart = reinterpret_cast<float*>(take((size_t)g.n * (g.D / 4) * 4));
     w.S = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.M = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
-    // bf16 copy of M: the A operand of the tensor-core memory projection
-    w.Mb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.M);
     w.Z = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
     w.C = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.G = take((size_t)g.n * g.D * g.es);
   } else {
-    w.hloc = w.G = w.Mb = nullptr;
+    w.hloc = w.G = nullptr;
     w.alpha = w.S = w.M = w.Z = w.C = w.spart = nullptr;
   }
   w.bytes = off;
@@ -196,7 +194,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 }
 
 struct BwdWs {
-  char *dU, *dH, *dHhat, *dqkv, *dPb;
+  char *dU, *dH, *dHhat, *dqkv;
   float *dP, *dM, *dS, *ds, *dwp_part, *Drow, *part;
   size_t bytes;
 };
@@ -214,13 +212,12 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dU = take((size_t)g.n * g.D * g.es);
     w.dH = take((size_t)g.n * g.D * g.es);
     w.dP = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
-    w.dPb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.dP);
     w.dM = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
   } else {
-    w.dU = w.dH = w.dPb = nullptr;
+    w.dU = w.dH = nullptr;
     w.dP = w.dM = w.dS = w.ds = w.dwp_part = nullptr;
   }
   w.dHhat = take((size_t)g.n * g.D * g.es);
@@ -396,21 +393,11 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
-    // Sec. 3.5: exponential causal memory (scan), then projection and shift.
-    pr.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C, g.B,
-                        g.Nb, D);
+    // Sec. 3.5: exponential causal memory, projection and shift in one kernel.
+    pr.begin("memory_fwd");
+    e = memory_fwd(lc, g.dtype, w.S, decay, w_m, w.M, w.Z, w.C, g.B, g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "causal memory");
-    {
-      EpiArgs ea;
-      ea.out = w.C;
-      ea.ldo = D;
-      ea.Nb = g.Nb;
-      e = run_gemm(lc, pr, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
-                   EPI_SHIFT, ea);
-      if (e != cudaSuccess) return cuda_fail(e, "memory projection");
-    }
     // Sec. 3.7-3.8: gate and injection fused into the W_g GEMM.
     EpiArgs ea;
     ea.H = w.hloc;
@@ -475,31 +462,22 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   if (!g.honly) {
     // Sec. 3.8 reversed: dU and the per-block memory gradient (shifted: dP).
     pr.begin("gate_bwd");
-    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.dtype == BCMT_BF16 ? bw.dPb : nullptr,
-                 g.B, g.T, D, g.L);
+    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "gate backward");
     // Sec. 3.5 reversed: dM = dP W_m^T, reverse decayed scan -> dS; dW_m = M^T dP.
-    {
-      EpiArgs ea;
-      ea.out = bw.dM;
-      ea.ldo = D;
-      e = run_gemm(lc, pr, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
-                   EPI_STORE, ea);
-      if (e != cudaSuccess) return cuda_fail(e, "dM");
-    }
+    pr.begin("memory_dm");
+    e = small_gemm(lc, g.dtype, 0, g.B * g.Nb, D, D, bw.dP, D, 1, w_m, 1, D, bw.dM, D);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dM");
     pr.begin("memory_scan_bwd");
     e = memory_scan_bwd(lc, bw.dM, decay, w.Z, bw.dS, g.B, g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
-    {
-      EpiArgs ea;
-      ea.out = dw_m;
-      ea.ldo = D;
-      e = run_gemm(lc, pr, "gemm_dwm", g.dtype, g.dtype, D, D, g.B * g.Nb, w.Mb, 1, D, bw.dPb, D, 1,
-                   EPI_STORE, ea);
-      if (e != cudaSuccess) return cuda_fail(e, "dW_m");
-    }
+    pr.begin("memory_dwm");
+    e = small_gemm(lc, 0, g.dtype, D, D, g.B * g.Nb, w.M, 1, D, bw.dP, D, 1, dw_m, D);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_m");
     // Sec. 3.4 reversed: pooling scores and dW_p.
     pr.begin("summary_bwd");
     e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);

@@ -9,11 +9,22 @@
 
 namespace bcmt {
 
+// Besides operator() (any n, used by the SIMT GEMM), every epilogue offers a
+// two-phase form for the tcgen05 GEMM's 32-column TMEM chunks: load() fetches
+// the chunk's extra inputs into registers (issued a chunk ahead, and for the
+// first chunk before the accumulator is ready), apply() consumes them.
+struct NoPre {};
+
 template <class TO>
 struct EpiStoreF {
+  using Pre = NoPre;
   TO* out;
   long ldo;
   long split_stride;
+  __device__ __forceinline__ void load(int, int, Pre&) const {}
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int z) const {
+    (*this)(row, col, v, 32, z);
+  }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int z) const {
     TO* p = out + (long)z * split_stride + (long)row * ldo + col;
     if (n % 8 == 0) {
@@ -32,11 +43,28 @@ struct EpiStoreF {
 // stores would serialise one memory round trip per vector.
 template <class TO>
 struct EpiStoreScoreF {
+  struct Pre {
+    float w[32];
+  };
   TO* out;
   long ldo;
   const TO* w_p;
   float* spart;
   long n_rows;
+  __device__ __forceinline__ void load(int, int col, Pre& pre) const {
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) load8(w_p + col + j, pre.w + j);
+  }
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
+                                        int) const {
+    TO* p = out + (long)row * ldo + col;
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) s = fmaf(to_f(from_f<TO>(v[j])), pre.w[j], s);
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store8(p + j, v + j);
+    spart[(long)(col / 32) * n_rows + row] = s;
+  }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     float w[32];
     for (int j = 0; j < n; j += 4) load4(w_p + col + j, w + j);
@@ -55,9 +83,14 @@ struct EpiStoreScoreF {
 // Sec. 3.5 shift: row m = b*Nb + i of M W_m becomes the memory row of block
 // i+1 of the same sequence; the last block's row is dropped.
 struct EpiShiftF {
+  using Pre = NoPre;
   float* out;
   long ldo;
   int Nb;
+  __device__ __forceinline__ void load(int, int, Pre&) const {}
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int z) const {
+    (*this)(row, col, v, 32, z);
+  }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     if ((row % Nb) + 1 >= Nb) return;
     float* p = out + (long)(row + 1) * ldo + col;
@@ -68,11 +101,39 @@ struct EpiShiftF {
 // Sec. 3.8: G = sigmoid(H W_g), Y = H + G * M_tokens, M_tokens row = Cmem[b, t/L].
 template <class T>
 struct EpiGateInjectF {
+  struct Pre {
+    float h[32], c[32];
+  };
   const T* H;
   const float* Cmem;
   T* G;
   T* Y;
   int Tlen, L, Nb, D;
+  __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
+    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
+    const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
+    const T* h = H + (long)row * D + col;
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      load8(h + j, pre.h + j);
+      load8(cm + j, pre.c + j);
+    }
+  }
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
+                                        int) const {
+    const long o = (long)row * D + col;
+    float g[32], y[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      g[j] = sigmoidf_(v[j]);
+      y[j] = fmaf(g[j], pre.c[j], pre.h[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      store8(G + o + j, g + j);
+      store8(Y + o + j, y + j);
+    }
+  }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
@@ -105,6 +166,10 @@ struct EpiGateInjectF {
 // Y = H + ...) + alpha_t dS_blk (pooling S = H^T alpha) + ds_t w_p (scores).
 template <class T>
 struct EpiDHF {
+  struct Pre {
+    float dy[32], sv[32], wp[32];
+    float at, st;
+  };
   const T* dY;
   const float* alpha;
   const float* dS;
@@ -112,6 +177,28 @@ struct EpiDHF {
   const T* w_p;
   T* out;
   int Tlen, L, Nb, D;
+  __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
+    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
+    const float* dsb = dS + ((long)b * Nb + blk) * D + col;
+    const T* dy = dY + (long)row * D + col;
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      load8(dy + j, pre.dy + j);
+      load8(dsb + j, pre.sv + j);
+      load8(w_p + col + j, pre.wp + j);
+    }
+    pre.at = alpha[row];
+    pre.st = ds[row];
+  }
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
+                                        int) const {
+    const long o = (long)row * D + col;
+    float r[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) r[j] = v[j] + pre.dy[j] + pre.at * pre.sv[j] + pre.st * pre.wp[j];
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store8(out + o + j, r + j);
+  }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* dsb = dS + ((long)b * Nb + blk) * D + col;

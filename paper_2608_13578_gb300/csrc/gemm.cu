@@ -299,16 +299,23 @@ __global__ void __launch_bounds__(192, 1)
       const int m_blk = tile % tiles_m, rest = tile / tiles_m;
       const int n_blk = rest % tiles_n, z = rest / tiles_n;
       const int acc = j & 1, use = j >> 1;
-      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
-      tc::fence_after_sync();
       const int row = m_blk * kBM + q * 32 + lane;
       const int n0 = n_blk * BN;
+      const bool row_ok = row < M;
+      // The epilogue's own inputs do not depend on the accumulator: fetch the
+      // first chunk's before waiting for it, and each next chunk's one ahead.
+      typename Epi::Pre pre[2];
+      if (row_ok && n0 < N) epi.load(row, n0, pre[0]);
+      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
+      tc::fence_after_sync();
       const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-#pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
+#pragma unroll
+      for (int ci = 0; ci < BN / 32; ++ci) {
+        const int c = ci * 32;
+        if (ci + 1 < BN / 32 && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
         float v[32];
         tc::tmem_ld32(base + (uint32_t)c, v);
-        if (ok && row < M && n0 + c < N) epi(row, n0 + c, v, 32, z);
+        if (ok && row_ok && n0 + c < N) epi.apply(row, n0 + c, v, pre[ci & 1], z);
       }
       tc::fence_before_sync();
       __syncwarp();

@@ -116,15 +116,19 @@ bool attn_tc_supported(int dtype, int dh, int L);
 // spart[j * B*T + token]), alpha = softmax(s), S = H^T alpha.
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
                         float* alpha, float* S, int B, int T, int D, int L);
-// Sec. 3.5: M = normalised decayed scan of S over blocks (fp32, plus a bf16
-// copy in Mb when non-null), Z its denominator [Nb, D], C[b, 0] = 0.  The
-// projection C[b, i+1] = M_i W_m is a GEMM with the EPI_SHIFT epilogue.
-cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D);
+// Sec. 3.5: M = normalised decayed scan of S over blocks, Z its denominator
+// [Nb, D], and the projected, shifted memory C[b, 0] = 0, C[b, i+1] = M_i W_m.
+cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
+                       const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D);
+// out[m, n] = sum_k A(m,k) B(k,n) on CUDA cores in 16 x 32 tiles (small
+// products of the memory stage); A fp32, B of dtype_b, out of dtype_out.
+cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int N, int K,
+                       const float* A, long sam, long sak, const void* B, long sbk, long sbn,
+                       void* out, long ldo);
 // Backward of the gate and injection: dU = dY*C*G*(1-G); dP[b,i-1] = sum over
-// block i of dY*G (also as bf16 in dPb when non-null); dP[b,Nb-1] = 0.
+// block i of dY*G; dP[b,Nb-1] = 0.
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, void* dPb, int B, int T, int D, int L);
+                     void* dU, float* dP, int B, int T, int D, int L);
 // Backward of the memory scan: dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i, given
 // dM = dP W_m^T.
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,

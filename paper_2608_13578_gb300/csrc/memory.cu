@@ -101,49 +101,165 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 }
 
 // -------------------------------------------------------------- Sec. 3.5
-// One thread per (batch b, channel c): the decayed scan over blocks
-//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i,
-// the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j).
-// Writes M (fp32, and a bf16 copy for the tensor-core projection when Mb is
-// given), Z (batch 0 only; it does not depend on b) and the first block's
-// memory row C[b, 0] = 0.  The projection C[b, i+1] = M_i W_m follows as a GEMM.
-__global__ void __launch_bounds__(128)
-    memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
-                           float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
-                           float* __restrict__ Cmem, int Nb, int D) {
+// Memory rows for blocks i0 .. i0+15 of batch b, projected and shifted:
+// C[b, i+1, n0 .. n0+31] = M_i W_m[:, n0 .. n0+31] (and C[b, 0] = 0).
+// The decayed scan
+//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i
+// (the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j)) is
+// recomputed per CTA from block 0 for every channel straight into shared
+// memory, so the projection needs no separate pass.  The CTAs of the first
+// column tile also store M (for dW_m) and, for batch 0, Z (for the backward
+// scan).  Grid (D/32, ceil(Nb/16), B), 256 threads; thread (r, p) computes
+// output row i0+r, columns n0+2p and n0+2p+1.
+template <class TW>
+__global__ void __launch_bounds__(256)
+    memory_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
+                      const TW* __restrict__ w_m, float* __restrict__ M, float* __restrict__ Z,
+                      float* __restrict__ Cmem, int Nb, int D) {
   pdl_enter();
-  const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
-  if (c >= D) return;
-  const float a = decay[c];
-  const long base = (long)b * Nb * D + c;
-  float Nn = 0.f, Zz = 0.f;
-  constexpr int U = 8;
-  for (int i0 = 0; i0 < Nb; i0 += U) {
-    float sv[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) sv[u] = (i0 + u < Nb) ? S[base + (long)(i0 + u) * D] : 0.f;
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u;
-      if (i < Nb) {
-        Nn = fmaf(a, Nn, sv[u]);
-        Zz = fmaf(a, Zz, 1.0f);
+  extern __shared__ float Ms[];  // [16][D + 1]
+  __shared__ float Ws[64][33];
+  const int n0 = blockIdx.x * 32, i0 = blockIdx.y * 16, b = blockIdx.z;
+  const int i1 = min(Nb, i0 + 16);
+  const int ld = D + 1;
+  const bool keep = blockIdx.x == 0;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    const float a = decay[k];
+    float Nn = 0.f, Zz = 0.f;
+    for (int i = 0; i < i1; ++i) {
+      Nn = fmaf(a, Nn, S[((long)b * Nb + i) * D + k]);
+      Zz = fmaf(a, Zz, 1.0f);
+      if (i >= i0) {
         const float m = Nn / Zz;
-        M[base + (long)i * D] = m;
-        if (Mb) Mb[base + (long)i * D] = __float2bfloat16_rn(m);
-        if (b == 0) Z[(long)i * D + c] = Zz;
+        Ms[(i - i0) * ld + k] = m;
+        if (keep) {
+          M[((long)b * Nb + i) * D + k] = m;
+          if (b == 0) Z[(long)i * D + k] = Zz;
+        }
       }
     }
+    for (int i = i1; i < i0 + 16; ++i) Ms[(i - i0) * ld + k] = 0.f;
   }
-  Cmem[base] = 0.f;
+  const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
+  float acc0 = 0.f, acc1 = 0.f;
+  for (int k0 = 0; k0 < D; k0 += 64) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < 64 * 32; e += blockDim.x) {
+      const int kk = e >> 5, nn = e & 31;
+      Ws[kk][nn] = to_f(w_m[(long)(k0 + kk) * D + n0 + nn]);
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int kk = 0; kk < 64; ++kk) {
+      const float m = Ms[r * ld + k0 + kk];
+      acc0 = fmaf(m, Ws[kk][2 * p], acc0);
+      acc1 = fmaf(m, Ws[kk][2 * p + 1], acc1);
+    }
+  }
+  const int i = i0 + r;
+  if (i + 1 < Nb) {
+    float* c = Cmem + ((long)b * Nb + i + 1) * D + n0 + 2 * p;
+    c[0] = acc0;
+    c[1] = acc1;
+  }
+  if (i0 == 0 && r == 0) {
+    float* c = Cmem + (long)b * Nb * D + n0 + 2 * p;
+    c[0] = 0.f;
+    c[1] = 0.f;
+  }
 }
 
-cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D) {
-  dim3 grid((D + 127) / 128, B);
-  launch_k(memory_scan_fwd_kernel, dim3(grid), dim3(128), 0, lc.stream,
-S, decay, M, (bf16*)Mb, Z, Cmem, Nb, D);
-  return cudaGetLastError();
+cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
+                       const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D) {
+  if (D % 64 != 0) return cudaErrorInvalidValue;
+  dim3 grid(D / 32, (Nb + 15) / 16, B);
+  const size_t smem = (size_t)16 * (D + 1) * sizeof(float);
+  static size_t attr_bytes[2] = {0, 0};  // largest dynamic smem opted into, per instantiation
+  cudaError_t e = cudaSuccess;
+  if (dtype == 0) {
+    if (smem > attr_bytes[0]) {
+      e = cudaFuncSetAttribute(memory_fwd_kernel<float>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess) attr_bytes[0] = smem;
+    }
+    if (e == cudaSuccess)
+      e = launch_k(memory_fwd_kernel<float>, grid, dim3(256), smem, lc.stream, S, decay,
+                   (const float*)w_m, M, Z, Cmem, Nb, D);
+  } else {
+    if (smem > attr_bytes[1]) {
+      e = cudaFuncSetAttribute(memory_fwd_kernel<bf16>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess) attr_bytes[1] = smem;
+    }
+    if (e == cudaSuccess)
+      e = launch_k(memory_fwd_kernel<bf16>, grid, dim3(256), smem, lc.stream, S, decay,
+                   (const bf16*)w_m, M, Z, Cmem, Nb, D);
+  }
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Small products of the memory stage's backward on CUDA cores, in 16 x 32
+// output tiles so even a [128 x 512] result spreads over 128 CTAs:
+// out[m, n] = sum_k A(m, k) B(k, n) with A(m,k) = A[m*sam + k*sak] (fp32) and
+// B(k,n) = B[k*sbk + n*sbn] (fp32 or bf16), stored as TO.
+template <class TB, class TO>
+__global__ void __launch_bounds__(256)
+    small_gemm_kernel(int Mr, int N, int K, const float* __restrict__ A, long sam, long sak,
+                      const TB* __restrict__ Bm, long sbk, long sbn, TO* __restrict__ out,
+                      long ldo) {
+  pdl_enter();
+  __shared__ float As[16][65];
+  __shared__ float Bs[64][33];
+  const int n0 = blockIdx.x * 32, m0 = blockIdx.y * 16;
+  const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
+  float acc0 = 0.f, acc1 = 0.f;
+  for (int k0 = 0; k0 < K; k0 += 64) {
+    for (int e = threadIdx.x; e < 16 * 64; e += blockDim.x) {
+      int mm, kk;
+      if (sak == 1) { mm = e >> 6; kk = e & 63; } else { kk = e >> 4; mm = e & 15; }
+      const int m = m0 + mm, k = k0 + kk;
+      As[mm][kk] = (m < Mr && k < K) ? A[(long)m * sam + (long)k * sak] : 0.f;
+    }
+    for (int e = threadIdx.x; e < 64 * 32; e += blockDim.x) {
+      int kk, nn;
+      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 6; kk = e & 63; }
+      const int n = n0 + nn, k = k0 + kk;
+      Bs[kk][nn] = (n < N && k < K) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int kk = 0; kk < 64; ++kk) {
+      const float a = As[r][kk];
+      acc0 = fmaf(a, Bs[kk][2 * p], acc0);
+      acc1 = fmaf(a, Bs[kk][2 * p + 1], acc1);
+    }
+    __syncthreads();
+  }
+  const int m = m0 + r, n = n0 + 2 * p;
+  if (m < Mr) {
+    if (n < N) out[(long)m * ldo + n] = from_f<TO>(acc0);
+    if (n + 1 < N) out[(long)m * ldo + n + 1] = from_f<TO>(acc1);
+  }
+}
+
+cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int N, int K,
+                       const float* A, long sam, long sak, const void* B, long sbk, long sbn,
+                       void* out, long ldo) {
+  dim3 grid((N + 31) / 32, (M + 15) / 16);
+  cudaError_t e;
+  if (dtype_b == 0 && dtype_out == 0)
+    e = launch_k(small_gemm_kernel<float, float>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
+                 sak, (const float*)B, sbk, sbn, (float*)out, ldo);
+  else if (dtype_b == 0)
+    e = launch_k(small_gemm_kernel<float, bf16>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
+                 sak, (const float*)B, sbk, sbn, (bf16*)out, ldo);
+  else if (dtype_out == 0)
+    e = launch_k(small_gemm_kernel<bf16, float>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
+                 sak, (const bf16*)B, sbk, sbn, (float*)out, ldo);
+  else
+    e = launch_k(small_gemm_kernel<bf16, bf16>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
+                 sak, (const bf16*)B, sbk, sbn, (bf16*)out, ldo);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // ----------------------------------------------------- Sec. 3.8 backward
@@ -155,7 +271,7 @@ template <class T>
 __global__ void __launch_bounds__(256)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
                     const float* __restrict__ Cmem, T* __restrict__ dU, float* __restrict__ dP,
-                    bf16* __restrict__ dPb, int Tlen, int D, int L) {
+                    int Tlen, int D, int L) {
   pdl_enter();
   // 8 row groups x 32 threads of 4 channels: 128 channels per CTA.
   __shared__ float part[8][128 + 4];
@@ -193,23 +309,22 @@ __global__ void __launch_bounds__(256)
       const long o = (i > 0) ? ((long)b * Nb + i - 1) * D + cc : ((long)b * Nb + Nb - 1) * D + cc;
       if (i == 0) t = 0.f;
       dP[o] = t;
-      if (dPb) dPb[o] = __float2bfloat16_rn(t);
     }
   }
 }
 
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
+                     void* dU, float* dP, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
   dim3 grid((D + 127) / 128, Nb, B);
   if (dtype == 0)
     launch_k(gate_bwd_kernel<float>, dim3(grid), dim3(256), 0, lc.stream,
 (const float*)dY, (const float*)G, Cmem,
-                                                        (float*)dU, dP, (bf16*)dPb, T, D, L);
+                                                        (float*)dU, dP, T, D, L);
   else
     launch_k(gate_bwd_kernel<bf16>, dim3(grid), dim3(256), 0, lc.stream,
 (const bf16*)dY, (const bf16*)G, Cmem,
-                                                       (bf16*)dU, dP, (bf16*)dPb, T, D, L);
+                                                       (bf16*)dU, dP, T, D, L);
   return cudaGetLastError();
 }
 
