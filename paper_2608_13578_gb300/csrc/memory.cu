@@ -101,40 +101,89 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 }
 
 // -------------------------------------------------------------- Sec. 3.5
+// Small products of the memory stage on CUDA cores, in 16 x 32 output tiles
+// so even a [128 x 512] result spreads over 128 CTAs.  K is consumed in
+// chunks of kKC; every load of a chunk is issued into registers before the
+// first one is used, so a chunk costs one memory round trip, not one per
+// element.  Thread (r, p) of 256 owns output row r and columns 2p, 2p+1.
+constexpr int kKC = 256;
+
+template <class TB>
+__device__ __forceinline__ void stage_b_chunk(float (*Bs)[33], const TB* __restrict__ Bm, long sbk,
+                                              long sbn, int k0, int K, int n0, int N) {
+  // kKC x 32 elements, 32 per thread, all loads first
+  float v[32];
+#pragma unroll
+  for (int q = 0; q < 32; ++q) {
+    const int e = threadIdx.x + q * 256;
+    int kk, nn;
+    if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
+    const int k = k0 + kk, n = n0 + nn;
+    v[q] = (k < K && n < N) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
+  }
+#pragma unroll
+  for (int q = 0; q < 32; ++q) {
+    const int e = threadIdx.x + q * 256;
+    int kk, nn;
+    if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
+    Bs[kk][nn] = v[q];
+  }
+}
+
+__device__ __forceinline__ void mac_chunk(const float* __restrict__ arow, float (*Bs)[33], int p,
+                                          float& acc0, float& acc1) {
+#pragma unroll 16
+  for (int kk = 0; kk < kKC; ++kk) {
+    const float a = arow[kk];
+    acc0 = fmaf(a, Bs[kk][2 * p], acc0);
+    acc1 = fmaf(a, Bs[kk][2 * p + 1], acc1);
+  }
+}
+
 // Memory rows for blocks i0 .. i0+15 of batch b, projected and shifted:
-// C[b, i+1, n0 .. n0+31] = M_i W_m[:, n0 .. n0+31] (and C[b, 0] = 0).
-// The decayed scan
+// C[b, i+1, n0 .. n0+31] = M_i W_m[:, n0 .. n0+31] (and C[b, 0] = 0).  The
+// decayed scan
 //   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i
 // (the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j)) is
 // recomputed per CTA from block 0 for every channel straight into shared
 // memory, so the projection needs no separate pass.  The CTAs of the first
 // column tile also store M (for dW_m) and, for batch 0, Z (for the backward
-// scan).  Grid (D/32, ceil(Nb/16), B), 256 threads; thread (r, p) computes
-// output row i0+r, columns n0+2p and n0+2p+1.
+// scan).  Grid (D/32, ceil(Nb/16), B).
 template <class TW>
 __global__ void __launch_bounds__(256)
     memory_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                       const TW* __restrict__ w_m, float* __restrict__ M, float* __restrict__ Z,
                       float* __restrict__ Cmem, int Nb, int D) {
   pdl_enter();
-  extern __shared__ float Ms[];  // [16][D + 1]
-  __shared__ float Ws[64][33];
+  extern __shared__ float dyn[];
+  float* Ms = dyn;                                         // [16][D + 1]
+  float(*Bs)[33] = reinterpret_cast<float(*)[33]>(dyn + 16 * (D + 1));  // [kKC][33]
   const int n0 = blockIdx.x * 32, i0 = blockIdx.y * 16, b = blockIdx.z;
   const int i1 = min(Nb, i0 + 16);
   const int ld = D + 1;
   const bool keep = blockIdx.x == 0;
   for (int k = threadIdx.x; k < D; k += blockDim.x) {
     const float a = decay[k];
+    const float* Sk = S + (long)b * Nb * D + k;
     float Nn = 0.f, Zz = 0.f;
-    for (int i = 0; i < i1; ++i) {
-      Nn = fmaf(a, Nn, S[((long)b * Nb + i) * D + k]);
-      Zz = fmaf(a, Zz, 1.0f);
-      if (i >= i0) {
-        const float m = Nn / Zz;
-        Ms[(i - i0) * ld + k] = m;
-        if (keep) {
-          M[((long)b * Nb + i) * D + k] = m;
-          if (b == 0) Z[(long)i * D + k] = Zz;
+    for (int c0 = 0; c0 < i1; c0 += 16) {
+      float sv[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) sv[u] = (c0 + u < i1) ? Sk[(long)(c0 + u) * D] : 0.f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int i = c0 + u;
+        if (i < i1) {
+          Nn = fmaf(a, Nn, sv[u]);
+          Zz = fmaf(a, Zz, 1.0f);
+          if (i >= i0) {
+            const float m = Nn / Zz;
+            Ms[(i - i0) * ld + k] = m;
+            if (keep) {
+              M[((long)b * Nb + i) * D + k] = m;
+              if (b == 0) Z[(long)i * D + k] = Zz;
+            }
+          }
         }
       }
     }
@@ -142,19 +191,11 @@ __global__ void __launch_bounds__(256)
   }
   const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
   float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < D; k0 += 64) {
+  for (int k0 = 0; k0 < D; k0 += kKC) {
     __syncthreads();
-    for (int e = threadIdx.x; e < 64 * 32; e += blockDim.x) {
-      const int kk = e >> 5, nn = e & 31;
-      Ws[kk][nn] = to_f(w_m[(long)(k0 + kk) * D + n0 + nn]);
-    }
+    stage_b_chunk<TW>(Bs, w_m, D, 1, k0, D, n0, D);
     __syncthreads();
-#pragma unroll 8
-    for (int kk = 0; kk < 64; ++kk) {
-      const float m = Ms[r * ld + k0 + kk];
-      acc0 = fmaf(m, Ws[kk][2 * p], acc0);
-      acc1 = fmaf(m, Ws[kk][2 * p + 1], acc1);
-    }
+    mac_chunk(Ms + r * ld + k0, Bs, p, acc0, acc1);
   }
   const int i = i0 + r;
   if (i + 1 < Nb) {
@@ -169,28 +210,27 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+static cudaError_t opt_in_smem(const void* kern, size_t bytes, size_t* cached) {
+  if (bytes <= *cached) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess) *cached = bytes;
+  return e;
+}
+
 cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float* decay,
                        const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D) {
   if (D % 64 != 0) return cudaErrorInvalidValue;
   dim3 grid(D / 32, (Nb + 15) / 16, B);
-  const size_t smem = (size_t)16 * (D + 1) * sizeof(float);
-  static size_t attr_bytes[2] = {0, 0};  // largest dynamic smem opted into, per instantiation
-  cudaError_t e = cudaSuccess;
+  const size_t smem = ((size_t)16 * (D + 1) + (size_t)kKC * 33) * sizeof(float);
+  static size_t attr_bytes[2] = {0, 0};
+  cudaError_t e;
   if (dtype == 0) {
-    if (smem > attr_bytes[0]) {
-      e = cudaFuncSetAttribute(memory_fwd_kernel<float>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess) attr_bytes[0] = smem;
-    }
+    e = opt_in_smem((const void*)memory_fwd_kernel<float>, smem, &attr_bytes[0]);
     if (e == cudaSuccess)
       e = launch_k(memory_fwd_kernel<float>, grid, dim3(256), smem, lc.stream, S, decay,
                    (const float*)w_m, M, Z, Cmem, Nb, D);
   } else {
-    if (smem > attr_bytes[1]) {
-      e = cudaFuncSetAttribute(memory_fwd_kernel<bf16>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess) attr_bytes[1] = smem;
-    }
+    e = opt_in_smem((const void*)memory_fwd_kernel<bf16>, smem, &attr_bytes[1]);
     if (e == cudaSuccess)
       e = launch_k(memory_fwd_kernel<bf16>, grid, dim3(256), smem, lc.stream, S, decay,
                    (const bf16*)w_m, M, Z, Cmem, Nb, D);
@@ -198,9 +238,7 @@ cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float*
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-// Small products of the memory stage's backward on CUDA cores, in 16 x 32
-// output tiles so even a [128 x 512] result spreads over 128 CTAs:
-// out[m, n] = sum_k A(m, k) B(k, n) with A(m,k) = A[m*sam + k*sak] (fp32) and
+// out[m, n] = sum_k A(m, k) B(k, n), A(m,k) = A[m*sam + k*sak] (fp32),
 // B(k,n) = B[k*sbk + n*sbn] (fp32 or bf16), stored as TO.
 template <class TB, class TO>
 __global__ void __launch_bounds__(256)
@@ -208,32 +246,35 @@ __global__ void __launch_bounds__(256)
                       const TB* __restrict__ Bm, long sbk, long sbn, TO* __restrict__ out,
                       long ldo) {
   pdl_enter();
-  __shared__ float As[16][65];
-  __shared__ float Bs[64][33];
+  extern __shared__ float dyn[];
+  float* As = dyn;                                              // [16][kKC + 1]
+  float(*Bs)[33] = reinterpret_cast<float(*)[33]>(dyn + 16 * (kKC + 1));
   const int n0 = blockIdx.x * 32, m0 = blockIdx.y * 16;
   const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
   float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < K; k0 += 64) {
-    for (int e = threadIdx.x; e < 16 * 64; e += blockDim.x) {
-      int mm, kk;
-      if (sak == 1) { mm = e >> 6; kk = e & 63; } else { kk = e >> 4; mm = e & 15; }
-      const int m = m0 + mm, k = k0 + kk;
-      As[mm][kk] = (m < Mr && k < K) ? A[(long)m * sam + (long)k * sak] : 0.f;
-    }
-    for (int e = threadIdx.x; e < 64 * 32; e += blockDim.x) {
-      int kk, nn;
-      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 6; kk = e & 63; }
-      const int n = n0 + nn, k = k0 + kk;
-      Bs[kk][nn] = (n < N && k < K) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
-    }
+  for (int k0 = 0; k0 < K; k0 += kKC) {
     __syncthreads();
-#pragma unroll 8
-    for (int kk = 0; kk < 64; ++kk) {
-      const float a = As[r][kk];
-      acc0 = fmaf(a, Bs[kk][2 * p], acc0);
-      acc1 = fmaf(a, Bs[kk][2 * p + 1], acc1);
+    {
+      float v[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        const int e = threadIdx.x + q * 256;
+        int mm, kk;
+        if (sak == 1) { mm = e >> 8; kk = e & 255; } else { kk = e >> 4; mm = e & 15; }
+        const int m = m0 + mm, k = k0 + kk;
+        v[q] = (m < Mr && k < K) ? A[(long)m * sam + (long)k * sak] : 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        const int e = threadIdx.x + q * 256;
+        int mm, kk;
+        if (sak == 1) { mm = e >> 8; kk = e & 255; } else { kk = e >> 4; mm = e & 15; }
+        As[mm * (kKC + 1) + kk] = v[q];
+      }
     }
+    stage_b_chunk<TB>(Bs, Bm, sbk, sbn, k0, K, n0, N);
     __syncthreads();
+    mac_chunk(As + r * (kKC + 1), Bs, p, acc0, acc1);
   }
   const int m = m0 + r, n = n0 + 2 * p;
   if (m < Mr) {
@@ -246,19 +287,30 @@ cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int 
                        const float* A, long sam, long sak, const void* B, long sbk, long sbn,
                        void* out, long ldo) {
   dim3 grid((N + 31) / 32, (M + 15) / 16);
+  const size_t smem = ((size_t)16 * (kKC + 1) + (size_t)kKC * 33) * sizeof(float);
+  static size_t attr_bytes[4] = {0, 0, 0, 0};
   cudaError_t e;
-  if (dtype_b == 0 && dtype_out == 0)
-    e = launch_k(small_gemm_kernel<float, float>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
-                 sak, (const float*)B, sbk, sbn, (float*)out, ldo);
-  else if (dtype_b == 0)
-    e = launch_k(small_gemm_kernel<float, bf16>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
-                 sak, (const float*)B, sbk, sbn, (bf16*)out, ldo);
-  else if (dtype_out == 0)
-    e = launch_k(small_gemm_kernel<bf16, float>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
-                 sak, (const bf16*)B, sbk, sbn, (float*)out, ldo);
-  else
-    e = launch_k(small_gemm_kernel<bf16, bf16>, grid, dim3(256), 0, lc.stream, M, N, K, A, sam,
-                 sak, (const bf16*)B, sbk, sbn, (bf16*)out, ldo);
+  if (dtype_b == 0 && dtype_out == 0) {
+    e = opt_in_smem((const void*)small_gemm_kernel<float, float>, smem, &attr_bytes[0]);
+    if (e == cudaSuccess)
+      e = launch_k(small_gemm_kernel<float, float>, grid, dim3(256), smem, lc.stream, M, N, K, A,
+                   sam, sak, (const float*)B, sbk, sbn, (float*)out, ldo);
+  } else if (dtype_b == 0) {
+    e = opt_in_smem((const void*)small_gemm_kernel<float, bf16>, smem, &attr_bytes[1]);
+    if (e == cudaSuccess)
+      e = launch_k(small_gemm_kernel<float, bf16>, grid, dim3(256), smem, lc.stream, M, N, K, A,
+                   sam, sak, (const float*)B, sbk, sbn, (bf16*)out, ldo);
+  } else if (dtype_out == 0) {
+    e = opt_in_smem((const void*)small_gemm_kernel<bf16, float>, smem, &attr_bytes[2]);
+    if (e == cudaSuccess)
+      e = launch_k(small_gemm_kernel<bf16, float>, grid, dim3(256), smem, lc.stream, M, N, K, A,
+                   sam, sak, (const bf16*)B, sbk, sbn, (float*)out, ldo);
+  } else {
+    e = opt_in_smem((const void*)small_gemm_kernel<bf16, bf16>, smem, &attr_bytes[3]);
+    if (e == cudaSuccess)
+      e = launch_k(small_gemm_kernel<bf16, bf16>, grid, dim3(256), smem, lc.stream, M, N, K, A,
+                   sam, sak, (const bf16*)B, sbk, sbn, (bf16*)out, ldo);
+  }
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
