@@ -69,6 +69,26 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 __device__ __forceinline__ float sigmoidf_(float u) { return 1.0f / (1.0f + expf(-u)); }
+// Hardware-approximate sigmoid (ex2.approx and an approximate divide, a few
+// ulp in fp32) for results stored in bf16, whose rounding is ~1000x coarser.
+__device__ __forceinline__ float sigmoid_bf16out(float u) {
+  return __fdividef(1.0f, 1.0f + __expf(-u));
+}
+
+// Raw bf16 pairs, converted when used.
+__device__ __forceinline__ void load8_raw(const bf16* p, uint4& raw) {
+  raw = *reinterpret_cast<const uint4*>(p);
+}
+__device__ __forceinline__ void unpack8(const uint4& raw, float* v) {
+  const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+    float2 f = __bfloat1622float2(h);
+    v[2 * i] = f.x;
+    v[2 * i + 1] = f.y;
+  }
+}
 
 // Vector load/store of 4 consecutive elements (16 B for fp32, 8 B for bf16).
 // The address must be aligned to the vector width.

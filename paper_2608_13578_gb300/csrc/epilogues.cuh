@@ -43,8 +43,9 @@ struct EpiStoreF {
 // stores would serialise one memory round trip per vector.
 template <class TO>
 struct EpiStoreScoreF {
+  // tcgen05 path (bf16 only): w_p as raw bf16 pairs
   struct Pre {
-    float w[32];
+    uint4 w[4];
   };
   TO* out;
   long ldo;
@@ -52,17 +53,23 @@ struct EpiStoreScoreF {
   float* spart;
   long n_rows;
   __device__ __forceinline__ void load(int, int col, Pre& pre) const {
+    const bf16* wp = reinterpret_cast<const bf16*>(w_p) + col;
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) load8(w_p + col + j, pre.w + j);
+    for (int j = 0; j < 4; ++j) load8_raw(wp + 8 * j, pre.w[j]);
   }
   __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
                                         int) const {
-    TO* p = out + (long)row * ldo + col;
+    bf16* p = reinterpret_cast<bf16*>(out) + (long)row * ldo + col;
     float s = 0.f;
 #pragma unroll
-    for (int j = 0; j < 32; ++j) s = fmaf(to_f(from_f<TO>(v[j])), pre.w[j], s);
+    for (int q = 0; q < 4; ++q) {
+      float w[8];
+      unpack8(pre.w[q], w);
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) store8(p + j, v + j);
+      for (int e = 0; e < 8; ++e)
+        s = fmaf(__bfloat162float(__float2bfloat16_rn(v[8 * q + e])), w[e], s);
+      store8(p + 8 * q, v + 8 * q);
+    }
     spart[(long)(col / 32) * n_rows + row] = s;
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
@@ -101,8 +108,10 @@ struct EpiShiftF {
 // Sec. 3.8: G = sigmoid(H W_g), Y = H + G * M_tokens, M_tokens row = Cmem[b, t/L].
 template <class T>
 struct EpiGateInjectF {
+  // tcgen05 path (bf16 only): H as raw bf16 pairs, C in fp32
   struct Pre {
-    float h[32], c[32];
+    uint4 h[4];
+    float c[32];
   };
   const T* H;
   const float* Cmem;
@@ -112,26 +121,26 @@ struct EpiGateInjectF {
   __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
-    const T* h = H + (long)row * D + col;
+    const bf16* h = reinterpret_cast<const bf16*>(H) + (long)row * D + col;
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) {
-      load8(h + j, pre.h + j);
-      load8(cm + j, pre.c + j);
-    }
+    for (int j = 0; j < 4; ++j) load8_raw(h + 8 * j, pre.h[j]);
+#pragma unroll
+    for (int j = 0; j < 32; j += 4) load4(cm + j, pre.c + j);
   }
   __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
                                         int) const {
     const long o = (long)row * D + col;
-    float g[32], y[32];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      g[j] = sigmoidf_(v[j]);
-      y[j] = fmaf(g[j], pre.c[j], pre.h[j]);
-    }
+    for (int q = 0; q < 4; ++q) {
+      float h[8], g[8], y[8];
+      unpack8(pre.h[q], h);
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) {
-      store8(G + o + j, g + j);
-      store8(Y + o + j, y + j);
+      for (int e = 0; e < 8; ++e) {
+        g[e] = sigmoid_bf16out(v[8 * q + e]);
+        y[e] = fmaf(g[e], pre.c[8 * q + e], h[e]);
+      }
+      store8(reinterpret_cast<bf16*>(G) + o + 8 * q, g);
+      store8(reinterpret_cast<bf16*>(Y) + o + 8 * q, y);
     }
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
@@ -166,8 +175,10 @@ struct EpiGateInjectF {
 // Y = H + ...) + alpha_t dS_blk (pooling S = H^T alpha) + ds_t w_p (scores).
 template <class T>
 struct EpiDHF {
+  // tcgen05 path (bf16 only): dY and w_p as raw bf16 pairs, dS in fp32
   struct Pre {
-    float dy[32], sv[32], wp[32];
+    uint4 dy[4], wp[4];
+    float sv[32];
     float at, st;
   };
   const T* dY;
@@ -180,24 +191,31 @@ struct EpiDHF {
   __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
     const float* dsb = dS + ((long)b * Nb + blk) * D + col;
-    const T* dy = dY + (long)row * D + col;
+    const bf16* dy = reinterpret_cast<const bf16*>(dY) + (long)row * D + col;
+    const bf16* wp = reinterpret_cast<const bf16*>(w_p) + col;
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) {
-      load8(dy + j, pre.dy + j);
-      load8(dsb + j, pre.sv + j);
-      load8(w_p + col + j, pre.wp + j);
+    for (int j = 0; j < 4; ++j) {
+      load8_raw(dy + 8 * j, pre.dy[j]);
+      load8_raw(wp + 8 * j, pre.wp[j]);
     }
+#pragma unroll
+    for (int j = 0; j < 32; j += 4) load4(dsb + j, pre.sv + j);
     pre.at = alpha[row];
     pre.st = ds[row];
   }
   __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
                                         int) const {
     const long o = (long)row * D + col;
-    float r[32];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) r[j] = v[j] + pre.dy[j] + pre.at * pre.sv[j] + pre.st * pre.wp[j];
+    for (int q = 0; q < 4; ++q) {
+      float dy[8], wp[8], r[8];
+      unpack8(pre.dy[q], dy);
+      unpack8(pre.wp[q], wp);
 #pragma unroll
-    for (int j = 0; j < 32; j += 8) store8(out + o + j, r + j);
+      for (int e = 0; e < 8; ++e)
+        r[e] = v[8 * q + e] + dy[e] + pre.at * pre.sv[8 * q + e] + pre.st * wp[e];
+      store8(reinterpret_cast<bf16*>(out) + o + 8 * q, r);
+    }
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
     const int b = row / Tlen, t = row - b * Tlen, blk = t / L;

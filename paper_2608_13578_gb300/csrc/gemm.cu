@@ -174,11 +174,13 @@ int sm_count() {
 // blocks (optionally one K-split each), taken round-robin by the CTAs, m
 // fastest.  Warp 0 / lane 0 streams 64-deep K slices of A and B into a
 // STAGES-deep ring with TMA; warp 1 / lane 0 issues the MMAs into one of two
-// TMEM accumulators; warps 2-5 drain the other accumulator through the
-// epilogue at the same time, so a tile's epilogue overlaps the next tile's
+// TMEM accumulators; warps 2-9 drain the other accumulator through the
+// epilogue at the same time (two warps per TMEM lane quarter, each taking
+// half of the tile's columns), so a tile's epilogue overlaps the next tile's
 // main loop.
+constexpr int kGemmThreads = 320;
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    int M, int N, int kps, int nkb, int tiles_m, int tiles_n, int n_tiles, Epi epi,
                    unsigned* status) {
@@ -201,7 +203,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&tfull[a], 1);
-      tc::mbar_init(&tempty[a], 4);
+      tc::mbar_init(&tempty[a], 8);
     }
     tc::fence_mbar_init();
     tc::prefetch_tmap(&mA);
@@ -292,8 +294,10 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else {
-    // ---- epilogue warps 2..5: warp w reads TMEM lanes 32*(w%4) .. +31
+    // ---- epilogue warps 2..9: warp w reads TMEM lanes 32*(w%4) .. +31 and
+    // the columns of half (w-2)/4 of the tile
     const int q = warp & 3;
+    const int c_beg = ((warp - 2) >> 2) * (BN / 2);
     int j = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++j) {
       const int m_blk = tile % tiles_m, rest = tile / tiles_m;
@@ -304,15 +308,16 @@ __global__ void __launch_bounds__(192, 1)
       const bool row_ok = row < M;
       // The epilogue's own inputs do not depend on the accumulator: fetch the
       // first chunk's before waiting for it, and each next chunk's one ahead.
+      constexpr int NCH = BN / 64;  // 32-column chunks per epilogue warp
       typename Epi::Pre pre[2];
-      if (row_ok && n0 < N) epi.load(row, n0, pre[0]);
+      if (row_ok && n0 + c_beg < N) epi.load(row, n0 + c_beg, pre[0]);
       const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
       tc::fence_after_sync();
       const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll
-      for (int ci = 0; ci < BN / 32; ++ci) {
-        const int c = ci * 32;
-        if (ci + 1 < BN / 32 && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
+      for (int ci = 0; ci < NCH; ++ci) {
+        const int c = c_beg + ci * 32;
+        if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
         float v[32];
         tc::tmem_ld32(base + (uint32_t)c, v);
         if (ok && row_ok && n0 + c < N) epi.apply(row, n0 + c, v, pre[ci & 1], z);
@@ -370,7 +375,7 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
     attr_set = true;
   }
   const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
-  launch_k(kern, dim3(grid), dim3(192), Cfg::SMEM, lc.stream,
+  launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream,
 mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
                                             lc.status);
   return cudaGetLastError();

@@ -109,9 +109,9 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 constexpr int kKC = 256;
 
 template <class TB>
-__device__ __forceinline__ void stage_b_chunk(float (*Bs)[33], const TB* __restrict__ Bm, long sbk,
+__device__ __forceinline__ void stage_b_chunk(float* Bs, const TB* __restrict__ Bm, long sbk,
                                               long sbn, int k0, int K, int n0, int N) {
-  // kKC x 32 elements, 32 per thread, all loads first
+  // kKC x 32 elements (row stride 32), 32 per thread, all loads first
   float v[32];
 #pragma unroll
   for (int q = 0; q < 32; ++q) {
@@ -126,17 +126,29 @@ __device__ __forceinline__ void stage_b_chunk(float (*Bs)[33], const TB* __restr
     const int e = threadIdx.x + q * 256;
     int kk, nn;
     if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
-    Bs[kk][nn] = v[q];
+    Bs[kk * 32 + nn] = v[q];
   }
 }
 
-__device__ __forceinline__ void mac_chunk(const float* __restrict__ arow, float (*Bs)[33], int p,
-                                          float& acc0, float& acc1) {
-#pragma unroll 16
-  for (int kk = 0; kk < kKC; ++kk) {
-    const float a = arow[kk];
-    acc0 = fmaf(a, Bs[kk][2 * p], acc0);
-    acc1 = fmaf(a, Bs[kk][2 * p + 1], acc1);
+// acc += sum over the chunk's k of arow[k] * Bs[k][2p .. 2p+1]; arow 16-byte
+// aligned.  One 16-byte and four 8-byte shared loads per eight FMAs.
+__device__ __forceinline__ void mac_chunk(const float* __restrict__ arow, const float* Bs, int p,
+                                          int kn, float& acc0, float& acc1) {
+#pragma unroll 4
+  for (int kk = 0; kk < kn; kk += 4) {
+    const float4 a = *reinterpret_cast<const float4*>(arow + kk);
+    const float2 b0 = *reinterpret_cast<const float2*>(Bs + (kk + 0) * 32 + 2 * p);
+    const float2 b1 = *reinterpret_cast<const float2*>(Bs + (kk + 1) * 32 + 2 * p);
+    const float2 b2 = *reinterpret_cast<const float2*>(Bs + (kk + 2) * 32 + 2 * p);
+    const float2 b3 = *reinterpret_cast<const float2*>(Bs + (kk + 3) * 32 + 2 * p);
+    acc0 = fmaf(a.x, b0.x, acc0);
+    acc1 = fmaf(a.x, b0.y, acc1);
+    acc0 = fmaf(a.y, b1.x, acc0);
+    acc1 = fmaf(a.y, b1.y, acc1);
+    acc0 = fmaf(a.z, b2.x, acc0);
+    acc1 = fmaf(a.z, b2.y, acc1);
+    acc0 = fmaf(a.w, b3.x, acc0);
+    acc1 = fmaf(a.w, b3.y, acc1);
   }
 }
 
@@ -155,12 +167,12 @@ __global__ void __launch_bounds__(256)
                       const TW* __restrict__ w_m, float* __restrict__ M, float* __restrict__ Z,
                       float* __restrict__ Cmem, int Nb, int D) {
   pdl_enter();
-  extern __shared__ float dyn[];
-  float* Ms = dyn;                                         // [16][D + 1]
-  float(*Bs)[33] = reinterpret_cast<float(*)[33]>(dyn + 16 * (D + 1));  // [kKC][33]
+  extern __shared__ __align__(16) float dyn[];
+  const int ld = D + 4;                                    // keeps rows 16-byte aligned
+  float* Ms = dyn;                                         // [16][D + 4]
+  float* Bs = dyn + 16 * ld;                               // [kKC][32]
   const int n0 = blockIdx.x * 32, i0 = blockIdx.y * 16, b = blockIdx.z;
   const int i1 = min(Nb, i0 + 16);
-  const int ld = D + 1;
   const bool keep = blockIdx.x == 0;
   for (int k = threadIdx.x; k < D; k += blockDim.x) {
     const float a = decay[k];
@@ -195,7 +207,7 @@ __global__ void __launch_bounds__(256)
     __syncthreads();
     stage_b_chunk<TW>(Bs, w_m, D, 1, k0, D, n0, D);
     __syncthreads();
-    mac_chunk(Ms + r * ld + k0, Bs, p, acc0, acc1);
+    mac_chunk(Ms + r * ld + k0, Bs, p, min(kKC, D - k0), acc0, acc1);
   }
   const int i = i0 + r;
   if (i + 1 < Nb) {
@@ -221,7 +233,7 @@ cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float*
                        const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D) {
   if (D % 64 != 0) return cudaErrorInvalidValue;
   dim3 grid(D / 32, (Nb + 15) / 16, B);
-  const size_t smem = ((size_t)16 * (D + 1) + (size_t)kKC * 33) * sizeof(float);
+  const size_t smem = ((size_t)16 * (D + 4) + (size_t)kKC * 32) * sizeof(float);
   static size_t attr_bytes[2] = {0, 0};
   cudaError_t e;
   if (dtype == 0) {
@@ -246,9 +258,10 @@ __global__ void __launch_bounds__(256)
                       const TB* __restrict__ Bm, long sbk, long sbn, TO* __restrict__ out,
                       long ldo) {
   pdl_enter();
-  extern __shared__ float dyn[];
-  float* As = dyn;                                              // [16][kKC + 1]
-  float(*Bs)[33] = reinterpret_cast<float(*)[33]>(dyn + 16 * (kKC + 1));
+  extern __shared__ __align__(16) float dyn[];
+  constexpr int lda = kKC + 4;                                  // 16-byte aligned rows
+  float* As = dyn;                                              // [16][kKC + 4]
+  float* Bs = dyn + 16 * lda;                                   // [kKC][32]
   const int n0 = blockIdx.x * 32, m0 = blockIdx.y * 16;
   const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
   float acc0 = 0.f, acc1 = 0.f;
@@ -269,12 +282,12 @@ __global__ void __launch_bounds__(256)
         const int e = threadIdx.x + q * 256;
         int mm, kk;
         if (sak == 1) { mm = e >> 8; kk = e & 255; } else { kk = e >> 4; mm = e & 15; }
-        As[mm * (kKC + 1) + kk] = v[q];
+        As[mm * lda + kk] = v[q];
       }
     }
     stage_b_chunk<TB>(Bs, Bm, sbk, sbn, k0, K, n0, N);
     __syncthreads();
-    mac_chunk(As + r * (kKC + 1), Bs, p, acc0, acc1);
+    mac_chunk(As + r * lda, Bs, p, (min(kKC, K - k0) + 3) & ~3, acc0, acc1);
   }
   const int m = m0 + r, n = n0 + 2 * p;
   if (m < Mr) {
@@ -287,7 +300,7 @@ cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int 
                        const float* A, long sam, long sak, const void* B, long sbk, long sbn,
                        void* out, long ldo) {
   dim3 grid((N + 31) / 32, (M + 15) / 16);
-  const size_t smem = ((size_t)16 * (kKC + 1) + (size_t)kKC * 33) * sizeof(float);
+  const size_t smem = ((size_t)16 * (kKC + 4) + (size_t)kKC * 32) * sizeof(float);
   static size_t attr_bytes[4] = {0, 0, 0, 0};
   cudaError_t e;
   if (dtype_b == 0 && dtype_out == 0) {
