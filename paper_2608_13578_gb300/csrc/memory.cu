@@ -108,39 +108,47 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 // element.  Thread (r, p) of 256 owns output row r and columns 2p, 2p+1.
 constexpr int kKC = 256;
 
+// Column swizzle of the staged B chunk: XOR with an even value keeps the
+// (2p, 2p+1) pairs adjacent for the 8-byte reads, and spreads a column of
+// 16 consecutive k over 16 banks for the transposed stores.
+__device__ __forceinline__ int bsw(int kk, int nn) { return kk * 32 + (nn ^ ((kk & 15) << 1)); }
+
 template <class TB>
 __device__ __forceinline__ void stage_b_chunk(float* Bs, const TB* __restrict__ Bm, long sbk,
                                               long sbn, int k0, int K, int n0, int N) {
-  // kKC x 32 elements (row stride 32), 32 per thread, all loads first
-  float v[32];
+  // kKC x 32 elements, 32 per thread, in two halves of 16 loads issued before use
 #pragma unroll
-  for (int q = 0; q < 32; ++q) {
-    const int e = threadIdx.x + q * 256;
-    int kk, nn;
-    if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
-    const int k = k0 + kk, n = n0 + nn;
-    v[q] = (k < K && n < N) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
-  }
+  for (int h = 0; h < 2; ++h) {
+    float v[16];
 #pragma unroll
-  for (int q = 0; q < 32; ++q) {
-    const int e = threadIdx.x + q * 256;
-    int kk, nn;
-    if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
-    Bs[kk * 32 + nn] = v[q];
+    for (int q = 0; q < 16; ++q) {
+      const int e = threadIdx.x + (h * 16 + q) * 256;
+      int kk, nn;
+      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
+      const int k = k0 + kk, n = n0 + nn;
+      v[q] = (k < K && n < N) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int e = threadIdx.x + (h * 16 + q) * 256;
+      int kk, nn;
+      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
+      Bs[bsw(kk, nn)] = v[q];
+    }
   }
 }
 
-// acc += sum over the chunk's k of arow[k] * Bs[k][2p .. 2p+1]; arow 16-byte
+// acc += sum over the chunk's k of arow[k] * B[k][2p .. 2p+1]; arow 16-byte
 // aligned.  One 16-byte and four 8-byte shared loads per eight FMAs.
 __device__ __forceinline__ void mac_chunk(const float* __restrict__ arow, const float* Bs, int p,
                                           int kn, float& acc0, float& acc1) {
 #pragma unroll 4
   for (int kk = 0; kk < kn; kk += 4) {
     const float4 a = *reinterpret_cast<const float4*>(arow + kk);
-    const float2 b0 = *reinterpret_cast<const float2*>(Bs + (kk + 0) * 32 + 2 * p);
-    const float2 b1 = *reinterpret_cast<const float2*>(Bs + (kk + 1) * 32 + 2 * p);
-    const float2 b2 = *reinterpret_cast<const float2*>(Bs + (kk + 2) * 32 + 2 * p);
-    const float2 b3 = *reinterpret_cast<const float2*>(Bs + (kk + 3) * 32 + 2 * p);
+    const float2 b0 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 0, 2 * p));
+    const float2 b1 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 1, 2 * p));
+    const float2 b2 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 2, 2 * p));
+    const float2 b3 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 3, 2 * p));
     acc0 = fmaf(a.x, b0.x, acc0);
     acc1 = fmaf(a.x, b0.y, acc1);
     acc0 = fmaf(a.y, b1.x, acc0);
@@ -253,7 +261,7 @@ cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float*
 // out[m, n] = sum_k A(m, k) B(k, n), A(m,k) = A[m*sam + k*sak] (fp32),
 // B(k,n) = B[k*sbk + n*sbn] (fp32 or bf16), stored as TO.
 template <class TB, class TO>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 2)
     small_gemm_kernel(int Mr, int N, int K, const float* __restrict__ A, long sam, long sak,
                       const TB* __restrict__ Bm, long sbk, long sbn, TO* __restrict__ out,
                       long ldo) {
