@@ -101,30 +101,51 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 }
 
 // -------------------------------------------------------------- Sec. 3.5
-// Small products of the memory stage on CUDA cores, in 16 x 32 output tiles
-// so even a [128 x 512] result spreads over 128 CTAs.  K is consumed in
-// chunks of kKC; every load of a chunk is issued into registers before the
-// first one is used, so a chunk costs one memory round trip, not one per
-// element.  Thread (r, p) of 256 owns output row r and columns 2p, 2p+1.
-constexpr int kKC = 256;
+// Small products of the memory stage on CUDA cores (at most a few hundred rows
+// of output, K <= a few thousand).  A CTA owns a 16 x 32 output tile and splits
+// K over its 8 warps: lane l of warp w accumulates output column l for all 16
+// rows over k = w, w+8, ...; the A values of a k are one 64-byte broadcast,
+// the B value one conflict-free word.  K is staged in slices of kKS (all of a
+// slice's loads are issued before the first use), and the 8 partial tiles are
+// added in warp order at the end, so results are deterministic.
+constexpr int kKS = 512;
 
-// Column swizzle of the staged B chunk: XOR with an even value keeps the
-// (2p, 2p+1) pairs adjacent for the 8-byte reads, and spreads a column of
-// 16 consecutive k over 16 banks for the transposed stores.
-__device__ __forceinline__ int bsw(int kk, int nn) { return kk * 32 + (nn ^ ((kk & 15) << 1)); }
-
-template <class TB>
-__device__ __forceinline__ void stage_b_chunk(float* Bs, const TB* __restrict__ Bm, long sbk,
-                                              long sbn, int k0, int K, int n0, int N) {
-  // kKC x 32 elements, 32 per thread, in two halves of 16 loads issued before use
+// A slice: As[kk*16 + mm] = A(m0+mm, k0+kk) for kk < kKS (zero outside).
+__device__ __forceinline__ void stage_a(float* As, const float* __restrict__ A, long sam, long sak,
+                                        int m0, int Mr, int k0, int K) {
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     float v[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int e = threadIdx.x + (h * 16 + q) * 256;
+      int mm, kk;
+      if (sak == 1) { mm = e >> 9; kk = e & (kKS - 1); } else { kk = e >> 4; mm = e & 15; }
+      const int m = m0 + mm, k = k0 + kk;
+      v[q] = (m < Mr && k < K) ? A[(long)m * sam + (long)k * sak] : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int e = threadIdx.x + (h * 16 + q) * 256;
+      int mm, kk;
+      if (sak == 1) { mm = e >> 9; kk = e & (kKS - 1); } else { kk = e >> 4; mm = e & 15; }
+      As[kk * 16 + mm] = v[q];
+    }
+  }
+}
+
+// B slice: Bs[kk*33 + nn] = B(k0+kk, n0+nn) (zero outside).
+template <class TB>
+__device__ __forceinline__ void stage_b(float* Bs, const TB* __restrict__ Bm, long sbk, long sbn,
+                                        int k0, int K, int n0, int N) {
+#pragma unroll
+  for (int h = 0; h < 4; ++h) {
+    float v[16];
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int e = threadIdx.x + (h * 16 + q) * 256;
       int kk, nn;
-      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
+      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 9; kk = e & (kKS - 1); }
       const int k = k0 + kk, n = n0 + nn;
       v[q] = (k < K && n < N) ? to_f(Bm[(long)k * sbk + (long)n * sbn]) : 0.f;
     }
@@ -132,43 +153,59 @@ __device__ __forceinline__ void stage_b_chunk(float* Bs, const TB* __restrict__ 
     for (int q = 0; q < 16; ++q) {
       const int e = threadIdx.x + (h * 16 + q) * 256;
       int kk, nn;
-      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 8; kk = e & 255; }
-      Bs[bsw(kk, nn)] = v[q];
+      if (sbn == 1) { kk = e >> 5; nn = e & 31; } else { nn = e >> 9; kk = e & (kKS - 1); }
+      Bs[kk * 33 + nn] = v[q];
     }
   }
 }
 
-// acc += sum over the chunk's k of arow[k] * B[k][2p .. 2p+1]; arow 16-byte
-// aligned.  One 16-byte and four 8-byte shared loads per eight FMAs.
-__device__ __forceinline__ void mac_chunk(const float* __restrict__ arow, const float* Bs, int p,
-                                          int kn, float& acc0, float& acc1) {
-#pragma unroll 4
-  for (int kk = 0; kk < kn; kk += 4) {
-    const float4 a = *reinterpret_cast<const float4*>(arow + kk);
-    const float2 b0 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 0, 2 * p));
-    const float2 b1 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 1, 2 * p));
-    const float2 b2 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 2, 2 * p));
-    const float2 b3 = *reinterpret_cast<const float2*>(Bs + bsw(kk + 3, 2 * p));
-    acc0 = fmaf(a.x, b0.x, acc0);
-    acc1 = fmaf(a.x, b0.y, acc1);
-    acc0 = fmaf(a.y, b1.x, acc0);
-    acc1 = fmaf(a.y, b1.y, acc1);
-    acc0 = fmaf(a.z, b2.x, acc0);
-    acc1 = fmaf(a.z, b2.y, acc1);
-    acc0 = fmaf(a.w, b3.x, acc0);
-    acc1 = fmaf(a.w, b3.y, acc1);
+// acc[r] += sum over this warp's k of As[k][r] * Bs[k][lane]
+__device__ __forceinline__ void mac_slice(const float* As, const float* Bs, int kn, int warp,
+                                          int lane, float* acc) {
+#pragma unroll 2
+  for (int kk = warp; kk < kn; kk += 8) {
+    const float4* a4 = reinterpret_cast<const float4*>(As + kk * 16);
+    const float b = Bs[kk * 33 + lane];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 a = a4[q];
+      acc[4 * q + 0] = fmaf(a.x, b, acc[4 * q + 0]);
+      acc[4 * q + 1] = fmaf(a.y, b, acc[4 * q + 1]);
+      acc[4 * q + 2] = fmaf(a.z, b, acc[4 * q + 2]);
+      acc[4 * q + 3] = fmaf(a.w, b, acc[4 * q + 3]);
+    }
   }
 }
+
+// The 8 warps' partial tiles added in warp order; thread t ends with output
+// elements 2t and 2t+1 of the 16 x 32 tile (row (2t)/32, columns (2t)%32, +1).
+__device__ __forceinline__ void reduce_tile(float* red, const float* acc, int warp, int lane,
+                                            float& o0, float& o1) {
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 16; ++r) red[warp * 512 + r * 32 + lane] = acc[r];
+  __syncthreads();
+  const int e = 2 * threadIdx.x;
+  o0 = 0.f;
+  o1 = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) {
+    o0 += red[w * 512 + e];
+    o1 += red[w * 512 + e + 1];
+  }
+}
+
+constexpr size_t kSmallSmem = (size_t)(kKS * 16 + kKS * 33) * sizeof(float);
 
 // Memory rows for blocks i0 .. i0+15 of batch b, projected and shifted:
 // C[b, i+1, n0 .. n0+31] = M_i W_m[:, n0 .. n0+31] (and C[b, 0] = 0).  The
 // decayed scan
 //   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i
 // (the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j)) is
-// recomputed per CTA from block 0 for every channel straight into shared
-// memory, so the projection needs no separate pass.  The CTAs of the first
-// column tile also store M (for dW_m) and, for batch 0, Z (for the backward
-// scan).  Grid (D/32, ceil(Nb/16), B).
+// recomputed per CTA from block 0 for each channel of the K slice straight
+// into the A operand, so the projection needs no separate pass.  The CTAs of
+// the first column tile also store M (for dW_m) and, for batch 0, Z (for the
+// backward scan).  Grid (D/32, ceil(Nb/16), B).
 template <class TW>
 __global__ void __launch_bounds__(256)
     memory_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
@@ -176,57 +213,70 @@ __global__ void __launch_bounds__(256)
                       float* __restrict__ Cmem, int Nb, int D) {
   pdl_enter();
   extern __shared__ __align__(16) float dyn[];
-  const int ld = D + 4;                                    // keeps rows 16-byte aligned
-  float* Ms = dyn;                                         // [16][D + 4]
-  float* Bs = dyn + 16 * ld;                               // [kKC][32]
+  float* As = dyn;
+  float* Bs = dyn + kKS * 16;
   const int n0 = blockIdx.x * 32, i0 = blockIdx.y * 16, b = blockIdx.z;
   const int i1 = min(Nb, i0 + 16);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool keep = blockIdx.x == 0;
-  for (int k = threadIdx.x; k < D; k += blockDim.x) {
-    const float a = decay[k];
-    const float* Sk = S + (long)b * Nb * D + k;
-    float Nn = 0.f, Zz = 0.f;
-    for (int c0 = 0; c0 < i1; c0 += 16) {
-      float sv[16];
+  float acc[16];
 #pragma unroll
-      for (int u = 0; u < 16; ++u) sv[u] = (c0 + u < i1) ? Sk[(long)(c0 + u) * D] : 0.f;
+  for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+  for (int k0 = 0; k0 < D; k0 += kKS) {
+    const int kn = min(kKS, D - k0);
+    __syncthreads();
+    stage_b<TW>(Bs, w_m, D, 1, k0, D, n0, D);  // W_m rows k0.., columns n0..n0+31
+    for (int kk = threadIdx.x; kk < kKS; kk += blockDim.x) {
+      const int k = k0 + kk;
+      float mrow[16];
 #pragma unroll
-      for (int u = 0; u < 16; ++u) {
-        const int i = c0 + u;
-        if (i < i1) {
-          Nn = fmaf(a, Nn, sv[u]);
-          Zz = fmaf(a, Zz, 1.0f);
-          if (i >= i0) {
-            const float m = Nn / Zz;
-            Ms[(i - i0) * ld + k] = m;
-            if (keep) {
-              M[((long)b * Nb + i) * D + k] = m;
-              if (b == 0) Z[(long)i * D + k] = Zz;
+      for (int r = 0; r < 16; ++r) mrow[r] = 0.f;
+      if (kk < kn) {
+        const float a = decay[k];
+        const float* Sk = S + (long)b * Nb * D + k;
+        float Nn = 0.f, Zz = 0.f;
+        for (int c0 = 0; c0 < i1; c0 += 16) {
+          float sv[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) sv[u] = (c0 + u < i1) ? Sk[(long)(c0 + u) * D] : 0.f;
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int i = c0 + u;
+            if (i < i1) {
+              Nn = fmaf(a, Nn, sv[u]);
+              Zz = fmaf(a, Zz, 1.0f);
+              if (i >= i0) {
+                const float m = Nn / Zz;
+                mrow[u] = m;  // c0 == i0 whenever i >= i0 (i0 is a multiple of 16)
+                if (keep) {
+                  M[((long)b * Nb + i) * D + k] = m;
+                  if (b == 0) Z[(long)i * D + k] = Zz;
+                }
+              }
             }
           }
         }
       }
+      float4* dst = reinterpret_cast<float4*>(As + kk * 16);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        dst[q] = make_float4(mrow[4 * q], mrow[4 * q + 1], mrow[4 * q + 2], mrow[4 * q + 3]);
     }
-    for (int i = i1; i < i0 + 16; ++i) Ms[(i - i0) * ld + k] = 0.f;
-  }
-  const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
-  float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < D; k0 += kKC) {
     __syncthreads();
-    stage_b_chunk<TW>(Bs, w_m, D, 1, k0, D, n0, D);
-    __syncthreads();
-    mac_chunk(Ms + r * ld + k0, Bs, p, min(kKC, D - k0), acc0, acc1);
+    mac_slice(As, Bs, kn, warp, lane, acc);
   }
+  float o0, o1;
+  reduce_tile(dyn, acc, warp, lane, o0, o1);
+  const int r = (2 * threadIdx.x) >> 5, c = (2 * threadIdx.x) & 31;
   const int i = i0 + r;
+  float* cb = Cmem + (long)b * Nb * D + n0 + c;
   if (i + 1 < Nb) {
-    float* c = Cmem + ((long)b * Nb + i + 1) * D + n0 + 2 * p;
-    c[0] = acc0;
-    c[1] = acc1;
+    cb[(long)(i + 1) * D] = o0;
+    cb[(long)(i + 1) * D + 1] = o1;
   }
   if (i0 == 0 && r == 0) {
-    float* c = Cmem + (long)b * Nb * D + n0 + 2 * p;
-    c[0] = 0.f;
-    c[1] = 0.f;
+    cb[0] = 0.f;
+    cb[1] = 0.f;
   }
 }
 
@@ -241,18 +291,17 @@ cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float*
                        const void* w_m, float* M, float* Z, float* Cmem, int B, int Nb, int D) {
   if (D % 64 != 0) return cudaErrorInvalidValue;
   dim3 grid(D / 32, (Nb + 15) / 16, B);
-  const size_t smem = ((size_t)16 * (D + 4) + (size_t)kKC * 32) * sizeof(float);
   static size_t attr_bytes[2] = {0, 0};
   cudaError_t e;
   if (dtype == 0) {
-    e = opt_in_smem((const void*)memory_fwd_kernel<float>, smem, &attr_bytes[0]);
+    e = opt_in_smem((const void*)memory_fwd_kernel<float>, kSmallSmem, &attr_bytes[0]);
     if (e == cudaSuccess)
-      e = launch_k(memory_fwd_kernel<float>, grid, dim3(256), smem, lc.stream, S, decay,
+      e = launch_k(memory_fwd_kernel<float>, grid, dim3(256), kSmallSmem, lc.stream, S, decay,
                    (const float*)w_m, M, Z, Cmem, Nb, D);
   } else {
-    e = opt_in_smem((const void*)memory_fwd_kernel<bf16>, smem, &attr_bytes[1]);
+    e = opt_in_smem((const void*)memory_fwd_kernel<bf16>, kSmallSmem, &attr_bytes[1]);
     if (e == cudaSuccess)
-      e = launch_k(memory_fwd_kernel<bf16>, grid, dim3(256), smem, lc.stream, S, decay,
+      e = launch_k(memory_fwd_kernel<bf16>, grid, dim3(256), kSmallSmem, lc.stream, S, decay,
                    (const bf16*)w_m, M, Z, Cmem, Nb, D);
   }
   return e != cudaSuccess ? e : cudaGetLastError();
@@ -261,46 +310,32 @@ cudaError_t memory_fwd(const Launch& lc, int dtype, const float* S, const float*
 // out[m, n] = sum_k A(m, k) B(k, n), A(m,k) = A[m*sam + k*sak] (fp32),
 // B(k,n) = B[k*sbk + n*sbn] (fp32 or bf16), stored as TO.
 template <class TB, class TO>
-__global__ void __launch_bounds__(256, 2)
+__global__ void __launch_bounds__(256)
     small_gemm_kernel(int Mr, int N, int K, const float* __restrict__ A, long sam, long sak,
                       const TB* __restrict__ Bm, long sbk, long sbn, TO* __restrict__ out,
                       long ldo) {
   pdl_enter();
   extern __shared__ __align__(16) float dyn[];
-  constexpr int lda = kKC + 4;                                  // 16-byte aligned rows
-  float* As = dyn;                                              // [16][kKC + 4]
-  float* Bs = dyn + 16 * lda;                                   // [kKC][32]
+  float* As = dyn;
+  float* Bs = dyn + kKS * 16;
   const int n0 = blockIdx.x * 32, m0 = blockIdx.y * 16;
-  const int r = threadIdx.x >> 4, p = threadIdx.x & 15;
-  float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < K; k0 += kKC) {
-    __syncthreads();
-    {
-      float v[16];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float acc[16];
 #pragma unroll
-      for (int q = 0; q < 16; ++q) {
-        const int e = threadIdx.x + q * 256;
-        int mm, kk;
-        if (sak == 1) { mm = e >> 8; kk = e & 255; } else { kk = e >> 4; mm = e & 15; }
-        const int m = m0 + mm, k = k0 + kk;
-        v[q] = (m < Mr && k < K) ? A[(long)m * sam + (long)k * sak] : 0.f;
-      }
-#pragma unroll
-      for (int q = 0; q < 16; ++q) {
-        const int e = threadIdx.x + q * 256;
-        int mm, kk;
-        if (sak == 1) { mm = e >> 8; kk = e & 255; } else { kk = e >> 4; mm = e & 15; }
-        As[mm * lda + kk] = v[q];
-      }
-    }
-    stage_b_chunk<TB>(Bs, Bm, sbk, sbn, k0, K, n0, N);
+  for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += kKS) {
     __syncthreads();
-    mac_chunk(As + r * lda, Bs, p, (min(kKC, K - k0) + 3) & ~3, acc0, acc1);
+    stage_a(As, A, sam, sak, m0, Mr, k0, K);
+    stage_b<TB>(Bs, Bm, sbk, sbn, k0, K, n0, N);
+    __syncthreads();
+    mac_slice(As, Bs, min(kKS, K - k0), warp, lane, acc);
   }
-  const int m = m0 + r, n = n0 + 2 * p;
+  float o0, o1;
+  reduce_tile(dyn, acc, warp, lane, o0, o1);
+  const int m = m0 + ((2 * threadIdx.x) >> 5), n = n0 + ((2 * threadIdx.x) & 31);
   if (m < Mr) {
-    if (n < N) out[(long)m * ldo + n] = from_f<TO>(acc0);
-    if (n + 1 < N) out[(long)m * ldo + n + 1] = from_f<TO>(acc1);
+    if (n < N) out[(long)m * ldo + n] = from_f<TO>(o0);
+    if (n + 1 < N) out[(long)m * ldo + n + 1] = from_f<TO>(o1);
   }
 }
 
@@ -308,8 +343,8 @@ cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int 
                        const float* A, long sam, long sak, const void* B, long sbk, long sbn,
                        void* out, long ldo) {
   dim3 grid((N + 31) / 32, (M + 15) / 16);
-  const size_t smem = ((size_t)16 * (kKC + 4) + (size_t)kKC * 32) * sizeof(float);
   static size_t attr_bytes[4] = {0, 0, 0, 0};
+  const size_t smem = kSmallSmem;
   cudaError_t e;
   if (dtype_b == 0 && dtype_out == 0) {
     e = opt_in_smem((const void*)small_gemm_kernel<float, float>, smem, &attr_bytes[0]);
