@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <memory>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -50,6 +51,66 @@ unsigned* status_ptr() {
   }
   return per_dev[dev];
 }
+
+// A second stream per device for the weight gradients of the backward pass,
+// which no later step of the pass reads: they run beside the dependent chain
+// (forked and joined with events, so the pair can also be captured into a
+// CUDA graph).  Streams and events are host-side objects: no device memory.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t ev[8] = {};
+  std::mutex mu;  // one backward at a time may use the events
+};
+
+SideStream* side_stream() {
+  static std::mutex mu;
+  static std::vector<SideStream*> per_dev;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if ((int)per_dev.size() <= dev) per_dev.resize(dev + 1, nullptr);
+  if (!per_dev[dev]) {
+    SideStream* ss = new SideStream();
+    bool ok = cudaStreamCreateWithFlags(&ss->s, cudaStreamNonBlocking) == cudaSuccess;
+    for (int i = 0; i < 8 && ok; ++i)
+      ok = cudaEventCreateWithFlags(&ss->ev[i], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      delete ss;  // fall back to one stream
+      return nullptr;
+    }
+    per_dev[dev] = ss;
+  }
+  return per_dev[dev];
+}
+
+// Fork/join of the side stream for one call; joins on destruction so every
+// return path leaves the side stream merged back into the caller's stream.
+struct Fork {
+  SideStream* ss;
+  cudaStream_t main;
+  int next = 0;
+  bool forked = false;
+  Fork(SideStream* side, cudaStream_t m) : ss(side), main(m) {
+    if (ss) ss->mu.lock();
+  }
+  cudaStream_t side() const { return ss ? ss->s : main; }
+  // the side stream waits for everything enqueued on the main stream so far
+  void point() {
+    if (!ss || next >= 7) return;
+    cudaEventRecord(ss->ev[next], main);
+    cudaStreamWaitEvent(ss->s, ss->ev[next], 0);
+    ++next;
+    forked = true;
+  }
+  ~Fork() {
+    if (!ss) return;
+    if (forked) {
+      cudaEventRecord(ss->ev[7], ss->s);
+      cudaStreamWaitEvent(main, ss->ev[7], 0);
+    }
+    ss->mu.unlock();
+  }
+};
 
 // Tensor-core paths of the layer (switchable only through bcmt_testing.h).
 bool g_use_tc_gemm = true;
@@ -451,8 +512,15 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   unsigned* sp = status_ptr();
   if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool profiling = (p->flags & BCMT_FLAG_PROFILE) != 0;
   Launch lc{s, sp};
-  Prof pr{(p->flags & BCMT_FLAG_PROFILE) != 0, s};
+  Prof pr{profiling, s};
+  // Weight gradients go to the side stream (kept on one stream while
+  // profiling, so every kernel is timed alone).
+  std::unique_ptr<Fork> fork_holder(new Fork(profiling ? nullptr : side_stream(), s));
+  Fork& fork = *fork_holder;
+  Launch lcs{fork.side(), sp};
+  Prof prs{profiling, fork.side()};
   FwdWs w = fwd_layout(g, const_cast<void*>(workspace));
   BwdWs bw = bwd_layout(g, scratch);
   const int D = g.D, n = (int)g.n;
@@ -474,23 +542,24 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     e = memory_scan_bwd(lc, bw.dM, decay, w.Z, bw.dS, g.B, g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
-    pr.begin("memory_dwm");
-    e = small_gemm(lc, 0, g.dtype, D, D, g.B * g.Nb, w.M, 1, D, bw.dP, D, 1, dw_m, D);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_m");
     // Sec. 3.4 reversed: pooling scores and dW_p.
     pr.begin("summary_bwd");
     e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");
-    pr.begin("reduce_rows");
-    e = reduce_rows(lc, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_p");
-    // dW_g = H^T dU
-    e = weight_grad(lc, pr, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D, bw.part,
-                    dw_g);
+    // side stream: dW_m = M^T dP, dW_g = H^T dU, dW_p
+    fork.point();
+    prs.begin("memory_dwm");
+    e = small_gemm(lcs, 0, g.dtype, D, D, g.B * g.Nb, w.M, 1, D, bw.dP, D, 1, dw_m, D);
+    prs.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_m");
+    e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
+                    bw.part, dw_g);
     if (e != cudaSuccess) return cuda_fail(e, "dW_g");
+    prs.begin("reduce_rows");
+    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
+    prs.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_p");
     // dH = dY + dU W_g^T + alpha dS + ds w_p
     EpiArgs ea;
     ea.out = bw.dH;
@@ -517,12 +586,13 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     EpiArgs ea;
     ea.out = bw.dHhat;
     ea.ldo = D;
+    fork.point();  // dH is final
+    e = weight_grad(lcs, prs, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part,
+                    dw_o);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_O");
     e = run_gemm(lc, pr, "gemm_dhhat", g.dtype, g.dtype, n, D, D, dH, D, 1, w_o, 1, D, EPI_STORE,
                  ea);
     if (e != cudaSuccess) return cuda_fail(e, "dHhat");
-    e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part,
-                    dw_o);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_O");
   }
   // Attention backward -> dQ, dK, dV.
   {
@@ -566,13 +636,15 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     EpiArgs ea;
     ea.out = dx_or_dq;
     ea.ldo = D;
+    fork.point();  // dQKV is final
+    e = weight_grad(lcs, prs, "gemm_dw_qkv", g.dtype, g.dtype, D, 3 * D, g.n, x_or_q, D, bw.dqkv,
+                    3 * D, bw.part, dw_qkv);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_qkv");
     e = run_gemm(lc, pr, "gemm_dx", g.dtype, g.dtype, n, D, 3 * D, bw.dqkv, 3 * D, 1, w_qkv, 1,
                  3 * D, EPI_STORE, ea);
     if (e != cudaSuccess) return cuda_fail(e, "dX");
-    e = weight_grad(lc, pr, "gemm_dw_qkv", g.dtype, g.dtype, D, 3 * D, g.n, x_or_q, D, bw.dqkv,
-                    3 * D, bw.part, dw_qkv);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_qkv");
   }
+  fork_holder.reset();  // join the side stream before any status read
   return finish(p, s);
 }
 
