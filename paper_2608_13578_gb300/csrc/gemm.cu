@@ -381,11 +381,14 @@ mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
   return cudaGetLastError();
 }
 
-template <bool A_MN, bool B_MN>
+// Output tile widths: 128 x 256 tiles move 48 KB per 64-deep K slice for
+// 4.2 MFLOP (87 FLOP per L2 byte), 128 x 128 tiles 32 KB for 2.1 MFLOP (64).
+// The wide tile is used when it still gives most SMs a tile.
+template <int BN, bool A_MN, bool B_MN>
 static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                           long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                           const EpiArgs& ea, int splits) {
-  constexpr int BN = 128, ST = 6;
+  constexpr int ST = BN == 256 ? 4 : 6;
   switch (epi) {
     case EPI_STORE:
       if (dtype_out == 0)
@@ -397,28 +400,50 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,
           EpiStoreF<float>{(float*)ea.out, ea.ldo, ea.split_stride}, splits);
-    case EPI_GATE_INJECT:
-      return tc_launch<BN, ST, A_MN, B_MN>(
-          lc, M, N, K, A, sam, sak, B, sbk, sbn,
-          EpiGateInjectF<bf16>{(const bf16*)ea.H, ea.Cmem, (bf16*)ea.G, (bf16*)ea.Y, ea.T, ea.L,
-                               ea.Nb, ea.D},
-          1);
-    case EPI_STORE_SCORE:
-      return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                                           EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
-                                                                (const bf16*)ea.w_p, ea.spart, M},
-                                           1);
-    case EPI_SHIFT:
-      return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                                           EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
-    case EPI_DH:
+    default:
+      break;
+  }
+  // fused epilogues, instantiated only for the operand layouts the layer uses
+  if constexpr (!A_MN && B_MN) {
+    switch (epi) {
+      case EPI_GATE_INJECT:
+        return tc_launch<BN, ST, A_MN, B_MN>(
+            lc, M, N, K, A, sam, sak, B, sbk, sbn,
+            EpiGateInjectF<bf16>{(const bf16*)ea.H, ea.Cmem, (bf16*)ea.G, (bf16*)ea.Y, ea.T, ea.L,
+                                 ea.Nb, ea.D},
+            1);
+      case EPI_STORE_SCORE:
+        return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                             EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
+                                                                  (const bf16*)ea.w_p, ea.spart, M},
+                                             1);
+      case EPI_SHIFT:
+        return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                             EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
+      default:
+        break;
+    }
+  }
+  if constexpr (!A_MN && !B_MN) {
+    if (epi == EPI_DH)
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,
           EpiDHF<bf16>{(const bf16*)ea.dY, ea.alpha, ea.dS, ea.ds, (const bf16*)ea.w_p,
                        (bf16*)ea.out, ea.T, ea.L, ea.Nb, ea.D},
           1);
   }
-  return cudaErrorInvalidValue;
+  return cudaErrorNotSupported;
+}
+
+template <bool A_MN, bool B_MN>
+static cudaError_t tc_pick(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
+                           long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                           const EpiArgs& ea, int splits) {
+  const long tiles256 = (long)((M + kBM - 1) / kBM) * ((N + 255) / 256) * splits;
+  if (N % 256 == 0 && tiles256 * 4 >= (long)sm_count() * 3)
+    return tc_epi<256, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea,
+                                   splits);
+  return tc_epi<128, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
 }
 
 cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
@@ -428,10 +453,10 @@ cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const 
   splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
   const bool a_k = (sak == 1), a_m = (sam == 1) && !a_k;
   const bool b_k = (sbk == 1), b_n = (sbn == 1) && !b_k;
-  if (a_k && b_n) return tc_epi<false, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
-  if (a_k && b_k) return tc_epi<false, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
-  if (a_m && b_n) return tc_epi<true, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
-  if (a_m && b_k) return tc_epi<true, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_k && b_n) return tc_pick<false, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_k && b_k) return tc_pick<false, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_m && b_n) return tc_pick<true, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (a_m && b_k) return tc_pick<true, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
   return cudaErrorNotSupported;
 }
 

@@ -36,7 +36,9 @@ def _operand(rows, cols, major_rows: bool, dtype, gen, pad=8):
     return store, 1, ld, logical
 
 
-GEMM_SHAPES = [(128, 64, 64), (200, 128, 100), (256, 192, 512), (1000, 512, 320), (77, 256, 1536)]
+# the last two shapes have enough 128 x 256 tiles to take the wide-tile kernel
+GEMM_SHAPES = [(128, 64, 64), (200, 128, 100), (256, 192, 512), (1000, 512, 320), (77, 256, 1536),
+               (4096, 1024, 256), (4000, 768, 200)]
 LAYOUTS = [("k", "n"), ("k", "k"), ("m", "n"), ("m", "k")]
 
 
