@@ -187,16 +187,13 @@ def kernel_model(w):
         # read Q, K, V, dO, O and the log-sum-exp; write dQ, dK, dV
         "attn_bwd_tc": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
         "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
-        # read H; write pooling weights and summaries
-        "summary_fwd": ("hbm", n * D * es + n * 4 + B * Nb * D * 4),
-        # read S, W_m; write M, Z and the projected, shifted memory C
-        "memory_fwd": ("hbm", B * Nb * D * 4 * 3 + Nb * D * 4 + D * D * es),
-        # read dY, G, C; write dU and the shifted memory gradient
-        "gate_bwd": ("hbm", 3 * n * D * es + 2 * B * Nb * D * 4),
-        "memory_dm": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
-        "memory_scan_bwd": ("hbm", B * Nb * D * 8 + Nb * D * 4),
+        # summaries (read H and the score partials, write alpha and S), then the
+        # scan and projection (read S and W_m, write M, Z and C)
+        "memory_fwd": ("hbm", n * D * es + n * 4 * (D // 32 + 1) + B * Nb * D * 4 * 4
+                       + Nb * D * 4 + D * D * es),
+        # gate backward (read dY, G; write dU), dM, scan, pooling backward (read H)
+        "memory_bwd": ("hbm", 4 * n * D * es + 3 * n * 4 + B * Nb * D * 4 * 6 + D * D * es),
         "memory_dwm": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
-        "summary_bwd": ("hbm", n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
     }
 
 

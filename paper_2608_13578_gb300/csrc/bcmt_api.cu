@@ -221,6 +221,7 @@ int dw_splits(int M, int N, long K) {
 struct FwdWs {
   char *qkv, *hhat, *hloc, *G;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
+  unsigned* gbar;
   size_t bytes;
 };
 
@@ -233,6 +234,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     off += al256(bytes);
     return r;
   };
+  w.gbar = reinterpret_cast<unsigned*>(take(64));  // grid barrier of the memory kernel
   w.qkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
   w.lse = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
   w.hhat = take((size_t)g.n * g.D * g.es);
@@ -257,6 +259,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 struct BwdWs {
   char *dU, *dH, *dHhat, *dqkv;
   float *dP, *dM, *dS, *ds, *dwp_part, *Drow, *part;
+  unsigned* gbar;
   size_t bytes;
 };
 
@@ -269,6 +272,7 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     off += al256(bytes);
     return r;
   };
+  w.gbar = reinterpret_cast<unsigned*>(take(64));  // grid barrier of the memory kernel
   if (!g.honly) {
     w.dU = take((size_t)g.n * g.D * g.es);
     w.dH = take((size_t)g.n * g.D * g.es);
@@ -449,16 +453,13 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // Sec. 3.4: adaptive block summaries.
-    pr.begin("summary_fwd");
-    e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "block summaries");
-    // Sec. 3.5: exponential causal memory, projection and shift in one kernel.
+    // Sec. 3.4-3.5: adaptive block summaries, exponential causal memory,
+    // projection and shift: one cooperative kernel.
     pr.begin("memory_fwd");
-    e = memory_fwd(lc, g.dtype, w.S, decay, w_m, w.M, w.Z, w.C, g.B, g.Nb, D);
+    e = memory_fwd_phase(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, decay, w_m, w.M, w.Z,
+                         w.C, w.gbar, g.B, g.T, D, g.L);
     pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "causal memory");
+    if (e != cudaSuccess) return cuda_fail(e, "block summaries and causal memory");
     // Sec. 3.7-3.8: gate and injection fused into the W_g GEMM.
     EpiArgs ea;
     ea.H = w.hloc;
@@ -528,25 +529,14 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
 
   const void* dH = dy;  // HOnly: Y = H
   if (!g.honly) {
-    // Sec. 3.8 reversed: dU and the per-block memory gradient (shifted: dP).
-    pr.begin("gate_bwd");
-    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.B, g.T, D, g.L);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "gate backward");
-    // Sec. 3.5 reversed: dM = dP W_m^T, reverse decayed scan -> dS; dW_m = M^T dP.
-    pr.begin("memory_dm");
-    e = small_gemm(lc, g.dtype, 0, g.B * g.Nb, D, D, bw.dP, D, 1, w_m, 1, D, bw.dM, D);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "dM");
-    pr.begin("memory_scan_bwd");
-    e = memory_scan_bwd(lc, bw.dM, decay, w.Z, bw.dS, g.B, g.Nb, D);
+    // Sec. 3.8, 3.5, 3.4 reversed in one cooperative kernel: dU and the shifted
+    // per-block memory gradient dP; dM = dP W_m^T; the reverse decayed scan
+    // -> dS; the pooling backward -> ds and the dW_p partials.
+    pr.begin("memory_bwd");
+    e = memory_bwd_phase(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, w_m, bw.dM, decay, w.Z, bw.dS,
+                         w.hloc, w.alpha, bw.ds, bw.dwp_part, bw.gbar, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
-    // Sec. 3.4 reversed: pooling scores and dW_p.
-    pr.begin("summary_bwd");
-    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     // side stream: dW_m = M^T dP, dW_g = H^T dU, dW_p
     fork.point();
     prs.begin("memory_dwm");

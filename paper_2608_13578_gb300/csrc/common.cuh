@@ -75,6 +75,15 @@ __device__ __forceinline__ float sigmoid_bf16out(float u) {
   return __fdividef(1.0f, 1.0f + __expf(-u));
 }
 
+// Loads that bypass L1 (ld.global.cg): for data written earlier in the same
+// kernel by other CTAs (the phases of a cooperative kernel).
+__device__ __forceinline__ void load8_cg(const float* p, float* v) {
+  const float4 a = __ldcg(reinterpret_cast<const float4*>(p));
+  const float4 b = __ldcg(reinterpret_cast<const float4*>(p) + 1);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
 // Raw bf16 pairs, converted when used.
 __device__ __forceinline__ void load8_raw(const bf16* p, uint4& raw) {
   raw = *reinterpret_cast<const uint4*>(p);
