@@ -80,6 +80,7 @@ __device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* _
   const long row0 = (long)b * Tlen + t0;
   for (int r = threadIdx.x; r < n; r += kThreads) {
     float s = 0.f;
+#pragma unroll 16
     for (int j = 0; j < npart; ++j) s += spart[(long)j * n_tok + row0 + r];
     sc[r] = s;
   }
@@ -341,17 +342,32 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
   if (c < D) {
     float cm[4];
     load4(Cmem + ((long)b * Nb + i) * D + c, cm);
-    for (int r = rg; r < n; r += 8) {
-      const long o = ((long)b * Tlen + t0 + r) * D + c;
-      float dy[4], g[4], du[4];
-      load4(dY + o, dy);
-      load4(G + o, g);
+    // rows rg, rg+8, ... in batches of 8: every load of a batch is issued
+    // before its first store
+    for (int r0 = rg; r0 < n; r0 += 64) {
+      float dy[8][4], g[8][4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        du[e] = dy[e] * cm[e] * g[e] * (1.0f - g[e]);
-        acc[e] = fmaf(dy[e], g[e], acc[e]);
+      for (int u = 0; u < 8; ++u) {
+        const int r = r0 + 8 * u;
+        if (r < n) {
+          const long o = ((long)b * Tlen + t0 + r) * D + c;
+          load4(dY + o, dy[u]);
+          load4(G + o, g[u]);
+        }
       }
-      store4(dU + o, du);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int r = r0 + 8 * u;
+        if (r < n) {
+          float du[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            du[e] = dy[u][e] * cm[e] * g[u][e] * (1.0f - g[u][e]);
+            acc[e] = fmaf(dy[u][e], g[u][e], acc[e]);
+          }
+          store4(dU + ((long)b * Tlen + t0 + r) * D + c, du);
+        }
+      }
     }
   }
 #pragma unroll
@@ -417,17 +433,29 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   const T* Hb = Hm + ((long)b * Tlen + t0) * D;
   const float* dSi = dS + ((long)b * Nb + i) * D;
   const float* ab = alpha + (long)b * Tlen + t0;
-  for (int r = warp; r < n; r += 8) {
-    float d = 0.f;
+  // g_t = H_t . dS_i: warp w takes rows w, w+8, ... four at a time; all the
+  // loads of a 256-channel chunk for the four rows go out together
+  for (int r0 = warp; r0 < n; r0 += 32) {
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
     for (int c = lane * 8; c < D; c += 256) {
-      float h[8], sv[8];
-      load8(Hb + (long)r * D + c, h);
+      float sv[8], h[4][8];
       load8_cg(dSi + c, sv);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) d = fmaf(h[e], sv[e], d);
+      for (int u = 0; u < 4; ++u)
+        if (r0 + 8 * u < n) load8(Hb + (long)(r0 + 8 * u) * D + c, h[u]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (r0 + 8 * u < n) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) d[u] = fmaf(h[u][e], sv[e], d[u]);
+        }
     }
-    d = warp_sum(d);
-    if (lane == 0) g[r] = d;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float t = warp_sum(d[u]);
+      if (lane == 0 && r0 + 8 * u < n) g[r0 + 8 * u] = t;
+    }
   }
   __syncthreads();
   if (warp == 0) {
