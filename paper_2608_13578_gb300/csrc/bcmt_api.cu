@@ -219,9 +219,8 @@ int dw_splits(int M, int N, long K) {
 }
 
 struct FwdWs {
-  char *qkv, *hhat, *hloc, *G;
+  char *qkv, *hhat, *hloc, *G, *Mb;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
-  unsigned* gbar;
   size_t bytes;
 };
 
@@ -234,7 +233,6 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     off += al256(bytes);
     return r;
   };
-  w.gbar = reinterpret_cast<unsigned*>(take(64));  // grid barrier of the memory kernel
   w.qkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
   w.lse = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
   w.hhat = take((size_t)g.n * g.D * g.es);
@@ -245,11 +243,13 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     w.spart = reinterpret_cast<float*>(take((size_t)g.n * (g.D / 4) * 4));
     w.S = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.M = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    // M in the storage dtype: the A operand of the memory projection (and of dW_m)
+    w.Mb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.M);
     w.Z = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
     w.C = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.G = take((size_t)g.n * g.D * g.es);
   } else {
-    w.hloc = w.G = nullptr;
+    w.hloc = w.G = w.Mb = nullptr;
     w.alpha = w.S = w.M = w.Z = w.C = w.spart = nullptr;
   }
   w.bytes = off;
@@ -257,9 +257,8 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 }
 
 struct BwdWs {
-  char *dU, *dH, *dHhat, *dqkv;
+  char *dU, *dH, *dHhat, *dqkv, *dPb;
   float *dP, *dM, *dS, *ds, *dwp_part, *Drow, *part;
-  unsigned* gbar;
   size_t bytes;
 };
 
@@ -272,17 +271,17 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     off += al256(bytes);
     return r;
   };
-  w.gbar = reinterpret_cast<unsigned*>(take(64));  // grid barrier of the memory kernel
   if (!g.honly) {
     w.dU = take((size_t)g.n * g.D * g.es);
     w.dH = take((size_t)g.n * g.D * g.es);
     w.dP = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.dPb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.dP);
     w.dM = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
   } else {
-    w.dU = w.dH = nullptr;
+    w.dU = w.dH = w.dPb = nullptr;
     w.dP = w.dM = w.dS = w.ds = w.dwp_part = nullptr;
   }
   w.dHhat = take((size_t)g.n * g.D * g.es);
@@ -453,13 +452,26 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // Sec. 3.4-3.5: adaptive block summaries, exponential causal memory,
-    // projection and shift: one cooperative kernel.
-    pr.begin("memory_fwd");
-    e = memory_fwd_phase(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, decay, w_m, w.M, w.Z,
-                         w.C, w.gbar, g.B, g.T, D, g.L);
+    // Sec. 3.4: adaptive block summaries.
+    pr.begin("summary_fwd");
+    e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
     pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "block summaries and causal memory");
+    if (e != cudaSuccess) return cuda_fail(e, "block summaries");
+    // Sec. 3.5: exponential causal memory (scan), then projection and shift.
+    pr.begin("memory_scan_fwd");
+    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C, g.B,
+                        g.Nb, D);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "causal memory");
+    {
+      EpiArgs ea;
+      ea.out = w.C;
+      ea.ldo = D;
+      ea.Nb = g.Nb;
+      e = run_gemm(lc, pr, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
+                   EPI_SHIFT, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "memory projection");
+    }
     // Sec. 3.7-3.8: gate and injection fused into the W_g GEMM.
     EpiArgs ea;
     ea.H = w.hloc;
@@ -529,20 +541,40 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
 
   const void* dH = dy;  // HOnly: Y = H
   if (!g.honly) {
-    // Sec. 3.8, 3.5, 3.4 reversed in one cooperative kernel: dU and the shifted
-    // per-block memory gradient dP; dM = dP W_m^T; the reverse decayed scan
-    // -> dS; the pooling backward -> ds and the dW_p partials.
-    pr.begin("memory_bwd");
-    e = memory_bwd_phase(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, w_m, bw.dM, decay, w.Z, bw.dS,
-                         w.hloc, w.alpha, bw.ds, bw.dwp_part, bw.gbar, g.B, g.T, D, g.L);
+    // Sec. 3.8 reversed: dU and the per-block memory gradient (shifted: dP).
+    pr.begin("gate_bwd");
+    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.dtype == BCMT_BF16 ? bw.dPb : nullptr,
+                 g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "gate backward");
+    // Sec. 3.5 reversed: dM = dP W_m^T, reverse decayed scan -> dS.
+    {
+      EpiArgs ea;
+      ea.out = bw.dM;
+      ea.ldo = D;
+      e = run_gemm(lc, pr, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
+                   EPI_STORE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "dM");
+    }
+    pr.begin("memory_scan_bwd");
+    e = memory_scan_bwd(lc, bw.dM, decay, w.Z, bw.dS, g.B, g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
+    // Sec. 3.4 reversed: pooling scores and the dW_p partials.
+    pr.begin("summary_bwd");
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     // side stream: dW_m = M^T dP, dW_g = H^T dU, dW_p
     fork.point();
-    prs.begin("memory_dwm");
-    e = small_gemm(lcs, 0, g.dtype, D, D, g.B * g.Nb, w.M, 1, D, bw.dP, D, 1, dw_m, D);
-    prs.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_m");
+    {
+      EpiArgs ea;
+      ea.out = dw_m;
+      ea.ldo = D;
+      e = run_gemm(lcs, prs, "gemm_dwm", g.dtype, g.dtype, D, D, g.B * g.Nb, w.Mb, 1, D, bw.dPb, D,
+                   1, EPI_STORE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "dW_m");
+    }
     e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
                     bw.part, dw_g);
     if (e != cudaSuccess) return cuda_fail(e, "dW_g");

@@ -383,12 +383,13 @@ mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
 
 // Output tile widths: 128 x 256 tiles move 48 KB per 64-deep K slice for
 // 4.2 MFLOP (87 FLOP per L2 byte), 128 x 128 tiles 32 KB for 2.1 MFLOP (64).
-// The wide tile is used when it still gives most SMs a tile.
+// The wide tile is used when it still gives most SMs a tile; 128 x 64 tiles
+// (an 8-deep ring) when even 128-wide tiles would leave most SMs idle.
 template <int BN, bool A_MN, bool B_MN>
 static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                           long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                           const EpiArgs& ea, int splits) {
-  constexpr int ST = BN == 256 ? 4 : 6;
+  constexpr int ST = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
   switch (epi) {
     case EPI_STORE:
       if (dtype_out == 0)
@@ -439,10 +440,17 @@ template <bool A_MN, bool B_MN>
 static cudaError_t tc_pick(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                            long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                            const EpiArgs& ea, int splits) {
-  const long tiles256 = (long)((M + kBM - 1) / kBM) * ((N + 255) / 256) * splits;
+  const long tm = (M + kBM - 1) / kBM;
+  const long tiles256 = tm * ((N + 255) / 256) * splits;
+  const long tiles128 = tm * ((N + 127) / 128) * splits;
   if (N % 256 == 0 && tiles256 * 4 >= (long)sm_count() * 3)
     return tc_epi<256, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea,
                                    splits);
+  // few tiles (the memory stage's [B*Nb x D] products): narrow tiles spread the
+  // operand traffic over more SMs
+  if (tiles128 * 4 < (long)sm_count())
+    return tc_epi<64, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea,
+                                  splits);
   return tc_epi<128, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
 }
 

@@ -112,27 +112,27 @@ cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
 bool attn_tc_supported(int dtype, int dh, int L);
 
 // ------------------------------------------------ summary, memory, gate
-// Forward of Sec. 3.4-3.5 as one cooperative kernel: pooling scores (summed
-// from npart partials spart[j * B*T + token]), alpha = softmax per block,
-// S = H^T alpha; then the decayed scan M (and its denominator Z [Nb, D]) and
-// the projected, shifted memory C[b, 0] = 0, C[b, i+1] = M_i W_m.  gbar: two
-// words of device memory for the grid barrier.
-cudaError_t memory_fwd_phase(const Launch& lc, int dtype, const void* Hm, const float* spart,
-                             int npart, float* alpha, float* S, const float* decay,
-                             const void* w_m, float* M, float* Z, float* Cmem, unsigned* gbar,
-                             int B, int T, int D, int L);
-// Backward of Sec. 3.8 (dU, dP), 3.5 (dM = dP W_m^T, dS by the reverse scan)
-// and 3.4 (ds, per-block dW_p partials) as one cooperative kernel.
-cudaError_t memory_bwd_phase(const Launch& lc, int dtype, const void* dY, const void* G,
-                             const float* Cmem, void* dU, float* dP, const void* w_m, float* dM,
-                             const float* decay, const float* Z, float* dS, const void* Hm,
-                             const float* alpha, float* ds, float* dwp_part, unsigned* gbar, int B,
-                             int T, int D, int L);
-// out[m, n] = sum_k A(m,k) B(k,n) on CUDA cores in 16 x 32 tiles (small
-// products of the memory stage); A fp32, B of dtype_b, out of dtype_out.
-cudaError_t small_gemm(const Launch& lc, int dtype_b, int dtype_out, int M, int N, int K,
-                       const float* A, long sam, long sak, const void* B, long sbk, long sbn,
-                       void* out, long ldo);
+// Sec. 3.4: per block, s = H w_p (summed from npart partial dot products
+// spart[j * B*T + token]), alpha = softmax(s), S = H^T alpha.
+cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
+                        float* alpha, float* S, int B, int T, int D, int L);
+// Sec. 3.5: M = normalised decayed scan of S over blocks (fp32, plus a bf16
+// copy in Mb when non-null), Z its denominator [Nb, D], C[b, 0] = 0.  The
+// projection C[b, i+1] = M_i W_m is a GEMM with the EPI_SHIFT epilogue.
+cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
+                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D);
+// Backward of the gate and injection: dU = dY*C*G*(1-G); dP[b,i-1] = sum over
+// block i of dY*G (also in bf16 in dPb when non-null); dP[b,Nb-1] = 0.
+cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
+                     void* dU, float* dP, void* dPb, int B, int T, int D, int L);
+// Backward of the memory scan: dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i, given
+// dM = dP W_m^T.
+cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
+                            float* dS, int B, int Nb, int D);
+// Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
+// dwp_part[b*Nb+i] = sum_t ds_t H_t.
+cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
+                        const float* dS, float* ds, float* dwp_part, int B, int T, int D, int L);
 // Column sums of an fp32 [rows, cols] matrix in row order, stored in dtype_out.
 cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, int dtype_out,
                         void* out);
