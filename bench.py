@@ -170,6 +170,7 @@ def kernel_model(w):
     amount in flops for tensor-core GEMMs and bytes for HBM-bound kernels."""
     n, D, H, Nb, B = w.B * w.T, w.D, w.H, w.n_blocks, w.B
     es = 2 if w.dtype == "bf16" else 4
+    npart = D // 32 if w.dtype == "bf16" else D // 4  # score partials per token
     g = lambda m, nn, k: ("tensor", 2.0 * m * nn * k)
     return {
         "gemm_qkv": g(n, 3 * D, D),
@@ -187,13 +188,20 @@ def kernel_model(w):
         # read Q, K, V, dO, O and the log-sum-exp; write dQ, dK, dV
         "attn_bwd_tc": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
         "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
-        # summaries (read H and the score partials, write alpha and S), then the
-        # scan and projection (read S and W_m, write M, Z and C)
-        "memory_fwd": ("hbm", n * D * es + n * 4 * (D // 32 + 1) + B * Nb * D * 4 * 4
-                       + Nb * D * 4 + D * D * es),
-        # gate backward (read dY, G; write dU), dM, scan, pooling backward (read H)
-        "memory_bwd": ("hbm", 4 * n * D * es + 3 * n * 4 + B * Nb * D * 4 * 6 + D * D * es),
-        "memory_dwm": ("hbm", 2 * B * Nb * D * 4 + D * D * es),
+        # Sec. 3.4 summaries: read H and the score partials, write alpha and S
+        "summary_fwd": ("hbm", n * D * es + n * 4 * npart + n * 4 + B * Nb * D * 4),
+        # Sec. 3.5 scan: read S, write M (fp32 and the bf16 operand copy), Z, C[:, 0]
+        "memory_scan_fwd": ("hbm", B * Nb * D * (4 + 4 + 2) + Nb * D * 4 + B * D * 4),
+        "gemm_wm": g(B * Nb, D, D),
+        # Sec. 3.8 reversed: read dY, G and C; write dU and dP (fp32 + bf16)
+        "gate_bwd": ("hbm", 3 * n * D * es + B * Nb * D * (4 + 4 + 2)),
+        "gemm_dm": g(B * Nb, D, D),
+        # reverse scan: read dM and Z, write dS
+        "memory_scan_bwd": ("hbm", 2 * B * Nb * D * 4 + Nb * D * 4),
+        # pooling backward: read H, alpha and dS; write ds and the dW_p partials
+        "summary_bwd": ("hbm", n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
+        "gemm_dwm": g(D, D, B * Nb),
+        "reduce_rows": ("hbm", B * Nb * D * 4 + D * es),
     }
 
 

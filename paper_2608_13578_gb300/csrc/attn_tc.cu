@@ -57,7 +57,14 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 }
 }  // namespace
 
+// Both kernels are instantiated for NCH = the number of 32-key chunks of a
+// block that one warp's 32 query rows can reach (1 for L <= 32, L / 32
+// otherwise); a warp reads only the chunks up to its own last row's key, the
+// rest of its P and dS rows are causal zeros.
+__device__ __forceinline__ int chunks_needed(int warp, int wbs) { return (warp * 32 - wbs) / 32 + 1; }
+
 // ====================================================================== forward
+template <int NCH>
 __global__ void __launch_bounds__(128)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mO,
@@ -119,46 +126,54 @@ __global__ void __launch_bounds__(128)
   bool ok = tc::mbar_wait(&bar[1], 0, status);
   tc::fence_after_sync();
 
-  // ---- masked softmax, thread = query row r of the tile
+  // ---- masked softmax, thread = query row r of the tile: the row's scores
+  // (at most 128 keys) come out of TMEM in one batch of loads
   const int r = warp * 32 + lane;
-  const int nc = L < 32 ? 32 : L;                           // columns this warp reads
-  const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;  // first of them
+  const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;  // first key column read
+  const int nld = chunks_needed(warp, wbs);                    // 32-column chunks read
   const int rbs = (r / L) * L;                              // first key row r may see
   const float sl2 = scale * kLog2e;
+  uint32_t sr[NCH][32];
+#pragma unroll
+  for (int ci = 0; ci < NCH; ++ci)
+    if (ci < nld) tc::tmem_ld32_issue(trow + (uint32_t)(wbs + ci * 32), sr[ci]);
+  tc::tmem_wait();
   float mx = -INFINITY;
-  for (int c = 0; c < nc; c += 32) {
-    float v[32];
-    tc::tmem_ld32(trow + (uint32_t)(wbs + c), v);
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      const int kk = wbs + c + j;
-      if (kk >= rbs && kk <= r) mx = fmaxf(mx, v[j]);
+  for (int ci = 0; ci < NCH; ++ci)
+    if (ci < nld) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const int kk = wbs + ci * 32 + j;
+        if (kk >= rbs && kk <= r) mx = fmaxf(mx, __uint_as_float(sr[ci][j]));
+      }
     }
-  }
   float sum = 0.f;
-  for (int c = 0; c < nc; c += 32) {
-    float v[32];
-    tc::tmem_ld32(trow + (uint32_t)(wbs + c), v);
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      const int kk = wbs + c + j;
-      const float p = (kk >= rbs && kk <= r) ? exp2f((v[j] - mx) * sl2) : 0.f;
-      v[j] = p;
-      sum += p;
-    }
+  for (int ci = 0; ci < NCH; ++ci)
+    if (ci < nld) {
+      float v[32];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      uint4 q;
-      q.x = pack2(v[8 * u + 0], v[8 * u + 1]);
-      q.y = pack2(v[8 * u + 2], v[8 * u + 3]);
-      q.z = pack2(v[8 * u + 4], v[8 * u + 5]);
-      q.w = pack2(v[8 * u + 6], v[8 * u + 7]);
-      put_unit(sP, r, (wbs + c) / 8 + u, q);
+      for (int j = 0; j < 32; ++j) {
+        const int kk = wbs + ci * 32 + j;
+        const float p =
+            (kk >= rbs && kk <= r) ? exp2f((__uint_as_float(sr[ci][j]) - mx) * sl2) : 0.f;
+        v[j] = p;
+        sum += p;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        uint4 q;
+        q.x = pack2(v[8 * u + 0], v[8 * u + 1]);
+        q.y = pack2(v[8 * u + 2], v[8 * u + 3]);
+        q.z = pack2(v[8 * u + 4], v[8 * u + 5]);
+        q.w = pack2(v[8 * u + 6], v[8 * u + 7]);
+        put_unit(sP, r, (wbs + ci * 32) / 8 + u, q);
+      }
     }
-  }
   const uint4 zero = make_uint4(0, 0, 0, 0);
   for (int u = 0; u < 16; ++u)
-    if (u * 8 < wbs || u * 8 >= wbs + nc) put_unit(sP, r, u, zero);
+    if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
@@ -179,10 +194,13 @@ __global__ void __launch_bounds__(128)
 
   // ---- epilogue: O = (P V) / sum, staged in the (now free) Q/P tile
   const float inv = 1.0f / sum;
-  for (int half = 0; half < 2; ++half) {
-    float v[32];
-    tc::tmem_ld32(trow + (uint32_t)(half * 32), v);
-    stage_half(sQ, r, half, v, inv);
+  {
+    uint32_t o[2][32];
+    tc::tmem_ld32_issue(trow, o[0]);
+    tc::tmem_ld32_issue(trow + 32u, o[1]);
+    tc::tmem_wait();
+    stage_half(sQ, r, 0, reinterpret_cast<const float*>(o[0]), inv);
+    stage_half(sQ, r, 1, reinterpret_cast<const float*>(o[1]), inv);
   }
   if (ok && t0 + r < Tlen) lse[((long)b * H + h) * Tlen + t0 + r] = mx * scale + logf(sum);
   tc::fence_proxy_async_smem();
@@ -201,6 +219,7 @@ __global__ void __launch_bounds__(128)
 // Shared memory: Q, K, dO (16 KB each) and a 32 KB region that holds V, then
 // P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in registers
 // until the dV product has consumed P.  80 KB per CTA: two CTAs per SM.
+template <int NCH>
 __global__ void __launch_bounds__(128)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
@@ -294,18 +313,27 @@ __global__ void __launch_bounds__(128)
 
   // ---- P = exp(S*scale - lse) to shared memory; scale * P * (dP - Drow) kept
   // packed in registers (up to 128 keys: 64 words)
-  const int nc = L < 32 ? 32 : L;
   const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;
+  const int nld = chunks_needed(warp, wbs);
   const int rbs = (r / L) * L;
   const float sl2 = scale * kLog2e, ll2 = lr * kLog2e;
-  uint32_t dsp[64];
+  uint32_t dsp[NCH * 16];
 #pragma unroll
-  for (int ci = 0; ci < 4; ++ci) {
-    if (ci * 32 < nc) {
+  for (int ci = 0; ci < NCH; ++ci) {
+    if (ci < nld) {
       const int c = ci * 32;
       float s[32], dp[32];
-      tc::tmem_ld32(trow + (uint32_t)(wbs + c), s);
-      tc::tmem_ld32(trow + 128u + (uint32_t)(wbs + c), dp);
+      {
+        uint32_t rs[32], rd[32];
+        tc::tmem_ld32_issue(trow + (uint32_t)(wbs + c), rs);
+        tc::tmem_ld32_issue(trow + 128u + (uint32_t)(wbs + c), rd);
+        tc::tmem_wait();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          s[j] = __uint_as_float(rs[j]);
+          dp[j] = __uint_as_float(rd[j]);
+        }
+      }
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
         const int kk = wbs + c + j;
@@ -328,7 +356,7 @@ __global__ void __launch_bounds__(128)
   }
   const uint4 zero = make_uint4(0, 0, 0, 0);
   for (int u = 0; u < 16; ++u)
-    if (u * 8 < wbs || u * 8 >= wbs + nc) put_unit(sP, r, u, zero);
+    if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
@@ -348,8 +376,8 @@ __global__ void __launch_bounds__(128)
   ok = tc::mbar_wait(&bar[2], 0, status) && ok;
   tc::fence_after_sync();
 #pragma unroll
-  for (int ci = 0; ci < 4; ++ci) {
-    if (ci * 32 < nc) {
+  for (int ci = 0; ci < NCH; ++ci) {
+    if (ci < nld) {
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const uint4 d = make_uint4(dsp[ci * 16 + 4 * u], dsp[ci * 16 + 4 * u + 1],
@@ -385,19 +413,16 @@ __global__ void __launch_bounds__(128)
 
   // ---- epilogue: rows of dV, dK (key r) and dQ (query r) through staging tiles
   {
-    float v[32];
-    tc::tmem_ld32(trow + 0u, v);
-    stage_half(sdO, r, 0, v, 1.0f);
-    tc::tmem_ld32(trow + 32u, v);
-    stage_half(sdO, r, 1, v, 1.0f);
-    tc::tmem_ld32(trow + 64u, v);
-    stage_half(sK, r, 0, v, 1.0f);
-    tc::tmem_ld32(trow + 96u, v);
-    stage_half(sK, r, 1, v, 1.0f);
-    tc::tmem_ld32(trow + 128u, v);
-    stage_half(sQ, r, 0, v, 1.0f);
-    tc::tmem_ld32(trow + 160u, v);
-    stage_half(sQ, r, 1, v, 1.0f);
+    uint8_t* const dst[3] = {sdO, sK, sQ};  // dV, dK, dQ staging tiles
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      uint32_t o[2][32];
+      tc::tmem_ld32_issue(trow + (uint32_t)(64 * q), o[0]);
+      tc::tmem_ld32_issue(trow + (uint32_t)(64 * q + 32), o[1]);
+      tc::tmem_wait();
+      stage_half(dst[q], r, 0, reinterpret_cast<const float*>(o[0]), 1.0f);
+      stage_half(dst[q], r, 1, reinterpret_cast<const float*>(o[1]), 1.0f);
+    }
   }
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
@@ -429,51 +454,74 @@ static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, in
 static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
 static constexpr int kBwdSmem = 5 * kTB + 1024 + 64;
 
-cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
-  if (!attn_tc_supported(1, a.dh, a.L)) return cudaErrorNotSupported;
-  const int D = a.H * kDh;
-  CUtensorMap mQ, mK, mV, mO;
-  if (!head_map(&mQ, a.Q, a.ld_qkv, D, a.T, a.B) || !head_map(&mK, a.K, a.ld_qkv, D, a.T, a.B) ||
-      !head_map(&mV, a.V, a.ld_qkv, D, a.T, a.B) || !head_map(&mO, a.O, a.ld_o, D, a.T, a.B))
-    return cudaErrorInvalidValue;
+static int chunks_for(int L) { return L <= 32 ? 1 : L / 32; }
+
+template <class K>
+static cudaError_t opt_in(K* kern, int bytes) {
+  return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+template <int NCH>
+static cudaError_t fwd_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kFwdSmem);
+    cudaError_t e = opt_in(attn_fwd_tc_kernel<NCH>, kFwdSmem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
-  launch_k(attn_fwd_tc_kernel, dim3(grid), dim3(128), kFwdSmem, lc.stream,
-mQ, mK, mV, mO, a.lse, a.T, a.H, a.L,
-                                                         1.0f / sqrtf((float)a.dh), lc.status);
-  return cudaGetLastError();
+  cudaError_t e = launch_k(attn_fwd_tc_kernel<NCH>, grid, dim3(128), kFwdSmem, lc.stream, m[0],
+                           m[1], m[2], m[3], a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)a.dh),
+                           lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
+  if (!attn_tc_supported(1, a.dh, a.L)) return cudaErrorNotSupported;
+  const int D = a.H * kDh;
+  CUtensorMap m[4];
+  if (!head_map(&m[0], a.Q, a.ld_qkv, D, a.T, a.B) || !head_map(&m[1], a.K, a.ld_qkv, D, a.T, a.B) ||
+      !head_map(&m[2], a.V, a.ld_qkv, D, a.T, a.B) || !head_map(&m[3], a.O, a.ld_o, D, a.T, a.B))
+    return cudaErrorInvalidValue;
+  switch (chunks_for(a.L)) {
+    case 1: return fwd_launch<1>(lc, a, m);
+    case 2: return fwd_launch<2>(lc, a, m);
+    default: return fwd_launch<4>(lc, a, m);
+  }
+}
+
+template <int NCH>
+static cudaError_t bwd_launch(const Launch& lc, const AttnBwdArgs& a, const CUtensorMap* m) {
+  const AttnArgs& f = a.f;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = opt_in(attn_bwd_tc_kernel<NCH>, kBwdSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
+  cudaError_t e = launch_k(attn_bwd_tc_kernel<NCH>, grid, dim3(128), kBwdSmem, lc.stream, m[0],
+                           m[1], m[2], m[3], m[4], m[5], m[6], (const bf16*)f.O, f.ld_o, f.lse,
+                           f.T, f.H, f.L, 1.0f / sqrtf((float)f.dh), lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
   const AttnArgs& f = a.f;
   if (!attn_tc_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
   const int D = f.H * kDh;
-  CUtensorMap mQ, mK, mV, mdO, mdQ, mdK, mdV;
-  if (!head_map(&mQ, f.Q, f.ld_qkv, D, f.T, f.B) || !head_map(&mK, f.K, f.ld_qkv, D, f.T, f.B) ||
-      !head_map(&mV, f.V, f.ld_qkv, D, f.T, f.B) || !head_map(&mdO, a.dO, f.ld_o, D, f.T, f.B) ||
-      !head_map(&mdQ, a.dQ, a.ld_dqkv, D, f.T, f.B) ||
-      !head_map(&mdK, a.dK, a.ld_dqkv, D, f.T, f.B) ||
-      !head_map(&mdV, a.dV, a.ld_dqkv, D, f.T, f.B))
+  CUtensorMap m[7];
+  if (!head_map(&m[0], f.Q, f.ld_qkv, D, f.T, f.B) || !head_map(&m[1], f.K, f.ld_qkv, D, f.T, f.B) ||
+      !head_map(&m[2], f.V, f.ld_qkv, D, f.T, f.B) || !head_map(&m[3], a.dO, f.ld_o, D, f.T, f.B) ||
+      !head_map(&m[4], a.dQ, a.ld_dqkv, D, f.T, f.B) ||
+      !head_map(&m[5], a.dK, a.ld_dqkv, D, f.T, f.B) ||
+      !head_map(&m[6], a.dV, a.ld_dqkv, D, f.T, f.B))
     return cudaErrorInvalidValue;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
+  switch (chunks_for(f.L)) {
+    case 1: return bwd_launch<1>(lc, a, m);
+    case 2: return bwd_launch<2>(lc, a, m);
+    default: return bwd_launch<4>(lc, a, m);
   }
-  dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
-  launch_k(attn_bwd_tc_kernel, dim3(grid), dim3(128), kBwdSmem, lc.stream,
-
-      mQ, mK, mV, mdO, mdQ, mdK, mdV, (const bf16*)f.O, f.ld_o, f.lse, f.T, f.H, f.L,
-      1.0f / sqrtf((float)f.dh), lc.status);
-  return cudaGetLastError();
 }
 
 }  // namespace bcmt
