@@ -474,6 +474,132 @@ def bench_dense(w, t, stream, flush, args):
             "what": "x W_qkv -> torch SDPA(is_causal) over the full sequence -> W_O, fwd+bwd, bf16"}
 
 
+# ------------------------------------------------ whole-model training steps
+# Config 5 of the benchmark set (a 6-layer GPT-style decoder with the BCMT
+# mixer), and the paper's own throughput shape (Tables 1-2: D 128, 8 heads,
+# 6 layers, batch 16) for BCMT, its HOnly ablation and dense attention.
+MODEL_WORKLOADS = {
+    "gpt6_v32000_d512_h8_mlp2048_l64_t1024_b16": dict(
+        B=16, vocab=32000, D=512, H=8, layers=6, mlp=2048, runs=[("bcmt", 64, 1024)]),
+    "paper_d128_h8_6l_b16_sweep": dict(
+        B=16, vocab=50257, D=128, H=8, layers=6, mlp=512,
+        runs=[(m, L, T) for T in (128, 256, 512, 1024) for L in (64, 128, 256, 512) if L <= T
+              for m in ("bcmt", "honly")] + [("dense", 0, T) for T in (128, 256, 512, 1024)]),
+}
+
+
+def bench_models(args):
+    """Training-step tokens/s of whole models (embedding, 6 blocks, LM head,
+    cross-entropy, AdamW) with the BCMT mixer from this library and the rest
+    from PyTorch; the dense-attention model of the same shape beside it."""
+    import torch
+    from paper_2608_13578_gb300 import build
+    build.build()
+    from paper_2608_13578_gb300 import bcmt as C
+    from paper_2608_13578_gb300 import gpt, layer
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        if rank != 0:
+            return None  # model steps are measured on one GPU
+    torch.cuda.set_device(local_rank)
+    name = args.workload
+    spec = MODEL_WORKLOADS[name]
+    B = spec["B"]
+    stream = torch.cuda.current_stream()
+
+    def run(mixer, L, T, steps, warmup):
+        c = gpt.GPTConfig(vocab=spec["vocab"], D=spec["D"], H=spec["H"], layers=spec["layers"],
+                          mlp=spec["mlp"], L=max(L, 1), T=T,
+                          mixer="dense" if mixer == "dense" else "bcmt", honly=mixer == "honly")
+        model = gpt.build(c)
+        opt = gpt.make_optimizer(model)
+        g = torch.Generator().manual_seed(rank_seed(0, rank))
+        ids_h = torch.randint(0, c.vocab, (B, T + 1), generator=g).pin_memory()
+        ids = ids_h.cuda()
+        inp, tgt = ids[:, :-1].contiguous(), ids[:, 1:].contiguous()
+        for _ in range(max(3, warmup)):
+            gpt.train_step(model, opt, inp, tgt)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for i in range(steps):
+            ev[i][0].record(stream)
+            gpt.train_step(model, opt, inp, tgt)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        ms = sum(a.elapsed_time(b) for a, b in ev)
+        # end to end: the step's token ids copied in from pinned host memory and
+        # its loss read back, every step
+        d_ids = torch.empty_like(ids)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        losses = []
+        for _ in range(steps):
+            d_ids.copy_(ids_h, non_blocking=True)
+            loss = gpt.train_step(model, opt, d_ids[:, :-1], d_ids[:, 1:])
+            losses.append(loss.item())
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1)
+        tok = B * T * steps
+        r = {"mixer": mixer, "L": L if mixer != "dense" else None, "T": T,
+             "tokens_per_s": round(tok / (ms / 1e3), 1), "ms_per_step": round(ms / steps, 3),
+             "e2e_tokens_per_s": round(tok / (e2e_ms / 1e3), 1),
+             "tflops": round(gpt.flops_per_token(c) * tok / (ms / 1e3) / 1e12, 1),
+             "loss_first_last": [round(losses[0], 4), round(losses[-1], 4)],
+             "h2d_bytes_per_step": ids_h.numel() * ids_h.element_size(), "d2h_bytes_per_step": 4}
+        del model, opt
+        torch.cuda.empty_cache()
+        return r
+
+    def mixer_launches(L, T, honly):
+        """Our kernels per mixer forward+backward at this shape (profiled call)."""
+        D, H = spec["D"], spec["H"]
+        p = layer.params_for(B, T, D, H, L, "bf16", True, honly, flags=C.BCMT_FLAG_PROFILE)
+        t = {"x": torch.randn(B, T, D, device="cuda").bfloat16(),
+             "w_qkv": torch.randn(D, 3 * D, device="cuda").bfloat16(),
+             "decay": torch.full((D,), 0.8, device="cuda")}
+        for n in ("w_o", "w_m", "w_g"):
+            t[n] = torch.randn(D, D, device="cuda").bfloat16()
+        t["w_p"] = torch.randn(D, device="cuda").bfloat16()
+        C.bcmt_profile_reset()
+        y, ws = layer.forward(p, t)
+        layer.backward(p, t, ws, torch.randn_like(y))
+        n = sum(c for c, _ in C.bcmt_profile_read().values())
+        C.bcmt_profile_reset()
+        return n
+
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    rows = [run(m, L, T, args.steps, args.warmup) for m, L, T in spec["runs"]]
+    clk = clocks.stop()
+    head = rows[0]
+    dense = None
+    if name.startswith("gpt"):
+        dense = run("dense", 0, spec["runs"][0][2], args.steps, args.warmup)
+    launches = sum(mixer_launches(L, T, m == "honly") * spec["layers"] * args.steps
+                   for m, L, T in spec["runs"][:1] if m != "dense")
+    out = {"metric": "training-step tokens/s of a 6-layer decoder with the BCMT mixer",
+           "value": head["tokens_per_s"], "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+           "warmup": max(3, args.warmup), "ms_per_step": head["ms_per_step"],
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+           "data": "synthetic token ids uniform over the vocabulary, random init",
+           "config": {"workload": name, "B": B, "T": head["T"], "L": head["L"], "D": spec["D"],
+                      "H": spec["H"], "layers": spec["layers"], "mlp": spec["mlp"],
+                      "vocab": spec["vocab"], "optimizer": "AdamW (fused, bf16 params)",
+                      "l2": "working set (weights, activations, optimizer state) > L2"},
+           "clocks": clk,
+           "e2e": {"value": head["e2e_tokens_per_s"], "unit": UNIT,
+                   "h2d_bytes_per_step": head["h2d_bytes_per_step"],
+                   "d2h_bytes_per_step": head["d2h_bytes_per_step"]},
+           "gpu_launches": launches, "model_tflops": head["tflops"], "runs": rows,
+           "dense_model": dense}
+    print(json.dumps(out))
+    return out
+
+
 # ------------------------------------------------------ reference arm (oracle)
 def bench_reference(args):
     rank, _, world = dist_env()
@@ -481,9 +607,13 @@ def bench_reference(args):
         return None
     from paper_2608_13578_gb300.inputs import HEADLINE, WORKLOADS
     name = args.workload or HEADLINE
+    if name in MODEL_WORKLOADS:
+        out = {"impl": "reference", "unavailable": "the oracle covers the mixer layer only; "
+                                                   "whole-model steps have no CPU reference"}
+        print(json.dumps(out))
+        return out
     w = WORKLOADS[name]
     # each step: the oracle's fwd+bwd on one batch element of the workload
-    budget = max(5.0, 150.0 / max(1, args.steps + args.warmup))
     d = run_oracle_sample(name, budget_s=0.0, max_reps=args.warmup + args.steps)
     times = d["times"][args.warmup:] or d["times"]
     secs = sum(times)
@@ -500,7 +630,6 @@ def bench_reference(args):
            "cpu_baseline": cpu,
            "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
-    del budget
     print(json.dumps(out))
     return out
 
@@ -509,6 +638,8 @@ def main():
     args = parse()
     if args.impl == "reference":
         bench_reference(args)
+    elif args.workload in MODEL_WORKLOADS:
+        bench_models(args)
     else:
         bench_ours(args)
 

@@ -31,7 +31,7 @@
  *    bf16); arithmetic accumulates in fp32.  `decay` is always fp32 [D], each
  *    entry in [0, 1); pass 0.8 in every entry for the paper's setting.
  *  - Pointers must be 16-byte aligned.  Requirements on shapes: B, T >= 1;
- *    H >= 1 and D % H == 0; dh = D / H a multiple of 32 and <= 128; D a
+ *    H >= 1 and D % H == 0; dh = D / H a multiple of 8 and <= 128; D a
  *    multiple of 64; 1 <= L <= 1024.  Any T is accepted: the last block may be
  *    ragged (Sec. 3.2).  bf16 shapes with dh == 64 and L a power of two in
  *    [16, 128] run the tcgen05 tensor-core attention; other valid shapes run a
@@ -112,7 +112,9 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
 
 /* Backward pass: gradients of sum(dy * Y) with respect to the layer inputs
  * and weights, given the workspace of the matching bcmt_forward (same p and
- * same inputs).  The decay is fixed (Sec. 3.5) and gets no gradient.
+ * same inputs).  The paper keeps the decay fixed (Sec. 3.5); its gradient,
+ * for a learned per-channel decay (named as future work in Sec. 5), is
+ * returned only when d_decay is non-NULL.
  *   dy       [B,T,D]
  *   x_or_q   the forward's x when input_is_x, else its q
  *   k, v     the forward's k and v iff !input_is_x (else may be NULL)
@@ -124,14 +126,16 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
  *   dk, dv   [B,T,D]  used iff !input_is_x
  *   dw_qkv   [D,3D]   used iff input_is_x
  *   dw_o [D,D], dw_p [D], dw_m [D,D], dw_g [D,D]
+ *   d_decay  [D] fp32, optional (NULL: not computed)
  * Every output is overwritten (not accumulated).  With BCMT_FLAG_HONLY,
- * dw_p, dw_m and dw_g are set to zero. */
+ * dw_p, dw_m, dw_g and d_decay are set to zero. */
 bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or_q,
                           const void* k, const void* v, const void* w_qkv, const void* w_o,
                           const void* w_p, const void* w_m, const void* w_g,
                           const float* decay, const void* workspace,
                           void* scratch, void* dx_or_dq, void* dk, void* dv, void* dw_qkv,
-                          void* dw_o, void* dw_p, void* dw_m, void* dw_g, void* stream);
+                          void* dw_o, void* dw_p, void* dw_m, void* dw_g, float* d_decay,
+                          void* stream);
 
 /* Allocation-free backward of the intra-block attention alone (the SIMT
  * kernels of the layer's backward; the paper has no counterpart -- it is an

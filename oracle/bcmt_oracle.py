@@ -31,8 +31,11 @@ reverse order; the tests pin them with central finite differences.
 
 Readings where the paper is silent (each also listed in the design notes):
   * the decay ``a`` is a per-channel vector a[D] in [0,1); the paper's fixed
-    scalar 0.8 (Sec. 3.5) is the broadcast case; it is not learned, so it has
-    no gradient;
+    scalar 0.8 (Sec. 3.5) is the broadcast case.  The paper does not learn it;
+    its gradient d_decay (for the learned per-channel decay that Sec. 5 names
+    as future work) is the derivative of the double sum of Sec. 3.5 itself:
+    with num_i = sum_j a^(i-j) S_j and den_i = sum_j a^(i-j),
+      dM_i/da = (sum_j (i-j) a^(i-j-1) S_j - M_i sum_j (i-j) a^(i-j-1)) / den_i;
   * no biases anywhere, no scale on the pooling scores s;
   * the pooling and attention softmaxes of a ragged last block run over its
     L_i real tokens; the memory denominator counts blocks, not tokens;
@@ -175,7 +178,7 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
     """Hand-derived gradients of the forward above, in reverse order.
 
     Returns dx (or dq, dk, dv when the layer started from Q, K, V) and
-    dw_qkv (when it started from x), dw_o, dw_p, dw_m, dw_g.
+    dw_qkv (when it started from x), dw_o, dw_p, dw_m, dw_g, d_decay.
     """
     inp = fw["_in"]
     w_qkv, w_o, w_p, w_m, w_g = (inp[n] for n in ("w_qkv", "w_o", "w_p", "w_m", "w_g"))
@@ -190,6 +193,7 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
     dw_g = np.zeros((D, D))
     dw_m = np.zeros((D, D))
     dw_p = np.zeros(D)
+    d_decay = np.zeros(D)
     dw_o = np.zeros((D, D))
     dQ = np.zeros((B, T, D))
     dK = np.zeros((B, T, D))
@@ -219,6 +223,15 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
             for j in range(n_b):
                 for i in range(j, n_b):
                     dS[j] += (a ** (i - j)) * dM[i] / Z[i]
+            # d M_i / d a from the same double sum (terms j < i; j = i has a^0)
+            for i in range(n_b):
+                dnum = np.zeros(D)
+                dden = np.zeros(D)
+                for j in range(i):
+                    w = (i - j) * a ** (i - j - 1)
+                    dnum += w * fw["S"][b, j]
+                    dden += w
+                d_decay += dM[i] * (dnum - M[b, i] * dden) / Z[i]
 
             # Sec. 3.4 reversed: S_i = sum_t alpha_t H_t, alpha = softmax(s), s = H w_p.
             for i, (t0, t1) in enumerate(blocks):
@@ -246,7 +259,7 @@ def backward(fw: Dict[str, np.ndarray], dY: np.ndarray) -> Dict[str, np.ndarray]
                 dQ[b, t0:t1, cols] = dScore @ Kb / math.sqrt(d_h)
                 dK[b, t0:t1, cols] = dScore.T @ Qb / math.sqrt(d_h)
 
-    out = dict(dw_o=dw_o, dw_p=dw_p, dw_m=dw_m, dw_g=dw_g)
+    out = dict(dw_o=dw_o, dw_p=dw_p, dw_m=dw_m, dw_g=dw_g, d_decay=d_decay)
     if inp["input_is_x"]:
         x = inp["x"]
         dQKV = np.concatenate([dQ, dK, dV], axis=2)       # [B,T,3D]

@@ -61,7 +61,7 @@ def _load():
     lib.bcmt_scratch_size.restype = ctypes.c_size_t
     lib.bcmt_forward.argtypes = [_P] + [_VP] * 13
     lib.bcmt_forward.restype = ctypes.c_int
-    lib.bcmt_backward.argtypes = [_P] + [_VP] * 20
+    lib.bcmt_backward.argtypes = [_P] + [_VP] * 21
     lib.bcmt_backward.restype = ctypes.c_int
     lib.bcmt_device_status.argtypes = [_VP]
     lib.bcmt_device_status.restype = ctypes.c_int
@@ -138,12 +138,14 @@ def bcmt_forward(p: bcmt_params, x, q, k, v, w_qkv, w_o, w_p, w_m, w_g, decay, y
 
 
 def bcmt_backward(p: bcmt_params, dy, x_or_q, k, v, w_qkv, w_o, w_p, w_m, w_g, decay, workspace,
-                  scratch, dx_or_dq, dk, dv, dw_qkv, dw_o, dw_p, dw_m, dw_g, stream=None) -> None:
+                  scratch, dx_or_dq, dk, dv, dw_qkv, dw_o, dw_p, dw_m, dw_g, stream=None,
+                  d_decay=None) -> None:
+    """d_decay (fp32 [D], optional): gradient for a learned per-channel decay."""
     _check(LIB.bcmt_backward(ctypes.byref(p), _ptr(dy), _ptr(x_or_q), _ptr(k), _ptr(v),
                              _ptr(w_qkv), _ptr(w_o), _ptr(w_p), _ptr(w_m), _ptr(w_g), _ptr(decay),
                              _ptr(workspace), _ptr(scratch), _ptr(dx_or_dq), _ptr(dk), _ptr(dv),
                              _ptr(dw_qkv), _ptr(dw_o), _ptr(dw_p), _ptr(dw_m), _ptr(dw_g),
-                             _stream(stream)))
+                             _ptr(d_decay), _stream(stream)))
 
 
 def bcmt_device_status(stream=None) -> None:

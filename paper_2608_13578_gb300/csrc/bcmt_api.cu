@@ -173,8 +173,8 @@ bcmt_status check_params(const bcmt_params* p) {
   if (p->D % 64 != 0) return fail(BCMT_ERR_SHAPE, "D = %d is not a multiple of 64", p->D);
   if (p->D % p->H != 0) return fail(BCMT_ERR_SHAPE, "D = %d is not divisible by H = %d", p->D, p->H);
   const int dh = p->D / p->H;
-  if (dh % 32 != 0 || dh > 128)
-    return fail(BCMT_ERR_SHAPE, "head width D/H = %d must be a multiple of 32 and <= 128", dh);
+  if (dh % 8 != 0 || dh > 128)
+    return fail(BCMT_ERR_SHAPE, "head width D/H = %d must be a multiple of 8 and <= 128", dh);
   if (p->L > 1024) return fail(BCMT_ERR_UNSUPPORTED, "block size L = %d > 1024", p->L);
   if ((long long)p->B * p->T > (1ll << 30))
     return fail(BCMT_ERR_SHAPE, "B*T = %lld tokens is too large", (long long)p->B * p->T);
@@ -258,7 +258,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 
 struct BwdWs {
   char *dU, *dH, *dHhat, *dqkv, *dPb;
-  float *dP, *dM, *dS, *ds, *dwp_part, *Drow, *part;
+  float *dP, *dM, *dS, *ds, *dwp_part, *da_part, *Drow, *part;
   size_t bytes;
 };
 
@@ -280,9 +280,10 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.da_part = reinterpret_cast<float*>(take((size_t)g.B * g.D * 4));
   } else {
     w.dU = w.dH = w.dPb = nullptr;
-    w.dP = w.dM = w.dS = w.ds = w.dwp_part = nullptr;
+    w.dP = w.dM = w.dS = w.ds = w.dwp_part = w.da_part = nullptr;
   }
   w.dHhat = take((size_t)g.n * g.D * g.es);
   w.dqkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
@@ -494,7 +495,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                           const void* w_o, const void* w_p, const void* w_m, const void* w_g,
                           const float* decay, const void* workspace, void* scratch, void* dx_or_dq,
                           void* dk, void* dv, void* dw_qkv, void* dw_o, void* dw_p, void* dw_m,
-                          void* dw_g, void* stream) {
+                          void* dw_g, float* d_decay, void* stream) {
   BCMT_TRY(check_params(p));
   Geometry g(p);
   BCMT_TRY(check_ptr(dy, "dy"));
@@ -557,7 +558,8 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
       if (e != cudaSuccess) return cuda_fail(e, "dM");
     }
     pr.begin("memory_scan_bwd");
-    e = memory_scan_bwd(lc, bw.dM, decay, w.Z, bw.dS, g.B, g.Nb, D);
+    e = memory_scan_bwd(lc, bw.dM, decay, w.Z, w.M, bw.dS, d_decay ? bw.da_part : nullptr, g.B,
+                        g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
     // Sec. 3.4 reversed: pooling scores and the dW_p partials.
@@ -582,6 +584,12 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
     prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "dW_p");
+    if (d_decay) {  // fp32, summed over the batch rows in order
+      prs.begin("reduce_rows");
+      e = reduce_rows(lcs, bw.da_part, g.B, D, 0, d_decay);
+      prs.end(nullptr);
+      if (e != cudaSuccess) return cuda_fail(e, "d_decay");
+    }
     // dH = dY + dU W_g^T + alpha dS + ds w_p
     EpiArgs ea;
     ea.out = bw.dH;
@@ -600,7 +608,8 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   } else {
     const size_t wb = (size_t)D * D * g.es;
     if ((e = fill_zero(lc, dw_m, wb)) != cudaSuccess || (e = fill_zero(lc, dw_g, wb)) != cudaSuccess ||
-        (e = fill_zero(lc, dw_p, (size_t)D * g.es)) != cudaSuccess)
+        (e = fill_zero(lc, dw_p, (size_t)D * g.es)) != cudaSuccess ||
+        (d_decay && (e = fill_zero(lc, d_decay, (size_t)D * 4)) != cudaSuccess))
       return cuda_fail(e, "zeroing HOnly gradients");
   }
   // Sec. 3.3 reversed: dHhat = dH W_O^T, dW_O = Hhat^T dH.

@@ -126,9 +126,10 @@ cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
                      void* dU, float* dP, void* dPb, int B, int T, int D, int L);
 // Backward of the memory scan: dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i, given
-// dM = dP W_m^T.
+// dM = dP W_m^T; when da_part is non-null also the decay gradient of each
+// batch row, da_part [B, D] (M is the forward's fp32 memory, read only then).
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
-                            float* dS, int B, int Nb, int D);
+                            const float* M, float* dS, float* da_part, int B, int Nb, int D);
 // Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
 // dwp_part[b*Nb+i] = sum_t ds_t H_t.
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,

@@ -148,32 +148,49 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
 // Sec. 3.5 reversed: item (x, b): channels 256x .. 256x+255.  With dM = dP W_m^T,
 // the reverse decayed scan of M_i = N_i / Z_i,
 //   R_i = dM_i / Z_i + a R_{i+1},  dS_i = R_i  (= sum_{i'>=i} a^(i'-i) dM_i' / Z_i').
+// When da_part is non-null the same pass also differentiates the decay (the
+// learned per-channel decay the paper names as future work, Sec. 5): with the
+// adjoint of Z, Q_i = -dM_i M_i / Z_i + a Q_{i+1}, and N_{i-1} = M_{i-1} Z_{i-1},
+//   d a = sum_{i>=1} (R_i N_{i-1} + Q_i Z_{i-1}) = sum_{i>=1} Z_{i-1} (R_i M_{i-1} + Q_i),
+// written per batch row (da_part[b, c]) and summed over b by the caller.
 __device__ void scan_bwd_item(const float* dM, const float* __restrict__ decay,
-                              const float* __restrict__ Z, float* dS, int Nb, int D,
-                              int x, int b) {
+                              const float* __restrict__ Z, const float* __restrict__ M,
+                              float* dS, float* __restrict__ da_part, int Nb, int D, int x,
+                              int b) {
   const int c = x * kThreads + threadIdx.x;
   if (c >= D) return;
   const float a = decay[c];
   const long base = (long)b * Nb * D + c;
-  float R = 0.f;
+  float R = 0.f, Qz = 0.f, da = 0.f;
   constexpr int U = 8;
   for (int i1 = Nb; i1 > 0; i1 -= U) {
-    float mv[U], zv[U];
+    float mv[U], zv[U], mi[U], mp[U], zp[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int i = i1 - 1 - u;
       mv[u] = (i >= 0) ? __ldcg(dM + base + (long)i * D) : 0.f;
       zv[u] = (i >= 0) ? Z[(long)i * D + c] : 1.f;
+      if (da_part) {
+        mi[u] = (i >= 0) ? M[base + (long)i * D] : 0.f;
+        mp[u] = (i >= 1) ? M[base + (long)(i - 1) * D] : 0.f;
+        zp[u] = (i >= 1) ? Z[(long)(i - 1) * D + c] : 0.f;
+      }
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int i = i1 - 1 - u;
       if (i >= 0) {
-        R = fmaf(a, R, mv[u] / zv[u]);
+        const float g = mv[u] / zv[u];
+        R = fmaf(a, R, g);
         dS[base + (long)i * D] = R;
+        if (da_part) {
+          Qz = fmaf(a, Qz, -g * mi[u]);
+          da = fmaf(zp[u], fmaf(R, mp[u], Qz), da);
+        }
       }
     }
   }
+  if (da_part) da_part[(long)b * D + c] = da;
 }
 
 // Sec. 3.4 reversed: item (i, b).  With S_i = sum_t alpha_t H_t and
@@ -320,9 +337,10 @@ __global__ void __launch_bounds__(kThreads)
 
 __global__ void __launch_bounds__(kThreads)
     memory_scan_bwd_kernel(const float* __restrict__ dM, const float* __restrict__ decay,
-                           const float* __restrict__ Z, float* __restrict__ dS, int Nb, int D) {
+                           const float* __restrict__ Z, const float* __restrict__ M,
+                           float* __restrict__ dS, float* __restrict__ da_part, int Nb, int D) {
   pdl_enter();
-  scan_bwd_item(dM, decay, Z, dS, Nb, D, blockIdx.x, blockIdx.y);
+  scan_bwd_item(dM, decay, Z, M, dS, da_part, Nb, D, blockIdx.x, blockIdx.y);
 }
 
 template <class T>
@@ -387,10 +405,10 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 }
 
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
-                            float* dS, int B, int Nb, int D) {
+                            const float* M, float* dS, float* da_part, int B, int Nb, int D) {
   dim3 grid((D + kThreads - 1) / kThreads, B);
   cudaError_t e = launch_k(memory_scan_bwd_kernel, grid, dim3(kThreads), 0, lc.stream, dM, decay,
-                           Z, dS, Nb, D);
+                           Z, M, dS, da_part, Nb, D);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 

@@ -42,8 +42,10 @@ def forward(p, t: Dict[str, torch.Tensor], stream=None, workspace: Optional[torc
 
 
 def backward(p, t: Dict[str, torch.Tensor], workspace: torch.Tensor, dy: torch.Tensor, stream=None,
-             scratch: Optional[torch.Tensor] = None, out: Optional[Dict[str, torch.Tensor]] = None):
-    """Runs bcmt_backward; returns a dict of gradients (dx or dq/dk/dv, dw_*)."""
+             scratch: Optional[torch.Tensor] = None, out: Optional[Dict[str, torch.Tensor]] = None,
+             decay_grad: bool = False):
+    """Runs bcmt_backward; returns a dict of gradients (dx or dq/dk/dv, dw_*, and
+    d_decay when ``decay_grad``)."""
     dev = dy.device
     if scratch is None:
         scratch = _buffer(C.bcmt_scratch_size(p), dev)
@@ -56,18 +58,21 @@ def backward(p, t: Dict[str, torch.Tensor], workspace: torch.Tensor, dy: torch.T
             g.setdefault(n, torch.empty_like(t[n[1]]))
     for n in ("w_o", "w_p", "w_m", "w_g"):
         g.setdefault("d" + n, torch.empty_like(t[n]))
+    if decay_grad:
+        g.setdefault("d_decay", torch.empty_like(t["decay"]))
     C.bcmt_backward(p, dy, t["x"] if p.input_is_x else t["q"],
                     None if p.input_is_x else t["k"], None if p.input_is_x else t["v"],
                     t.get("w_qkv") if p.input_is_x else None, t["w_o"], t["w_p"], t["w_m"],
                     t["w_g"], t["decay"], workspace, scratch,
                     g["dx"] if p.input_is_x else g["dq"], None if p.input_is_x else g["dk"],
                     None if p.input_is_x else g["dv"], g.get("dw_qkv"), g["dw_o"], g["dw_p"],
-                    g["dw_m"], g["dw_g"], stream)
+                    g["dw_m"], g["dw_g"], stream, g.get("d_decay"))
     return g
 
 
 class BCMTMixer(torch.autograd.Function):
-    """y = BCMT(x) with the weights as differentiable inputs (x-entry layer)."""
+    """y = BCMT(x) with the weights as differentiable inputs (x-entry layer).
+    The decay gets a gradient only when it requires one (learned decay)."""
 
     @staticmethod
     def forward(ctx, x, w_qkv, w_o, w_p, w_m, w_g, decay, L: int, H: int, honly: bool = False):
@@ -87,5 +92,6 @@ class BCMTMixer(torch.autograd.Function):
     def backward(ctx, dy):
         x, w_qkv, w_o, w_p, w_m, w_g, decay, ws = ctx.saved_tensors
         t = dict(x=x, w_qkv=w_qkv, w_o=w_o, w_p=w_p, w_m=w_m, w_g=w_g, decay=decay)
-        g = backward(ctx.p, t, ws, dy.contiguous())
-        return g["dx"], g["dw_qkv"], g["dw_o"], g["dw_p"], g["dw_m"], g["dw_g"], None, None, None, None
+        g = backward(ctx.p, t, ws, dy.contiguous(), decay_grad=ctx.needs_input_grad[6])
+        return (g["dx"], g["dw_qkv"], g["dw_o"], g["dw_p"], g["dw_m"], g["dw_g"], g.get("d_decay"),
+                None, None, None)

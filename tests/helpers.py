@@ -14,8 +14,8 @@ from paper_2608_13578_gb300.inputs import Workload, as_float64, make_inputs
 FP32_ABS = 1e-4
 BF16_REL = 2e-2
 
-GRAD_NAMES_X = ("dx", "dw_qkv", "dw_o", "dw_p", "dw_m", "dw_g")
-GRAD_NAMES_QKV = ("dq", "dk", "dv", "dw_o", "dw_p", "dw_m", "dw_g")
+GRAD_NAMES_X = ("dx", "dw_qkv", "dw_o", "dw_p", "dw_m", "dw_g", "d_decay")
+GRAD_NAMES_QKV = ("dq", "dk", "dv", "dw_o", "dw_p", "dw_m", "dw_g", "d_decay")
 
 
 def errors(gpu: torch.Tensor, ref: np.ndarray):
@@ -59,6 +59,6 @@ def gpu_run(w: Workload, t_dev: dict, backward: bool = True):
     p = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype, w.input_is_x, w.honly,
                          flags=layer.C.BCMT_FLAG_CHECK)
     y, ws = layer.forward(p, t_dev)
-    g = layer.backward(p, t_dev, ws, t_dev["dy"]) if backward else None
+    g = layer.backward(p, t_dev, ws, t_dev["dy"], decay_grad=True) if backward else None
     torch.cuda.synchronize()
     return y, g

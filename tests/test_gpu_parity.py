@@ -35,6 +35,8 @@ SMALL = [
     W(1, 300, 128, 2, 256, "bf16"),
     W(2, 150, 128, 2, 48, "bf16"),
     W(1, 96, 192, 2, 32, "bf16"),                       # dh = 96 -> SIMT attention
+    W(2, 300, 128, 8, 64, "bf16"),                      # dh = 16 (the paper's D128 h8)
+    W(1, 200, 128, 8, 32, "fp32"),
     W(2, 256, 128, 2, 64, "bf16", decay=(0.0, 0.0)),
 ]
 VARIANTS = [
@@ -61,7 +63,7 @@ def _check(w: Workload, backward=True, batch=None):
                     got = got[batch]
                 else:
                     continue
-            if w.honly and n in ("dw_p", "dw_m", "dw_g"):
+            if w.honly and n in ("dw_p", "dw_m", "dw_g", "d_decay"):
                 assert torch.count_nonzero(got).item() == 0
                 continue
             assert_close(n, got, gr[n], w.dtype)

@@ -32,6 +32,8 @@ MUTATIONS = {
     "bwd: reverse scan divides by Z_j": ("dS[j] += (a ** (i - j)) * dM[i] / Z[i]", "dS[j] += (a ** (i - j)) * dM[i] / Z[j]"),
     "bwd: shift not reversed": ("dP[i] = dC[i + 1]", "dP[i] = dC[i]"),
     "bwd: dK with untransposed scores": ("dK[b, t0:t1, cols] = dScore.T @ Qb", "dK[b, t0:t1, cols] = dScore @ Qb"),
+    "bwd: decay gradient without the denominator term": ("d_decay += dM[i] * (dnum - M[b, i] * dden) / Z[i]", "d_decay += dM[i] * dnum / Z[i]"),
+    "bwd: decay gradient exponent": ("w = (i - j) * a ** (i - j - 1)", "w = (i - j) * a ** (i - j)"),
     "bwd: gate derivative": ("dU[t0:t1] = dG * G[b, t0:t1] * (1.0 - G[b, t0:t1])", "dU[t0:t1] = dG * G[b, t0:t1]"),
 }
 

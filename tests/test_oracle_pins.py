@@ -258,7 +258,7 @@ def _fd_check(p, L, H, names, honly=False, qkv=None, eps=1e-6):
             lm = _loss(p, dY, L, H, honly, qkv)
             arr[idx] = old
             fd[idx] = (lp - lm) / (2 * eps)
-        g = gr["d" + n]
+        g = gr["d_decay" if n == "decay" else "d" + n]
         err = np.max(np.abs(g - fd)) / max(1e-12, np.max(np.abs(fd)))
         assert err < 1e-6, (n, err)
 
@@ -268,7 +268,7 @@ def test_backward_finite_differences():
     (ragged last block, per-channel decay including a = 0, two heads)."""
     p = rand_problem(B=2, T=10, D=8, H=2, seed=14)
     p["decay"][1] = 0.0
-    _fd_check(p, 4, 2, ["x", "w_qkv", "w_o", "w_p", "w_m", "w_g"])
+    _fd_check(p, 4, 2, ["x", "w_qkv", "w_o", "w_p", "w_m", "w_g", "decay"])
 
 
 def test_backward_finite_differences_qkv_entry():
@@ -281,7 +281,28 @@ def test_backward_finite_differences_qkv_entry():
 
 def test_backward_finite_differences_honly():
     p = rand_problem(B=1, T=6, D=4, H=1, seed=17)
-    _fd_check(p, 4, 1, ["x", "w_qkv", "w_o"], honly=True)
+    _fd_check(p, 4, 1, ["x", "w_qkv", "w_o", "decay"], honly=True)
+
+
+def test_decay_gradient_two_blocks_closed_form():
+    """Two blocks: M_1 = (a S_0 + S_1) / (1 + a), so dM_1/da = (S_0 - M_1) / (1 + a)
+    and d_decay = sum_b dM_1 * (S_0 - M_1) / (1 + a), with dM_1 = dP_1 W_m^T where
+    dP_1 = 0 (the last block's memory feeds no block): the decay gradient of two
+    blocks is exactly zero, and with three it is the closed form through M_1."""
+    p = rand_problem(B=2, T=8, D=6, H=2, seed=31)
+    dY = np.random.default_rng(32).standard_normal((2, 8, 6))
+    gr = O.backward(run(p, 4, 2), dY)
+    np.testing.assert_array_equal(gr["d_decay"], np.zeros(6))
+    # three blocks: only M_1 and M_0 get gradient; M_0 = S_0 has no decay
+    fw = run(p, 3, 2)   # T = 8, L = 3: blocks of 3, 3, 2 tokens
+    gr = O.backward(fw, dY)
+    a = p["decay"]
+    expect = np.zeros(6)
+    for b in range(2):
+        dC2 = np.sum(dY[b, 6:8] * fw["G"][b, 6:8], axis=0)   # dP_1 = dC_2
+        dM1 = dC2 @ p["w_m"].T
+        expect += dM1 * (fw["S"][b, 0] - fw["M"][b, 1]) / (1.0 + a)
+    np.testing.assert_allclose(gr["d_decay"], expect, rtol=1e-12, atol=1e-14)
 
 
 def test_block_never_sees_its_own_summary():
