@@ -137,6 +137,33 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                           void* dw_o, void* dw_p, void* dw_m, void* dw_g, float* d_decay,
                           void* stream);
 
+/* Incremental decoding (one new token per sequence per call).  The paper
+ * trains only; decoding follows from the causal structure of Sec. 3.3-3.8:
+ * token t of block i = t / L attends to the earlier tokens of its block, and
+ * Y_t = H_t + sigmoid(H_t W_g) * C_i with C_i = M_{i-1} W_m (zero in block 0).
+ * The state carries the current block's K/V cache, the block summary
+ * accumulated online (Sec. 3.4), the memory recurrence N_i = a N_{i-1} + S_i,
+ * Z_i = a Z_{i-1} + 1 (Sec. 3.5) and the current memory row.  Decoding the
+ * tokens 0..T-1 of a sequence in order gives the rows of bcmt_forward's Y.
+ *
+ * p: B sequences decoded in lockstep, D, H, L, dtype and flags as for the
+ * forward (BCMT_FLAG_HONLY: Y = H); input_is_x must be 1; p->T is ignored.
+ *   state  bcmt_decode_state_size(p) bytes of device memory, caller-owned;
+ *          bcmt_decode_reset zeroes it to start new sequences
+ *   pos    position t of the token being decoded (0, 1, 2, ... in order; the
+ *          state assumes the previous call decoded pos - 1)
+ *   x_t    [B, D] the token's input row per sequence
+ *   weights and decay as for bcmt_forward (x-entry: w_qkv [D, 3D])
+ *   y_t    [B, D] output row, written
+ * Calls are asynchronous on `stream`; consecutive steps of one state must be
+ * issued in order on one stream. */
+size_t bcmt_decode_state_size(const bcmt_params* p);
+bcmt_status bcmt_decode_reset(const bcmt_params* p, void* state, void* stream);
+bcmt_status bcmt_decode_step(const bcmt_params* p, void* state, long pos, const void* x_t,
+                             const void* w_qkv, const void* w_o, const void* w_p,
+                             const void* w_m, const void* w_g, const float* decay, void* y_t,
+                             void* stream);
+
 /* Allocation-free backward of the intra-block attention alone (the SIMT
  * kernels of the layer's backward; the paper has no counterpart -- it is an
  * interface for callers that cannot call cudaMalloc, such as a host framework

@@ -72,6 +72,12 @@ def _load():
     lib.bcmt_profile_read.restype = ctypes.c_int
     lib.bcmt_profile_reset.argtypes = []
     lib.bcmt_profile_reset.restype = None
+    lib.bcmt_decode_state_size.argtypes = [_P]
+    lib.bcmt_decode_state_size.restype = ctypes.c_size_t
+    lib.bcmt_decode_reset.argtypes = [_P, _VP, _VP]
+    lib.bcmt_decode_reset.restype = ctypes.c_int
+    lib.bcmt_decode_step.argtypes = [_P, _VP, ctypes.c_long] + [_VP] * 9
+    lib.bcmt_decode_step.restype = ctypes.c_int
     lib.bcmt_attention_backward_noalloc.argtypes = [_P, _VP, _VP, _VP, ctypes.c_long, _VP, _VP,
                                                     _VP, _VP, _VP, _VP, ctypes.c_long, _VP]
     lib.bcmt_attention_backward_noalloc.restype = ctypes.c_int
@@ -93,6 +99,7 @@ LIB = _load()
 EXPORTED = ("bcmt_workspace_size", "bcmt_scratch_size", "bcmt_forward", "bcmt_backward",
             "bcmt_device_status", "bcmt_last_error", "bcmt_profile_read", "bcmt_profile_reset",
             "bcmt_attention_backward_noalloc",
+            "bcmt_decode_state_size", "bcmt_decode_reset", "bcmt_decode_step",
             "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_attn")
 
 
@@ -150,6 +157,21 @@ def bcmt_backward(p: bcmt_params, dy, x_or_q, k, v, w_qkv, w_o, w_p, w_m, w_g, d
 
 def bcmt_device_status(stream=None) -> None:
     _check(LIB.bcmt_device_status(_stream(stream)))
+
+
+def bcmt_decode_state_size(p: bcmt_params) -> int:
+    return LIB.bcmt_decode_state_size(ctypes.byref(p))
+
+
+def bcmt_decode_reset(p: bcmt_params, state, stream=None) -> None:
+    _check(LIB.bcmt_decode_reset(ctypes.byref(p), _ptr(state), _stream(stream)))
+
+
+def bcmt_decode_step(p: bcmt_params, state, pos: int, x_t, w_qkv, w_o, w_p, w_m, w_g, decay, y_t,
+                     stream=None) -> None:
+    _check(LIB.bcmt_decode_step(ctypes.byref(p), _ptr(state), pos, _ptr(x_t), _ptr(w_qkv),
+                                _ptr(w_o), _ptr(w_p), _ptr(w_m), _ptr(w_g), _ptr(decay),
+                                _ptr(y_t), _stream(stream)))
 
 
 def bcmt_attention_backward_noalloc(p: bcmt_params, q, k, v, ld, o, lse, dO, dq, dk, dv, ld_d,

@@ -679,6 +679,102 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   return finish(p, s);
 }
 
+// ------------------------------------------------------------------ decoding
+namespace {
+DecodeState decode_layout(const Geometry& g, void* base, size_t* bytes) {
+  DecodeState st;
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    char* r = p ? p + off : nullptr;
+    off += al256(n);
+    return r;
+  };
+  auto f32 = [&](size_t n) { return reinterpret_cast<float*>(take(n * 4)); };
+  const size_t bd = (size_t)g.B * g.D;
+  st.Kc = take((size_t)g.B * g.L * g.D * g.es);
+  st.Vc = take((size_t)g.B * g.L * g.D * g.es);
+  st.xf = f32(bd);
+  st.qkv = f32(3 * bd);
+  st.hhat = f32(bd);
+  st.H = f32(bd);
+  st.U = f32(bd);
+  st.pm = f32(g.B);
+  st.pden = f32(g.B);
+  st.pnum = f32(bd);
+  st.N = f32(bd);
+  st.Z = f32(bd);
+  st.C = f32(bd);
+  st.Mr = f32(bd);
+  *bytes = off;
+  return st;
+}
+}  // namespace
+
+size_t bcmt_decode_state_size(const bcmt_params* p) {
+  if (check_params(p) != BCMT_OK) return 0;
+  Geometry g(p);
+  size_t bytes = 0;
+  decode_layout(g, nullptr, &bytes);
+  return bytes;
+}
+
+bcmt_status bcmt_decode_reset(const bcmt_params* p, void* state, void* stream) {
+  BCMT_TRY(check_params(p));
+  BCMT_TRY(check_ptr(state, "state"));
+  const size_t bytes = bcmt_decode_state_size(p);
+  cudaError_t e = cudaMemsetAsync(state, 0, bytes, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "decode state reset");
+  return finish(p, static_cast<cudaStream_t>(stream));
+}
+
+bcmt_status bcmt_decode_step(const bcmt_params* p, void* state, long pos, const void* x_t,
+                             const void* w_qkv, const void* w_o, const void* w_p,
+                             const void* w_m, const void* w_g, const float* decay, void* y_t,
+                             void* stream) {
+  BCMT_TRY(check_params(p));
+  if (!p->input_is_x)
+    return fail(BCMT_ERR_ARG, "decoding starts from the token rows x (input_is_x must be 1)");
+  if (pos < 0) return fail(BCMT_ERR_ARG, "pos = %ld must be >= 0", pos);
+  Geometry g(p);
+  BCMT_TRY(check_ptr(state, "state"));
+  BCMT_TRY(check_ptr(x_t, "x_t"));
+  BCMT_TRY(check_ptr(w_qkv, "w_qkv"));
+  BCMT_TRY(check_ptr(w_o, "w_o"));
+  BCMT_TRY(check_ptr(y_t, "y_t"));
+  if (!g.honly) {
+    BCMT_TRY(check_ptr(w_p, "w_p"));
+    BCMT_TRY(check_ptr(w_m, "w_m"));
+    BCMT_TRY(check_ptr(w_g, "w_g"));
+    BCMT_TRY(check_ptr(decay, "decay"));
+  }
+  unsigned* sp = status_ptr();
+  if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
+  Launch lc{static_cast<cudaStream_t>(stream), sp};
+  size_t bytes = 0;
+  DecodeArgs a;
+  a.s = decode_layout(g, state, &bytes);
+  a.B = g.B;
+  a.D = g.D;
+  a.H = g.H;
+  a.dh = g.dh;
+  a.L = g.L;
+  a.j = (int)(pos % g.L);
+  a.honly = g.honly;
+  a.x = a.s.xf;
+  a.w_qkv = w_qkv;
+  a.w_o = w_o;
+  a.w_p = w_p;
+  a.w_m = w_m;
+  a.w_g = w_g;
+  a.decay = decay;
+  a.y = y_t;
+  cudaError_t e = decode_widen(lc, g.dtype, x_t, a.s.xf, (long)g.B * g.D);
+  if (e == cudaSuccess) e = decode_step(lc, g.dtype, a);
+  if (e != cudaSuccess) return cuda_fail(e, "decode step");
+  return finish(p, lc.stream);
+}
+
 bcmt_status bcmt_attention_backward_noalloc(const bcmt_params* p, const void* q, const void* k,
                                             const void* v, long ld, const void* o,
                                             const float* lse, const void* dO, void* dq, void* dk,

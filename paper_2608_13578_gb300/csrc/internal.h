@@ -139,4 +139,30 @@ cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, i
                         void* out);
 cudaError_t fill_zero(const Launch& lc, void* p, size_t bytes);
 
+// ---------------------------------------------------------- decoding
+// The per-layer decoding state (caller-owned device memory, zeroed by
+// bcmt_decode_reset): the current block's K/V cache in the storage dtype, the
+// online block summary, the memory recurrence and the current memory row, and
+// the step's fp32 temporaries.
+struct DecodeState {
+  void *Kc, *Vc;                    // [B, L, D] storage dtype
+  float *xf, *qkv, *hhat, *H, *U;   // step temporaries: [B, D], [B, 3D], [B, D] x3
+  float *pm, *pden;                 // [B]: running max and denominator of the block's scores
+  float *pnum;                      // [B, D]: running numerator sum exp(s - m) H
+  float *N, *Z;                     // [B, D]: N_i, Z_i of the last completed block
+  float *C;                         // [B, D]: memory row of the current block
+  float *Mr;                        // [B, D]: M_i rounded to the storage dtype
+};
+struct DecodeArgs {
+  int B, D, H, dh, L, j;  // j = slot of the token in its block
+  bool honly;
+  const float* x;         // the token's input rows, fp32 [B, D]
+  const void *w_qkv, *w_o, *w_p, *w_m, *w_g;
+  const float* decay;
+  void* y;                // [B, D] storage dtype
+  DecodeState s;
+};
+cudaError_t decode_widen(const Launch& lc, int dtype, const void* x, float* out, long n);
+cudaError_t decode_step(const Launch& lc, int dtype, const DecodeArgs& a);
+
 }  // namespace bcmt

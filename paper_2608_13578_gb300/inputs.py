@@ -63,7 +63,7 @@ def _wl(name, B, T, D, H, L, dtype="bf16", backward=True, decay=(0.8, 0.8)):
                     backward=backward, decay=decay)
 
 
-# The five problem families the benchmark and the parity tests use.  Sizes and
+# The problem families the benchmark and the parity tests use.  Sizes and
 # value distributions mirror the paper's language-modelling runs (context up to
 # 1024 tokens, Sec. 4.1) plus longer block-size and sequence-length sweeps.
 WORKLOADS: Dict[str, Workload] = {}
@@ -75,6 +75,10 @@ for _w in [
       for L in (32, 64, 128, 256)],
     *[_wl(f"seqscale_bf16_b4_t{T}_l128_d1024_h16", 4, T, 1024, 16, 128,
           decay=(0.9, 0.999)) for T in (2048, 4096, 8192, 16384)],
+    # one layer of the paper's own model shape (Sec. 4.1: D 128, 8 heads of 16,
+    # batch 16, context 1024), block sizes of its Table 2
+    *[_wl(f"paper_bf16_b16_t1024_l{L}_d128_h8", 16, 1024, 128, 8, L)
+      for L in (64, 128, 256, 512)],
 ]:
     WORKLOADS[_w.name] = _w
 

@@ -95,3 +95,31 @@ class BCMTMixer(torch.autograd.Function):
         g = backward(ctx.p, t, ws, dy.contiguous(), decay_grad=ctx.needs_input_grad[6])
         return (g["dx"], g["dw_qkv"], g["dw_o"], g["dw_p"], g["dw_m"], g["dw_g"], g.get("d_decay"),
                 None, None, None)
+
+
+class Decoder:
+    """Incremental decoding of B sequences in lockstep through one BCMT layer
+    (``bcmt_decode_step``): ``step(x_t)`` takes the next token's input rows
+    [B, D] and returns the layer's output rows [B, D]."""
+
+    def __init__(self, weights: Dict[str, torch.Tensor], B: int, H: int, L: int,
+                 honly: bool = False):
+        D = weights["w_o"].shape[0]
+        dt = "bf16" if weights["w_o"].dtype == torch.bfloat16 else "fp32"
+        self.p = params_for(B, 1, D, H, L, dt, True, honly)
+        self.w = weights
+        self.state = _buffer(C.bcmt_decode_state_size(self.p), weights["w_o"].device)
+        self.reset()
+
+    def reset(self):
+        C.bcmt_decode_reset(self.p, self.state)
+        self.pos = 0
+
+    def step(self, x_t: torch.Tensor, stream=None) -> torch.Tensor:
+        w = self.w
+        x_t = x_t.contiguous()
+        y = torch.empty(x_t.shape, dtype=x_t.dtype, device=x_t.device)
+        C.bcmt_decode_step(self.p, self.state, self.pos, x_t, w["w_qkv"], w["w_o"],
+                           w.get("w_p"), w.get("w_m"), w.get("w_g"), w.get("decay"), y, stream)
+        self.pos += 1
+        return y
