@@ -1,0 +1,665 @@
+// Intra-block causal attention on the tcgen05 tensor cores (Sec. 3.3) for the
+// shapes the single-tile kernels of attn_tc.cu do not take: head widths
+// DH in {16, 32, 64} and block sizes L that divide 128 or are multiples of 128
+// (up to 1024), bf16 operands.
+//
+// A CTA owns a 128-token tile of one head and walks the key tiles its rows
+// can see: for L >= 128 the tiles of its block from the block start up to the
+// diagonal tile, for L < 128 the diagonal tile alone (whose mask is then
+// block-diagonal).  Q/K/V/dO tiles are [128 tokens x DH] slices brought in by
+// TMA with the swizzle whose span is one row (DH * 2 bytes: 32, 64 or 128),
+// so every operand is a canonical swizzled layout the MMA reads K-major or
+// MN-major.  Scores and products accumulate in TMEM.
+//
+//  * forward: per key tile S = Q K^T (N = 128), online softmax with the
+//    thread owning one query row (running max and sum in registers), P in
+//    bf16 to shared memory, P V into TMEM, O rescaled and accumulated in
+//    registers; O and the log-sum-exp are stored at the end.
+//  * backward, two kernels (no atomics, fixed summation order):
+//      dQ:  per query tile, Drow = dO . O, then per key tile and 64-key half
+//           S, dP (N = 64), dS = P (dP - Drow) scale, dQ += dS K (TMEM);
+//      dKV: per key tile, per query tile and 64-query half S^T = K Q^T,
+//           dP^T = V dO^T, dV += P^T dO, dK += dS^T Q (TMEM), with the query
+//           tile's log-sum-exp and Drow staged in shared memory.
+#include "attn_common.cuh"
+#include "common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+#include "tmap.h"
+
+namespace bcmt {
+using namespace attn;
+
+namespace {
+constexpr int kTile = 128;
+
+template <int DH>
+struct Geo {
+  static constexpr uint32_t span = DH * 2;                    // bytes per tile row
+  static constexpr uint32_t tile = kTile * span;              // one 128-row tile
+  static constexpr uint32_t sbo = 8 * span;                   // 8-row atom
+  static constexpr uint32_t layout = DH == 64 ? 2u : DH == 32 ? 4u : 6u;
+  // K-major [rows x DH] operand at row offset `row0`, K step kk (16 columns)
+  static __device__ __forceinline__ uint64_t kmaj(const uint8_t* t, int row0, int kk) {
+    return tc::sdesc_sw(tc::smem_u32(t) + row0 * span + kk * 32, 16, sbo, layout);
+  }
+  // the same tile read MN-major (DH contiguous = N), K = rows from row0, step kk
+  static __device__ __forceinline__ uint64_t mnmaj(const uint8_t* t, int row0, int kk) {
+    return tc::sdesc_sw(tc::smem_u32(t) + (row0 + kk * 16) * span, tile, sbo, layout);
+  }
+};
+
+// A [128 x 128] bf16 operand in two 64-column swizzle-128 halves (put_unit's
+// layout), read K-major from column 64*half, K step kk.  A single 64-column
+// half buffer is read with half = 0 and kk < 4.
+__device__ __forceinline__ uint64_t p_kmaj(const uint8_t* p, int half, int kk) {
+  return tc::sdesc(tc::smem_u32(p) + half * 16384 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+}
+
+// Loads TMEM columns col .. col+DH-1 of the warp's lane quarter (thread = row).
+template <int DH>
+__device__ __forceinline__ void tmem_row(uint32_t taddr, float* v) {
+  uint32_t r[2][32];
+  tc::tmem_ld32_issue(taddr, r[0]);
+  if (DH > 32) tc::tmem_ld32_issue(taddr + 32u, r[1]);
+  tc::tmem_wait();
+#pragma unroll
+  for (int c = 0; c < DH; ++c) v[c] = __uint_as_float(r[c >> 5][c & 31]);
+}
+
+template <int DH>
+__device__ __forceinline__ void store_row(bf16* dst, const float* v, float mul) {
+#pragma unroll
+  for (int u = 0; u < DH / 8; ++u) {
+    float t[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) t[e] = v[8 * u + e] * mul;
+    *reinterpret_cast<uint4*>(dst + 8 * u) = pack8(t);
+  }
+}
+
+// First key of the key-tile walk of the query tile at t0, and the tile count.
+__device__ __forceinline__ void key_walk(int t0, int L, int& kstart, int& nkt) {
+  kstart = L >= kTile ? (t0 / L) * L : t0;
+  nkt = (t0 - kstart) / kTile + 1;
+}
+}  // namespace
+
+// ====================================================================== forward
+template <int DH>
+__global__ void __launch_bounds__(128)
+    attn_fwd_fl_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
+                       const __grid_constant__ CUtensorMap mV, bf16* __restrict__ O, long ld_o,
+                       float* __restrict__ lse, int Tlen, int H, int L, float scale,
+                       unsigned* status) {
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sP = smem;                       // 32 KB: P [128 queries x 128 keys]
+  uint8_t* sQ = smem + 32768;
+  uint8_t* sK = sQ + G::tile;
+  uint8_t* sV = sK + G::tile;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);  // kv, s, o
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  int kstart, nkt;
+  key_walk(t0, L, kstart, nkt);
+
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 3 * G::tile);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart, b);
+  }
+  __syncwarp();
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, 256);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  const int r = warp * 32 + lane;
+  const float sl2 = scale * kLog2e;
+  float m = -INFINITY, l = 0.f;
+  float oacc[DH];
+#pragma unroll
+  for (int c = 0; c < DH; ++c) oacc[c] = 0.f;
+  bool ok = true;
+
+  for (int kt = 0; kt < nkt; ++kt) {
+    const bool diag = kt == nkt - 1;
+    if (tid == 0) {
+      const bool okk = tc::mbar_wait(&bar[0], kt & 1, status);
+      tc::fence_after_sync();
+      if (okk) {
+        constexpr uint32_t idS = tc::idesc_bf16(128, 128, 0, 0);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk)
+          tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 0, kk), idS, kk > 0 ? 1u : 0u);
+      }
+      tc::mma_commit(&bar[1]);
+    }
+    __syncwarp();
+    ok = tc::mbar_wait(&bar[1], kt & 1, status) && ok;
+    tc::fence_after_sync();
+
+    // ---- online softmax of this key tile (thread = query row r)
+    int wbs = 0, nld = 4, rbs = 0;
+    if (diag) {
+      if (L < kTile) {
+        wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;
+        rbs = (r / L) * L;
+      }
+      nld = chunks_needed(warp, wbs);
+    }
+    uint32_t sr[4][32];
+#pragma unroll
+    for (int ci = 0; ci < 4; ++ci)
+      if (ci < nld) tc::tmem_ld32_issue(trow + (uint32_t)(wbs + ci * 32), sr[ci]);
+    tc::tmem_wait();
+    float mt = -INFINITY;
+#pragma unroll
+    for (int ci = 0; ci < 4; ++ci)
+      if (ci < nld) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int kk = wbs + ci * 32 + j;
+          if (!diag || (kk >= rbs && kk <= r)) mt = fmaxf(mt, __uint_as_float(sr[ci][j]));
+        }
+      }
+    const float m_new = fmaxf(m, mt * sl2);
+    const float alpha = exp2f(m - m_new);  // 0 on the first tile (m = -inf)
+    float psum = 0.f;
+#pragma unroll
+    for (int ci = 0; ci < 4; ++ci)
+      if (ci < nld) {
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int kk = wbs + ci * 32 + j;
+          const bool valid = !diag || (kk >= rbs && kk <= r);
+          const float p = valid ? exp2f(__uint_as_float(sr[ci][j]) * sl2 - m_new) : 0.f;
+          v[j] = p;
+          psum += p;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) put_unit(sP, r, (wbs + ci * 32) / 8 + u, pack8(v + 8 * u));
+      }
+    const uint4 zero = make_uint4(0, 0, 0, 0);
+    for (int u = 0; u < 16; ++u)
+      if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
+    l = l * alpha + psum;
+    m = m_new;
+    tc::fence_proxy_async_smem();
+    tc::fence_before_sync();
+    __syncthreads();
+
+    if (tid == 0) {
+      tc::fence_after_sync();
+      constexpr uint32_t idO = tc::idesc_bf16(128, DH, 0, 1);
+#pragma unroll
+      for (int kk = 0; kk < kTile / 16; ++kk)
+        tc::mma_bf16(tmem + 128, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
+      tc::mma_commit(&bar[2]);
+    }
+    __syncwarp();
+    ok = tc::mbar_wait(&bar[2], kt & 1, status) && ok;
+    tc::fence_after_sync();
+    // K, V and P are free: fetch the next key tile while this one's P V is
+    // folded into the accumulator
+    if (tid == 0 && kt + 1 < nkt) {
+      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
+      tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+    }
+    float o[DH];
+    tmem_row<DH>(trow + 128u, o);
+#pragma unroll
+    for (int c = 0; c < DH; ++c) oacc[c] = fmaf(oacc[c], alpha, o[c]);
+  }
+
+  const int t = t0 + r;
+  if (ok && t < Tlen) {
+    store_row<DH>(O + ((long)b * Tlen + t) * ld_o + h * DH, oacc, 1.0f / l);
+    lse[((long)b * H + h) * Tlen + t] = m * kLn2 + logf(l);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+}
+
+// ================================================================ backward: dQ
+template <int DH>
+__global__ void __launch_bounds__(128)
+    attn_bwd_dq_fl_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
+                          const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
+                          const bf16* __restrict__ O, const bf16* __restrict__ dO, long ld_o,
+                          const float* __restrict__ lse, float* __restrict__ Drow,
+                          bf16* __restrict__ dQ, long ld_d, int Tlen, int H, int L, float scale,
+                          unsigned* status) {
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sdS = smem;                      // 16 KB: scale * dS, one 64-key half
+  uint8_t* sQ = smem + 16384;
+  uint8_t* sdO = sQ + G::tile;
+  uint8_t* sK = sdO + G::tile;
+  uint8_t* sV = sK + G::tile;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);  // kv, s, q
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  int kstart, nkt;
+  key_walk(t0, L, kstart, nkt);
+
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+    tc::prefetch_tmap(&mdO);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * G::tile);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart, b);
+  }
+  __syncwarp();
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, 256);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  // Drow_t = dO_t . O_t and the row's log-sum-exp (global rows)
+  const int r = warp * 32 + lane;
+  const int t = t0 + r;
+  const bool row_ok = t < Tlen;
+  float drow = 0.f, lse2 = 0.f;
+  if (row_ok) {
+    const bf16* orow = O + ((long)b * Tlen + t) * ld_o + h * DH;
+    const bf16* grow = dO + ((long)b * Tlen + t) * ld_o + h * DH;
+#pragma unroll
+    for (int u = 0; u < DH / 8; ++u) {
+      float ov[8], gv[8];
+      load8(orow + 8 * u, ov);
+      load8(grow + 8 * u, gv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) drow = fmaf(ov[e], gv[e], drow);
+    }
+    const long li = ((long)b * H + h) * Tlen + t;
+    Drow[li] = drow;
+    lse2 = lse[li] * kLog2e;
+  }
+  const float sl2 = scale * kLog2e;
+  const int rbs = L < kTile ? (r / L) * L : 0;
+  bool ok = true;
+  int ns = 0, nq = 0;  // commits to bar[1] and bar[2] so far
+
+  for (int kt = 0; kt < nkt; ++kt) {
+    const bool diag = kt == nkt - 1;
+    if (tid == 0) {
+      ok = tc::mbar_wait(&bar[0], kt & 1, status) && ok;
+      tc::fence_after_sync();
+    }
+    for (int hh = 0; hh < 2; ++hh) {
+      if (tid == 0) {
+        if (ok) {
+          constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)  // S half -> columns 0..63
+            tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)  // dP half -> columns 64..127
+            tc::mma_bf16(tmem + 64, G::kmaj(sdO, 0, kk), G::kmaj(sV, 64 * hh, kk), id64,
+                         kk > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[1]);
+      }
+      __syncwarp();
+      ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
+      ++ns;
+      tc::fence_after_sync();
+      uint32_t rs[2][32], rd[2][32];
+      tc::tmem_ld32_issue(trow, rs[0]);
+      tc::tmem_ld32_issue(trow + 32u, rs[1]);
+      tc::tmem_ld32_issue(trow + 64u, rd[0]);
+      tc::tmem_ld32_issue(trow + 96u, rd[1]);
+      tc::tmem_wait();
+      // the previous dQ product must be done with the dS buffer it reads
+      if (nq > 0) {
+        ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+        tc::fence_after_sync();
+      }
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int kk = 64 * hh + 32 * c + j;  // key column within the tile
+          const bool valid = row_ok && (!diag || (kk >= rbs && kk <= r));
+          const float p = valid ? exp2f(__uint_as_float(rs[c][j]) * sl2 - lse2) : 0.f;
+          v[j] = p * (__uint_as_float(rd[c][j]) - drow) * scale;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) put_unit(sdS, r, 4 * c + u, pack8(v + 8 * u));
+      }
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid == 0) {
+        tc::fence_after_sync();
+        if (ok) {
+          constexpr uint32_t idQ = tc::idesc_bf16(128, DH, 0, 1);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // dQ += dS[:, 64hh..] K[64hh.., :]
+            tc::mma_bf16(tmem + 128, p_kmaj(sdS, 0, kk), G::mnmaj(sK, 64 * hh, kk), idQ,
+                         (kt > 0 || hh > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[2]);
+      }
+      ++nq;
+    }
+    // the next key tile may overwrite K and V once this tile's products are done
+    if (tid == 0 && kt + 1 < nkt) {
+      ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
+      tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+    }
+    __syncwarp();
+  }
+  ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+  tc::fence_after_sync();
+  float q[DH];
+  tmem_row<DH>(trow + 128u, q);
+  if (ok && row_ok) store_row<DH>(dQ + ((long)b * Tlen + t) * ld_d + h * DH, q, 1.0f);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+}
+
+// =============================================================== backward: dKV
+template <int DH>
+__global__ void __launch_bounds__(128)
+    attn_bwd_dkv_fl_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
+                           const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
+                           const float* __restrict__ lse, const float* __restrict__ Drow,
+                           bf16* __restrict__ dK, bf16* __restrict__ dV, long ld_d, int Tlen, int H,
+                           int L, float scale, unsigned* status) {
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sPt = smem;                      // 16 KB: P^T, one 64-query half
+  uint8_t* sdSt = smem + 16384;             // 16 KB: scale * dS^T, the same half
+  uint8_t* sK = smem + 32768;
+  uint8_t* sV = sK + G::tile;
+  uint8_t* sQ = sV + G::tile;
+  uint8_t* sdO = sQ + G::tile;
+  float* slse = reinterpret_cast<float*>(sdO + G::tile);  // [128] lse * log2(e)
+  float* sdr = slse + kTile;                               // [128] Drow
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sdr + kTile);  // kv, s, q
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int k0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  // queries that see this key tile: to the end of its block (L >= 128) or of
+  // the tile itself (L < 128, block-diagonal mask)
+  const int qend = min(L >= kTile ? (k0 / L + 1) * L : k0 + kTile, Tlen);
+  const int nqt = (qend - k0 + kTile - 1) / kTile;
+
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+    tc::prefetch_tmap(&mdO);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * G::tile);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, k0, b);
+  }
+  __syncwarp();
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, 256);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  const int r = warp * 32 + lane;  // key row
+  const int key = k0 + r;
+  const float sl2 = scale * kLog2e;
+  // L < 128: key r's block ends at its block start + L (within the tile)
+  const int kbe = L < kTile ? (r / L) * L + L : kTile;
+  bool ok = true;
+  int ns = 0, nq = 0;
+
+  for (int qt = 0; qt < nqt; ++qt) {
+    const int q0 = k0 + qt * kTile;
+    const bool diag = qt == 0;
+    {
+      const int tq = q0 + tid;
+      const long li = ((long)b * H + h) * Tlen + tq;
+      slse[tid] = tq < Tlen ? lse[li] * kLog2e : 0.f;
+      sdr[tid] = tq < Tlen ? Drow[li] : 0.f;
+    }
+    if (tid == 0) {
+      ok = tc::mbar_wait(&bar[0], qt & 1, status) && ok;
+      tc::fence_after_sync();
+    }
+    __syncthreads();  // slse / sdr written
+    for (int hh = 0; hh < 2; ++hh) {
+      if (tid == 0) {
+        if (ok) {
+          constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)  // S^T half -> columns 0..63
+            tc::mma_bf16(tmem, G::kmaj(sK, 0, kk), G::kmaj(sQ, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)  // dP^T half -> columns 64..127
+            tc::mma_bf16(tmem + 64, G::kmaj(sV, 0, kk), G::kmaj(sdO, 64 * hh, kk), id64,
+                         kk > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[1]);
+      }
+      __syncwarp();
+      ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
+      ++ns;
+      tc::fence_after_sync();
+      uint32_t rs[2][32], rd[2][32];
+      tc::tmem_ld32_issue(trow, rs[0]);
+      tc::tmem_ld32_issue(trow + 32u, rs[1]);
+      tc::tmem_ld32_issue(trow + 64u, rd[0]);
+      tc::tmem_ld32_issue(trow + 96u, rd[1]);
+      tc::tmem_wait();
+      if (nq > 0) {  // the previous dV/dK products are done with P^T and dS^T
+        ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+        tc::fence_after_sync();
+      }
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        float pv[32], dv[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int jq = 64 * hh + 32 * c + j;  // query column within the tile
+          const int tq = q0 + jq;
+          const bool valid = tq < Tlen && (!diag || (jq >= r && jq < kbe));
+          const float p = valid ? exp2f(__uint_as_float(rs[c][j]) * sl2 - slse[jq]) : 0.f;
+          pv[j] = p;
+          dv[j] = p * (__uint_as_float(rd[c][j]) - sdr[jq]) * scale;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          put_unit(sPt, r, 4 * c + u, pack8(pv + 8 * u));
+          put_unit(sdSt, r, 4 * c + u, pack8(dv + 8 * u));
+        }
+      }
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid == 0) {
+        tc::fence_after_sync();
+        if (ok) {
+          constexpr uint32_t idKV = tc::idesc_bf16(128, DH, 0, 1);
+          const uint32_t acc0 = (qt > 0 || hh > 0) ? 1u : 0u;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // dV += P^T[:, 64hh..] dO[64hh.., :]
+            tc::mma_bf16(tmem + 128, p_kmaj(sPt, 0, kk), G::mnmaj(sdO, 64 * hh, kk), idKV,
+                         (acc0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // dK += dS^T[:, 64hh..] Q[64hh.., :]
+            tc::mma_bf16(tmem + 192, p_kmaj(sdSt, 0, kk), G::mnmaj(sQ, 64 * hh, kk), idKV,
+                         (acc0 || kk > 0) ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[2]);
+      }
+      ++nq;
+    }
+    if (tid == 0 && qt + 1 < nqt) {
+      ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
+      tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, q0 + kTile, b);
+      tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, q0 + kTile, b);
+    }
+    __syncthreads();  // slse / sdr are rewritten next
+  }
+  ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+  tc::fence_after_sync();
+  float v[DH];
+  tmem_row<DH>(trow + 128u, v);
+  if (ok && key < Tlen) store_row<DH>(dV + ((long)b * Tlen + key) * ld_d + h * DH, v, 1.0f);
+  tmem_row<DH>(trow + 192u, v);
+  if (ok && key < Tlen) store_row<DH>(dK + ((long)b * Tlen + key) * ld_d + h * DH, v, 1.0f);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+}
+
+// ========================================================================= host
+bool attn_fl_supported(int dtype, int dh, int L) {
+  const bool l_ok = (L >= 16 && kTile % L == 0) || (L % kTile == 0 && L <= 1024);
+  return dtype == 1 && (dh == 16 || dh == 32 || dh == 64) && l_ok && tmap_encoder() != nullptr;
+}
+
+namespace {
+template <int DH>
+bool head_map_fl(CUtensorMap* m, const void* base, long ld, int D, int T, int B) {
+  const uint64_t dims[3] = {(uint64_t)D, (uint64_t)T, (uint64_t)B};
+  const uint64_t st[2] = {(uint64_t)ld * 2, (uint64_t)ld * 2 * (uint64_t)T};
+  const uint32_t box[3] = {DH, kTile, 1};
+  const CUtensorMapSwizzle sw = DH == 64   ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : DH == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                           : CU_TENSOR_MAP_SWIZZLE_32B;
+  return make_tmap_bf16(m, base, 3, dims, st, box, sw);
+}
+
+// dynamic shared memory: 1 KB alignment slack + tiles + staging + barriers
+template <int DH> constexpr int fwd_smem() { return 1024 + 32768 + 3 * Geo<DH>::tile + 64; }
+template <int DH> constexpr int dq_smem() { return 1024 + 16384 + 4 * Geo<DH>::tile + 64; }
+template <int DH> constexpr int dkv_smem() {
+  return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
+}
+
+template <class K>
+cudaError_t opt_in(K* kern, int bytes, bool* done) {
+  if (*done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) *done = true;
+  return e;
+}
+
+template <int DH>
+cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
+  const int D = a.H * DH;
+  CUtensorMap mq, mk, mv;
+  if (!head_map_fl<DH>(&mq, a.Q, a.ld_qkv, D, a.T, a.B) ||
+      !head_map_fl<DH>(&mk, a.K, a.ld_qkv, D, a.T, a.B) ||
+      !head_map_fl<DH>(&mv, a.V, a.ld_qkv, D, a.T, a.B))
+    return cudaErrorInvalidValue;
+  static bool attr = false;
+  cudaError_t e = opt_in(attn_fwd_fl_kernel<DH>, fwd_smem<DH>(), &attr);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
+  e = launch_k(attn_fwd_fl_kernel<DH>, grid, dim3(128), fwd_smem<DH>(), lc.stream, mq, mk, mv,
+               (bf16*)a.O, a.ld_o, a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)DH), lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+template <int DH>
+cudaError_t bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
+  const AttnArgs& f = a.f;
+  const int D = f.H * DH;
+  CUtensorMap mq, mk, mv, mdo;
+  if (!head_map_fl<DH>(&mq, f.Q, f.ld_qkv, D, f.T, f.B) ||
+      !head_map_fl<DH>(&mk, f.K, f.ld_qkv, D, f.T, f.B) ||
+      !head_map_fl<DH>(&mv, f.V, f.ld_qkv, D, f.T, f.B) ||
+      !head_map_fl<DH>(&mdo, a.dO, f.ld_o, D, f.T, f.B))
+    return cudaErrorInvalidValue;
+  static bool attr_q = false, attr_kv = false;
+  cudaError_t e = opt_in(attn_bwd_dq_fl_kernel<DH>, dq_smem<DH>(), &attr_q);
+  if (e == cudaSuccess) e = opt_in(attn_bwd_dkv_fl_kernel<DH>, dkv_smem<DH>(), &attr_kv);
+  if (e != cudaSuccess) return e;
+  const float scale = 1.0f / sqrtf((float)DH);
+  dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
+  e = launch_k(attn_bwd_dq_fl_kernel<DH>, grid, dim3(128), dq_smem<DH>(), lc.stream, mq, mk, mv,
+               mdo, (const bf16*)f.O, (const bf16*)a.dO, f.ld_o, (const float*)f.lse, a.Drow,
+               (bf16*)a.dQ, a.ld_dqkv, f.T, f.H, f.L, scale, lc.status);
+  if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
+  e = launch_k(attn_bwd_dkv_fl_kernel<DH>, grid, dim3(128), dkv_smem<DH>(), lc.stream, mq, mk, mv,
+               mdo, (const float*)f.lse, (const float*)a.Drow, (bf16*)a.dK, (bf16*)a.dV,
+               a.ld_dqkv, f.T, f.H, f.L, scale, lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t attn_fwd_fl(const Launch& lc, const AttnArgs& a) {
+  if (!attn_fl_supported(1, a.dh, a.L)) return cudaErrorNotSupported;
+  switch (a.dh) {
+    case 16: return fwd_fl<16>(lc, a);
+    case 32: return fwd_fl<32>(lc, a);
+    default: return fwd_fl<64>(lc, a);
+  }
+}
+
+cudaError_t attn_bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
+  if (!attn_fl_supported(1, a.f.dh, a.f.L)) return cudaErrorNotSupported;
+  switch (a.f.dh) {
+    case 16: return bwd_fl<16>(lc, a);
+    case 32: return bwd_fl<32>(lc, a);
+    default: return bwd_fl<64>(lc, a);
+  }
+}
+
+}  // namespace bcmt

@@ -14,29 +14,19 @@
 // and runs the five products S = Q K^T, dP = dO V^T, dV = P^T dO,
 // dQ = dS K, dK = dS^T Q on the tensor cores, reading the same shared tiles
 // K-major or MN-major as each product needs.
+#include "attn_common.cuh"
 #include "common.cuh"
 #include "internal.h"
 #include "tc.cuh"
 #include "tmap.h"
 
 namespace bcmt {
+using namespace attn;
 
 namespace {
 constexpr int kTile = 128;
 constexpr int kDh = 64;
 constexpr uint32_t kTB = kTile * kDh * 2;  // one 128 x 64 bf16 tile: 16 KB
-constexpr float kLog2e = 1.4426950408889634f;
-
-// Writes 16-byte unit `u` (keys 8u .. 8u+7) of row r of a 128 x 128 bf16
-// K-major operand stored as two 128-row swizzle-128 atoms (keys 0-63, 64-127).
-__device__ __forceinline__ void put_unit(uint8_t* base, int r, int u, uint4 val) {
-  *reinterpret_cast<uint4*>(base + (u >> 3) * 16384 + tc::sw128_offset(r, u & 7)) = val;
-}
-
-__device__ __forceinline__ uint32_t pack2(float a, float b) {
-  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t*>(&t);
-}
 
 // Stores one 64-wide fp32 row (two 32-column halves) as bf16 into a
 // 128-row x 128-byte swizzled staging tile (the TMA store layout).
@@ -51,17 +41,12 @@ __device__ __forceinline__ void stage_half(uint8_t* tile, int r, int half, const
     *reinterpret_cast<uint4*>(tile + tc::sw128_offset(r, half * 4 + u)) = q;
   }
 }
-
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
 }  // namespace
 
 // Both kernels are instantiated for NCH = the number of 32-key chunks of a
 // block that one warp's 32 query rows can reach (1 for L <= 32, L / 32
 // otherwise); a warp reads only the chunks up to its own last row's key, the
 // rest of its P and dS rows are causal zeros.
-__device__ __forceinline__ int chunks_needed(int warp, int wbs) { return (warp * 32 - wbs) / 32 + 1; }
 
 // ====================================================================== forward
 template <int NCH>

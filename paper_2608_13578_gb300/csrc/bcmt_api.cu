@@ -333,8 +333,12 @@ cudaError_t run_gemm(const Launch& lc, Prof& pr, const char* name, int dtype, in
   return e;
 }
 
-bool use_attn_tc(const Geometry& g) {
-  return g_use_tc_attn && attn_tc_supported(g.dtype, g.dh, g.L);
+// Attention kernel for a shape: 1 = single-tile tcgen05 (head width 64,
+// L <= 128), 2 = key-tile-walking tcgen05, 0 = SIMT (fp32 and the rest).
+int attn_kind(const Geometry& g) {
+  if (!g_use_tc_attn) return 0;
+  if (attn_tc_supported(g.dtype, g.dh, g.L)) return 1;
+  return attn_fl_supported(g.dtype, g.dh, g.L) ? 2 : 0;
 }
 
 bcmt_status finish(const bcmt_params* p, cudaStream_t s) {
@@ -429,9 +433,12 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   }
   // Sec. 3.3: intra-block causal attention -> Concat(heads).
   AttnArgs aa{Qp, Kp, Vp, ld, w.hhat, D, w.lse, g.B, g.T, g.H, g.dh, g.L};
-  if (use_attn_tc(g)) {
+  if (attn_kind(g) == 1) {
     pr.begin("attn_fwd_tc");
     e = attn_fwd_tc(lc, aa);
+  } else if (attn_kind(g) == 2) {
+    pr.begin("attn_fwd_fl");
+    e = attn_fwd_fl(lc, aa);
   } else {
     pr.begin("attn_fwd_simt");
     e = attn_fwd_simt(lc, g.dtype, aa);
@@ -652,9 +659,12 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     }
     AttnBwdArgs ab{{Qp, Kp, Vp, ld, w.hhat, D, w.lse, g.B, g.T, g.H, g.dh, g.L},
                    bw.dHhat, bw.Drow, dQ, dK, dV, ldd};
-    if (use_attn_tc(g)) {
+    if (attn_kind(g) == 1) {
       pr.begin("attn_bwd_tc");
       e = attn_bwd_tc(lc, ab);
+    } else if (attn_kind(g) == 2) {
+      pr.begin("attn_bwd_fl");
+      e = attn_bwd_fl(lc, ab);
     } else {
       pr.begin("attn_bwd_simt");
       e = attn_bwd_simt(lc, g.dtype, ab);
@@ -882,10 +892,14 @@ int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, 
   AttnArgs aa{q, k, v, ld, o, g.D, lse, g.B, g.T, g.H, g.dh, g.L};
   cudaError_t e;
   if (!backward) {
-    e = impl == 1 ? attn_fwd_tc(lc, aa) : attn_fwd_simt(lc, g.dtype, aa);
+    e = impl == 1 ? attn_fwd_tc(lc, aa)
+        : impl == 2 ? attn_fwd_fl(lc, aa)
+                    : attn_fwd_simt(lc, g.dtype, aa);
   } else {
     AttnBwdArgs ab{aa, dO, drow, dq, dk, dv, ld_d};
-    e = impl == 1 ? attn_bwd_tc(lc, ab) : attn_bwd_simt(lc, g.dtype, ab);
+    e = impl == 1 ? attn_bwd_tc(lc, ab)
+        : impl == 2 ? attn_bwd_fl(lc, ab)
+                    : attn_bwd_simt(lc, g.dtype, ab);
   }
   if (e != cudaSuccess) {
     fail(BCMT_ERR_CUDA, "test attention: %s", cudaGetErrorString(e));

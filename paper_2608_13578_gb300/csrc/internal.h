@@ -110,6 +110,11 @@ cudaError_t attn_bwd_simt_noalloc(const Launch& lc, int dtype, const AttnBwdArgs
 cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a);
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
 bool attn_tc_supported(int dtype, int dh, int L);
+// tcgen05 attention that walks key tiles (head widths 16/32/64, L dividing or
+// a multiple of 128); the backward writes Drow itself (dQ kernel first).
+bool attn_fl_supported(int dtype, int dh, int L);
+cudaError_t attn_fwd_fl(const Launch& lc, const AttnArgs& a);
+cudaError_t attn_bwd_fl(const Launch& lc, const AttnBwdArgs& a);
 
 // ------------------------------------------------ summary, memory, gate
 // Sec. 3.4: per block, s = H w_p (summed from npart partial dot products

@@ -98,9 +98,28 @@ ATTN_CASES = [
     (1, 384, 3, 64, 128, "bf16"),
     (2, 130, 2, 64, 16, "bf16"),
     (1, 300, 2, 64, 256, "bf16"),
+    (1, 600, 2, 64, 256, "bf16"),     # ragged last block, 1-3 key tiles per query tile
+    (1, 1100, 1, 64, 512, "bf16"),
+    (1, 1024, 1, 64, 1024, "bf16"),
+    (2, 300, 4, 16, 64, "bf16"),      # the paper's 16-wide heads
+    (2, 200, 8, 16, 128, "bf16"),
+    (1, 520, 4, 16, 512, "bf16"),
+    (2, 130, 4, 16, 16, "bf16"),
+    (1, 520, 2, 32, 256, "bf16"),
+    (2, 150, 2, 32, 32, "bf16"),
     (2, 100, 2, 32, 24, "fp32"),
     (1, 256, 4, 32, 32, "fp32"),
 ]
+
+
+def _impl_ok(impl, dh, L, dtype):
+    if impl == 0:
+        return True
+    if dtype != "bf16":
+        return False
+    if impl == 1:
+        return dh == 64 and L in (16, 32, 64, 128)
+    return dh in (16, 32, 64) and ((L >= 16 and 128 % L == 0) or (L % 128 == 0 and L <= 1024))
 
 
 def _attn_ref(q, k, v, L, H, dO):
@@ -123,12 +142,11 @@ def _attn_ref(q, k, v, L, H, dO):
     return fw["Hhat"], lse, gr["dq"], gr["dk"], gr["dv"]
 
 
-@pytest.mark.parametrize("impl", [0, 1], ids=["simt", "tc"])
+@pytest.mark.parametrize("impl", [0, 1, 2], ids=["simt", "tc", "tc_walk"])
 @pytest.mark.parametrize("B,T,H,dh,L,dtype", ATTN_CASES)
 def test_attention_fwd_bwd(C, impl, B, T, H, dh, L, dtype):
-    tc_ok = dtype == "bf16" and dh == 64 and L in (16, 32, 64, 128)
-    if impl == 1 and not tc_ok:
-        pytest.skip("shape outside the tcgen05 attention kernel (served by the SIMT kernel)")
+    if not _impl_ok(impl, dh, L, dtype):
+        pytest.skip("shape outside this attention kernel")
     D = H * dh
     tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
     gen = torch.Generator().manual_seed(B * 1000 + T + L)

@@ -36,6 +36,8 @@ SMALL = [
     W(2, 150, 128, 2, 48, "bf16"),
     W(1, 96, 192, 2, 32, "bf16"),                       # dh = 96 -> SIMT attention
     W(2, 300, 128, 8, 64, "bf16"),                      # dh = 16 (the paper's D128 h8)
+    W(1, 700, 128, 4, 256, "bf16"),                     # dh = 32, key-tile walk
+    W(2, 600, 256, 4, 512, "bf16"),                     # dh = 64, L = 512
     W(1, 200, 128, 8, 32, "fp32"),
     W(2, 256, 128, 2, 64, "bf16", decay=(0.0, 0.0)),
 ]
