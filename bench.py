@@ -175,7 +175,9 @@ def kernel_model(w):
     return {
         "gemm_qkv": g(n, 3 * D, D),
         "gemm_wo": g(n, D, D),
-        "gemm_gate_inject": g(n, D, D),
+        "gemm_gate": g(n, D, D),
+        # Sec. 3.8 injection: read H, G and C; write Y
+        "inject": ("hbm", 3 * n * D * es + B * Nb * D * 4),
         "gemm_dh": g(n, D, D),
         "gemm_dhhat": g(n, D, D),
         "gemm_dx": g(n, D, 3 * D),
@@ -198,8 +200,9 @@ def kernel_model(w):
         "gemm_dm": g(B * Nb, D, D),
         # reverse scan: read dM and Z, write dS
         "memory_scan_bwd": ("hbm", 2 * B * Nb * D * 4 + Nb * D * 4),
-        # pooling backward: read H, alpha and dS; write ds and the dW_p partials
-        "summary_bwd": ("hbm", n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
+        # pooling backward: read H, alpha and dS; write ds and the dW_p partials;
+        # complete dH in place (read and write)
+        "summary_bwd": ("hbm", 3 * n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
         "gemm_dwm": g(D, D, B * Nb),
         "reduce_rows": ("hbm", B * Nb * D * 4 + D * es),
     }

@@ -56,10 +56,11 @@ unsigned* status_ptr() {
 // which no later step of the pass reads: they run beside the dependent chain
 // (forked and joined with events, so the pair can also be captured into a
 // CUDA graph).  Streams and events are host-side objects: no device memory.
+constexpr int kSideEvents = 12;
 struct SideStream {
   cudaStream_t s = nullptr;
-  cudaEvent_t ev[8] = {};
-  std::mutex mu;  // one backward at a time may use the events
+  cudaEvent_t ev[kSideEvents] = {};
+  std::mutex mu;  // one call at a time may use the events
 };
 
 SideStream* side_stream() {
@@ -72,7 +73,7 @@ SideStream* side_stream() {
   if (!per_dev[dev]) {
     SideStream* ss = new SideStream();
     bool ok = cudaStreamCreateWithFlags(&ss->s, cudaStreamNonBlocking) == cudaSuccess;
-    for (int i = 0; i < 8 && ok; ++i)
+    for (int i = 0; i < kSideEvents && ok; ++i)
       ok = cudaEventCreateWithFlags(&ss->ev[i], cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
       delete ss;  // fall back to one stream
@@ -95,18 +96,30 @@ struct Fork {
   }
   cudaStream_t side() const { return ss ? ss->s : main; }
   // the side stream waits for everything enqueued on the main stream so far
-  void point() {
-    if (!ss || next >= 7) return;
+  // (false when the events are used up: the caller then stays on one stream)
+  bool point() {
+    if (!ss || next >= kSideEvents - 1) return false;
     cudaEventRecord(ss->ev[next], main);
     cudaStreamWaitEvent(ss->s, ss->ev[next], 0);
     ++next;
     forked = true;
+    return true;
+  }
+  // records what the side stream has been given so far; wait_mark(m) later
+  // makes the main stream wait for exactly that
+  int mark() {
+    if (!ss || !forked || next >= kSideEvents - 1) return -1;
+    cudaEventRecord(ss->ev[next], ss->s);
+    return next++;
+  }
+  void wait_mark(int m) {
+    if (ss && m >= 0) cudaStreamWaitEvent(main, ss->ev[m], 0);
   }
   ~Fork() {
     if (!ss) return;
     if (forked) {
-      cudaEventRecord(ss->ev[7], ss->s);
-      cudaStreamWaitEvent(main, ss->ev[7], 0);
+      cudaEventRecord(ss->ev[kSideEvents - 1], ss->s);
+      cudaStreamWaitEvent(main, ss->ev[kSideEvents - 1], 0);
     }
     ss->mu.unlock();
   }
@@ -410,8 +423,16 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   unsigned* sp = status_ptr();
   if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool profiling = (p->flags & BCMT_FLAG_PROFILE) != 0;
   Launch lc{s, sp};
-  Prof pr{(p->flags & BCMT_FLAG_PROFILE) != 0, s};
+  Prof pr{profiling, s};
+  // The memory stage runs on the side stream beside the gate GEMM (one
+  // stream while profiling).
+  std::unique_ptr<Fork> fork_holder(
+      new Fork(profiling || g.honly ? nullptr : side_stream(), s));
+  Fork& fork = *fork_holder;
+  Launch lcs{fork.side(), sp};
+  Prof prs{profiling, fork.side()};
   FwdWs w = fwd_layout(g, workspace);
   const int D = g.D, n = (int)g.n;
   cudaError_t e;
@@ -460,40 +481,45 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // Sec. 3.4: adaptive block summaries.
-    pr.begin("summary_fwd");
-    e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
-    pr.end(nullptr);
+    // side stream: Sec. 3.4 adaptive block summaries, Sec. 3.5 exponential
+    // causal memory (scan), then its projection and one-block shift -> C
+    fork.point();
+    prs.begin("summary_fwd");
+    e = summary_fwd(lcs, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
+    prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
-    // Sec. 3.5: exponential causal memory (scan), then projection and shift.
-    pr.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C, g.B,
-                        g.Nb, D);
-    pr.end(nullptr);
+    prs.begin("memory_scan_fwd");
+    e = memory_scan_fwd(lcs, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C,
+                        g.B, g.Nb, D);
+    prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "causal memory");
     {
       EpiArgs ea;
       ea.out = w.C;
       ea.ldo = D;
       ea.Nb = g.Nb;
-      e = run_gemm(lc, pr, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
+      e = run_gemm(lcs, prs, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
                    EPI_SHIFT, ea);
       if (e != cudaSuccess) return cuda_fail(e, "memory projection");
     }
-    // Sec. 3.7-3.8: gate and injection fused into the W_g GEMM.
-    EpiArgs ea;
-    ea.H = w.hloc;
-    ea.Cmem = w.C;
-    ea.G = w.G;
-    ea.Y = y;
-    ea.T = g.T;
-    ea.L = g.L;
-    ea.Nb = g.Nb;
-    ea.D = D;
-    e = run_gemm(lc, pr, "gemm_gate_inject", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
-                 EPI_GATE_INJECT, ea);
-    if (e != cudaSuccess) return cuda_fail(e, "gated injection");
+    const int memory_done = fork.mark();
+    // main stream, meanwhile: Sec. 3.8 gate G = sigmoid(H W_g)
+    {
+      EpiArgs ea;
+      ea.out = w.G;
+      ea.ldo = D;
+      e = run_gemm(lc, pr, "gemm_gate", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
+                   EPI_GATE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "gate");
+    }
+    // Sec. 3.7-3.8: Y = H + G * M_tokens once the memory rows are ready
+    fork.wait_mark(memory_done);
+    pr.begin("inject");
+    e = inject(lc, g.dtype, w.hloc, w.G, w.C, y, g.B, g.T, D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "injection");
   }
+  fork_holder.reset();  // join the side stream before any status read
   return finish(p, s);
 }
 
@@ -555,27 +581,24 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                  g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "gate backward");
-    // Sec. 3.5 reversed: dM = dP W_m^T, reverse decayed scan -> dS.
+    // side stream: Sec. 3.5 reversed, dM = dP W_m^T and the reverse decayed
+    // scan -> dS (and the decay gradient's batch rows)
+    fork.point();
     {
       EpiArgs ea;
       ea.out = bw.dM;
       ea.ldo = D;
-      e = run_gemm(lc, pr, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
+      e = run_gemm(lcs, prs, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
                    EPI_STORE, ea);
       if (e != cudaSuccess) return cuda_fail(e, "dM");
     }
-    pr.begin("memory_scan_bwd");
-    e = memory_scan_bwd(lc, bw.dM, decay, w.Z, w.M, bw.dS, d_decay ? bw.da_part : nullptr, g.B,
+    prs.begin("memory_scan_bwd");
+    e = memory_scan_bwd(lcs, bw.dM, decay, w.Z, w.M, bw.dS, d_decay ? bw.da_part : nullptr, g.B,
                         g.Nb, D);
-    pr.end(nullptr);
+    prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
-    // Sec. 3.4 reversed: pooling scores and the dW_p partials.
-    pr.begin("summary_bwd");
-    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, bw.ds, bw.dwp_part, g.B, g.T, D, g.L);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "summary backward");
-    // side stream: dW_m = M^T dP, dW_g = H^T dU, dW_p
-    fork.point();
+    const int scan_done = fork.mark();
+    // side stream, then: dW_m = M^T dP and dW_g = H^T dU
     {
       EpiArgs ea;
       ea.out = dw_m;
@@ -587,6 +610,25 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
                     bw.part, dw_g);
     if (e != cudaSuccess) return cuda_fail(e, "dW_g");
+    // main stream, meanwhile: dH = dY + dU W_g^T (the identity and gate paths)
+    {
+      EpiArgs ea;
+      ea.out = bw.dH;
+      ea.ldo = D;
+      ea.add = dy;
+      e = run_gemm(lc, pr, "gemm_dh", g.dtype, g.dtype, n, D, D, bw.dU, D, 1, w_g, 1, D, EPI_ADD,
+                   ea);
+      if (e != cudaSuccess) return cuda_fail(e, "dH");
+    }
+    // Sec. 3.4 reversed once dS is ready: pooling scores, the dW_p partials,
+    // and dH += alpha dS + ds w_p
+    fork.wait_mark(scan_done);
+    pr.begin("summary_bwd");
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part, g.B, g.T,
+                    D, g.L);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "summary backward");
+    fork.point();
     prs.begin("reduce_rows");
     e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
     prs.end(nullptr);
@@ -597,20 +639,6 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
       prs.end(nullptr);
       if (e != cudaSuccess) return cuda_fail(e, "d_decay");
     }
-    // dH = dY + dU W_g^T + alpha dS + ds w_p
-    EpiArgs ea;
-    ea.out = bw.dH;
-    ea.dY = dy;
-    ea.alpha = w.alpha;
-    ea.dS = bw.dS;
-    ea.ds = bw.ds;
-    ea.w_p = w_p;
-    ea.T = g.T;
-    ea.L = g.L;
-    ea.Nb = g.Nb;
-    ea.D = D;
-    e = run_gemm(lc, pr, "gemm_dh", g.dtype, g.dtype, n, D, D, bw.dU, D, 1, w_g, 1, D, EPI_DH, ea);
-    if (e != cudaSuccess) return cuda_fail(e, "dH");
     dH = bw.dH;
   } else {
     const size_t wb = (size_t)D * D * g.es;
@@ -624,7 +652,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     EpiArgs ea;
     ea.out = bw.dHhat;
     ea.ldo = D;
-    fork.point();  // dH is final
+    if (g.honly) fork.point();  // dH (= dY) is final; otherwise forked after summary_bwd
     e = weight_grad(lcs, prs, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part,
                     dw_o);
     if (e != cudaSuccess) return cuda_fail(e, "dW_O");

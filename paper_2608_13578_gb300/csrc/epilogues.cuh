@@ -105,134 +105,74 @@ struct EpiShiftF {
   }
 };
 
-// Sec. 3.8: G = sigmoid(H W_g), Y = H + G * M_tokens, M_tokens row = Cmem[b, t/L].
+// Sec. 3.8 gate: G = sigmoid(H W_g) in the storage dtype.  The injection
+// Y = H + G * C_blk runs as its own pass once the memory rows C are ready, so
+// that this GEMM does not wait for the memory stage.
 template <class T>
-struct EpiGateInjectF {
-  // tcgen05 path (bf16 only): H as raw bf16 pairs, C in fp32
-  struct Pre {
-    uint4 h[4];
-    float c[32];
-  };
-  const T* H;
-  const float* Cmem;
+struct EpiGateF {
+  using Pre = NoPre;
   T* G;
-  T* Y;
-  int Tlen, L, Nb, D;
-  __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
-    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
-    const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
-    const bf16* h = reinterpret_cast<const bf16*>(H) + (long)row * D + col;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) load8_raw(h + 8 * j, pre.h[j]);
-#pragma unroll
-    for (int j = 0; j < 32; j += 4) load4(cm + j, pre.c + j);
-  }
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
-                                        int) const {
-    const long o = (long)row * D + col;
+  long ldo;
+  __device__ __forceinline__ void load(int, int, Pre&) const {}
+  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int) const {
+    bf16* p = reinterpret_cast<bf16*>(G) + (long)row * ldo + col;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      float h[8], g[8], y[8];
-      unpack8(pre.h[q], h);
+      float g[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        g[e] = sigmoid_bf16out(v[8 * q + e]);
-        y[e] = fmaf(g[e], pre.c[8 * q + e], h[e]);
-      }
-      store8(reinterpret_cast<bf16*>(G) + o + 8 * q, g);
-      store8(reinterpret_cast<bf16*>(Y) + o + 8 * q, y);
+      for (int e = 0; e < 8; ++e) g[e] = sigmoid_bf16out(v[8 * q + e]);
+      store8(p + 8 * q, g);
     }
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
-    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
-    const float* cm = Cmem + ((long)b * Nb + blk) * D + col;
-    const long o = (long)row * D + col;
-    float h[32], c[32];
-    for (int j = 0; j < n; j += 4) {
-      load4(H + o + j, h + j);
-      load4(cm + j, c + j);
-    }
+    T* p = G + (long)row * ldo + col;
     float g[32];
-    for (int j = 0; j < n; ++j) {
-      g[j] = sigmoidf_(v[j]);
-      h[j] = fmaf(g[j], c[j], h[j]);
-    }
+    for (int j = 0; j < n; ++j) g[j] = sigmoidf_(v[j]);
     if (n % 8 == 0) {
-      for (int j = 0; j < n; j += 8) {
-        store8(G + o + j, g + j);
-        store8(Y + o + j, h + j);
-      }
+      for (int j = 0; j < n; j += 8) store8(p + j, g + j);
     } else {
-      for (int j = 0; j < n; j += 4) {
-        store4(G + o + j, g + j);
-        store4(Y + o + j, h + j);
-      }
+      for (int j = 0; j < n; j += 4) store4(p + j, g + j);
     }
   }
 };
 
-// Backward into H: dH = dU W_g^T (the accumulator) + dY (identity path of
-// Y = H + ...) + alpha_t dS_blk (pooling S = H^T alpha) + ds_t w_p (scores).
+// out = acc + add, same row-major layout (e.g. dU W_g^T + dY: the identity
+// path of Y = H + ... joins the gate path's gradient).
 template <class T>
-struct EpiDHF {
-  // tcgen05 path (bf16 only): dY and w_p as raw bf16 pairs, dS in fp32
+struct EpiAddF {
+  // tcgen05 path (bf16 only): the addend as raw bf16 pairs
   struct Pre {
-    uint4 dy[4], wp[4];
-    float sv[32];
-    float at, st;
+    uint4 a[4];
   };
-  const T* dY;
-  const float* alpha;
-  const float* dS;
-  const float* ds;
-  const T* w_p;
+  const T* add;
   T* out;
-  int Tlen, L, Nb, D;
+  long ldo;
   __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
-    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
-    const float* dsb = dS + ((long)b * Nb + blk) * D + col;
-    const bf16* dy = reinterpret_cast<const bf16*>(dY) + (long)row * D + col;
-    const bf16* wp = reinterpret_cast<const bf16*>(w_p) + col;
+    const bf16* a = reinterpret_cast<const bf16*>(add) + (long)row * ldo + col;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      load8_raw(dy + 8 * j, pre.dy[j]);
-      load8_raw(wp + 8 * j, pre.wp[j]);
-    }
-#pragma unroll
-    for (int j = 0; j < 32; j += 4) load4(dsb + j, pre.sv + j);
-    pre.at = alpha[row];
-    pre.st = ds[row];
+    for (int j = 0; j < 4; ++j) load8_raw(a + 8 * j, pre.a[j]);
   }
   __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
                                         int) const {
-    const long o = (long)row * D + col;
+    bf16* p = reinterpret_cast<bf16*>(out) + (long)row * ldo + col;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      float dy[8], wp[8], r[8];
-      unpack8(pre.dy[q], dy);
-      unpack8(pre.wp[q], wp);
+      float a[8], r[8];
+      unpack8(pre.a[q], a);
 #pragma unroll
-      for (int e = 0; e < 8; ++e)
-        r[e] = v[8 * q + e] + dy[e] + pre.at * pre.sv[8 * q + e] + pre.st * wp[e];
-      store8(reinterpret_cast<bf16*>(out) + o + 8 * q, r);
+      for (int e = 0; e < 8; ++e) r[e] = v[8 * q + e] + a[e];
+      store8(p + 8 * q, r);
     }
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
-    const int b = row / Tlen, t = row - b * Tlen, blk = t / L;
-    const float* dsb = dS + ((long)b * Nb + blk) * D + col;
-    const long o = (long)row * D + col;
-    const float at = alpha[row], st = ds[row];
-    float dy[32], sv[32], wp[32];
-    for (int j = 0; j < n; j += 4) {
-      load4(dY + o + j, dy + j);
-      load4(dsb + j, sv + j);
-      load4(w_p + col + j, wp + j);
-    }
-    for (int j = 0; j < n; ++j) dy[j] = v[j] + dy[j] + at * sv[j] + st * wp[j];
+    const long o = (long)row * ldo + col;
+    float a[32];
+    for (int j = 0; j < n; j += 4) load4(add + o + j, a + j);
+    for (int j = 0; j < n; ++j) a[j] += v[j];
     if (n % 8 == 0) {
-      for (int j = 0; j < n; j += 8) store8(out + o + j, dy + j);
+      for (int j = 0; j < n; j += 8) store8(out + o + j, a + j);
     } else {
-      for (int j = 0; j < n; j += 4) store4(out + o + j, dy + j);
+      for (int j = 0; j < n; j += 4) store4(out + o + j, a + j);
     }
   }
 };

@@ -108,11 +108,9 @@ static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int
     case EPI_PARTIAL:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                              EpiStoreF<float>{(float*)ea.out, ea.ldo, ea.split_stride}, splits);
-    case EPI_GATE_INJECT:
+    case EPI_GATE:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                             EpiGateInjectF<TI>{(const TI*)ea.H, ea.Cmem, (TI*)ea.G, (TI*)ea.Y,
-                                                ea.T, ea.L, ea.Nb, ea.D},
-                             1);
+                             EpiGateF<TI>{(TI*)ea.out, ea.ldo}, 1);
     case EPI_STORE_SCORE:
       if (dtype_out == 0)
         return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
@@ -126,11 +124,9 @@ static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int
     case EPI_SHIFT:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                              EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
-    case EPI_DH:
+    case EPI_ADD:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                             EpiDHF<TI>{(const TI*)ea.dY, ea.alpha, ea.dS, ea.ds,
-                                        (const TI*)ea.w_p, (TI*)ea.out, ea.T, ea.L, ea.Nb, ea.D},
-                             1);
+                             EpiAddF<TI>{(const TI*)ea.add, (TI*)ea.out, ea.ldo}, 1);
   }
   return cudaErrorInvalidValue;
 }
@@ -407,12 +403,9 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
   // fused epilogues, instantiated only for the operand layouts the layer uses
   if constexpr (!A_MN && B_MN) {
     switch (epi) {
-      case EPI_GATE_INJECT:
-        return tc_launch<BN, ST, A_MN, B_MN>(
-            lc, M, N, K, A, sam, sak, B, sbk, sbn,
-            EpiGateInjectF<bf16>{(const bf16*)ea.H, ea.Cmem, (bf16*)ea.G, (bf16*)ea.Y, ea.T, ea.L,
-                                 ea.Nb, ea.D},
-            1);
+      case EPI_GATE:
+        return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                             EpiGateF<bf16>{(bf16*)ea.out, ea.ldo}, 1);
       case EPI_STORE_SCORE:
         return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
@@ -426,12 +419,10 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
     }
   }
   if constexpr (!A_MN && !B_MN) {
-    if (epi == EPI_DH)
+    if (epi == EPI_ADD)
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,
-          EpiDHF<bf16>{(const bf16*)ea.dY, ea.alpha, ea.dS, ea.ds, (const bf16*)ea.w_p,
-                       (bf16*)ea.out, ea.T, ea.L, ea.Nb, ea.D},
-          1);
+          EpiAddF<bf16>{(const bf16*)ea.add, (bf16*)ea.out, ea.ldo}, 1);
   }
   return cudaErrorNotSupported;
 }

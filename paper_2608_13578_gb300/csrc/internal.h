@@ -20,8 +20,8 @@ struct Launch {
 enum EpiKind {
   EPI_STORE = 0,        // out[m*ldo + n] = acc                       (out dtype = dtype_out)
   EPI_PARTIAL = 1,      // out(fp32)[z*split_stride + m*ldo + n] = acc of K-split z
-  EPI_GATE_INJECT = 2,  // G = sigmoid(acc); Y = H + G * Cmem[b, blk(t)]      (Sec. 3.8)
-  EPI_DH = 3,           // dH = acc + dY + alpha_t dS[b, blk(t)] + ds_t w_p   (backward)
+  EPI_GATE = 2,         // out = G = sigmoid(acc) in the storage dtype        (Sec. 3.8)
+  EPI_ADD = 3,          // out[m*ldo + n] = acc + add[m*ldo + n] (storage dtype)
   EPI_SHIFT = 4,        // out(fp32)[m+1] = acc for row m = b*Nb + i with i+1 < Nb (Sec. 3.5 shift)
   EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
 };
@@ -30,19 +30,11 @@ struct EpiArgs {
   void* out = nullptr;
   long ldo = 0;
   long split_stride = 0;
-  // EPI_GATE_INJECT
-  const void* H = nullptr;
-  const float* Cmem = nullptr;
-  void* G = nullptr;
-  void* Y = nullptr;
-  // EPI_STORE_SCORE: partial pooling scores, [D / n, M] fp32
+  // EPI_STORE_SCORE: partial pooling scores, [D / n, M] fp32, and w_p
   float* spart = nullptr;
-  // EPI_DH
-  const void* dY = nullptr;
-  const float* alpha = nullptr;
-  const float* dS = nullptr;
-  const float* ds = nullptr;
   const void* w_p = nullptr;
+  // EPI_ADD: the addend, same layout as out
+  const void* add = nullptr;
   // token geometry: row m = b*T + t, block blk(t) = t / L, Nb blocks, width D
   int T = 1, L = 1, Nb = 1, D = 0;
 };
@@ -136,9 +128,13 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
                             const float* M, float* dS, float* da_part, int B, int Nb, int D);
 // Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
-// dwp_part[b*Nb+i] = sum_t ds_t H_t.
+// dwp_part[b*Nb+i] = sum_t ds_t H_t, and dH_t += alpha_t dS_blk + ds_t w_p in place.
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* dS, float* ds, float* dwp_part, int B, int T, int D, int L);
+                        const float* dS, const void* w_p, void* dH, float* ds, float* dwp_part,
+                        int B, int T, int D, int L);
+// Sec. 3.7-3.8 injection: Y = H + G * C[b, t / L].
+cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Cm,
+                   void* Y, int B, int T, int D, int L);
 // Column sums of an fp32 [rows, cols] matrix in row order, stored in dtype_out.
 cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, int dtype_out,
                         void* out);

@@ -4,6 +4,8 @@
 // cores.  (The memory's D x D projections run on the tensor cores, gemm.cu.)
 // Every kernel reads rows with 16-byte vector loads, issues a batch's loads
 // before its first use, and reduces in a fixed order (deterministic).
+#include <algorithm>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -195,10 +197,13 @@ __device__ void scan_bwd_item(const float* dM, const float* __restrict__ decay,
 
 // Sec. 3.4 reversed: item (i, b).  With S_i = sum_t alpha_t H_t and
 // alpha = softmax(s): g_t = H_t . dS_i, ds_t = alpha_t (g_t - sum_u alpha_u g_u),
-// and the block's share of dW_p = sum_t ds_t H_t.
+// and the block's share of dW_p = sum_t ds_t H_t.  The same pass completes the
+// gradient of H in place: dH_t += alpha_t dS_i + ds_t w_p (the pooling and the
+// score paths, added to dY + dU W_g^T already in dH).
 template <class T>
 __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
                                  const float* __restrict__ alpha, const float* dS,
+                                 const T* __restrict__ w_p, T* dH,
                                  float* __restrict__ ds_out, float* __restrict__ dwp_part,
                                  int Tlen, int D, int L, int Nb, int i, int b) {
   float* g = sm;                   // [kMaxL]
@@ -249,16 +254,40 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   }
   __syncthreads();
   const int rg = warp, co = lane;
+  T* dHb = dH + ((long)b * Tlen + t0) * D;
   for (int c0 = 0; c0 < D; c0 += 256) {
     const int c = c0 + co * 8;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     if (c < D) {
-      for (int r = rg; r < n; r += 8) {
-        float h[8];
-        load8(Hb + (long)r * D + c, h);
-        const float w = g[r];
+      float sv[8], wp[8];
+      load8_cg(dSi + c, sv);
+      load8(w_p + c, wp);
+      // rows rg, rg+8, ... two at a time: all loads of a pair before its stores
+      for (int r = rg; r < n; r += 16) {
+        const bool two = r + 8 < n;
+        float h0[8], h1[8], d0[8], d1[8];
+        load8(Hb + (long)r * D + c, h0);
+        load8(dHb + (long)r * D + c, d0);
+        if (two) {
+          load8(Hb + (long)(r + 8) * D + c, h1);
+          load8(dHb + (long)(r + 8) * D + c, d1);
+        }
+        const float w0 = g[r], a0 = ab[r];
+        const float w1 = two ? g[r + 8] : 0.f, a1 = two ? ab[r + 8] : 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] = fmaf(w, h[e], acc[e]);
+        for (int e = 0; e < 8; ++e) {
+          acc[e] = fmaf(w0, h0[e], acc[e]);
+          d0[e] += a0 * sv[e] + w0 * wp[e];
+        }
+        store8(dHb + (long)r * D + c, d0);
+        if (two) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            acc[e] = fmaf(w1, h1[e], acc[e]);
+            d1[e] += a1 * sv[e] + w1 * wp[e];
+          }
+          store8(dHb + (long)(r + 8) * D + c, d1);
+        }
       }
     }
 #pragma unroll
@@ -346,11 +375,54 @@ __global__ void __launch_bounds__(kThreads)
 template <class T>
 __global__ void __launch_bounds__(kThreads)
     summary_bwd_kernel(const T* __restrict__ Hm, const float* __restrict__ alpha,
-                       const float* __restrict__ dS, float* __restrict__ ds,
-                       float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
+                       const float* __restrict__ dS, const T* __restrict__ w_p, T* dH,
+                       float* __restrict__ ds, float* __restrict__ dwp_part, int Tlen, int D,
+                       int L, int Nb) {
   pdl_enter();
   extern __shared__ __align__(16) float sm[];
-  summary_bwd_item<T>(sm, Hm, alpha, dS, ds, dwp_part, Tlen, D, L, Nb, blockIdx.x, blockIdx.y);
+  summary_bwd_item<T>(sm, Hm, alpha, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb, blockIdx.x,
+                      blockIdx.y);
+}
+
+// Sec. 3.7-3.8: Y = H + G * C[b, t / L], the memory row of the token's block
+// broadcast by index.  Each thread takes two runs of 8 channels and issues
+// all their loads before its stores.
+template <class T>
+__global__ void __launch_bounds__(kThreads)
+    inject_kernel(const T* __restrict__ Hm, const T* __restrict__ G, const float* __restrict__ Cm,
+                  T* __restrict__ Y, long n_rows, int Tlen, int D, int L, int Nb) {
+  pdl_enter();
+  const int runs = D / 8;
+  const long total = n_rows * runs;
+  const long stride = (long)gridDim.x * kThreads;
+  for (long i0 = (long)blockIdx.x * kThreads + threadIdx.x; i0 < total; i0 += 2 * stride) {
+    float h[2][8], g[2][8], c[2][8];
+    long o[2];
+    bool live[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const long i = i0 + u * stride;
+      live[u] = i < total;
+      if (!live[u]) continue;
+      const long row = i / runs;
+      const int cc = (int)(i - row * runs) * 8;
+      const int b = (int)(row / Tlen), t = (int)(row - (long)b * Tlen);
+      o[u] = row * D + cc;
+      load8(Hm + o[u], h[u]);
+      load8(G + o[u], g[u]);
+      const float* cm = Cm + ((long)b * Nb + t / L) * D + cc;
+      load4(cm, c[u]);
+      load4(cm + 4, c[u] + 4);
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      if (!live[u]) continue;
+      float y[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) y[e] = fmaf(g[u][e], c[u][e], h[u][e]);
+      store8(Y + o[u], y);
+    }
+  }
 }
 
 // ============================================================== host side
@@ -413,17 +485,37 @@ cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* deca
 }
 
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* dS, float* ds, float* dwp_part, int B, int T, int D, int L) {
+                        const float* dS, const void* w_p, void* dH, float* ds, float* dwp_part,
+                        int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
   dim3 grid(Nb, B);
   cudaError_t e;
   if (dtype == 0)
     e = launch_k(summary_bwd_kernel<float>, grid, dim3(kThreads), kSummarySmem, lc.stream,
-                 (const float*)Hm, alpha, dS, ds, dwp_part, T, D, L, Nb);
+                 (const float*)Hm, alpha, dS, (const float*)w_p, (float*)dH, ds, dwp_part, T, D,
+                 L, Nb);
   else
     e = launch_k(summary_bwd_kernel<bf16>, grid, dim3(kThreads), kSummarySmem, lc.stream,
-                 (const bf16*)Hm, alpha, dS, ds, dwp_part, T, D, L, Nb);
+                 (const bf16*)Hm, alpha, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T, D, L,
+                 Nb);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Cm,
+                   void* Y, int B, int T, int D, int L) {
+  const int Nb = (T + L - 1) / L;
+  const long n_rows = (long)B * T;
+  const long work = n_rows * (D / 8);
+  const int blocks = (int)std::max<long>(1, std::min<long>((work + 2 * kThreads - 1) / (2 * kThreads),
+                                                           1L << 16));
+  cudaError_t e;
+  if (dtype == 0)
+    e = launch_k(inject_kernel<float>, dim3(blocks), dim3(kThreads), 0, lc.stream,
+                 (const float*)Hm, (const float*)G, Cm, (float*)Y, n_rows, T, D, L, Nb);
+  else
+    e = launch_k(inject_kernel<bf16>, dim3(blocks), dim3(kThreads), 0, lc.stream,
+                 (const bf16*)Hm, (const bf16*)G, Cm, (bf16*)Y, n_rows, T, D, L, Nb);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
