@@ -899,9 +899,11 @@ int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, cons
   ea.ldo = ldc;
   ea.split_stride = (long)M * ldc;
   const EpiKind ek = splits > 1 ? EPI_PARTIAL : EPI_STORE;
-  cudaError_t e = impl == 1 ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
-                            : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek,
-                                        ea, splits);
+  cudaError_t e =
+      impl == 1   ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
+      : impl == 2 ? gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
+                  : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea,
+                              splits);
   if (e != cudaSuccess) {
     fail(BCMT_ERR_CUDA, "test gemm: %s", cudaGetErrorString(e));
     return -1;

@@ -13,18 +13,21 @@ namespace bcmt {
 // two-phase form for the tcgen05 GEMM's 32-column TMEM chunks: load() fetches
 // the chunk's extra inputs into registers (issued a chunk ahead, and for the
 // first chunk before the accumulator is ready), apply() consumes them.
+// Epilogues with kTma = true only transform the 32 values in place in
+// apply(); the GEMM then stages them in shared memory and writes the output
+// tile (out, ldo, split_stride, element type OutT) with TMA stores.
 struct NoPre {};
 
 template <class TO>
 struct EpiStoreF {
   using Pre = NoPre;
+  using OutT = TO;
+  static constexpr bool kTma = true;
   TO* out;
   long ldo;
   long split_stride;
   __device__ __forceinline__ void load(int, int, Pre&) const {}
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int z) const {
-    (*this)(row, col, v, 32, z);
-  }
+  __device__ __forceinline__ void apply(int, int, float*, const Pre&, int) const {}
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int z) const {
     TO* p = out + (long)z * split_stride + (long)row * ldo + col;
     if (n % 8 == 0) {
@@ -47,6 +50,9 @@ struct EpiStoreScoreF {
   struct Pre {
     uint4 w[4];
   };
+  using OutT = TO;
+  static constexpr bool kTma = true;
+  static constexpr long split_stride = 0;
   TO* out;
   long ldo;
   const TO* w_p;
@@ -57,9 +63,7 @@ struct EpiStoreScoreF {
 #pragma unroll
     for (int j = 0; j < 4; ++j) load8_raw(wp + 8 * j, pre.w[j]);
   }
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
-                                        int) const {
-    bf16* p = reinterpret_cast<bf16*>(out) + (long)row * ldo + col;
+  __device__ __forceinline__ void apply(int row, int col, float* v, const Pre& pre, int) const {
     float s = 0.f;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -68,7 +72,6 @@ struct EpiStoreScoreF {
 #pragma unroll
       for (int e = 0; e < 8; ++e)
         s = fmaf(__bfloat162float(__float2bfloat16_rn(v[8 * q + e])), w[e], s);
-      store8(p + 8 * q, v + 8 * q);
     }
     spart[(long)(col / 32) * n_rows + row] = s;
   }
@@ -91,11 +94,14 @@ struct EpiStoreScoreF {
 // i+1 of the same sequence; the last block's row is dropped.
 struct EpiShiftF {
   using Pre = NoPre;
+  using OutT = float;
+  static constexpr bool kTma = false;  // rows move: stored directly
+  static constexpr long split_stride = 0;
   float* out;
   long ldo;
   int Nb;
   __device__ __forceinline__ void load(int, int, Pre&) const {}
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int z) const {
+  __device__ __forceinline__ void apply(int row, int col, float* v, const Pre&, int z) const {
     (*this)(row, col, v, 32, z);
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
@@ -111,21 +117,18 @@ struct EpiShiftF {
 template <class T>
 struct EpiGateF {
   using Pre = NoPre;
-  T* G;
+  using OutT = T;
+  static constexpr bool kTma = true;
+  static constexpr long split_stride = 0;
+  T* out;
   long ldo;
   __device__ __forceinline__ void load(int, int, Pre&) const {}
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre&, int) const {
-    bf16* p = reinterpret_cast<bf16*>(G) + (long)row * ldo + col;
+  __device__ __forceinline__ void apply(int, int, float* v, const Pre&, int) const {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      float g[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) g[e] = sigmoid_bf16out(v[8 * q + e]);
-      store8(p + 8 * q, g);
-    }
+    for (int e = 0; e < 32; ++e) v[e] = sigmoid_bf16out(v[e]);
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
-    T* p = G + (long)row * ldo + col;
+    T* p = out + (long)row * ldo + col;
     float g[32];
     for (int j = 0; j < n; ++j) g[j] = sigmoidf_(v[j]);
     if (n % 8 == 0) {
@@ -144,6 +147,9 @@ struct EpiAddF {
   struct Pre {
     uint4 a[4];
   };
+  using OutT = T;
+  static constexpr bool kTma = true;
+  static constexpr long split_stride = 0;
   const T* add;
   T* out;
   long ldo;
@@ -152,16 +158,13 @@ struct EpiAddF {
 #pragma unroll
     for (int j = 0; j < 4; ++j) load8_raw(a + 8 * j, pre.a[j]);
   }
-  __device__ __forceinline__ void apply(int row, int col, const float* v, const Pre& pre,
-                                        int) const {
-    bf16* p = reinterpret_cast<bf16*>(out) + (long)row * ldo + col;
+  __device__ __forceinline__ void apply(int, int, float* v, const Pre& pre, int) const {
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      float a[8], r[8];
+      float a[8];
       unpack8(pre.a[q], a);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) r[e] = v[8 * q + e] + a[e];
-      store8(p + 8 * q, r);
+      for (int e = 0; e < 8; ++e) v[8 * q + e] += a[e];
     }
   }
   __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {

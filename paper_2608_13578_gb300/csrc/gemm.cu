@@ -11,6 +11,9 @@
 //  * gemm_simt: true-fp32 FMA, used for fp32 tensors (a TF32 tensor-core
 //    product cannot meet a 1e-4 absolute error bound).
 #include <stdio.h>
+#include <string.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "epilogues.cuh"
@@ -144,13 +147,81 @@ cudaError_t gemm_simt(const Launch& lc, int dtype, int dtype_out, int M, int N, 
 // ===================================================================== tcgen05
 namespace {
 constexpr int kBM = 128, kBK = 64;
+constexpr int kEpiWarps = 8;
+constexpr int kOutStage = 4096;  // per epilogue warp: two 32x32 bf16 or one 32x32 fp32 chunk
+
+__device__ __forceinline__ uint4 pack8_bf16(const float* v) {
+  uint4 q;
+  __nv_bfloat162 t0 = __floats2bfloat162_rn(v[0], v[1]), t1 = __floats2bfloat162_rn(v[2], v[3]);
+  __nv_bfloat162 t2 = __floats2bfloat162_rn(v[4], v[5]), t3 = __floats2bfloat162_rn(v[6], v[7]);
+  q.x = *reinterpret_cast<uint32_t*>(&t0);
+  q.y = *reinterpret_cast<uint32_t*>(&t1);
+  q.z = *reinterpret_cast<uint32_t*>(&t2);
+  q.w = *reinterpret_cast<uint32_t*>(&t3);
+  return q;
+}
+
+// Epilogue output of one warp: 32 rows (thread = row) x 32 columns, after the
+// functor's in-place transform.  TMA-stored epilogues stage the chunk in the
+// warp's shared buffer in the swizzled layout of the output tensor map (64-byte
+// swizzle for bf16 rows of 64 bytes, 128-byte swizzle for fp32 rows of 128) and
+// lane 0 stores it with one bulk copy; bf16 chunks alternate between two
+// buffers.  Other epilogues store from registers.
+// apply: this thread's row is valid; store: lane 0 issues the chunk's store
+// (rows past M are clipped by the tensor map).  Called by the whole warp.
+template <class Epi>
+__device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC, uint8_t* sbuf,
+                                          int& nout, int lane, int row, int row0, int col, int z,
+                                          float* v, const typename Epi::Pre& pre, bool apply,
+                                          bool store) {
+  if constexpr (Epi::kTma) {
+    using OT = typename Epi::OutT;
+    if (apply) epi.apply(row, col, v, pre, z);
+    constexpr bool kBf = sizeof(OT) == 2;
+    uint8_t* buf = sbuf + (kBf ? (nout & 1) * 2048 : 0);
+    if (lane == 0) {
+      if (kBf)
+        tc::tma_store_wait_read<1>();
+      else
+        tc::tma_store_wait_read<0>();
+    }
+    __syncwarp();
+    if (kBf) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        *reinterpret_cast<uint4*>(buf + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) =
+            pack8_bf16(v + 8 * u);
+    } else {
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        *reinterpret_cast<float4*>(buf + lane * 128 + ((u ^ (lane & 7)) << 4)) =
+            make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+    }
+    tc::fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0 && store) {
+      tc::tma_store_3d(mC, buf, col, row0, z);
+      tc::tma_store_commit();
+    }
+    ++nout;
+  } else {
+    (void)mC;
+    (void)sbuf;
+    (void)nout;
+    (void)row0;
+    (void)store;
+    if (apply) epi.apply(row, col, v, pre, z);
+  }
+}
 
 template <int BN, int STAGES>
 struct TcCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_BYTES = BN * kBK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr int OUT_OFF = STAGES * STAGE_BYTES;          // output staging
+  static constexpr int BAR_OFF = OUT_OFF + kEpiWarps * kOutStage;
+  static constexpr int SMEM = BAR_OFF + 1024 + 256;
   static constexpr int TMEM_COLS = 2 * BN;  // two accumulators
 };
 
@@ -178,13 +249,13 @@ constexpr int kGemmThreads = 320;
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   int M, int N, int kps, int nkb, int tiles_m, int tiles_n, int n_tiles, Epi epi,
-                   unsigned* status) {
+                   const __grid_constant__ CUtensorMap mC, int M, int N, int kps, int nkb,
+                   int tiles_m, int tiles_n, int n_tiles, Epi epi, unsigned* status) {
   using Cfg = TcCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Cfg::BAR_OFF);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;   // accumulator ready for the epilogue
   uint64_t* tempty = tfull + 2;       // accumulator drained by the epilogue
@@ -294,12 +365,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // the columns of half (w-2)/4 of the tile
     const int q = warp & 3;
     const int c_beg = ((warp - 2) >> 2) * (BN / 2);
-    int j = 0;
+    uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
+    int j = 0, nout = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++j) {
       const int m_blk = tile % tiles_m, rest = tile / tiles_m;
       const int n_blk = rest % tiles_n, z = rest / tiles_n;
       const int acc = j & 1, use = j >> 1;
-      const int row = m_blk * kBM + q * 32 + lane;
+      const int row0 = m_blk * kBM + q * 32;
+      const int row = row0 + lane;
       const int n0 = n_blk * BN;
       const bool row_ok = row < M;
       // The epilogue's own inputs do not depend on the accumulator: fetch the
@@ -316,13 +389,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
         float v[32];
         tc::tmem_ld32(base + (uint32_t)c, v);
-        if (ok && row_ok && n0 + c < N) epi.apply(row, n0 + c, v, pre[ci & 1], z);
+        if (n0 + c < N)
+          epi_chunk(epi, &mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1],
+                    ok && row_ok, ok);
       }
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&tempty[acc]);
       if (!ok) break;
     }
+    if (lane == 0) tc::tma_store_wait_all();  // output stores done before exit
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -334,6 +410,26 @@ bool g_tc_ok = true;
 }
 
 bool gemm_tc_available() { return g_tc_ok && tmap_encoder() != nullptr; }
+
+// Tensor map of an epilogue's output for its TMA stores: [splits][M][N] with
+// row stride ldo, 32 x 32 boxes (64-byte swizzle for bf16, 128-byte for fp32).
+template <class Epi>
+static bool out_map(CUtensorMap* m, const Epi& epi, int M, int N, int splits) {
+  memset(m, 0, sizeof(*m));
+  if constexpr (!Epi::kTma) {
+    return true;
+  } else {
+    using OT = typename Epi::OutT;
+    const uint64_t es = sizeof(OT);
+    const long ss = epi.split_stride > 0 ? epi.split_stride : (long)M * epi.ldo;
+    const uint64_t d[3] = {(uint64_t)N, (uint64_t)M, (uint64_t)splits};
+    const uint64_t st[2] = {(uint64_t)epi.ldo * es, (uint64_t)ss * es};
+    const uint32_t box[3] = {32, 32, 1};
+    return make_tmap(m, es == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                     epi.out, 3, d, st, box,
+                     es == 2 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
+  }
+}
 
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
 static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
@@ -370,11 +466,269 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  CUtensorMap mC;
+  if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
   const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
-  launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream,
-mA, mB, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi,
-                                            lc.status);
-  return cudaGetLastError();
+  cudaError_t e = launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream, mA, mB, mC,
+                           M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// ============================================================ CTA-pair GEMM
+// The same persistent, warp-specialised GEMM on pairs of CTAs (a cluster of
+// two): one tcgen05.mma.cta_group::2 computes a 256 x BN tile, each CTA
+// holding 128 rows of A and BN/2 of the N columns of B, so per SM a 64-deep K
+// slice brings 128x64 + (BN/2)x64 operands for a 128 x BN product: with
+// BN = 256 one and a half times the flops per byte of a single-CTA 128 x 256
+// tile, and a 32 KB stage that allows a 6-deep ring.  Both CTAs stream their
+// halves by TMA, counted on the even CTA's stage barrier; the even CTA issues
+// the MMAs and its commits arrive on the stage and accumulator barriers of
+// both CTAs; each CTA's epilogue warps drain their own 128 accumulator rows
+// and report back to the even CTA.
+template <int BN, int STAGES, int ACC>
+struct Tc2Cfg {
+  static constexpr int A_BYTES = kBM * kBK * 2;          // 16 KB
+  static constexpr int B_BYTES = (BN / 2) * kBK * 2;     // this CTA's half of B
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int OUT_OFF = STAGES * STAGE_BYTES;
+  static constexpr int BAR_OFF = OUT_OFF + kEpiWarps * kOutStage;
+  static constexpr int SMEM = BAR_OFF + 1024 + 256;
+  static constexpr int TMEM_COLS = ACC * BN;
+};
+
+template <int BN, int STAGES, int ACC, bool A_MN, bool B_MN, class Epi>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+                    const __grid_constant__ CUtensorMap mC, int M, int N, int kps, int nkb,
+                    int tiles_m, int tiles_n, int n_tiles, Epi epi, unsigned* status) {
+  using Cfg = Tc2Cfg<BN, STAGES, ACC>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Cfg::BAR_OFF);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;   // accumulator ready for the epilogue
+  uint64_t* tempty = tfull + ACC;     // accumulator drained by both CTAs' epilogues
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tempty + ACC);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = tc::cluster_rank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+  if (warp == 0 && lane == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < ACC; ++a) {
+      tc::mbar_init(&tfull[a], 1);
+      tc::mbar_init(&tempty[a], 16);  // 8 epilogue warps in each CTA
+    }
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mA);
+    tc::prefetch_tmap(&mB);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc_pair(tslot, Cfg::TMEM_COLS);
+    tc::tmem_relinquish_pair();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrive
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  pdl_enter();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer (both CTAs): this CTA's rows of A and half of B
+      int it = 0;
+      bool ok = true;
+      for (int tile = pair; tile < n_tiles && ok; tile += npairs) {
+        const int m_blk = tile % tiles_m, rest = tile / tiles_m;
+        const int n_blk = rest % tiles_n, z = rest / tiles_n;
+        const int m0 = m_blk * 2 * kBM + (int)rank * kBM;
+        const int n0 = n_blk * BN + (int)rank * (BN / 2);
+        const int kb0 = z * kps;
+        const int nk = min(nkb, kb0 + kps) - kb0;
+        for (int i = 0; i < nk; ++i, ++it) {
+          const int s = it % STAGES;
+          if (it >= STAGES && !tc::mbar_wait(&empty[s], ((it / STAGES) - 1) & 1, status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + s * Cfg::STAGE_BYTES;
+          uint8_t* sb = sa + Cfg::A_BYTES;
+          const uint32_t fb = tc::mapa(tc::smem_u32(&full[s]), 0);
+          if (rank == 0) tc::mbar_arrive_expect_tx(&full[s], 2 * Cfg::STAGE_BYTES);
+          const int k0 = (kb0 + i) * kBK;
+          if (!A_MN) {
+            tc::tma_load_2d_pair(sa, &mA, fb, k0, m0);
+          } else {
+            tc::tma_load_2d_pair(sa, &mA, fb, m0, k0);
+            tc::tma_load_2d_pair(sa + 8192, &mA, fb, m0 + 64, k0);
+          }
+          if (!B_MN) {
+            tc::tma_load_2d_pair(sb, &mB, fb, k0, n0);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 128; ++j)
+              tc::tma_load_2d_pair(sb + j * 8192, &mB, fb, n0 + 64 * j, k0);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---- MMA issuer (even CTA only)
+      constexpr uint32_t idesc = tc::idesc_bf16(2 * kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+      int it = 0, j = 0;
+      bool ok = true;
+      for (int tile = pair; tile < n_tiles && ok; tile += npairs, ++j) {
+        const int z = (tile / tiles_m) / tiles_n;
+        const int kb0 = z * kps, nk = min(nkb, kb0 + kps) - kb0;
+        const int acc = j % ACC, use = j / ACC;
+        if (use > 0 && !tc::mbar_wait_cluster(&tempty[acc], (use - 1) & 1, status)) break;
+        tc::fence_after_sync();
+        const uint32_t d = tmem + (uint32_t)(acc * BN);
+        for (int i = 0; i < nk; ++i, ++it) {
+          const int s = it % STAGES;
+          if (!tc::mbar_wait_cluster(&full[s], (it / STAGES) & 1, status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE_BYTES);
+          const uint32_t sb = sa + Cfg::A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024)
+                                     : tc::sdesc(sa + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024)
+                                     : tc::sdesc(sb + kk * 32, 16, 1024);
+            tc::mma_bf16_pair(d, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
+          }
+          tc::mma_commit_pair(&empty[s]);
+        }
+        tc::mma_commit_pair(&tfull[acc]);
+      }
+    }
+  } else {
+    // ---- epilogue warps 2..9 (both CTAs): this CTA's 128 accumulator rows
+    const int q = warp & 3;
+    const int c_beg = ((warp - 2) >> 2) * (BN / 2);
+    const uint32_t te0 = tc::mapa(tc::smem_u32(&tempty[0]), 0);
+    uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
+    int j = 0, nout = 0;
+    for (int tile = pair; tile < n_tiles; tile += npairs, ++j) {
+      const int m_blk = tile % tiles_m, rest = tile / tiles_m;
+      const int n_blk = rest % tiles_n, z = rest / tiles_n;
+      const int acc = j % ACC, use = j / ACC;
+      const int row0 = m_blk * 2 * kBM + (int)rank * kBM + q * 32;
+      const int row = row0 + lane;
+      const int n0 = n_blk * BN;
+      const bool row_ok = row < M;
+      constexpr int NCH = BN / 64;
+      typename Epi::Pre pre[2];
+      if (row_ok && n0 + c_beg < N) epi.load(row, n0 + c_beg, pre[0]);
+      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
+      tc::fence_after_sync();
+      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll
+      for (int ci = 0; ci < NCH; ++ci) {
+        const int c = c_beg + ci * 32;
+        if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
+        float v[32];
+        tc::tmem_ld32(base + (uint32_t)c, v);
+        if (n0 + c < N)
+          epi_chunk(epi, &mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1],
+                    ok && row_ok, ok);
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive_cluster(te0 + (uint32_t)(acc * 8));
+      if (!ok) break;
+    }
+    if (lane == 0) tc::tma_store_wait_all();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::cluster_sync();  // the peer no longer reads this CTA's shared memory or TMEM
+  tc::fence_after_sync();
+  if (warp == 1) tc::tmem_dealloc_pair(tmem, Cfg::TMEM_COLS);
+}
+
+template <int BN, int STAGES, int ACC, bool A_MN, bool B_MN, class Epi>
+static cudaError_t tc2_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                              long sak, const void* B, long sbk, long sbn, const Epi& epi,
+                              int splits) {
+  using Cfg = Tc2Cfg<BN, STAGES, ACC>;
+  CUtensorMap mA, mB;
+  if (!A_MN) {
+    uint64_t d[2] = {(uint64_t)K, (uint64_t)M}, st[1] = {(uint64_t)sam * 2};
+    uint32_t box[2] = {64, 128};
+    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+  } else {
+    uint64_t d[2] = {(uint64_t)M, (uint64_t)K}, st[1] = {(uint64_t)sak * 2};
+    uint32_t box[2] = {64, 64};
+    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+  }
+  if (!B_MN) {
+    uint64_t d[2] = {(uint64_t)K, (uint64_t)N}, st[1] = {(uint64_t)sbn * 2};
+    uint32_t box[2] = {64, (uint32_t)(BN / 2)};
+    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+  } else {
+    uint64_t d[2] = {(uint64_t)N, (uint64_t)K}, st[1] = {(uint64_t)sbk * 2};
+    uint32_t box[2] = {64, 64};
+    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+  }
+  const int nkb = (K + kBK - 1) / kBK;
+  const int kps = (nkb + splits - 1) / splits;
+  const int tiles_m = (M + 2 * kBM - 1) / (2 * kBM), tiles_n = (N + BN - 1) / BN;
+  const int n_tiles = tiles_m * tiles_n * splits;
+  auto kern = gemm_tc2_kernel<BN, STAGES, ACC, A_MN, B_MN, Epi>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  CUtensorMap mC;
+  if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
+  const int pairs = n_tiles < sm_count() / 2 ? n_tiles : sm_count() / 2;
+  cudaError_t e = launch_k_cluster(kern, dim3(2 * pairs), dim3(kGemmThreads), Cfg::SMEM,
+                                   lc.stream, 2, mA, mB, mC, M, N, kps, nkb, tiles_m, tiles_n,
+                                   n_tiles, epi, lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Test path: the CTA-pair kernel with 256 x 256 tiles (plain and split-K stores).
+cudaError_t gemm_tc_pair(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
+                         long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
+                         const EpiArgs& ea, int splits) {
+  if (N % 256 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
+  splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
+  const bool a_k = (sak == 1), b_k = (sbk == 1);
+  constexpr int ST = 6, ACC = 2;
+  auto go = [&](auto am, auto bm) -> cudaError_t {
+    constexpr bool AM = decltype(am)::value, BM = decltype(bm)::value;
+    if (epi == EPI_PARTIAL)
+      return tc2_launch<256, ST, ACC, AM, BM>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                              EpiStoreF<float>{(float*)ea.out, ea.ldo, ea.split_stride},
+                                              splits);
+    if (dtype_out == 0)
+      return tc2_launch<256, ST, ACC, AM, BM>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                              EpiStoreF<float>{(float*)ea.out, ea.ldo, 0}, 1);
+    return tc2_launch<256, ST, ACC, AM, BM>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
+                                            EpiStoreF<bf16>{(bf16*)ea.out, ea.ldo, 0}, 1);
+  };
+  using F = std::false_type;
+  using T = std::true_type;
+  // B_MN: B is N-contiguous (not K-major)
+  if (a_k && !b_k) return go(F{}, T{});
+  if (a_k && b_k) return go(F{}, F{});
+  if (!a_k && !b_k) return go(T{}, T{});
+  return go(T{}, F{});
 }
 
 // Output tile widths: 128 x 256 tiles move 48 KB per 64-deep K slice for

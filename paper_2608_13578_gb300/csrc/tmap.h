@@ -30,9 +30,18 @@ inline PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
 // box[0] x box[1] (x box[2]) elements; 128-byte swizzle unless given (the
 // box's inner extent in bytes must not exceed the swizzle span), zero fill
 // outside.
+inline bool make_tmap(CUtensorMap* m, CUtensorMapDataType dt, const void* base, int rank,
+                      const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+                      CUtensorMapSwizzle swz);
 inline bool make_tmap_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                            const uint64_t* strides_bytes, const uint32_t* box,
                            CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
+  return make_tmap(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, rank, dims, strides_bytes, box, swz);
+}
+// Any element type (rank 2 or 3, as above).
+inline bool make_tmap(CUtensorMap* m, CUtensorMapDataType dt, const void* base, int rank,
+                      const uint64_t* dims, const uint64_t* strides_bytes, const uint32_t* box,
+                      CUtensorMapSwizzle swz) {
   auto enc = tmap_encoder();
   if (!enc) return false;
   cuuint64_t gd[3], gs[2];
@@ -42,7 +51,7 @@ inline bool make_tmap_bf16(CUtensorMap* m, const void* base, int rank, const uin
     bx[i] = box[i];
   }
   for (int i = 0; i < rank - 1; ++i) gs[i] = strides_bytes[i];
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base),
+  CUresult r = enc(m, dt, (cuuint32_t)rank, const_cast<void*>(base),
                    gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;

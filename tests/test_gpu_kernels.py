@@ -178,3 +178,39 @@ def test_attention_fwd_bwd(C, impl, B, T, H, dh, L, dtype):
     chk("dq", dq, ref_dq)
     chk("dk", dk, ref_dk)
     chk("dv", dv, ref_dv)
+
+
+PAIR_SHAPES = [(256, 256, 64), (1000, 512, 320), (4096, 1536, 512), (77, 256, 1536),
+               (4000, 768, 200), (520, 256, 64)]
+
+
+@pytest.mark.parametrize("la,lb", LAYOUTS)
+@pytest.mark.parametrize("M,N,K", PAIR_SHAPES)
+def test_gemm_cta_pair(C, la, lb, M, N, K):
+    """The CTA-pair (cta_group::2) GEMM against a float64 product."""
+    gen = torch.Generator().manual_seed(M * 5 + N + K)
+    dt = torch.bfloat16
+    A, sam, sak, Al = _operand(M, K, la == "k", dt, gen)
+    B, sbk, sbn, Bl = _operand(K, N, lb == "n", dt, gen)
+    ref = Al.double() @ Bl.double()
+    Ad, Bd = A.cuda(), B.cuda()
+    for dto, tol in ((0, 1e-5), (1, 8e-3)):
+        Cd = torch.full((M, N), float("nan"), dtype=torch.float32 if dto == 0 else dt, device="cuda")
+        C.bcmt_test_gemm(2, 1, dto, M, N, K, Ad, sam, sak, Bd, sbk, sbn, Cd, N)
+        C.bcmt_device_status()
+        torch.cuda.synchronize()
+        err = (Cd.double().cpu() - ref).abs().max().item() / ref.abs().max().item()
+        assert err < tol, (dto, err)
+
+
+def test_gemm_cta_pair_split_k(C):
+    M, N, K, splits = 512, 256, 4096, 6
+    gen = torch.Generator().manual_seed(6)
+    A, sam, sak, Al = _operand(M, K, False, torch.bfloat16, gen)
+    B, sbk, sbn, Bl = _operand(K, N, True, torch.bfloat16, gen)
+    part = torch.full((splits, M, N), float("nan"), dtype=torch.float32, device="cuda")
+    n = C.bcmt_test_gemm(2, 1, 0, M, N, K, A.cuda(), sam, sak, B.cuda(), sbk, sbn, part, N, splits)
+    torch.cuda.synchronize()
+    got = part[:n].double().sum(0).cpu()
+    ref = Al.double() @ Bl.double()
+    assert (got - ref).abs().max().item() / ref.abs().max().item() < 1e-5
