@@ -57,10 +57,14 @@ unsigned* status_ptr() {
 // (forked and joined with events, so the pair can also be captured into a
 // CUDA graph).  Streams and events are host-side objects: no device memory.
 constexpr int kSideEvents = 12;
+// Per device: the layer's critical path runs on `crit` (the highest stream
+// priority) and the work beside it (memory stage in the forward, weight
+// gradients in the backward) on `side` (the lowest), so that when both have
+// CTAs waiting the block scheduler places the critical ones first.
 struct SideStream {
-  cudaStream_t s = nullptr;
+  cudaStream_t crit = nullptr, side = nullptr;
   cudaEvent_t ev[kSideEvents] = {};
-  std::mutex mu;  // one call at a time may use the events
+  std::mutex mu;  // one call at a time may use the streams' events
 };
 
 SideStream* side_stream() {
@@ -72,11 +76,15 @@ SideStream* side_stream() {
   if ((int)per_dev.size() <= dev) per_dev.resize(dev + 1, nullptr);
   if (!per_dev[dev]) {
     SideStream* ss = new SideStream();
-    bool ok = cudaStreamCreateWithFlags(&ss->s, cudaStreamNonBlocking) == cudaSuccess;
+    int least = 0, greatest = 0;
+    bool ok = cudaDeviceGetStreamPriorityRange(&least, &greatest) == cudaSuccess &&
+              cudaStreamCreateWithPriority(&ss->crit, cudaStreamNonBlocking, greatest) ==
+                  cudaSuccess &&
+              cudaStreamCreateWithPriority(&ss->side, cudaStreamNonBlocking, least) == cudaSuccess;
     for (int i = 0; i < kSideEvents && ok; ++i)
       ok = cudaEventCreateWithFlags(&ss->ev[i], cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
-      delete ss;  // fall back to one stream
+      delete ss;  // fall back to the caller's stream alone
       return nullptr;
     }
     per_dev[dev] = ss;
@@ -84,43 +92,53 @@ SideStream* side_stream() {
   return per_dev[dev];
 }
 
-// Fork/join of the side stream for one call; joins on destruction so every
-// return path leaves the side stream merged back into the caller's stream.
+// Fork/join of one call: the critical stream starts after everything the
+// caller has enqueued, the side stream forks from it at point(), and on
+// destruction (every return path) both are joined back into the caller's
+// stream.  Plain event record/wait, so a CUDA graph capture of the caller's
+// stream captures all three.  Without a SideStream everything stays on the
+// caller's stream.
 struct Fork {
   SideStream* ss;
-  cudaStream_t main;
+  cudaStream_t user;
   int next = 0;
   bool forked = false;
-  Fork(SideStream* side, cudaStream_t m) : ss(side), main(m) {
-    if (ss) ss->mu.lock();
+  Fork(SideStream* s, cudaStream_t u) : ss(s), user(u) {
+    if (!ss) return;
+    ss->mu.lock();
+    cudaEventRecord(ss->ev[next], user);
+    cudaStreamWaitEvent(ss->crit, ss->ev[next], 0);
+    ++next;
   }
-  cudaStream_t side() const { return ss ? ss->s : main; }
-  // the side stream waits for everything enqueued on the main stream so far
-  // (false when the events are used up: the caller then stays on one stream)
+  cudaStream_t main() const { return ss ? ss->crit : user; }
+  cudaStream_t side() const { return ss ? ss->side : user; }
+  // the side stream waits for everything enqueued on the critical stream so far
   bool point() {
-    if (!ss || next >= kSideEvents - 1) return false;
-    cudaEventRecord(ss->ev[next], main);
-    cudaStreamWaitEvent(ss->s, ss->ev[next], 0);
+    if (!ss || next >= kSideEvents - 2) return false;
+    cudaEventRecord(ss->ev[next], ss->crit);
+    cudaStreamWaitEvent(ss->side, ss->ev[next], 0);
     ++next;
     forked = true;
     return true;
   }
   // records what the side stream has been given so far; wait_mark(m) later
-  // makes the main stream wait for exactly that
+  // makes the critical stream wait for exactly that
   int mark() {
-    if (!ss || !forked || next >= kSideEvents - 1) return -1;
-    cudaEventRecord(ss->ev[next], ss->s);
+    if (!ss || !forked || next >= kSideEvents - 2) return -1;
+    cudaEventRecord(ss->ev[next], ss->side);
     return next++;
   }
   void wait_mark(int m) {
-    if (ss && m >= 0) cudaStreamWaitEvent(main, ss->ev[m], 0);
+    if (ss && m >= 0) cudaStreamWaitEvent(ss->crit, ss->ev[m], 0);
   }
   ~Fork() {
     if (!ss) return;
     if (forked) {
-      cudaEventRecord(ss->ev[kSideEvents - 1], ss->s);
-      cudaStreamWaitEvent(main, ss->ev[kSideEvents - 1], 0);
+      cudaEventRecord(ss->ev[kSideEvents - 2], ss->side);
+      cudaStreamWaitEvent(ss->crit, ss->ev[kSideEvents - 2], 0);
     }
+    cudaEventRecord(ss->ev[kSideEvents - 1], ss->crit);
+    cudaStreamWaitEvent(user, ss->ev[kSideEvents - 1], 0);
     ss->mu.unlock();
   }
 };
@@ -222,13 +240,26 @@ struct Geometry {
         honly((p->flags & BCMT_FLAG_HONLY) != 0), from_x(p->input_is_x != 0), dtype(p->dtype) {}
 };
 
-// K-split count of a weight-gradient GEMM [M x N], K = tokens: about one
-// wave of 128 x 128 tiles on the GPU.
-int dw_splits(int M, int N, long K) {
-  const int tiles = ((M + 127) / 128) * ((N + 127) / 128);
-  int s = std::max(1, 148 / std::max(1, tiles));
+// Weight gradients dW[M,N] = A^T B over K = tokens run on the CTA-pair GEMM
+// (256 x 256 tiles) when both sides are multiples of 256, else on 128-wide
+// tiles.  K is split so that the tiles x splits fill about two thirds of the
+// GPU (the rest stays free for the critical path beside them), with at least
+// 8 K slices per split.
+bool dw_pair(int dtype, int M, int N) {
+  return dtype == BCMT_BF16 && g_use_tc_gemm && M % 256 == 0 && N % 256 == 0;
+}
+int dw_splits(int dtype, int M, int N, long K) {
   const int nkb = (int)((K + 63) / 64);
-  return std::min(s, nkb);
+  int target, tiles;
+  if (dw_pair(dtype, M, N)) {
+    tiles = (M / 256) * (N / 256);
+    target = 50;  // pairs: 100 of the 152 SMs
+  } else {
+    tiles = ((M + 127) / 128) * ((N + 127) / 128);
+    target = 100;
+  }
+  int s = std::max(1, target / std::max(1, tiles));
+  return std::max(1, std::min(s, nkb / 8));
 }
 
 struct FwdWs {
@@ -301,8 +332,9 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
   w.dHhat = take((size_t)g.n * g.D * g.es);
   w.dqkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
   w.Drow = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
-  size_t part = (size_t)dw_splits(g.D, g.D, g.n) * g.D * g.D * 4;
-  if (g.from_x) part = std::max(part, (size_t)dw_splits(g.D, 3 * g.D, g.n) * g.D * 3 * g.D * 4);
+  size_t part = (size_t)dw_splits(g.dtype, g.D, g.D, g.n) * g.D * g.D * 4;
+  if (g.from_x)
+    part = std::max(part, (size_t)dw_splits(g.dtype, g.D, 3 * g.D, g.n) * g.D * 3 * g.D * 4);
   w.part = reinterpret_cast<float*>(take(part));
   w.bytes = off;
   return w;
@@ -317,16 +349,18 @@ bcmt_status cuda_fail(cudaError_t e, const char* what) {
 cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype, int dtype_out,
                         int M, int N, long K,
                         const void* A, long lda, const void* B, long ldb, float* part, void* out) {
-  const int splits = dw_splits(M, N, K);
+  const int splits = dw_splits(dtype, M, N, K);
   EpiArgs ea;
   ea.out = part;
   ea.ldo = N;
   ea.split_stride = (long)M * N;
   pr.begin(name);
-  cudaError_t e = (dtype == 1 && g_use_tc_gemm)
-                      ? gemm_tc(lc, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits)
-                      : gemm_simt(lc, dtype, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea,
-                                  splits);
+  cudaError_t e =
+      dw_pair(dtype, M, N)
+          ? gemm_tc_pair(lc, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits)
+      : (dtype == 1 && g_use_tc_gemm)
+          ? gemm_tc(lc, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits)
+          : gemm_simt(lc, dtype, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits);
   pr.end(nullptr);
   if (e != cudaSuccess) return e;
   pr.begin("reduce_splits");
@@ -424,13 +458,12 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool profiling = (p->flags & BCMT_FLAG_PROFILE) != 0;
-  Launch lc{s, sp};
-  Prof pr{profiling, s};
   // The memory stage runs on the side stream beside the gate GEMM (one
   // stream while profiling).
-  std::unique_ptr<Fork> fork_holder(
-      new Fork(profiling || g.honly ? nullptr : side_stream(), s));
+  std::unique_ptr<Fork> fork_holder(new Fork(profiling ? nullptr : side_stream(), s));
   Fork& fork = *fork_holder;
+  Launch lc{fork.main(), sp};
+  Prof pr{profiling, fork.main()};
   Launch lcs{fork.side(), sp};
   Prof prs{profiling, fork.side()};
   FwdWs w = fwd_layout(g, workspace);
@@ -560,12 +593,12 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   if (!sp) return fail(BCMT_ERR_CUDA, "no CUDA device / device status word unavailable");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool profiling = (p->flags & BCMT_FLAG_PROFILE) != 0;
-  Launch lc{s, sp};
-  Prof pr{profiling, s};
   // Weight gradients go to the side stream (kept on one stream while
   // profiling, so every kernel is timed alone).
   std::unique_ptr<Fork> fork_holder(new Fork(profiling ? nullptr : side_stream(), s));
   Fork& fork = *fork_holder;
+  Launch lc{fork.main(), sp};
+  Prof pr{profiling, fork.main()};
   Launch lcs{fork.side(), sp};
   Prof prs{profiling, fork.side()};
   FwdWs w = fwd_layout(g, const_cast<void*>(workspace));
