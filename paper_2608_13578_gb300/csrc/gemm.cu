@@ -803,6 +803,10 @@ cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const 
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits) {
   if (N % 64 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
+  // long K: the CTA-pair kernel's 256 x 256 tiles need 2/3 of the operand
+  // bytes per flop of a single CTA's 128 x 256 tile
+  if (epi == EPI_STORE && N % 256 == 0 && M >= 512 && K >= 1024)
+    return gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
   splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
   const bool a_k = (sak == 1), a_m = (sam == 1) && !a_k;
   const bool b_k = (sbk == 1), b_n = (sbn == 1) && !b_k;
