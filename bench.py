@@ -187,9 +187,12 @@ def kernel_model(w):
         # read Q, K, V; write Concat(heads) and the log-sum-exp
         "attn_fwd_tc": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
         "attn_fwd_simt": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
+        "attn_fwd_fl": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
         # read Q, K, V, dO, O and the log-sum-exp; write dQ, dK, dV
         "attn_bwd_tc": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
         "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
+        # two kernels (dQ, then dK/dV); the row dot products Drow are written and re-read
+        "attn_bwd_fl": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es + 2 * n * H * 4),
         # Sec. 3.4 summaries: read H and the score partials, write alpha and S
         "summary_fwd": ("hbm", n * D * es + n * 4 * npart + n * 4 + B * Nb * D * 4),
         # Sec. 3.5 scan: read S, write M (fp32 and the bf16 operand copy), Z, C[:, 0]

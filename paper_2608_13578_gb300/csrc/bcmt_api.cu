@@ -240,11 +240,23 @@ struct Geometry {
         honly((p->flags & BCMT_FLAG_HONLY) != 0), from_x(p->input_is_x != 0), dtype(p->dtype) {}
 };
 
+int device_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 2)
+      n = 148;
+  }
+  return n;
+}
+
 // Weight gradients dW[M,N] = A^T B over K = tokens run on the CTA-pair GEMM
 // (256 x 256 tiles) when both sides are multiples of 256, else on 128-wide
-// tiles.  K is split so that the tiles x splits fill about two thirds of the
-// GPU (the rest stays free for the critical path beside them), with at least
-// 8 K slices per split.
+// tiles, with K split into ranges of at least 8 slices.  A large product
+// (at least 8 pair tiles: dW_qkv, the step's last GEMM) is split to fill one
+// round of CTA pairs; the D x D ones are split to about 50 pairs (at most 12
+// splits), leaving SMs to the critical path beside them.
 bool dw_pair(int dtype, int M, int N) {
   return dtype == BCMT_BF16 && g_use_tc_gemm && M % 256 == 0 && N % 256 == 0;
 }
@@ -253,7 +265,7 @@ int dw_splits(int dtype, int M, int N, long K) {
   int target, tiles;
   if (dw_pair(dtype, M, N)) {
     tiles = (M / 256) * (N / 256);
-    target = 50;  // pairs: 100 of the 152 SMs
+    target = tiles >= 8 ? device_sms() / 2 : std::min(50, 12 * tiles);
   } else {
     tiles = ((M + 127) / 128) * ((N + 127) / 128);
     target = 100;
