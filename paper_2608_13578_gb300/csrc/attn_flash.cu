@@ -86,6 +86,10 @@ __device__ __forceinline__ void key_walk(int t0, int L, int& kstart, int& nkt) {
 }  // namespace
 
 // ====================================================================== forward
+// Pipelined over the key tiles: K is double-buffered, so the score product of
+// tile kt+1 is issued as soon as every thread has read tile kt's scores out of
+// TMEM and runs under tile kt's softmax; K of tile kt+2 streams in meanwhile.
+// V (single buffer) is reloaded once tile kt's P V product has completed.
 template <int DH>
 __global__ void __launch_bounds__(128)
     attn_fwd_fl_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
@@ -97,10 +101,15 @@ __global__ void __launch_bounds__(128)
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sP = smem;                       // 32 KB: P [128 queries x 128 keys]
   uint8_t* sQ = smem + 32768;
-  uint8_t* sK = sQ + G::tile;
-  uint8_t* sV = sK + G::tile;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);  // kv, s, o
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
+  uint8_t* sK0 = sQ + G::tile;              // K, two buffers
+  uint8_t* sV = sK0 + 2 * G::tile;
+  // barriers: K buffer 0/1 loaded (buffer 0 also counts Q), V loaded, S ready, P V done
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);
+  uint64_t* bar_k = bar;
+  uint64_t* bar_v = bar + 2;
+  uint64_t* bar_s = bar + 3;
+  uint64_t* bar_o = bar + 4;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 5);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
@@ -108,7 +117,7 @@ __global__ void __launch_bounds__(128)
   key_walk(t0, L, kstart, nkt);
 
   if (tid == 0) {
-    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    for (int i = 0; i < 5; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
     tc::prefetch_tmap(&mQ);
     tc::prefetch_tmap(&mK);
@@ -116,10 +125,15 @@ __global__ void __launch_bounds__(128)
   }
   pdl_enter();
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 3 * G::tile);
-    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
-    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart, b);
-    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart, b);
+    tc::mbar_arrive_expect_tx(&bar_k[0], 2 * G::tile);
+    tc::tma_load_3d(sQ, &mQ, &bar_k[0], h * DH, t0, b);
+    tc::tma_load_3d(sK0, &mK, &bar_k[0], h * DH, kstart, b);
+    tc::mbar_arrive_expect_tx(bar_v, G::tile);
+    tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart, b);
+    if (nkt > 1) {
+      tc::mbar_arrive_expect_tx(&bar_k[1], G::tile);
+      tc::tma_load_3d(sK0 + G::tile, &mK, &bar_k[1], h * DH, kstart + kTile, b);
+    }
   }
   __syncwarp();
   if (warp == 0) {
@@ -131,6 +145,20 @@ __global__ void __launch_bounds__(128)
   tc::fence_after_sync();
   const uint32_t tmem = *tslot;
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  constexpr uint32_t idS = tc::idesc_bf16(128, 128, 0, 0);
+  constexpr uint32_t idO = tc::idesc_bf16(128, DH, 0, 1);
+
+  if (tid == 0) {  // S of the first key tile
+    const bool okk = tc::mbar_wait(&bar_k[0], 0, status);
+    tc::fence_after_sync();
+    if (okk) {
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)
+        tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK0, 0, kk), idS, kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(bar_s);
+  }
+  __syncwarp();
 
   const int r = warp * 32 + lane;
   const float sl2 = scale * kLog2e;
@@ -142,22 +170,10 @@ __global__ void __launch_bounds__(128)
 
   for (int kt = 0; kt < nkt; ++kt) {
     const bool diag = kt == nkt - 1;
-    if (tid == 0) {
-      const bool okk = tc::mbar_wait(&bar[0], kt & 1, status);
-      tc::fence_after_sync();
-      if (okk) {
-        constexpr uint32_t idS = tc::idesc_bf16(128, 128, 0, 0);
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk)
-          tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 0, kk), idS, kk > 0 ? 1u : 0u);
-      }
-      tc::mma_commit(&bar[1]);
-    }
-    __syncwarp();
-    ok = tc::mbar_wait(&bar[1], kt & 1, status) && ok;
+    ok = tc::mbar_wait(bar_s, kt & 1, status) && ok;
     tc::fence_after_sync();
 
-    // ---- online softmax of this key tile (thread = query row r)
+    // ---- this tile's scores out of TMEM (thread = query row r)
     int wbs = 0, nld = 4, rbs = 0;
     if (diag) {
       if (L < kTile) {
@@ -171,6 +187,30 @@ __global__ void __launch_bounds__(128)
     for (int ci = 0; ci < 4; ++ci)
       if (ci < nld) tc::tmem_ld32_issue(trow + (uint32_t)(wbs + ci * 32), sr[ci]);
     tc::tmem_wait();
+    tc::fence_before_sync();
+    __syncthreads();  // every thread has its scores: the S columns are free
+    if (tid == 0) {
+      tc::fence_after_sync();
+      if (kt + 1 < nkt) {  // next tile's scores, under this tile's softmax
+        const int nb = (kt + 1) & 1;
+        const bool okk = tc::mbar_wait(&bar_k[nb], ((kt + 1) >> 1) & 1, status);
+        tc::fence_after_sync();
+        if (okk) {
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)
+            tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK0 + nb * G::tile, 0, kk), idS,
+                         kk > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(bar_s);
+      }
+      if (kt + 2 < nkt) {  // K buffer kt & 1 was read by tile kt's (completed) product
+        const int cb = kt & 1;
+        tc::mbar_arrive_expect_tx(&bar_k[cb], G::tile);
+        tc::tma_load_3d(sK0 + cb * G::tile, &mK, &bar_k[cb], h * DH, kstart + (kt + 2) * kTile, b);
+      }
+    }
+
+    // ---- online softmax (P to shared memory; the previous P V has completed)
     float mt = -INFINITY;
 #pragma unroll
     for (int ci = 0; ci < 4; ++ci)
@@ -210,21 +250,22 @@ __global__ void __launch_bounds__(128)
 
     if (tid == 0) {
       tc::fence_after_sync();
-      constexpr uint32_t idO = tc::idesc_bf16(128, DH, 0, 1);
+      const bool okv = tc::mbar_wait(bar_v, kt & 1, status);
+      tc::fence_after_sync();
+      if (okv) {
 #pragma unroll
-      for (int kk = 0; kk < kTile / 16; ++kk)
-        tc::mma_bf16(tmem + 128, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
-      tc::mma_commit(&bar[2]);
+        for (int kk = 0; kk < kTile / 16; ++kk)
+          tc::mma_bf16(tmem + 128, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
+      }
+      tc::mma_commit(bar_o);
     }
     __syncwarp();
-    ok = tc::mbar_wait(&bar[2], kt & 1, status) && ok;
+    ok = tc::mbar_wait(bar_o, kt & 1, status) && ok;
     tc::fence_after_sync();
-    // K, V and P are free: fetch the next key tile while this one's P V is
-    // folded into the accumulator
+    // V and P are free: fetch the next tile's V while this P V is folded in
     if (tid == 0 && kt + 1 < nkt) {
-      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
-      tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
-      tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      tc::mbar_arrive_expect_tx(bar_v, G::tile);
+      tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart + (kt + 1) * kTile, b);
     }
     float o[DH];
     tmem_row<DH>(trow + 128u, o);
@@ -586,7 +627,7 @@ bool head_map_fl(CUtensorMap* m, const void* base, long ld, int D, int T, int B)
 }
 
 // dynamic shared memory: 1 KB alignment slack + tiles + staging + barriers
-template <int DH> constexpr int fwd_smem() { return 1024 + 32768 + 3 * Geo<DH>::tile + 64; }
+template <int DH> constexpr int fwd_smem() { return 1024 + 32768 + 4 * Geo<DH>::tile + 64; }
 template <int DH> constexpr int dq_smem() { return 1024 + 16384 + 4 * Geo<DH>::tile + 64; }
 template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
