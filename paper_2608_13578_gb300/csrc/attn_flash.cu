@@ -633,14 +633,6 @@ template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
 }
 
-template <class K>
-cudaError_t opt_in(K* kern, int bytes, bool* done) {
-  if (*done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e == cudaSuccess) *done = true;
-  return e;
-}
-
 template <int DH>
 cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
   const int D = a.H * DH;
@@ -649,8 +641,8 @@ cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
       !head_map_fl<DH>(&mk, a.K, a.ld_qkv, D, a.T, a.B) ||
       !head_map_fl<DH>(&mv, a.V, a.ld_qkv, D, a.T, a.B))
     return cudaErrorInvalidValue;
-  static bool attr = false;
-  cudaError_t e = opt_in(attn_fwd_fl_kernel<DH>, fwd_smem<DH>(), &attr);
+  static std::atomic<unsigned long long> opted{0};
+  cudaError_t e = smem_opt_in(attn_fwd_fl_kernel<DH>, fwd_smem<DH>(), &opted);
   if (e != cudaSuccess) return e;
   dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
   e = launch_k(attn_fwd_fl_kernel<DH>, grid, dim3(128), fwd_smem<DH>(), lc.stream, mq, mk, mv,
@@ -668,9 +660,9 @@ cudaError_t bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
       !head_map_fl<DH>(&mv, f.V, f.ld_qkv, D, f.T, f.B) ||
       !head_map_fl<DH>(&mdo, a.dO, f.ld_o, D, f.T, f.B))
     return cudaErrorInvalidValue;
-  static bool attr_q = false, attr_kv = false;
-  cudaError_t e = opt_in(attn_bwd_dq_fl_kernel<DH>, dq_smem<DH>(), &attr_q);
-  if (e == cudaSuccess) e = opt_in(attn_bwd_dkv_fl_kernel<DH>, dkv_smem<DH>(), &attr_kv);
+  static std::atomic<unsigned long long> opted_q{0}, opted_kv{0};
+  cudaError_t e = smem_opt_in(attn_bwd_dq_fl_kernel<DH>, dq_smem<DH>(), &opted_q);
+  if (e == cudaSuccess) e = smem_opt_in(attn_bwd_dkv_fl_kernel<DH>, dkv_smem<DH>(), &opted_kv);
   if (e != cudaSuccess) return e;
   const float scale = 1.0f / sqrtf((float)DH);
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);

@@ -441,19 +441,10 @@ static constexpr int kBwdSmem = 5 * kTB + 1024 + 64;
 
 static int chunks_for(int L) { return L <= 32 ? 1 : L / 32; }
 
-template <class K>
-static cudaError_t opt_in(K* kern, int bytes) {
-  return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-}
-
 template <int NCH>
 static cudaError_t fwd_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = opt_in(attn_fwd_tc_kernel<NCH>, kFwdSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  static std::atomic<unsigned long long> opted{0};
+  if (cudaError_t e = smem_opt_in(attn_fwd_tc_kernel<NCH>, kFwdSmem, &opted); e != cudaSuccess) return e;
   dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
   cudaError_t e = launch_k(attn_fwd_tc_kernel<NCH>, grid, dim3(128), kFwdSmem, lc.stream, m[0],
                            m[1], m[2], m[3], a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)a.dh),
@@ -478,12 +469,8 @@ cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
 template <int NCH>
 static cudaError_t bwd_launch(const Launch& lc, const AttnBwdArgs& a, const CUtensorMap* m) {
   const AttnArgs& f = a.f;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = opt_in(attn_bwd_tc_kernel<NCH>, kBwdSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  static std::atomic<unsigned long long> opted{0};
+  if (cudaError_t e = smem_opt_in(attn_bwd_tc_kernel<NCH>, kBwdSmem, &opted); e != cudaSuccess) return e;
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
   cudaError_t e = launch_k(attn_bwd_tc_kernel<NCH>, grid, dim3(128), kBwdSmem, lc.stream, m[0],
                            m[1], m[2], m[3], m[4], m[5], m[6], (const bf16*)f.O, f.ld_o, f.lse,

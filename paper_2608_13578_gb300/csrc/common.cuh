@@ -2,6 +2,8 @@
 // reductions, and the status bits a kernel sets when a bounded wait expires.
 #pragma once
 
+#include <atomic>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -52,6 +54,22 @@ inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, siz
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// Raises `kern`'s dynamic shared memory limit to `bytes` on the current device,
+// once per device (function attributes belong to a device's context): `done`
+// is the call site's bit set of devices already configured.
+template <typename... KArgs>
+inline cudaError_t smem_opt_in(void (*kern)(KArgs...), int bytes,
+                               std::atomic<unsigned long long>* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (done->load() & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done->fetch_or(bit);
+  return e;
 }
 
 // The same with thread-block clusters of `cluster_x` CTAs along x.

@@ -460,12 +460,8 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
   const int n_tiles = tiles_m * tiles_n * splits;
   auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static std::atomic<unsigned long long> opted{0};
+  if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
   CUtensorMap mC;
   if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
   const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
@@ -687,12 +683,8 @@ static cudaError_t tc2_launch(const Launch& lc, int M, int N, int K, const void*
   const int tiles_m = (M + 2 * kBM - 1) / (2 * kBM), tiles_n = (N + BN - 1) / BN;
   const int n_tiles = tiles_m * tiles_n * splits;
   auto kern = gemm_tc2_kernel<BN, STAGES, ACC, A_MN, B_MN, Epi>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static std::atomic<unsigned long long> opted{0};
+  if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
   CUtensorMap mC;
   if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
   const int pairs = n_tiles < sm_count() / 2 ? n_tiles : sm_count() / 2;

@@ -427,12 +427,6 @@ __global__ void __launch_bounds__(kThreads)
 
 // ============================================================== host side
 namespace {
-cudaError_t opt_in_smem(const void* kern, size_t bytes, size_t* cached) {
-  if (bytes <= *cached) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-  if (e == cudaSuccess) *cached = bytes;
-  return e;
-}
 // shared memory of the summary kernels: scores [kMaxL], two scalars, [8][260]
 constexpr size_t kSummarySmem = (size_t)(kMaxL + 4 + 8 * 260) * sizeof(float);
 constexpr size_t kGateSmem = (size_t)(8 * 132) * sizeof(float);

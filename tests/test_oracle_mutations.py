@@ -61,6 +61,7 @@ def _load_mutant(old, new):
 
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
+@pytest.mark.filterwarnings("ignore::RuntimeWarning")  # a mutant may divide by zero
 def test_pins_catch_mutation(name, monkeypatch):
     mutant = _load_mutant(*MUTATIONS[name])
     monkeypatch.setattr(pins, "O", mutant)
