@@ -486,7 +486,8 @@ def bench_dense(w, t, stream, flush, args):
 # 6 layers, batch 16) for BCMT, its HOnly ablation and dense attention.
 MODEL_WORKLOADS = {
     "gpt6_v32000_d512_h8_mlp2048_l64_t1024_b16": dict(
-        B=16, vocab=32000, D=512, H=8, layers=6, mlp=2048, runs=[("bcmt", 64, 1024)]),
+        B=16, vocab=32000, D=512, H=8, layers=6, mlp=2048,
+        runs=[("bcmt", 64, 1024), ("bcmt_learned_decay", 64, 1024)]),
     "paper_d128_h8_6l_b16_sweep": dict(
         B=16, vocab=50257, D=128, H=8, layers=6, mlp=512,
         runs=[(m, L, T) for T in (128, 256, 512, 1024) for L in (64, 128, 256, 512) if L <= T
@@ -516,8 +517,9 @@ def bench_models(args):
 
     def run(mixer, L, T, steps, warmup):
         c = gpt.GPTConfig(vocab=spec["vocab"], D=spec["D"], H=spec["H"], layers=spec["layers"],
-                          mlp=spec["mlp"], L=max(L, 1), T=T,
-                          mixer="dense" if mixer == "dense" else "bcmt", honly=mixer == "honly")
+                          mixer="dense" if mixer == "dense" else "bcmt", mlp=spec["mlp"],
+                          L=max(L, 1), T=T, honly=mixer == "honly",
+                          learn_decay=mixer == "bcmt_learned_decay")
         model = gpt.build(c)
         opt = gpt.make_optimizer(model)
         g = torch.Generator().manual_seed(rank_seed(0, rank))
@@ -550,6 +552,7 @@ def bench_models(args):
         e2e_ms = e0.elapsed_time(e1)
         tok = B * T * steps
         r = {"mixer": mixer, "L": L if mixer != "dense" else None, "T": T,
+             "flops_per_token": gpt.flops_per_token(c),
              "tokens_per_s": round(tok / (ms / 1e3), 1), "ms_per_step": round(ms / steps, 3),
              "e2e_tokens_per_s": round(tok / (e2e_ms / 1e3), 1),
              "tflops": round(gpt.flops_per_token(c) * tok / (ms / 1e3) / 1e12, 1),
@@ -606,6 +609,97 @@ def bench_models(args):
     return out
 
 
+# ------------------------------------------------------------- decoding
+# Incremental decoding through one layer: B sequences decoded in lockstep, one
+# token per call (bcmt_decode_step).  The L steps of a block are captured
+# once as a CUDA graph (a block's slots 0..L-1 repeat in every block; the
+# state carries the memory across blocks) and replayed block after block.
+DECODE_WORKLOADS = {
+    "decode_bf16_b16_t1024_l64_d512_h8": dict(B=16, T=1024, D=512, H=8, L=64, dtype="bf16"),
+    "decode_bf16_b1_t1024_l64_d512_h8": dict(B=1, T=1024, D=512, H=8, L=64, dtype="bf16"),
+}
+
+
+def bench_decode(args):
+    import torch
+    from paper_2608_13578_gb300 import build
+    build.build()
+    from paper_2608_13578_gb300 import bcmt as C
+    from paper_2608_13578_gb300 import layer
+    from paper_2608_13578_gb300.inputs import Workload, make_inputs
+
+    rank, local_rank, world = dist_env()
+    if rank != 0:
+        return None
+    torch.cuda.set_device(local_rank)
+    name = args.workload
+    sp = DECODE_WORKLOADS[name]
+    B, T, D, H, L = sp["B"], sp["T"], sp["D"], sp["H"], sp["L"]
+    w = Workload(name, B, T, D, H, L, sp["dtype"], False, (0.8, 0.8), rank_seed(0, rank))
+    t = {k: v.cuda() for k, v in make_inputs(w).items()}
+    x_all = t["x"].transpose(0, 1).contiguous()          # [T, B, D]: token i of every sequence
+    xin = torch.empty(L, B, D, dtype=x_all.dtype, device="cuda")  # the graph's input rows
+    yout = torch.empty(T, B, D, dtype=x_all.dtype, device="cuda")
+    ybuf = torch.empty(L, B, D, dtype=x_all.dtype, device="cuda")
+    dec = layer.Decoder(t, B, H, L)
+    stream = torch.cuda.current_stream()
+
+    def block(pos0):
+        for j in range(L):
+            C.bcmt_decode_step(dec.p, dec.state, pos0 + j, xin[j], t["w_qkv"], t["w_o"], t["w_p"],
+                               t["w_m"], t["w_g"], t["decay"], ybuf[j], None)
+
+    xin.copy_(x_all[:L])
+    for _ in range(2):  # warm-up: two blocks
+        block(0)
+    torch.cuda.synchronize()
+    C.bcmt_decode_reset(dec.p, dec.state)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        block(0)
+    C.bcmt_decode_reset(dec.p, dec.state)
+    torch.cuda.synchronize()
+
+    def run_all():
+        for k in range(T // L):
+            xin.copy_(x_all[k * L:(k + 1) * L])
+            graph.replay()
+            yout[k * L:(k + 1) * L].copy_(ybuf)
+
+    run_all()  # warm the graph
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    reps = max(1, args.steps // 4)
+    ms = []
+    for _ in range(reps):
+        C.bcmt_decode_reset(dec.p, dec.state)
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        run_all()
+        b_.record(stream)
+        torch.cuda.synchronize()
+        ms.append(a.elapsed_time(b_))
+    clk = clocks.stop()
+    C.bcmt_device_status(stream)
+    tot = statistics.median(ms)
+    tok_s = B * T / (tot / 1e3)
+    # our launches per token step: widen, Q/K/V, attention, W_O, W_g, post (+ W_m per block)
+    launches = T * 6 + T // L
+    out = {"metric": "incremental decoding tokens/s through one BCMT layer", "value": round(tok_s, 1),
+           "unit": UNIT, "n_gpus": 1, "steps": reps, "warmup": 2,
+           "ms_per_step": round(tot / T, 5), "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": sp["dtype"], "data": "synthetic (seeded N(0,1) tokens, N(0,1/D) weights, decay 0.8)",
+           "config": {"workload": name, "B": B, "T": T, "D": D, "H": H, "L": L,
+                      "launch": f"CUDA graph of one block's {L} decode steps, replayed per block",
+                      "note": "ms_per_step is per decoded position (B tokens)"},
+           "clocks": clk, "gpu_launches": launches * reps,
+           "e2e": None}
+    print(json.dumps(out))
+    return out
+
+
 # ------------------------------------------------------ reference arm (oracle)
 def bench_reference(args):
     rank, _, world = dist_env()
@@ -613,9 +707,9 @@ def bench_reference(args):
         return None
     from paper_2608_13578_gb300.inputs import HEADLINE, WORKLOADS
     name = args.workload or HEADLINE
-    if name in MODEL_WORKLOADS:
-        out = {"impl": "reference", "unavailable": "the oracle covers the mixer layer only; "
-                                                   "whole-model steps have no CPU reference"}
+    if name in MODEL_WORKLOADS or name in DECODE_WORKLOADS:
+        out = {"impl": "reference", "unavailable": "the reference arm times the layer's forward "
+                                                   "and backward only"}
         print(json.dumps(out))
         return out
     w = WORKLOADS[name]
@@ -646,6 +740,8 @@ def main():
         bench_reference(args)
     elif args.workload in MODEL_WORKLOADS:
         bench_models(args)
+    elif args.workload in DECODE_WORKLOADS:
+        bench_decode(args)
     else:
         bench_ours(args)
 

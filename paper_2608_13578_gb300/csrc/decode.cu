@@ -22,8 +22,6 @@
 namespace bcmt {
 
 namespace {
-constexpr int kGemvRows = 16;   // rows per CTA of the vector-matrix product
-constexpr int kGemvKc = 128;    // K chunk staged in shared memory
 constexpr int kMaxL = 1024;
 
 template <class T>
@@ -33,56 +31,57 @@ __device__ __forceinline__ float round_to(float v) {
 }  // namespace
 
 // out[m, n] = sum_k A[m, k] W[k, n] (fp32 accumulate), A fp32 [M, K], W [K, N]
-// row-major.  CTA: 64 columns x 16 rows; 8 groups of 32 lanes split K, each
-// lane owns 2 adjacent columns (one 4- or 8-byte load per k); the groups'
-// sums are added in group order.  With round_out the result is rounded to TW.
-template <class TW>
-__global__ void __launch_bounds__(256)
+// row-major.  CTA: 32 columns (lane = column) x R rows of A; its 32 warps
+// split K (warp g takes rows g, g+32, ...), each thread issuing all eight
+// weight loads of a 256-row chunk before using them, and the warps' sums are
+// added in warp order.  With round_out the result is rounded to TW.
+template <class TW, int R>
+__global__ void __launch_bounds__(1024)
     decode_gemv_kernel(const float* __restrict__ A, int M, int K, const TW* __restrict__ W, int N,
                        float* __restrict__ out, int round_out) {
   pdl_enter();
-  __shared__ float sA[kGemvRows][kGemvKc];
-  __shared__ float red[8][kGemvRows][65];
-  const int lane = threadIdx.x & 31, g = threadIdx.x >> 5;
-  const int n = blockIdx.x * 64 + lane * 2;
-  const int m0 = blockIdx.y * kGemvRows;
-  const int mc = min(kGemvRows, M - m0);
-  float acc[kGemvRows][2];
+  constexpr int KC = 256;  // K chunk staged in shared memory
+  __shared__ float sA[R][KC];
+  extern __shared__ float red[];  // [32 warps][R][33]
+  const int tid = threadIdx.x, lane = tid & 31, g = tid >> 5;
+  const int n = blockIdx.x * 32 + lane;
+  const int m0 = blockIdx.y * R;
+  const int mc = min(R, M - m0);
+  float acc[R];
 #pragma unroll
-  for (int m = 0; m < kGemvRows; ++m) acc[m][0] = acc[m][1] = 0.f;
-  for (int k0 = 0; k0 < K; k0 += kGemvKc) {
-    for (int i = threadIdx.x; i < kGemvRows * kGemvKc; i += 256) {
-      const int m = i / kGemvKc, k = i - m * kGemvKc;
+  for (int m = 0; m < R; ++m) acc[m] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += KC) {
+    for (int i = tid; i < R * KC; i += 1024) {
+      const int m = i / KC, k = i - m * KC;
       sA[m][k] = (m < mc && k0 + k < K) ? A[(long)(m0 + m) * K + k0 + k] : 0.f;
     }
     __syncthreads();
     if (n < N) {
-      const int kend = min(kGemvKc, K - k0);
-      for (int kk = g; kk < kend; kk += 8) {
-        const TW* wp = W + (long)(k0 + kk) * N + n;
-        const float w0 = to_f(wp[0]), w1 = to_f(wp[1]);
+      const int kend = min(KC, K - k0);
+      float wv[KC / 32];
 #pragma unroll
-        for (int m = 0; m < kGemvRows; ++m) {
-          acc[m][0] = fmaf(sA[m][kk], w0, acc[m][0]);
-          acc[m][1] = fmaf(sA[m][kk], w1, acc[m][1]);
-        }
+      for (int u = 0; u < KC / 32; ++u) {
+        const int kk = g + 32 * u;
+        wv[u] = kk < kend ? to_f(W[(long)(k0 + kk) * N + n]) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < KC / 32; ++u) {
+        const int kk = g + 32 * u;  // < KC; zero weight past kend
+#pragma unroll
+        for (int m = 0; m < R; ++m) acc[m] = fmaf(sA[m][kk], wv[u], acc[m]);
       }
     }
     __syncthreads();
   }
 #pragma unroll
-  for (int m = 0; m < kGemvRows; ++m) {
-    red[g][m][lane * 2] = acc[m][0];
-    red[g][m][lane * 2 + 1] = acc[m][1];
-  }
+  for (int m = 0; m < R; ++m) red[(g * R + m) * 33 + lane] = acc[m];
   __syncthreads();
-  for (int i = threadIdx.x; i < kGemvRows * 64; i += 256) {
-    const int m = i / 64, c = i - m * 64;
-    const int col = blockIdx.x * 64 + c;
+  for (int i = tid; i < R * 32; i += 1024) {
+    const int m = i / 32, c = i - m * 32;
+    const int col = blockIdx.x * 32 + c;
     if (m < mc && col < N) {
       float t = 0.f;
-#pragma unroll
-      for (int q = 0; q < 8; ++q) t += red[q][m][c];
+      for (int q = 0; q < 32; ++q) t += red[(q * R + m) * 33 + c];
       out[(long)(m0 + m) * N + col] = round_out ? round_to<TW>(t) : t;
     }
   }
@@ -102,6 +101,7 @@ __global__ void __launch_bounds__(128)
   const int warp = tid >> 5, lane = tid & 31;
   const float* row = qkv + (long)b * 3 * D;
   const long cache = (long)b * L * D;
+  if (tid >= dh) q[tid] = 0.f;  // channels past dh multiply zero-filled key values
   for (int c = tid; c < dh; c += 128) {
     const int col = h * dh + c;
     q[c] = round_to<T>(row[col]);
@@ -111,9 +111,23 @@ __global__ void __launch_bounds__(128)
   __syncthreads();
   float mx = -INFINITY;
   for (int u = tid; u <= j; u += 128) {
+    // key u's row, 32 channels at a time: the four 16-byte loads go out together
     const T* kr = Kc + cache + (long)u * D + h * dh;
     float s = 0.f;
-    for (int c = 0; c < dh; ++c) s = fmaf(q[c], to_f(kr[c]), s);
+    for (int c0 = 0; c0 < dh; c0 += 32) {
+      float kv[32];
+#pragma unroll
+      for (int q8 = 0; q8 < 4; ++q8) {
+        if (c0 + 8 * q8 < dh) {
+          load8(kr + c0 + 8 * q8, kv + 8 * q8);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) kv[8 * q8 + e] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int e = 0; e < 32; ++e) s = fmaf(q[min(c0 + e, 127)], kv[e], s);
+    }
     s *= scale;
     p[u] = s;
     mx = fmaxf(mx, s);
@@ -136,6 +150,7 @@ __global__ void __launch_bounds__(128)
   for (int c = tid; c < dh; c += 128) {
     const T* vc = Vc + cache + h * dh + c;
     float o = 0.f;
+#pragma unroll 8
     for (int u = 0; u <= j; ++u) o = fmaf(p[u], to_f(vc[(long)u * D]), o);
     hhat[(long)b * D + h * dh + c] = round_to<T>(o * inv);
   }
@@ -198,13 +213,27 @@ __global__ void __launch_bounds__(256)
 
 // ---------------------------------------------------------------- host side
 namespace {
+template <class TW, int R>
+cudaError_t gemv_r(const Launch& lc, const float* A, int M, int K, const void* W, int N, float* out,
+                   bool round_out) {
+  const int smem = 32 * R * 33 * (int)sizeof(float);
+  static std::atomic<unsigned long long> opted{0};
+  if (smem > 48 * 1024) {
+    if (cudaError_t e = smem_opt_in(decode_gemv_kernel<TW, R>, smem, &opted); e != cudaSuccess)
+      return e;
+  }
+  dim3 grid((N + 31) / 32, (M + R - 1) / R);
+  cudaError_t e = launch_k(decode_gemv_kernel<TW, R>, grid, dim3(1024), smem, lc.stream, A, M, K,
+                           (const TW*)W, N, out, round_out ? 1 : 0);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 template <class TW>
 cudaError_t gemv(const Launch& lc, const float* A, int M, int K, const void* W, int N, float* out,
                  bool round_out) {
-  dim3 grid((N + 63) / 64, (M + kGemvRows - 1) / kGemvRows);
-  cudaError_t e = launch_k(decode_gemv_kernel<TW>, grid, dim3(256), 0, lc.stream, A, M, K,
-                           (const TW*)W, N, out, round_out ? 1 : 0);
-  return e != cudaSuccess ? e : cudaGetLastError();
+  if (M == 1) return gemv_r<TW, 1>(lc, A, M, K, W, N, out, round_out);
+  if (M <= 4) return gemv_r<TW, 4>(lc, A, M, K, W, N, out, round_out);
+  return gemv_r<TW, 16>(lc, A, M, K, W, N, out, round_out);
 }
 
 template <class T>
