@@ -25,7 +25,9 @@ int bcmt_test_set_tensor_cores(int gemm_on, int attn_on);
 /* C[M,N] = A[M,K] B[K,N] with fp32 accumulation, element (m,k) of A at
  * A[m*sam + k*sak] and (k,n) of B at B[k*sbk + n*sbn] (elements, not bytes);
  * C row-major with leading dimension ldc, of type dtype_out.  impl: 0 SIMT,
- * 1 tcgen05 (bf16 inputs; A and B each K-major or MN-major).  With
+ * 1 tcgen05 (bf16 inputs; A and B each K-major or MN-major; tile chosen per
+ * shape), 2 the CTA-pair tcgen05 kernel (N % 256 == 0), 3 / 4 / 5 the
+ * single-CTA kernel with 128- / 256- / 64-wide tiles.  With
  * splits > 1, K is cut into ranges whose fp32 partial products go to
  * C + z*M*ldc (C must then be fp32 and hold every split).  N % 64 == 0.
  * Returns the number of K-splits written, or -1 on error. */

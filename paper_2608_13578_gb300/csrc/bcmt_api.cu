@@ -944,11 +944,15 @@ int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, cons
   ea.ldo = ldc;
   ea.split_stride = (long)M * ldc;
   const EpiKind ek = splits > 1 ? EPI_PARTIAL : EPI_STORE;
+  // impl 3, 4, 5: the single-CTA kernel with 128-, 256- or 64-wide tiles
+  g_force_bn = impl == 3 ? 128 : impl == 4 ? 256 : impl == 5 ? 64 : 0;
   cudaError_t e =
-      impl == 1   ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
+      (impl == 1 || impl >= 3)
+          ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
       : impl == 2 ? gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea, splits)
                   : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, ek, ea,
                               splits);
+  g_force_bn = 0;
   if (e != cudaSuccess) {
     fail(BCMT_ERR_CUDA, "test gemm: %s", cudaGetErrorString(e));
     return -1;

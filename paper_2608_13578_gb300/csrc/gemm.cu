@@ -773,10 +773,19 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
   return cudaErrorNotSupported;
 }
 
+// Tile width forced by the test entry point (0: chosen per shape below).
+int g_force_bn = 0;
+
 template <bool A_MN, bool B_MN>
 static cudaError_t tc_pick(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                            long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                            const EpiArgs& ea, int splits) {
+  if (g_force_bn == 64)
+    return tc_epi<64, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (g_force_bn == 128)
+    return tc_epi<128, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
+  if (g_force_bn == 256 && N % 256 == 0)
+    return tc_epi<256, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
   const long tm = (M + kBM - 1) / kBM;
   const long tiles256 = tm * ((N + 255) / 256) * splits;
   const long tiles128 = tm * ((N + 127) / 128) * splits;
@@ -795,9 +804,10 @@ cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const 
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits) {
   if (N % 64 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
-  // long K: the CTA-pair kernel's 256 x 256 tiles need 2/3 of the operand
-  // bytes per flop of a single CTA's 128 x 256 tile
-  if (epi == EPI_STORE && N % 256 == 0 && M >= 512 && K >= 1024)
+  // long K or wide N: the CTA-pair kernel's 256 x 256 tiles need 2/3 of the
+  // operand bytes per flop of a single CTA's 128 x 256 tile (measured faster
+  // from K = 1024, or K = 768 with N >= 1024; no slower at K = 512)
+  if (epi == EPI_STORE && N % 256 == 0 && M >= 512 && (K >= 1024 || (K >= 768 && N >= 1024)))
     return gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
   splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
   const bool a_k = (sak == 1), a_m = (sam == 1) && !a_k;

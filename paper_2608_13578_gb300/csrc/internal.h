@@ -57,6 +57,9 @@ cudaError_t gemm_simt(const Launch& lc, int dtype, int dtype_out, int M, int N, 
 // tcgen05 GEMM (bf16 inputs, fp32 TMEM accumulation).  A must be either
 // K-major (sak == 1) or M-major (sam == 1), B either K-major (sbk == 1) or
 // N-major (sbn == 1).  Returns cudaErrorNotSupported for other layouts.
+// Test hook: forces the single-CTA tcgen05 GEMM's tile width (64, 128, 256;
+// 0 = chosen per shape).
+extern int g_force_bn;
 // The CTA-pair tcgen05 GEMM (256 x 256 tiles), EPI_STORE / EPI_PARTIAL only.
 cudaError_t gemm_tc_pair(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                          long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
