@@ -314,7 +314,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 
 struct BwdWs {
   char *dU, *dH, *dHhat, *dqkv, *dPb;
-  float *dP, *dM, *dS, *ds, *dwp_part, *da_part, *Drow, *part;
+  float *dP, *dM, *dS, *ds, *dwp_part, *da_part, *Drow, *part, *part_o;
   size_t bytes;
 };
 
@@ -348,6 +348,9 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
   if (g.from_x)
     part = std::max(part, (size_t)dw_splits(g.dtype, g.D, 3 * g.D, g.n) * g.D * 3 * g.D * 4);
   w.part = reinterpret_cast<float*>(take(part));
+  // dW_O's K-split partials: its product runs on the critical stream while
+  // the side stream may still be reducing dW_g's partials
+  w.part_o = reinterpret_cast<float*>(take((size_t)dw_splits(g.dtype, g.D, g.D, g.n) * g.D * g.D * 4));
   w.bytes = off;
   return w;
 }
@@ -360,7 +363,9 @@ bcmt_status cuda_fail(cudaError_t e, const char* what) {
 // ordered reduction.
 cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype, int dtype_out,
                         int M, int N, long K,
-                        const void* A, long lda, const void* B, long ldb, float* part, void* out) {
+                        const void* A, long lda, const void* B, long ldb, float* part, void* out,
+                        Fork* reduce_beside = nullptr, const Launch* lcs = nullptr,
+                        Prof* prs = nullptr) {
   const int splits = dw_splits(dtype, M, N, K);
   EpiArgs ea;
   ea.out = part;
@@ -375,9 +380,13 @@ cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype,
           : gemm_simt(lc, dtype, 0, M, N, (int)K, A, 1, lda, B, ldb, 1, EPI_PARTIAL, ea, splits);
   pr.end(nullptr);
   if (e != cudaSuccess) return e;
-  pr.begin("reduce_splits");
-  e = reduce_splits(lc, part, effective_splits((int)K, splits), (long)M * N, dtype_out, out);
-  pr.end(nullptr);
+  // the ordered sum of the partials, on the side stream when asked
+  const Launch& lr = reduce_beside ? *lcs : lc;
+  Prof& prr = reduce_beside ? *prs : pr;
+  if (reduce_beside) reduce_beside->point();
+  prr.begin("reduce_splits");
+  e = reduce_splits(lr, part, effective_splits((int)K, splits), (long)M * N, dtype_out, out);
+  prr.end(nullptr);
   return e;
 }
 
@@ -697,13 +706,15 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     EpiArgs ea;
     ea.out = bw.dHhat;
     ea.ldo = D;
-    if (g.honly) fork.point();  // dH (= dY) is final; otherwise forked after summary_bwd
-    e = weight_grad(lcs, prs, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part,
-                    dw_o);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_O");
     e = run_gemm(lc, pr, "gemm_dhhat", g.dtype, g.dtype, n, D, D, dH, D, 1, w_o, 1, D, EPI_STORE,
                  ea);
     if (e != cudaSuccess) return cuda_fail(e, "dHhat");
+    // dW_O on the critical stream (beside the attention backward the side
+    // stream's weight-gradient GEMMs would find no free SM); its reduction on
+    // the side stream
+    e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part_o,
+                    dw_o, &fork, &lcs, &prs);
+    if (e != cudaSuccess) return cuda_fail(e, "dW_O");
   }
   // Attention backward -> dQ, dK, dV.
   {
