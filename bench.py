@@ -340,36 +340,60 @@ def bench_ours(args):
     tokens_per_step = w.B * w.T
     value = job_tokens_per_s(world, tokens_per_step, args.steps, total_ms)
 
-    # ---- end to end through the public API: pinned host inputs in, results out
+    # ---- end to end through the public API: every step copies its inputs in
+    # from pinned host memory and its output and every gradient back out.  The
+    # copies run on their own streams and overlap the previous/next step's
+    # compute (double-buffered device inputs and outputs), as a training loop
+    # that streams its batches would.
     x_h = t_cpu["x"].pin_memory()
     dy_h = t_cpu["dy"].pin_memory()
     outs_h = {"y": torch.empty_like(t_cpu["x"]).pin_memory()}
     for n, g_ in grads.items():
         outs_h[n] = torch.empty(g_.shape, dtype=g_.dtype).pin_memory()
-    x_d, dy_d = torch.empty_like(t["x"]), torch.empty_like(t["dy"])
+    x_d = [torch.empty_like(t["x"]) for _ in range(2)]
+    dy_d = [torch.empty_like(t["dy"]) for _ in range(2)]
+    y_d = [torch.empty_like(t["x"]) for _ in range(2)]
+    g_d = [{n: torch.empty_like(g_) for n, g_ in grads.items()} for _ in range(2)]
     h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
     d2h = sum(v.numel() * v.element_size() for v in outs_h.values())
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in range(2)]
+    ev_done = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(2)]
 
-    def e2e_step():
-        x_d.copy_(x_h, non_blocking=True)
-        dy_d.copy_(dy_h, non_blocking=True)
-        C.bcmt_forward(p, x_d, None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
-                       t["w_g"], t["decay"], y, ws, stream)
-        C.bcmt_backward(p, dy_d, x_d, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
-                        t["w_g"], t["decay"], ws, sc, grads["dx"], None, None, grads["dw_qkv"],
-                        grads["dw_o"], grads["dw_p"], grads["dw_m"], grads["dw_g"], stream)
-        outs_h["y"].copy_(y, non_blocking=True)
-        for n, g_ in grads.items():
-            outs_h[n].copy_(g_, non_blocking=True)
+    def e2e_steps(k_steps):
+        for i in range(k_steps):
+            b = i % 2
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(ev_done[b])  # step i-2 has read buffer b
+                x_d[b].copy_(x_h, non_blocking=True)
+                dy_d[b].copy_(dy_h, non_blocking=True)
+                ev_in[b].record(s_in)
+            stream.wait_event(ev_in[b])
+            if i >= 2:
+                stream.wait_event(ev_out[b])  # step i-2's outputs are on the host
+            gb = g_d[b]
+            C.bcmt_forward(p, x_d[b], None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                           t["w_g"], t["decay"], y_d[b], ws, stream)
+            C.bcmt_backward(p, dy_d[b], x_d[b], None, None, t["w_qkv"], t["w_o"], t["w_p"],
+                            t["w_m"], t["w_g"], t["decay"], ws, sc, gb["dx"], None, None,
+                            gb["dw_qkv"], gb["dw_o"], gb["dw_p"], gb["dw_m"], gb["dw_g"], stream)
+            ev_done[b].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_done[b])
+                outs_h["y"].copy_(y_d[b], non_blocking=True)
+                for n, g_ in gb.items():
+                    outs_h[n].copy_(g_, non_blocking=True)
+                ev_out[b].record(s_out)
 
-    for _ in range(3):
-        e2e_step()
+    e2e_steps(3)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        e2e_step()
-    e1.record(stream)
+    s_in.wait_event(e0)
+    e2e_steps(args.steps)
+    e1.record(s_out)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
