@@ -335,7 +335,8 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dM = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
-    w.dwp_part = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.dwp_part = reinterpret_cast<float*>(
+        take((size_t)g.B * g.Nb * summary_bwd_chunks(g.L) * g.D * 4));
     w.da_part = reinterpret_cast<float*>(take((size_t)g.B * g.D * 4));
   } else {
     w.dU = w.dH = w.dPb = nullptr;
@@ -678,13 +679,13 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     // and dH += alpha dS + ds w_p
     fork.wait_mark(scan_done);
     pr.begin("summary_bwd");
-    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part, g.B, g.T,
-                    D, g.L);
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, w.S, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part, g.B,
+                    g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     fork.point();
     prs.begin("reduce_rows");
-    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb, D, g.dtype, dw_p);
+    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb * summary_bwd_chunks(g.L), D, g.dtype, dw_p);
     prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "dW_p");
     if (d_decay) {  // fp32, summed over the batch rows in order

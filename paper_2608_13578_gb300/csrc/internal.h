@@ -134,11 +134,15 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 // batch row, da_part [B, D] (M is the forward's fp32 memory, read only then).
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
                             const float* M, float* dS, float* da_part, int B, int Nb, int D);
-// Backward of the pooling: g_t = H_t . dS_blk, ds_t = alpha_t (g_t - sum alpha g),
-// dwp_part[b*Nb+i] = sum_t ds_t H_t, and dH_t += alpha_t dS_blk + ds_t w_p in place.
+// Backward of the pooling, in chunks of 32 rows of a block (grid
+// summary_bwd_chunks(L) x Nb x B): g_t = H_t . dS_blk,
+// ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
+// dwp_part[(b*Nb + i) * chunks + c] = sum over the chunk of ds_t H_t, and
+// dH_t += alpha_t dS_blk + ds_t w_p in place.
+int summary_bwd_chunks(int L);
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* dS, const void* w_p, void* dH, float* ds, float* dwp_part,
-                        int B, int T, int D, int L);
+                        const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
+                        float* dwp_part, int B, int T, int D, int L);
 // Sec. 3.7-3.8 injection: Y = H + G * C[b, t / L].
 cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Cm,
                    void* Y, int B, int T, int D, int L);

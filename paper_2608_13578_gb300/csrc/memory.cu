@@ -195,59 +195,70 @@ __device__ void scan_bwd_item(const float* dM, const float* __restrict__ decay,
   if (da_part) da_part[(long)b * D + c] = da;
 }
 
-// Sec. 3.4 reversed: item (i, b).  With S_i = sum_t alpha_t H_t and
-// alpha = softmax(s): g_t = H_t . dS_i, ds_t = alpha_t (g_t - sum_u alpha_u g_u),
-// and the block's share of dW_p = sum_t ds_t H_t.  The same pass completes the
-// gradient of H in place: dH_t += alpha_t dS_i + ds_t w_p (the pooling and the
-// score paths, added to dY + dU W_g^T already in dH).
+// Sec. 3.4 reversed: item (c, i, b), rows 16c .. 16c+15 of block i of batch b.
+// With S_i = sum_t alpha_t H_t and alpha = softmax(s): g_t = H_t . dS_i and
+// ds_t = alpha_t (g_t - sum_u alpha_u g_u), where sum_u alpha_u g_u = S_i . dS_i
+// (the forward's block summary), so every row chunk of a block is independent.
+// The chunk's share of dW_p = sum_t ds_t H_t goes to dwp_part, and the same
+// pass completes the gradient of H in place: dH_t += alpha_t dS_i + ds_t w_p
+// (the pooling and score paths, added to dY + dU W_g^T already in dH).
+constexpr int kBwdRows = 16;
+constexpr int kBwdRowsPerWarp = kBwdRows / 8;
 template <class T>
 __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
-                                 const float* __restrict__ alpha, const float* dS,
-                                 const T* __restrict__ w_p, T* dH,
+                                 const float* __restrict__ alpha, const float* __restrict__ Sb,
+                                 const float* dS, const T* __restrict__ w_p, T* dH,
                                  float* __restrict__ ds_out, float* __restrict__ dwp_part,
-                                 int Tlen, int D, int L, int Nb, int i, int b) {
-  float* g = sm;                   // [kMaxL]
-  float* cdot = sm + kMaxL;        // [1]
-  float* part = sm + kMaxL + 4;    // [8][260]
+                                 int Tlen, int D, int L, int Nb, int c, int i, int b) {
+  float* g = sm;                      // [kBwdRows]
+  float* red = sm + kBwdRows;         // [8]: per-warp partial sums of S_i . dS_i
+  float* part = sm + kBwdRows + 8;    // [8][260]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t0 = i * L, n = min(L, Tlen - t0);
+  const int blen = min(L, Tlen - i * L);
+  const int t0 = i * L + c * kBwdRows, n = min(kBwdRows, blen - c * kBwdRows);
   const T* Hb = Hm + ((long)b * Tlen + t0) * D;
   const float* dSi = dS + ((long)b * Nb + i) * D;
+  const float* Si = Sb + ((long)b * Nb + i) * D;
   const float* ab = alpha + (long)b * Tlen + t0;
-  // g_t = H_t . dS_i: warp w takes rows w, w+8, ... four at a time; all the
-  // loads of a 256-channel chunk for the four rows go out together
-  for (int r0 = warp; r0 < n; r0 += 32) {
-    float d[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-    for (int c = lane * 8; c < D; c += 256) {
-      float sv[8], h[4][8];
-      load8_cg(dSi + c, sv);
+  // sum_u alpha_u g_u = S_i . dS_i
+  float cp = 0.f;
+  for (int k = threadIdx.x; k < D; k += kThreads) cp = fmaf(Si[k], __ldcg(dSi + k), cp);
+  cp = warp_sum(cp);
+  if (lane == 0) red[warp] = cp;
+  // g_t = H_t . dS_i: warp w takes rows w, w+8; all the loads of a
+  // 256-channel chunk for its rows go out together
+  constexpr int RW = kBwdRowsPerWarp;
+  {
+    float d[RW];
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (r0 + 8 * u < n) load8(Hb + (long)(r0 + 8 * u) * D + c, h[u]);
+    for (int u = 0; u < RW; ++u) d[u] = 0.f;
+#pragma unroll 2
+    for (int k = lane * 8; k < D; k += 256) {
+      float sv[8], h[RW][8];
+      load8_cg(dSi + k, sv);
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (r0 + 8 * u < n) {
+      for (int u = 0; u < RW; ++u)
+        if (warp + 8 * u < n) load8(Hb + (long)(warp + 8 * u) * D + k, h[u]);
+#pragma unroll
+      for (int u = 0; u < RW; ++u)
+        if (warp + 8 * u < n) {
 #pragma unroll
           for (int e = 0; e < 8; ++e) d[u] = fmaf(h[u][e], sv[e], d[u]);
         }
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < RW; ++u) {
       const float t = warp_sum(d[u]);
-      if (lane == 0 && r0 + 8 * u < n) g[r0 + 8 * u] = t;
+      if (lane == 0 && warp + 8 * u < n) g[warp + 8 * u] = t;
     }
   }
   __syncthreads();
-  if (warp == 0) {
-    float acc = 0.f;
-    for (int r = lane; r < n; r += 32) acc = fmaf(ab[r], g[r], acc);
-    acc = warp_sum(acc);
-    if (lane == 0) *cdot = acc;
-  }
-  __syncthreads();
-  const float cd = *cdot;
-  for (int r = threadIdx.x; r < n; r += kThreads) {
+  float cd = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) cd += red[w];
+  __syncthreads();  // everyone has read red before g is overwritten below
+  if (threadIdx.x < n) {
+    const int r = threadIdx.x;
     const float v = ab[r] * (g[r] - cd);
     ds_out[(long)b * Tlen + t0 + r] = v;
     g[r] = v;
@@ -255,40 +266,33 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   __syncthreads();
   const int rg = warp, co = lane;
   T* dHb = dH + ((long)b * Tlen + t0) * D;
+  const long prow = ((long)b * Nb + i) * ((L + kBwdRows - 1) / kBwdRows) + c;
   for (int c0 = 0; c0 < D; c0 += 256) {
-    const int c = c0 + co * 8;
+    const int k = c0 + co * 8;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    if (c < D) {
+    if (k < D) {
       float sv[8], wp[8];
-      load8_cg(dSi + c, sv);
-      load8(w_p + c, wp);
-      // rows rg, rg+8, ... two at a time: all loads of a pair before its stores
-      for (int r = rg; r < n; r += 16) {
-        const bool two = r + 8 < n;
-        float h0[8], h1[8], d0[8], d1[8];
-        load8(Hb + (long)r * D + c, h0);
-        load8(dHb + (long)r * D + c, d0);
-        if (two) {
-          load8(Hb + (long)(r + 8) * D + c, h1);
-          load8(dHb + (long)(r + 8) * D + c, d1);
-        }
-        const float w0 = g[r], a0 = ab[r];
-        const float w1 = two ? g[r + 8] : 0.f, a1 = two ? ab[r + 8] : 0.f;
+      load8_cg(dSi + k, sv);
+      load8(w_p + k, wp);
+      // rows rg, rg+8: all their loads before the first store
+      float h[RW][8], d[RW][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          acc[e] = fmaf(w0, h0[e], acc[e]);
-          d0[e] += a0 * sv[e] + w0 * wp[e];
+      for (int u = 0; u < RW; ++u)
+        if (rg + 8 * u < n) {
+          load8(Hb + (long)(rg + 8 * u) * D + k, h[u]);
+          load8(dHb + (long)(rg + 8 * u) * D + k, d[u]);
         }
-        store8(dHb + (long)r * D + c, d0);
-        if (two) {
+#pragma unroll
+      for (int u = 0; u < RW; ++u)
+        if (rg + 8 * u < n) {
+          const float w = g[rg + 8 * u], a = ab[rg + 8 * u];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            acc[e] = fmaf(w1, h1[e], acc[e]);
-            d1[e] += a1 * sv[e] + w1 * wp[e];
+            acc[e] = fmaf(w, h[u][e], acc[e]);
+            d[u][e] += a * sv[e] + w * wp[e];
           }
-          store8(dHb + (long)(r + 8) * D + c, d1);
+          store8(dHb + (long)(rg + 8 * u) * D + k, d[u]);
         }
-      }
     }
 #pragma unroll
     for (int e = 0; e < 8; ++e) part[rg * 260 + co * 8 + e] = acc[e];
@@ -298,7 +302,7 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
       float t = 0.f;
 #pragma unroll
       for (int q = 0; q < 8; ++q) t += part[q * 260 + threadIdx.x];
-      dwp_part[((long)b * Nb + i) * D + cc] = t;
+      dwp_part[prow * D + cc] = t;
     }
     __syncthreads();
   }
@@ -373,15 +377,22 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 template <class T>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 2)
     summary_bwd_kernel(const T* __restrict__ Hm, const float* __restrict__ alpha,
-                       const float* __restrict__ dS, const T* __restrict__ w_p, T* dH,
-                       float* __restrict__ ds, float* __restrict__ dwp_part, int Tlen, int D,
-                       int L, int Nb) {
+                       const float* __restrict__ Sb, const float* __restrict__ dS,
+                       const T* __restrict__ w_p, T* dH, float* __restrict__ ds,
+                       float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
   pdl_enter();
-  extern __shared__ __align__(16) float sm[];
-  summary_bwd_item<T>(sm, Hm, alpha, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb, blockIdx.x,
-                      blockIdx.y);
+  __shared__ __align__(16) float sm[kBwdRows + 8 + 8 * 260];
+  // a ragged last block has fewer chunks than the grid's x extent: its empty
+  // chunks contribute zero partials to dW_p
+  if ((int)blockIdx.x * kBwdRows >= min(L, Tlen - (int)blockIdx.y * L)) {
+    const long prow = ((long)blockIdx.z * Nb + blockIdx.y) * gridDim.x + blockIdx.x;
+    for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
+    return;
+  }
+  summary_bwd_item<T>(sm, Hm, alpha, Sb, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb, blockIdx.x,
+                      blockIdx.y, blockIdx.z);
 }
 
 // Sec. 3.7-3.8: Y = H + G * C[b, t / L], the memory row of the token's block
@@ -478,21 +489,21 @@ cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* deca
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+int summary_bwd_chunks(int L) { return (L + kBwdRows - 1) / kBwdRows; }
+
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* dS, const void* w_p, void* dH, float* ds, float* dwp_part,
-                        int B, int T, int D, int L) {
+                        const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
+                        float* dwp_part, int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
-  dim3 grid(Nb, B);
+  dim3 grid(summary_bwd_chunks(L), Nb, B);
   cudaError_t e;
   if (dtype == 0)
-    e = launch_k(summary_bwd_kernel<float>, grid, dim3(kThreads), kSummarySmem, lc.stream,
-                 (const float*)Hm, alpha, dS, (const float*)w_p, (float*)dH, ds, dwp_part, T, D,
-                 L, Nb);
+    e = launch_k(summary_bwd_kernel<float>, grid, dim3(kThreads), 0, lc.stream, (const float*)Hm,
+                 alpha, Sb, dS, (const float*)w_p, (float*)dH, ds, dwp_part, T, D, L, Nb);
   else
-    e = launch_k(summary_bwd_kernel<bf16>, grid, dim3(kThreads), kSummarySmem, lc.stream,
-                 (const bf16*)Hm, alpha, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T, D, L,
-                 Nb);
+    e = launch_k(summary_bwd_kernel<bf16>, grid, dim3(kThreads), 0, lc.stream, (const bf16*)Hm,
+                 alpha, Sb, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T, D, L, Nb);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
