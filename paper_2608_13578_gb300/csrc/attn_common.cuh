@@ -16,6 +16,14 @@ __device__ __forceinline__ void put_unit(uint8_t* base, int r, int u, uint4 val)
   *reinterpret_cast<uint4*>(base + (u >> 3) * 16384 + tc::sw128_offset(r, u & 7)) = val;
 }
 
+// 2^x by the ex2.approx.ftz instruction (relative error near 2^-22, 2^-inf =
+// +0): for probabilities that are rounded to bf16 or summed in fp32.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
   __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&t);

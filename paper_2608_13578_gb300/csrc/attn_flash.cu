@@ -210,38 +210,71 @@ __global__ void __launch_bounds__(128)
       }
     }
 
-    // ---- online softmax (P to shared memory; the previous P V has completed)
-    float mt = -INFINITY;
+    // ---- online softmax (P to shared memory; the previous P V has completed).
+    // Tiles left of the diagonal need no mask: their max, exponentials and
+    // sum run with independent partial accumulators.
+    float m_new, psum;
+    if (!diag) {
+      float mx[8];
 #pragma unroll
-    for (int ci = 0; ci < 4; ++ci)
-      if (ci < nld) {
+      for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int kk = wbs + ci * 32 + j;
-          if (!diag || (kk >= rbs && kk <= r)) mt = fmaxf(mt, __uint_as_float(sr[ci][j]));
+      for (int ci = 0; ci < 4; ++ci)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) mx[j & 7] = fmaxf(mx[j & 7], __uint_as_float(sr[ci][j]));
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      m_new = fmaxf(m, mt * sl2);
+      const float nm = -m_new;
+      float ps[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          v[e] = ex2(fmaf(__uint_as_float(sr[u >> 2][(u & 3) * 8 + e]), sl2, nm));
+          ps[e & 3] += v[e];
         }
+        put_unit(sP, r, u, pack8(v));
       }
-    const float m_new = fmaxf(m, mt * sl2);
-    const float alpha = exp2f(m - m_new);  // 0 on the first tile (m = -inf)
-    float psum = 0.f;
+      psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
+    } else {
+      float mt = -INFINITY;
 #pragma unroll
-    for (int ci = 0; ci < 4; ++ci)
-      if (ci < nld) {
-        float v[32];
+      for (int ci = 0; ci < 4; ++ci)
+        if (ci < nld) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int kk = wbs + ci * 32 + j;
-          const bool valid = !diag || (kk >= rbs && kk <= r);
-          const float p = valid ? exp2f(__uint_as_float(sr[ci][j]) * sl2 - m_new) : 0.f;
-          v[j] = p;
-          psum += p;
+          for (int j = 0; j < 32; ++j) {
+            const int kk = wbs + ci * 32 + j;
+            if (kk >= rbs && kk <= r) mt = fmaxf(mt, __uint_as_float(sr[ci][j]));
+          }
         }
+      m_new = fmaxf(m, mt * sl2);
+      const float nm = -m_new;
+      float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int u = 0; u < 4; ++u) put_unit(sP, r, (wbs + ci * 32) / 8 + u, pack8(v + 8 * u));
-      }
-    const uint4 zero = make_uint4(0, 0, 0, 0);
-    for (int u = 0; u < 16; ++u)
-      if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
+      for (int ci = 0; ci < 4; ++ci)
+        if (ci < nld) {
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int kk = wbs + ci * 32 + u * 8 + e;
+              v[e] = (kk >= rbs && kk <= r)
+                         ? ex2(fmaf(__uint_as_float(sr[ci][u * 8 + e]), sl2, nm))
+                         : 0.f;
+              ps[e & 3] += v[e];
+            }
+            put_unit(sP, r, (wbs + ci * 32) / 8 + u, pack8(v));
+          }
+        }
+      psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
+      const uint4 zero = make_uint4(0, 0, 0, 0);
+      for (int u = 0; u < 16; ++u)
+        if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
+    }
+    const float alpha = ex2(m - m_new);  // 0 on the first tile (m = -inf)
     l = l * alpha + psum;
     m = m_new;
     tc::fence_proxy_async_smem();
@@ -356,6 +389,7 @@ __global__ void __launch_bounds__(128)
     lse2 = lse[li] * kLog2e;
   }
   const float sl2 = scale * kLog2e;
+  const float nl2 = -lse2, ndr = -drow * scale;
   const int rbs = L < kTile ? (r / L) * L : 0;
   bool ok = true;
   int ns = 0, nq = 0;  // commits to bar[1] and bar[2] so far
@@ -395,15 +429,25 @@ __global__ void __launch_bounds__(128)
         ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
         tc::fence_after_sync();
       }
+      // dS = P (dP - Drow) scale; rows past the end see zero-filled Q and dO
+      // (P finite, dP = Drow = 0), so only the diagonal tile needs a mask
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         float v[32];
+        if (!diag) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int kk = 64 * hh + 32 * c + j;  // key column within the tile
-          const bool valid = row_ok && (!diag || (kk >= rbs && kk <= r));
-          const float p = valid ? exp2f(__uint_as_float(rs[c][j]) * sl2 - lse2) : 0.f;
-          v[j] = p * (__uint_as_float(rd[c][j]) - drow) * scale;
+          for (int j = 0; j < 32; ++j)
+            v[j] = ex2(fmaf(__uint_as_float(rs[c][j]), sl2, nl2)) *
+                   fmaf(__uint_as_float(rd[c][j]), scale, ndr);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int kk = 64 * hh + 32 * c + j;  // key column within the tile
+            const bool valid = row_ok && kk >= rbs && kk <= r;
+            v[j] = valid ? ex2(fmaf(__uint_as_float(rs[c][j]), sl2, nl2)) *
+                               fmaf(__uint_as_float(rd[c][j]), scale, ndr)
+                         : 0.f;
+          }
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) put_unit(sdS, r, 4 * c + u, pack8(v + 8 * u));
@@ -460,8 +504,8 @@ __global__ void __launch_bounds__(128)
   uint8_t* sV = sK + G::tile;
   uint8_t* sQ = sV + G::tile;
   uint8_t* sdO = sQ + G::tile;
-  float* slse = reinterpret_cast<float*>(sdO + G::tile);  // [128] lse * log2(e)
-  float* sdr = slse + kTile;                               // [128] Drow
+  float* slse = reinterpret_cast<float*>(sdO + G::tile);  // [128] -lse * log2(e)
+  float* sdr = slse + kTile;                               // [128] -Drow * scale
   uint64_t* bar = reinterpret_cast<uint64_t*>(sdr + kTile);  // kv, s, q
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
 
@@ -513,8 +557,8 @@ __global__ void __launch_bounds__(128)
     {
       const int tq = q0 + tid;
       const long li = ((long)b * H + h) * Tlen + tq;
-      slse[tid] = tq < Tlen ? lse[li] * kLog2e : 0.f;
-      sdr[tid] = tq < Tlen ? Drow[li] : 0.f;
+      slse[tid] = tq < Tlen ? -lse[li] * kLog2e : 0.f;
+      sdr[tid] = tq < Tlen ? -Drow[li] * scale : 0.f;
     }
     if (tid == 0) {
       ok = tc::mbar_wait(&bar[0], qt & 1, status) && ok;
@@ -549,17 +593,27 @@ __global__ void __launch_bounds__(128)
         ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
         tc::fence_after_sync();
       }
+      // P^T and dS^T = P^T (dP^T - Drow) scale.  Query columns past the end
+      // see zero-filled Q and dO (P finite, dO = dP = Drow = 0: no
+      // contribution), so only the diagonal tile needs a mask.
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         float pv[32], dv[32];
+        const float4* nl4 = reinterpret_cast<const float4*>(slse + 64 * hh + 32 * c);
+        const float4* nd4 = reinterpret_cast<const float4*>(sdr + 64 * hh + 32 * c);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int jq = 64 * hh + 32 * c + j;  // query column within the tile
-          const int tq = q0 + jq;
-          const bool valid = tq < Tlen && (!diag || (jq >= r && jq < kbe));
-          const float p = valid ? exp2f(__uint_as_float(rs[c][j]) * sl2 - slse[jq]) : 0.f;
-          pv[j] = p;
-          dv[j] = p * (__uint_as_float(rd[c][j]) - sdr[jq]) * scale;
+        for (int j4 = 0; j4 < 8; ++j4) {
+          const float4 a = nl4[j4], d = nd4[j4];
+          const float na[4] = {a.x, a.y, a.z, a.w}, nd[4] = {d.x, d.y, d.z, d.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int j = 4 * j4 + e;
+            const int jq = 64 * hh + 32 * c + j;  // query column within the tile
+            const bool valid = !diag || (q0 + jq < Tlen && jq >= r && jq < kbe);
+            const float p = valid ? ex2(fmaf(__uint_as_float(rs[c][j]), sl2, na[e])) : 0.f;
+            pv[j] = p;
+            dv[j] = p * fmaf(__uint_as_float(rd[c][j]), scale, nd[e]);
+          }
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {

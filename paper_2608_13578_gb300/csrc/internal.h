@@ -134,7 +134,7 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 // batch row, da_part [B, D] (M is the forward's fp32 memory, read only then).
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
                             const float* M, float* dS, float* da_part, int B, int Nb, int D);
-// Backward of the pooling, in chunks of 32 rows of a block (grid
+// Backward of the pooling, in chunks of 16 rows of a block (grid
 // summary_bwd_chunks(L) x Nb x B): g_t = H_t . dS_blk,
 // ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
 // dwp_part[(b*Nb + i) * chunks + c] = sum over the chunk of ds_t H_t, and
