@@ -123,39 +123,37 @@ __global__ void __launch_bounds__(128)
   for (int ci = 0; ci < NCH; ++ci)
     if (ci < nld) tc::tmem_ld32_issue(trow + (uint32_t)(wbs + ci * 32), sr[ci]);
   tc::tmem_wait();
-  float mx = -INFINITY;
+  // the max and the sum run in independent partials (short dependency chains)
+  float mxp[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
   for (int ci = 0; ci < NCH; ++ci)
     if (ci < nld) {
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
         const int kk = wbs + ci * 32 + j;
-        if (kk >= rbs && kk <= r) mx = fmaxf(mx, __uint_as_float(sr[ci][j]));
+        if (kk >= rbs && kk <= r) mxp[j & 3] = fmaxf(mxp[j & 3], __uint_as_float(sr[ci][j]));
       }
     }
-  float sum = 0.f;
+  const float mx = fmaxf(fmaxf(mxp[0], mxp[1]), fmaxf(mxp[2], mxp[3]));
+  const float nm = -mx * sl2;
+  float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
   for (int ci = 0; ci < NCH; ++ci)
     if (ci < nld) {
-      float v[32];
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const int kk = wbs + ci * 32 + j;
-        const float p =
-            (kk >= rbs && kk <= r) ? exp2f((__uint_as_float(sr[ci][j]) - mx) * sl2) : 0.f;
-        v[j] = p;
-        sum += p;
-      }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        uint4 q;
-        q.x = pack2(v[8 * u + 0], v[8 * u + 1]);
-        q.y = pack2(v[8 * u + 2], v[8 * u + 3]);
-        q.z = pack2(v[8 * u + 4], v[8 * u + 5]);
-        q.w = pack2(v[8 * u + 6], v[8 * u + 7]);
-        put_unit(sP, r, (wbs + ci * 32) / 8 + u, q);
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const int kk = wbs + ci * 32 + u * 8 + e;
+          v[e] = (kk >= rbs && kk <= r) ? ex2(fmaf(__uint_as_float(sr[ci][u * 8 + e]), sl2, nm))
+                                        : 0.f;
+          ps[e & 3] += v[e];
+        }
+        put_unit(sP, r, (wbs + ci * 32) / 8 + u, pack8(v));
       }
     }
+  const float sum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
   const uint4 zero = make_uint4(0, 0, 0, 0);
   for (int u = 0; u < 16; ++u)
     if (u * 8 < wbs || u * 8 >= wbs + nld * 32) put_unit(sP, r, u, zero);
@@ -301,7 +299,7 @@ __global__ void __launch_bounds__(128)
   const int wbs = L < 32 ? warp * 32 : ((warp * 32) / L) * L;
   const int nld = chunks_needed(warp, wbs);
   const int rbs = (r / L) * L;
-  const float sl2 = scale * kLog2e, ll2 = lr * kLog2e;
+  const float sl2 = scale * kLog2e, nl2 = -lr * kLog2e, ndr = -drow * scale;
   uint32_t dsp[NCH * 16];
 #pragma unroll
   for (int ci = 0; ci < NCH; ++ci) {
@@ -322,9 +320,9 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
         const int kk = wbs + c + j;
-        const float p = (row_ok && kk >= rbs && kk <= r) ? exp2f(s[j] * sl2 - ll2) : 0.f;
+        const float p = (row_ok && kk >= rbs && kk <= r) ? ex2(fmaf(s[j], sl2, nl2)) : 0.f;
         s[j] = p;
-        dp[j] = p * (dp[j] - drow) * scale;
+        dp[j] = p * fmaf(dp[j], scale, ndr);
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
