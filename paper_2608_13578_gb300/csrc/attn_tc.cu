@@ -192,7 +192,7 @@ __global__ void __launch_bounds__(128)
   if (tid == 0 && ok) {
     tc::tma_store_3d(&mO, sQ, h * kDh, t0, b);
     tc::tma_store_commit();
-    tc::tma_store_wait_all();
+    tc::tma_store_wait_read<0>();  // the staging is read; the writes finish with the grid
   }
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 128);
@@ -415,7 +415,7 @@ __global__ void __launch_bounds__(128)
     tc::tma_store_3d(&mdK, sK, h * kDh, t0, b);
     tc::tma_store_3d(&mdV, sdO, h * kDh, t0, b);
     tc::tma_store_commit();
-    tc::tma_store_wait_all();
+    tc::tma_store_wait_read<0>();  // the staging is read; the writes finish with the grid
   }
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 256);

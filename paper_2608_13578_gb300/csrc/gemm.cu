@@ -398,7 +398,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       if (lane == 0) tc::mbar_arrive(&tempty[acc]);
       if (!ok) break;
     }
-    if (lane == 0) tc::tma_store_wait_all();  // output stores done before exit
+    if (lane == 0) tc::tma_store_wait_read<0>();  // staging read; the writes finish with the grid
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -645,7 +645,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       if (lane == 0) tc::mbar_arrive_cluster(te0 + (uint32_t)(acc * 8));
       if (!ok) break;
     }
-    if (lane == 0) tc::tma_store_wait_all();
+    if (lane == 0) tc::tma_store_wait_read<0>();  // staging read; the writes finish with the grid
   }
   tc::fence_before_sync();
   __syncthreads();

@@ -97,6 +97,10 @@ ATTN_CASES = [
     (2, 200, 2, 64, 32, "bf16"),
     (1, 384, 3, 64, 128, "bf16"),
     (2, 130, 2, 64, 16, "bf16"),
+    # more (tile, head) items than resident CTAs: several rounds per SM
+    (4, 1024, 12, 64, 64, "bf16"),
+    (3, 1000, 16, 64, 32, "bf16"),
+    (2, 1280, 16, 64, 128, "bf16"),
     (1, 300, 2, 64, 256, "bf16"),
     (1, 600, 2, 64, 256, "bf16"),     # ragged last block, 1-3 key tiles per query tile
     (1, 1100, 1, 64, 512, "bf16"),
