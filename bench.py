@@ -211,12 +211,38 @@ def kernel_model(w):
     }
 
 
-def csrc_digest():
+# The sources each timed kernel is built from (its translation unit and the
+# headers every kernel shares): an ncu figure stays valid while they do.
+SHARED_SOURCES = ("common.cuh", "tc.cuh", "tmap.h", "internal.h")
+KERNEL_SOURCES = {
+    "attn_fwd_tc": ("attn_tc.cu", "attn_common.cuh"),
+    "attn_bwd_tc": ("attn_tc.cu", "attn_common.cuh"),
+    "attn_fwd_fl": ("attn_flash.cu", "attn_common.cuh"),
+    "attn_bwd_fl": ("attn_flash.cu", "attn_common.cuh"),
+    "attn_fwd_simt": ("attn_simt.cu",),
+    "attn_bwd_simt": ("attn_simt.cu",),
+}
+
+
+def kernel_sources(kernel: str):
+    if kernel in KERNEL_SOURCES:
+        own = KERNEL_SOURCES[kernel]
+    elif kernel.startswith("gemm"):
+        own = ("gemm.cu", "epilogues.cuh")
+    else:
+        own = ("memory.cu",)
+    return own + SHARED_SOURCES
+
+
+def csrc_digest(kernel: str):
+    """Hash of the sources `kernel` is compiled from."""
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2608_13578_gb300", "csrc")
-    for f in sorted(os.listdir(d)):
-        with open(os.path.join(d, f), "rb") as fh:
-            h.update(f.encode() + fh.read())
+    for f in sorted(kernel_sources(kernel)):
+        path = os.path.join(d, f)
+        if os.path.exists(path):
+            with open(path, "rb") as fh:
+                h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
 
 
@@ -238,7 +264,7 @@ def ncu_traffic(kernel: str):
         with open(path) as f:
             d = json.load(f)
         e = d.get(kernel)
-        if e and e.get("csrc_digest") == csrc_digest():
+        if e and e.get("sources_digest") == csrc_digest(kernel):
             return e.get("dram_bytes_per_launch")
     except (OSError, ValueError):
         pass

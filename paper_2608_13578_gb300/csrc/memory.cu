@@ -63,13 +63,20 @@ __device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* _
   const int c = z * 256 + co * 8;
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   if (c < D) {
+    // the thread's rows rg, rg+8, ... four at a time, all loads first
     const T* Hc = Hm + row0 * D + c;
-    for (int r = rg; r < n; r += 8) {
-      float h[8];
-      load8(Hc + (long)r * D, h);
-      const float a = sc[r];
+    for (int r = rg; r < n; r += 32) {
+      float h[4][8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[e], acc[e]);
+      for (int u = 0; u < 4; ++u)
+        if (r + 8 * u < n) load8(Hc + (long)(r + 8 * u) * D, h[u]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (r + 8 * u < n) {
+          const float a = sc[r + 8 * u];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[u][e], acc[e]);
+        }
     }
   }
 #pragma unroll
