@@ -260,12 +260,13 @@ int device_sms() {
 bool dw_pair(int dtype, int M, int N) {
   return dtype == BCMT_BF16 && g_use_tc_gemm && M % 256 == 0 && N % 256 == 0;
 }
-int dw_splits(int dtype, int M, int N, long K) {
+int dw_splits(int dtype, int M, int N, long K, int max_pairs = 0) {
   const int nkb = (int)((K + 63) / 64);
   int target, tiles;
   if (dw_pair(dtype, M, N)) {
     tiles = (M / 256) * (N / 256);
     target = tiles >= 8 ? device_sms() / 2 : std::min(50, 12 * tiles);
+    if (max_pairs > 0) target = std::min(target, max_pairs);
   } else {
     tiles = ((M + 127) / 128) * ((N + 127) / 128);
     target = 100;
@@ -366,8 +367,8 @@ cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype,
                         int M, int N, long K,
                         const void* A, long lda, const void* B, long ldb, float* part, void* out,
                         Fork* reduce_beside = nullptr, const Launch* lcs = nullptr,
-                        Prof* prs = nullptr) {
-  const int splits = dw_splits(dtype, M, N, K);
+                        Prof* prs = nullptr, int max_pairs = 0) {
+  const int splits = dw_splits(dtype, M, N, K, max_pairs);
   EpiArgs ea;
   ea.out = part;
   ea.ldo = N;
@@ -536,39 +537,41 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // side stream: Sec. 3.4 adaptive block summaries, Sec. 3.5 exponential
-    // causal memory (scan), then its projection and one-block shift -> C
+    // side stream: Sec. 3.8 gate G = sigmoid(H W_g), independent of the memory
     fork.point();
-    prs.begin("summary_fwd");
-    e = summary_fwd(lcs, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
-    prs.end(nullptr);
+    {
+      EpiArgs ea;
+      ea.out = w.G;
+      ea.ldo = D;
+      ea.max_ctas = device_sms() / 2;  // half the SMs stay with the memory chain
+      e = run_gemm(lcs, prs, "gemm_gate", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
+                   EPI_GATE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "gate");
+    }
+    const int gate_done = fork.mark();
+    // critical stream, meanwhile: Sec. 3.4 adaptive block summaries, Sec. 3.5
+    // exponential causal memory (scan), then its projection and one-block
+    // shift -> C (a chain of small kernels: the longer of the two paths)
+    pr.begin("summary_fwd");
+    e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
+    pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
-    prs.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lcs, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C,
+    pr.begin("memory_scan_fwd");
+    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C,
                         g.B, g.Nb, D);
-    prs.end(nullptr);
+    pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "causal memory");
     {
       EpiArgs ea;
       ea.out = w.C;
       ea.ldo = D;
       ea.Nb = g.Nb;
-      e = run_gemm(lcs, prs, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
+      e = run_gemm(lc, pr, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
                    EPI_SHIFT, ea);
       if (e != cudaSuccess) return cuda_fail(e, "memory projection");
     }
-    const int memory_done = fork.mark();
-    // main stream, meanwhile: Sec. 3.8 gate G = sigmoid(H W_g)
-    {
-      EpiArgs ea;
-      ea.out = w.G;
-      ea.ldo = D;
-      e = run_gemm(lc, pr, "gemm_gate", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
-                   EPI_GATE, ea);
-      if (e != cudaSuccess) return cuda_fail(e, "gate");
-    }
-    // Sec. 3.7-3.8: Y = H + G * M_tokens once the memory rows are ready
-    fork.wait_mark(memory_done);
+    // Sec. 3.7-3.8: Y = H + G * M_tokens once the gate is ready too
+    fork.wait_mark(gate_done);
     pr.begin("inject");
     e = inject(lc, g.dtype, w.hloc, w.G, w.C, y, g.B, g.T, D, g.L);
     pr.end(nullptr);
@@ -662,8 +665,10 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                    1, EPI_STORE, ea);
       if (e != cudaSuccess) return cuda_fail(e, "dW_m");
     }
+    // (on a few SM pairs: it runs beside the pooling backward, which needs
+    // the rest, and has until the end of the backward)
     e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
-                    bw.part, dw_g);
+                    bw.part, dw_g, nullptr, nullptr, nullptr, device_sms() / 8);
     if (e != cudaSuccess) return cuda_fail(e, "dW_g");
     // main stream, meanwhile: dH = dY + dU W_g^T (the identity and gate paths)
     {

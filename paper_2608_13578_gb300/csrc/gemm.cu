@@ -434,7 +434,7 @@ static bool out_map(CUtensorMap* m, const Epi& epi, int M, int N, int splits) {
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
 static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
                              long sak, const void* B, long sbk, long sbn, const Epi& epi,
-                             int splits) {
+                             int splits, int max_ctas = 0) {
   using Cfg = TcCfg<BN, STAGES>;
   CUtensorMap mA, mB;
   if (!A_MN) {
@@ -464,7 +464,8 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
   CUtensorMap mC;
   if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
-  const int grid = n_tiles < sm_count() ? n_tiles : sm_count();
+  int grid = n_tiles < sm_count() ? n_tiles : sm_count();
+  if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   cudaError_t e = launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream, mA, mB, mC,
                            M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
@@ -751,7 +752,8 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
     switch (epi) {
       case EPI_GATE:
         return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                                             EpiGateF<bf16>{(bf16*)ea.out, ea.ldo}, 1);
+                                             EpiGateF<bf16>{(bf16*)ea.out, ea.ldo}, 1,
+                                             ea.max_ctas);
       case EPI_STORE_SCORE:
         return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,

@@ -37,6 +37,9 @@ struct EpiArgs {
   const void* add = nullptr;
   // token geometry: row m = b*T + t, block blk(t) = t / L, Nb blocks, width D
   int T = 1, L = 1, Nb = 1, D = 0;
+  // EPI_GATE on the tensor cores: at most this many persistent CTAs (0: one
+  // per SM), to leave SMs to a concurrent chain of small kernels
+  int max_ctas = 0;
 };
 
 // Number of non-empty K-splits when K (in 64-deep slices) is cut into
