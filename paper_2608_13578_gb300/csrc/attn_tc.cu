@@ -199,15 +199,16 @@ __global__ void __launch_bounds__(128)
 }
 
 // ===================================================================== backward
-// Shared memory: Q, K, dO (16 KB each) and a 32 KB region that holds V, then
-// P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in registers
-// until the dV product has consumed P.  80 KB per CTA: two CTAs per SM.
+// Shared memory: Q, K, dO, O (16 KB each) and a 32 KB region that holds V,
+// then P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in
+// registers until the dV product has consumed P.  96 KB per CTA: two CTAs per
+// SM.  O comes in by TMA with the other tiles (for Drow = dO . O).
 template <int NCH>
 __global__ void __launch_bounds__(128)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
                        const __grid_constant__ CUtensorMap mdQ, const __grid_constant__ CUtensorMap mdK,
-                       const __grid_constant__ CUtensorMap mdV, const bf16* __restrict__ O, long ld_o,
+                       const __grid_constant__ CUtensorMap mdV, const __grid_constant__ CUtensorMap mO,
                        const float* __restrict__ lse, int Tlen, int H, int L, float scale,
                        unsigned* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -217,7 +218,8 @@ __global__ void __launch_bounds__(128)
   uint8_t* sdO = smem + 2 * kTB;   // dO; then dV staging
   uint8_t* sV = smem + 3 * kTB;    // V, then (with the next 16 KB) P, then scale * dS
   uint8_t* sP = sV;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 5 * kTB);
+  uint8_t* sO = smem + 5 * kTB;    // O
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 6 * kTB);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -230,14 +232,16 @@ __global__ void __launch_bounds__(128)
     tc::prefetch_tmap(&mK);
     tc::prefetch_tmap(&mV);
     tc::prefetch_tmap(&mdO);
+    tc::prefetch_tmap(&mO);
   }
   pdl_enter();
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 4 * kTB);
+    tc::mbar_arrive_expect_tx(&bar[0], 5 * kTB);
     tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
     tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
     tc::tma_load_3d(sdO, &mdO, &bar[0], h * kDh, t0, b);
     tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
+    tc::tma_load_3d(sO, &mO, &bar[0], h * kDh, t0, b);
   }
   __syncwarp();
   if (warp == 0) {
@@ -270,23 +274,16 @@ __global__ void __launch_bounds__(128)
 
   const int r = warp * 32 + lane;
   const bool row_ok = (t0 + r) < Tlen;
-  // Drow = dO_r . O_r: the O row (global) is fetched before waiting for the tiles
-  uint4 ov[8];
-  float lr = 0.f;
-  if (row_ok) {
-    const bf16* orow = O + ((long)b * Tlen + t0 + r) * ld_o + h * kDh;
-#pragma unroll
-    for (int u = 0; u < 8; ++u) ov[u] = *reinterpret_cast<const uint4*>(orow + 8 * u);
-    lr = lse[((long)b * H + h) * Tlen + t0 + r];
-  }
+  const float lr = row_ok ? lse[((long)b * H + h) * Tlen + t0 + r] : 0.f;
   bool ok = tc::mbar_wait(&bar[0], 0, status);
-  float drow = 0.f;
+  float drow = 0.f;  // Drow = dO_r . O_r from the staged tiles
   if (row_ok) {
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       const uint4 gv = *reinterpret_cast<const uint4*>(sdO + tc::sw128_offset(r, u));
+      const uint4 ov = *reinterpret_cast<const uint4*>(sO + tc::sw128_offset(r, u));
       const bf16* gp = reinterpret_cast<const bf16*>(&gv);
-      const bf16* op = reinterpret_cast<const bf16*>(&ov[u]);
+      const bf16* op = reinterpret_cast<const bf16*>(&ov);
 #pragma unroll
       for (int e = 0; e < 8; ++e) drow = fmaf(__bfloat162float(gp[e]), __bfloat162float(op[e]), drow);
     }
@@ -435,7 +432,7 @@ static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, in
 }
 
 static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
-static constexpr int kBwdSmem = 5 * kTB + 1024 + 64;
+static constexpr int kBwdSmem = 6 * kTB + 1024 + 64;
 
 static int chunks_for(int L) { return L <= 32 ? 1 : L / 32; }
 
@@ -471,7 +468,7 @@ static cudaError_t bwd_launch(const Launch& lc, const AttnBwdArgs& a, const CUte
   if (cudaError_t e = smem_opt_in(attn_bwd_tc_kernel<NCH>, kBwdSmem, &opted); e != cudaSuccess) return e;
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
   cudaError_t e = launch_k(attn_bwd_tc_kernel<NCH>, grid, dim3(128), kBwdSmem, lc.stream, m[0],
-                           m[1], m[2], m[3], m[4], m[5], m[6], (const bf16*)f.O, f.ld_o, f.lse,
+                           m[1], m[2], m[3], m[4], m[5], m[6], m[7], f.lse,
                            f.T, f.H, f.L, 1.0f / sqrtf((float)f.dh), lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -480,12 +477,12 @@ cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
   const AttnArgs& f = a.f;
   if (!attn_tc_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
   const int D = f.H * kDh;
-  CUtensorMap m[7];
+  CUtensorMap m[8];
   if (!head_map(&m[0], f.Q, f.ld_qkv, D, f.T, f.B) || !head_map(&m[1], f.K, f.ld_qkv, D, f.T, f.B) ||
       !head_map(&m[2], f.V, f.ld_qkv, D, f.T, f.B) || !head_map(&m[3], a.dO, f.ld_o, D, f.T, f.B) ||
       !head_map(&m[4], a.dQ, a.ld_dqkv, D, f.T, f.B) ||
       !head_map(&m[5], a.dK, a.ld_dqkv, D, f.T, f.B) ||
-      !head_map(&m[6], a.dV, a.ld_dqkv, D, f.T, f.B))
+      !head_map(&m[6], a.dV, a.ld_dqkv, D, f.T, f.B) || !head_map(&m[7], f.O, f.ld_o, D, f.T, f.B))
     return cudaErrorInvalidValue;
   switch (chunks_for(f.L)) {
     case 1: return bwd_launch<1>(lc, a, m);
