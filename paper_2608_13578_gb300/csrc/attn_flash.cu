@@ -90,8 +90,12 @@ __device__ __forceinline__ void key_walk(int t0, int L, int& kstart, int& nkt) {
 // tile kt+1 is issued as soon as every thread has read tile kt's scores out of
 // TMEM and runs under tile kt's softmax; K of tile kt+2 streams in meanwhile.
 // V (single buffer) is reloaded once tile kt's P V product has completed.
-template <int DH>
-__global__ void __launch_bounds__(128)
+// NCH = the 32-key chunks a warp's rows can reach (1 or 2 for L < 128, else
+// 4); ONE: every query tile sees one key tile (L <= 128), so O can take the
+// columns of the consumed scores and the CTA needs 128 TMEM columns, not 256
+// (with fewer registers for NCH <= 2, three to four CTAs share an SM).
+template <int DH, int NCH, bool ONE>
+__global__ void __launch_bounds__(128, NCH <= 2 ? 3 : 2)
     attn_fwd_fl_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, bf16* __restrict__ O, long ld_o,
                        float* __restrict__ lse, int Tlen, int H, int L, float scale,
@@ -136,8 +140,10 @@ __global__ void __launch_bounds__(128)
     }
   }
   __syncwarp();
+  constexpr uint32_t kCols = ONE ? 128 : 256;  // S; O at kOcol
+  constexpr uint32_t kOcol = ONE ? 0 : 128;
   if (warp == 0) {
-    tc::tmem_alloc(tslot, 256);
+    tc::tmem_alloc(tslot, kCols);
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
@@ -182,9 +188,9 @@ __global__ void __launch_bounds__(128)
       }
       nld = chunks_needed(warp, wbs);
     }
-    uint32_t sr[4][32];
+    uint32_t sr[NCH][32];
 #pragma unroll
-    for (int ci = 0; ci < 4; ++ci)
+    for (int ci = 0; ci < NCH; ++ci)
       if (ci < nld) tc::tmem_ld32_issue(trow + (uint32_t)(wbs + ci * 32), sr[ci]);
     tc::tmem_wait();
     tc::fence_before_sync();
@@ -214,12 +220,12 @@ __global__ void __launch_bounds__(128)
     // Tiles left of the diagonal need no mask: their max, exponentials and
     // sum run with independent partial accumulators.
     float m_new, psum;
-    if (!diag) {
+    if (!ONE && !diag) {
       float mx[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
 #pragma unroll
-      for (int ci = 0; ci < 4; ++ci)
+      for (int ci = 0; ci < NCH; ++ci)
 #pragma unroll
         for (int j = 0; j < 32; ++j) mx[j & 7] = fmaxf(mx[j & 7], __uint_as_float(sr[ci][j]));
       const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
@@ -228,7 +234,7 @@ __global__ void __launch_bounds__(128)
       const float nm = -m_new;
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int u = 0; u < 16; ++u) {
+      for (int u = 0; u < 4 * NCH; ++u) {
         float v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -241,7 +247,7 @@ __global__ void __launch_bounds__(128)
     } else {
       float mt = -INFINITY;
 #pragma unroll
-      for (int ci = 0; ci < 4; ++ci)
+      for (int ci = 0; ci < NCH; ++ci)
         if (ci < nld) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -253,7 +259,7 @@ __global__ void __launch_bounds__(128)
       const float nm = -m_new;
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int ci = 0; ci < 4; ++ci)
+      for (int ci = 0; ci < NCH; ++ci)
         if (ci < nld) {
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -288,7 +294,7 @@ __global__ void __launch_bounds__(128)
       if (okv) {
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
-          tc::mma_bf16(tmem + 128, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
+          tc::mma_bf16(tmem + kOcol, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
       }
       tc::mma_commit(bar_o);
     }
@@ -301,7 +307,7 @@ __global__ void __launch_bounds__(128)
       tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart + (kt + 1) * kTile, b);
     }
     float o[DH];
-    tmem_row<DH>(trow + 128u, o);
+    tmem_row<DH>(trow + kOcol, o);
 #pragma unroll
     for (int c = 0; c < DH; ++c) oacc[c] = fmaf(oacc[c], alpha, o[c]);
   }
@@ -313,7 +319,7 @@ __global__ void __launch_bounds__(128)
   }
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
 }
 
 // ================================================================ backward: dQ
@@ -687,21 +693,30 @@ template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
 }
 
+template <int DH, int NCH, bool ONE>
+cudaError_t fwd_fl_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
+  static std::atomic<unsigned long long> opted{0};
+  auto kern = attn_fwd_fl_kernel<DH, NCH, ONE>;
+  cudaError_t e = smem_opt_in(kern, fwd_smem<DH>(), &opted);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
+  e = launch_k(kern, grid, dim3(128), fwd_smem<DH>(), lc.stream, m[0], m[1], m[2], (bf16*)a.O,
+               a.ld_o, a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)DH), lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 template <int DH>
 cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
   const int D = a.H * DH;
-  CUtensorMap mq, mk, mv;
-  if (!head_map_fl<DH>(&mq, a.Q, a.ld_qkv, D, a.T, a.B) ||
-      !head_map_fl<DH>(&mk, a.K, a.ld_qkv, D, a.T, a.B) ||
-      !head_map_fl<DH>(&mv, a.V, a.ld_qkv, D, a.T, a.B))
+  CUtensorMap m[3];
+  if (!head_map_fl<DH>(&m[0], a.Q, a.ld_qkv, D, a.T, a.B) ||
+      !head_map_fl<DH>(&m[1], a.K, a.ld_qkv, D, a.T, a.B) ||
+      !head_map_fl<DH>(&m[2], a.V, a.ld_qkv, D, a.T, a.B))
     return cudaErrorInvalidValue;
-  static std::atomic<unsigned long long> opted{0};
-  cudaError_t e = smem_opt_in(attn_fwd_fl_kernel<DH>, fwd_smem<DH>(), &opted);
-  if (e != cudaSuccess) return e;
-  dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
-  e = launch_k(attn_fwd_fl_kernel<DH>, grid, dim3(128), fwd_smem<DH>(), lc.stream, mq, mk, mv,
-               (bf16*)a.O, a.ld_o, a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)DH), lc.status);
-  return e != cudaSuccess ? e : cudaGetLastError();
+  if (a.L > kTile) return fwd_fl_launch<DH, 4, false>(lc, a, m);
+  if (a.L <= 32) return fwd_fl_launch<DH, 1, true>(lc, a, m);
+  if (a.L == 64) return fwd_fl_launch<DH, 2, true>(lc, a, m);
+  return fwd_fl_launch<DH, 4, true>(lc, a, m);
 }
 
 template <int DH>
