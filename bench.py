@@ -450,10 +450,12 @@ def bench_ours(args):
                    "share": round(ms / sum(v[1] for v in prof.values()), 4)}
                for k, (c, ms) in sorted(prof.items(), key=lambda kv: -kv[1][1])}
 
-    # ---- dense causal attention of the same shape (library SDPA), context only
-    dense = None
+    # ---- dense causal attention of the same shape (library SDPA), and the same
+    # BCMT layer written with eager torch ops: context only
+    dense = eager_bcmt = None
     if not args.no_dense and rank == 0:
         dense = bench_dense(w, t, stream, flush, args)
+        eager_bcmt = bench_torch_bcmt(w, t, stream, flush, args)
 
     out = None
     if rank == 0:
@@ -489,6 +491,7 @@ def bench_ours(args):
                               "note": "per-kernel times come from this second pass of the "
                                       "same steps; value comes from the pass without them"},
             "dense_causal_baseline": dense,
+            "torch_eager_bcmt_baseline": eager_bcmt,
         }
         print(json.dumps(out))
     if world > 1:
@@ -528,6 +531,73 @@ def bench_dense(w, t, stream, flush, args):
         tot += a.elapsed_time(b)
     return {"value": round(B * T * args.steps / (tot / 1e3), 1), "unit": UNIT,
             "what": "x W_qkv -> torch SDPA(is_causal) over the full sequence -> W_O, fwd+bwd, bf16"}
+
+
+def torch_bcmt_layer(x, w_qkv, w_o, w_p, w_m, w_g, decay, L, H):
+    """The BCMT layer (Sec. 3.3-3.8) written with eager torch ops, as a
+    framework-level implementation would: blocks folded into the batch for
+    torch's SDPA (is_causal), the pooling softmax per block, the decayed memory
+    as a masked weight matrix over blocks, the shifted projection, the gate.
+    A baseline for context, differentiable by autograd."""
+    import torch
+    import torch.nn.functional as F
+    B, T, D = x.shape
+    dh = D // H
+    Nb = (T + L - 1) // L
+    Tp = Nb * L
+    qkv = x @ w_qkv
+    if Tp != T:
+        qkv = F.pad(qkv, (0, 0, 0, Tp - T))
+    q, k, v = qkv.view(B, Nb, L, 3, H, dh).permute(3, 0, 1, 4, 2, 5).reshape(3, B * Nb, H, L, dh)
+    o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+    hhat = o.view(B, Nb, H, L, dh).permute(0, 1, 3, 2, 4).reshape(B, Tp, D)[:, :T]
+    hm = hhat @ w_o
+    s = (hm @ w_p.unsqueeze(1)).squeeze(-1).float()
+    hp = hm.float()
+    if Tp != T:
+        s = F.pad(s, (0, Tp - T), value=float("-inf"))
+        hp = F.pad(hp, (0, 0, 0, Tp - T))
+    alpha = torch.softmax(s.view(B, Nb, L), dim=-1)
+    S = torch.einsum("bnl,bnld->bnd", alpha, hp.view(B, Nb, L, D))
+    idx = torch.arange(Nb, device=x.device)
+    e = (idx[:, None] - idx[None, :]).clamp(min=0).to(torch.float32)
+    lower = (idx[:, None] >= idx[None, :]).to(torch.float32)
+    wts = decay.float()[None, None, :] ** e[:, :, None] * lower[:, :, None]
+    M = torch.einsum("ijd,bjd->bid", wts, S) / wts.sum(1)
+    P = M.to(x.dtype) @ w_m
+    C = torch.cat([torch.zeros_like(P[:, :1]), P[:, :-1]], dim=1)
+    G = torch.sigmoid(hm @ w_g)
+    return hm + G * C.repeat_interleave(L, dim=1)[:, :T]
+
+
+def bench_torch_bcmt(w, t, stream, flush, args):
+    """The same layer in eager torch (torch_bcmt_layer), fwd+bwd tokens/s."""
+    import torch
+    names = ("w_qkv", "w_o", "w_p", "w_m", "w_g")
+    params = {n: t[n].detach().clone().requires_grad_(True) for n in names}
+    x = t["x"].detach().clone().requires_grad_(True)
+    dy, decay = t["dy"], t["decay"]
+
+    def step():
+        y = torch_bcmt_layer(x, params["w_qkv"], params["w_o"], params["w_p"], params["w_m"],
+                             params["w_g"], decay, w.L, w.H)
+        y.backward(dy)
+
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    tot = 0.0
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        tot += a.elapsed_time(b)
+    return {"value": round(w.B * w.T * args.steps / (tot / 1e3), 1), "unit": UNIT,
+            "what": "the BCMT layer in eager torch ops (blocks folded into the batch for SDPA, "
+                    "pooling, masked decay weights, shifted W_m, gate), fwd+bwd, autograd"}
 
 
 # ------------------------------------------------ whole-model training steps
