@@ -138,3 +138,10 @@ def test_sequence_scaling(cuda_ok, T):
     # Full comparison at the shortest length; batch element 0 of Y and dX at the
     # longer ones (the mixer is independent across the batch).
     _check(w, backward=True, batch=None if T == 2048 else slice(0, 1))
+
+
+@pytest.mark.parametrize("L", [64, 128, 256, 512])
+def test_paper_shape(cuda_ok, L):
+    """One layer of the paper's model shape (Sec. 4.1: D 128, 8 heads of 16,
+    batch 16, context 1024) at the block sizes of its Table 2, full size."""
+    _check(WORKLOADS[f"paper_bf16_b16_t1024_l{L}_d128_h8"], backward=True)
