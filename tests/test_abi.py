@@ -58,6 +58,7 @@ def test_workspace_sizes_host_only(C):
     ("L", 0, "BCMT_ERR_SHAPE"),
     ("L", 4096, "BCMT_ERR_UNSUPPORTED"),
     ("T", 0, "BCMT_ERR_SHAPE"),
+    ("B", 0, "BCMT_ERR_SHAPE"),
     ("dtype", 7, "BCMT_ERR_ARG"),
     ("flags", 64, "BCMT_ERR_ARG"),
 ])

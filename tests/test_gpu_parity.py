@@ -40,6 +40,14 @@ SMALL = [
     W(2, 600, 256, 4, 512, "bf16"),                     # dh = 64, L = 512
     W(1, 200, 128, 8, 32, "fp32"),
     W(2, 256, 128, 2, 64, "bf16", decay=(0.0, 0.0)),
+    # degenerate shapes
+    W(1, 1, 128, 4, 16, "fp32"),                         # a single token
+    W(2, 1, 64, 1, 64, "bf16"),                          # single token, one 64-wide head
+    W(1, 33, 128, 2, 1, "fp32"),                         # L = 1: every token its own block
+    W(2, 50, 128, 2, 8, "bf16"),                         # L = 8 (SIMT attention in bf16)
+    W(2, 64, 128, 2, 64, "bf16"),                        # T = L: one full block, no memory
+    W(1, 40, 128, 1, 8, "fp32"),                         # the widest head, d_h = 128
+    W(1, 1100, 64, 1, 1024, "bf16"),                     # the largest block, ragged tail
 ]
 VARIANTS = [
     W(2, 100, 128, 4, 16, "fp32", input_is_x=False),
