@@ -715,11 +715,17 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     e = run_gemm(lc, pr, "gemm_dhhat", g.dtype, g.dtype, n, D, D, dH, D, 1, w_o, 1, D, EPI_STORE,
                  ea);
     if (e != cudaSuccess) return cuda_fail(e, "dHhat");
-    // dW_O on the critical stream (beside the attention backward the side
-    // stream's weight-gradient GEMMs would find no free SM); its reduction on
-    // the side stream
-    e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D, bw.part_o,
-                    dw_o, &fork, &lcs, &prs);
+    // dW_O: a small one (at most 8 GFLOP) goes to the side stream on a few SM
+    // pairs and runs beside the tail of the step (dx, dW_QKV); a large one
+    // stays on the critical stream with its reduction beside
+    if (2.0 * D * D * (double)g.n <= 8e9) {
+      fork.point();
+      e = weight_grad(lcs, prs, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D,
+                      bw.part_o, dw_o, nullptr, nullptr, nullptr, device_sms() / 12);
+    } else {
+      e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D,
+                      bw.part_o, dw_o, &fork, &lcs, &prs);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "dW_O");
   }
   // Attention backward -> dQ, dK, dV.
