@@ -56,13 +56,14 @@ unsigned* status_ptr() {
 // which no later step of the pass reads: they run beside the dependent chain
 // (forked and joined with events, so the pair can also be captured into a
 // CUDA graph).  Streams and events are host-side objects: no device memory.
-constexpr int kSideEvents = 12;
+constexpr int kSideEvents = 16;
 // Per device: the layer's critical path runs on `crit` (the highest stream
 // priority) and the work beside it (memory stage in the forward, weight
 // gradients in the backward) on `side` (the lowest), so that when both have
-// CTAs waiting the block scheduler places the critical ones first.
+// CTAs waiting the block scheduler places the critical ones first.  `side2`
+// (also lowest) takes work that must not hold up what is queued on `side`.
 struct SideStream {
-  cudaStream_t crit = nullptr, side = nullptr;
+  cudaStream_t crit = nullptr, side = nullptr, side2 = nullptr;
   cudaEvent_t ev[kSideEvents] = {};
   std::mutex mu;  // one call at a time may use the streams' events
 };
@@ -80,7 +81,8 @@ SideStream* side_stream() {
     bool ok = cudaDeviceGetStreamPriorityRange(&least, &greatest) == cudaSuccess &&
               cudaStreamCreateWithPriority(&ss->crit, cudaStreamNonBlocking, greatest) ==
                   cudaSuccess &&
-              cudaStreamCreateWithPriority(&ss->side, cudaStreamNonBlocking, least) == cudaSuccess;
+              cudaStreamCreateWithPriority(&ss->side, cudaStreamNonBlocking, least) == cudaSuccess &&
+              cudaStreamCreateWithPriority(&ss->side2, cudaStreamNonBlocking, least) == cudaSuccess;
     for (int i = 0; i < kSideEvents && ok; ++i)
       ok = cudaEventCreateWithFlags(&ss->ev[i], cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
@@ -102,7 +104,7 @@ struct Fork {
   SideStream* ss;
   cudaStream_t user;
   int next = 0;
-  bool forked = false;
+  bool forked = false, forked2 = false;
   Fork(SideStream* s, cudaStream_t u) : ss(s), user(u) {
     if (!ss) return;
     ss->mu.lock();
@@ -112,19 +114,29 @@ struct Fork {
   }
   cudaStream_t main() const { return ss ? ss->crit : user; }
   cudaStream_t side() const { return ss ? ss->side : user; }
+  cudaStream_t side2() const { return ss ? ss->side2 : user; }
   // the side stream waits for everything enqueued on the critical stream so far
   bool point() {
-    if (!ss || next >= kSideEvents - 2) return false;
+    if (!ss || next >= kSideEvents - 3) return false;
     cudaEventRecord(ss->ev[next], ss->crit);
     cudaStreamWaitEvent(ss->side, ss->ev[next], 0);
     ++next;
     forked = true;
     return true;
   }
+  // the same for the second side stream
+  bool point2() {
+    if (!ss || next >= kSideEvents - 3) return false;
+    cudaEventRecord(ss->ev[next], ss->crit);
+    cudaStreamWaitEvent(ss->side2, ss->ev[next], 0);
+    ++next;
+    forked2 = true;
+    return true;
+  }
   // records what the side stream has been given so far; wait_mark(m) later
   // makes the critical stream wait for exactly that
   int mark() {
-    if (!ss || !forked || next >= kSideEvents - 2) return -1;
+    if (!ss || !forked || next >= kSideEvents - 3) return -1;
     cudaEventRecord(ss->ev[next], ss->side);
     return next++;
   }
@@ -133,6 +145,10 @@ struct Fork {
   }
   ~Fork() {
     if (!ss) return;
+    if (forked2) {
+      cudaEventRecord(ss->ev[kSideEvents - 3], ss->side2);
+      cudaStreamWaitEvent(ss->crit, ss->ev[kSideEvents - 3], 0);
+    }
     if (forked) {
       cudaEventRecord(ss->ev[kSideEvents - 2], ss->side);
       cudaStreamWaitEvent(ss->crit, ss->ev[kSideEvents - 2], 0);
@@ -715,12 +731,15 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     e = run_gemm(lc, pr, "gemm_dhhat", g.dtype, g.dtype, n, D, D, dH, D, 1, w_o, 1, D, EPI_STORE,
                  ea);
     if (e != cudaSuccess) return cuda_fail(e, "dHhat");
-    // dW_O: a small one (at most 8 GFLOP) goes to the side stream on a few SM
-    // pairs and runs beside the tail of the step (dx, dW_QKV); a large one
-    // stays on the critical stream with its reduction beside
+    // dW_O: a small one (at most 8 GFLOP) goes to the second side stream on a
+    // few SM pairs and runs beside the tail of the step (dx, dW_QKV) without
+    // holding up dW_QKV; a large one stays on the critical stream with its
+    // reduction beside
     if (2.0 * D * D * (double)g.n <= 8e9) {
-      fork.point();
-      e = weight_grad(lcs, prs, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D,
+      fork.point2();
+      Launch lcs2{fork.side2(), sp};
+      Prof prs2{profiling, fork.side2()};
+      e = weight_grad(lcs2, prs2, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D,
                       bw.part_o, dw_o, nullptr, nullptr, nullptr, device_sms() / 12);
     } else {
       e = weight_grad(lc, pr, "gemm_dw_o", g.dtype, g.dtype, D, D, g.n, w.hhat, D, dH, D,
