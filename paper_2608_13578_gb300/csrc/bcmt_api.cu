@@ -681,10 +681,11 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                    1, EPI_STORE, ea);
       if (e != cudaSuccess) return cuda_fail(e, "dW_m");
     }
-    // (on a few SM pairs: it runs beside the pooling backward, which needs
-    // the rest, and has until the end of the backward)
+    // (up to 32 GFLOP on a few SM pairs: it runs beside the pooling backward,
+    // which needs the rest, and has until the end of the backward)
     e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
-                    bw.part, dw_g, nullptr, nullptr, nullptr, device_sms() / 8);
+                    bw.part, dw_g, nullptr, nullptr, nullptr,
+                    2.0 * D * D * (double)g.n <= 32e9 ? device_sms() / 8 : 0);
     if (e != cudaSuccess) return cuda_fail(e, "dW_g");
     // main stream, meanwhile: dH = dY + dU W_g^T (the identity and gate paths)
     {
