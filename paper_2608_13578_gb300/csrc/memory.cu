@@ -17,6 +17,40 @@ constexpr int kThreads = 256;
 }  // namespace
 
 // ======================================================== work items (device)
+// Four or eight consecutive values of a row, held as loaded: bf16 stays packed
+// until it is used, so that a batch of rows' loads can be in flight with few
+// registers.
+template <class T> struct Raw4 { float4 v; };
+template <> struct Raw4<bf16> { uint2 v; };
+__device__ __forceinline__ void ld_raw(const float* p, Raw4<float>& r) {
+  r.v = *reinterpret_cast<const float4*>(p);
+}
+__device__ __forceinline__ void ld_raw(const bf16* p, Raw4<bf16>& r) {
+  r.v = *reinterpret_cast<const uint2*>(p);
+}
+__device__ __forceinline__ void unraw(const Raw4<float>& r, float* v) {
+  v[0] = r.v.x; v[1] = r.v.y; v[2] = r.v.z; v[3] = r.v.w;
+}
+__device__ __forceinline__ void unraw(const Raw4<bf16>& r, float* v) {
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.v.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.v.y));
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+}
+template <class T> struct Raw8 { float4 lo, hi; };
+template <> struct Raw8<bf16> { uint4 v; };
+__device__ __forceinline__ void ld_raw(const float* p, Raw8<float>& r) {
+  r.lo = *reinterpret_cast<const float4*>(p);
+  r.hi = *reinterpret_cast<const float4*>(p + 4);
+}
+__device__ __forceinline__ void ld_raw(const bf16* p, Raw8<bf16>& r) {
+  r.v = *reinterpret_cast<const uint4*>(p);
+}
+__device__ __forceinline__ void unraw(const Raw8<float>& r, float* v) {
+  v[0] = r.lo.x; v[1] = r.lo.y; v[2] = r.lo.z; v[3] = r.lo.w;
+  v[4] = r.hi.x; v[5] = r.hi.y; v[6] = r.hi.z; v[7] = r.hi.w;
+}
+__device__ __forceinline__ void unraw(const Raw8<bf16>& r, float* v) { unpack8(r.v, v); }
+
 // Sec. 3.4: item (i, b, z): pooling scores of block i of batch b summed from
 // the npart partial dot products the W_O epilogue wrote, alpha = softmax over
 // the block (stored by z == 0), S_i[256 z .. 256 z + 255] = sum_t alpha_t H_t.
@@ -109,32 +143,35 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
   if (c < D) {
     float cm[4];
     load4(Cmem + ((long)b * Nb + i) * D + c, cm);
-    // rows rg, rg+8, ... in batches of 8: every load of a batch is issued
-    // before its first store
-    for (int r0 = rg; r0 < n; r0 += 64) {
-      float dy[8][4], g[8][4];
+    // rows rg, rg+8, ... in batches of 4 (loads held packed): every load of
+    // a batch is issued before its first store
+    const long step = 8L * D;
+    const long o0 = ((long)b * Tlen + t0 + rg) * D + c;
+    const T* dyp = dY + o0;
+    const T* gp = G + o0;
+    T* dup = dU + o0;
+#pragma unroll 1
+    for (int r0 = rg; r0 < n; r0 += 32, dyp += 4 * step, gp += 4 * step, dup += 4 * step) {
+      Raw4<T> rdy[4], rgt[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int r = r0 + 8 * u;
-        if (r < n) {
-          const long o = ((long)b * Tlen + t0 + r) * D + c;
-          load4(dY + o, dy[u]);
-          load4(G + o, g[u]);
+      for (int u = 0; u < 4; ++u)
+        if (r0 + 8 * u < n) {
+          ld_raw(dyp + u * step, rdy[u]);
+          ld_raw(gp + u * step, rgt[u]);
         }
-      }
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int r = r0 + 8 * u;
-        if (r < n) {
-          float du[4];
+      for (int u = 0; u < 4; ++u)
+        if (r0 + 8 * u < n) {
+          float dy[4], g[4], du[4];
+          unraw(rdy[u], dy);
+          unraw(rgt[u], g);
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            du[e] = dy[u][e] * cm[e] * g[u][e] * (1.0f - g[u][e]);
-            acc[e] = fmaf(dy[u][e], g[u][e], acc[e]);
+            du[e] = dy[e] * cm[e] * g[e] * (1.0f - g[e]);
+            acc[e] = fmaf(dy[e], g[e], acc[e]);
           }
-          store4(dU + ((long)b * Tlen + t0 + r) * D + c, du);
+          store4(dup + u * step, du);
         }
-      }
     }
   }
 #pragma unroll
@@ -406,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 // broadcast by index.  Each thread takes two runs of 8 channels and issues
 // all their loads before its stores.
 template <class T>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 3)
     inject_kernel(const T* __restrict__ Hm, const T* __restrict__ G, const float* __restrict__ Cm,
                   T* __restrict__ Y, long n_rows, int Tlen, int D, int L, int Nb) {
   pdl_enter();
@@ -414,7 +451,8 @@ __global__ void __launch_bounds__(kThreads)
   const long total = n_rows * runs;
   const long stride = (long)gridDim.x * kThreads;
   for (long i0 = (long)blockIdx.x * kThreads + threadIdx.x; i0 < total; i0 += 2 * stride) {
-    float h[2][8], g[2][8], c[2][8];
+    Raw8<T> rh[2], rgt[2];
+    Raw8<float> rc[2];
     long o[2];
     bool live[2];
 #pragma unroll
@@ -426,18 +464,19 @@ __global__ void __launch_bounds__(kThreads)
       const int cc = (int)(i - row * runs) * 8;
       const int b = (int)(row / Tlen), t = (int)(row - (long)b * Tlen);
       o[u] = row * D + cc;
-      load8(Hm + o[u], h[u]);
-      load8(G + o[u], g[u]);
-      const float* cm = Cm + ((long)b * Nb + t / L) * D + cc;
-      load4(cm, c[u]);
-      load4(cm + 4, c[u] + 4);
+      ld_raw(Hm + o[u], rh[u]);
+      ld_raw(G + o[u], rgt[u]);
+      ld_raw(Cm + ((long)b * Nb + t / L) * D + cc, rc[u]);
     }
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
       if (!live[u]) continue;
-      float y[8];
+      float h[8], g[8], c[8], y[8];
+      unraw(rh[u], h);
+      unraw(rgt[u], g);
+      unraw(rc[u], c);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) y[e] = fmaf(g[u][e], c[u][e], h[u][e]);
+      for (int e = 0; e < 8; ++e) y[e] = fmaf(g[e], c[e], h[e]);
       store8(Y + o[u], y);
     }
   }
