@@ -87,7 +87,8 @@ while True:
     O.backward(fw, t["dy"])
     times.append(time.perf_counter() - s)
     reps += 1
-    if time.perf_counter() - t0 > budget or reps >= {max_reps}:
+    # a budget of 0 runs exactly max_reps repetitions
+    if reps >= {max_reps} or (budget > 0 and time.perf_counter() - t0 > budget):
         break
 print(json.dumps({{"tokens": w.T, "reps": reps, "seconds": sum(times), "times": times}}))
 """
