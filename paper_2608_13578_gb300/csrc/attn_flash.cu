@@ -33,51 +33,6 @@ using namespace attn;
 namespace {
 constexpr int kTile = 128;
 
-template <int DH>
-struct Geo {
-  static constexpr uint32_t span = DH * 2;                    // bytes per tile row
-  static constexpr uint32_t tile = kTile * span;              // one 128-row tile
-  static constexpr uint32_t sbo = 8 * span;                   // 8-row atom
-  static constexpr uint32_t layout = DH == 64 ? 2u : DH == 32 ? 4u : 6u;
-  // K-major [rows x DH] operand at row offset `row0`, K step kk (16 columns)
-  static __device__ __forceinline__ uint64_t kmaj(const uint8_t* t, int row0, int kk) {
-    return tc::sdesc_sw(tc::smem_u32(t) + row0 * span + kk * 32, 16, sbo, layout);
-  }
-  // the same tile read MN-major (DH contiguous = N), K = rows from row0, step kk
-  static __device__ __forceinline__ uint64_t mnmaj(const uint8_t* t, int row0, int kk) {
-    return tc::sdesc_sw(tc::smem_u32(t) + (row0 + kk * 16) * span, tile, sbo, layout);
-  }
-};
-
-// A [128 x 128] bf16 operand in two 64-column swizzle-128 halves (put_unit's
-// layout), read K-major from column 64*half, K step kk.  A single 64-column
-// half buffer is read with half = 0 and kk < 4.
-__device__ __forceinline__ uint64_t p_kmaj(const uint8_t* p, int half, int kk) {
-  return tc::sdesc(tc::smem_u32(p) + half * 16384 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-}
-
-// Loads TMEM columns col .. col+DH-1 of the warp's lane quarter (thread = row).
-template <int DH>
-__device__ __forceinline__ void tmem_row(uint32_t taddr, float* v) {
-  uint32_t r[2][32];
-  tc::tmem_ld32_issue(taddr, r[0]);
-  if (DH > 32) tc::tmem_ld32_issue(taddr + 32u, r[1]);
-  tc::tmem_wait();
-#pragma unroll
-  for (int c = 0; c < DH; ++c) v[c] = __uint_as_float(r[c >> 5][c & 31]);
-}
-
-template <int DH>
-__device__ __forceinline__ void store_row(bf16* dst, const float* v, float mul) {
-#pragma unroll
-  for (int u = 0; u < DH / 8; ++u) {
-    float t[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) t[e] = v[8 * u + e] * mul;
-    *reinterpret_cast<uint4*>(dst + 8 * u) = pack8(t);
-  }
-}
-
 // First key of the key-tile walk of the query tile at t0, and the tile count.
 __device__ __forceinline__ void key_walk(int t0, int L, int& kstart, int& nkt) {
   kstart = L >= kTile ? (t0 / L) * L : t0;

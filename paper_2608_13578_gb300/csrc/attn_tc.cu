@@ -199,11 +199,26 @@ __global__ void __launch_bounds__(128)
 }
 
 // ===================================================================== backward
-// Shared memory: Q, K, dO, O (16 KB each) and a 32 KB region that holds V,
-// then P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in
-// registers until the dV product has consumed P.  96 KB per CTA: two CTAs per
-// SM.  O comes in by TMA with the other tiles (for Drow = dO . O).
-template <int NCH>
+// For head widths DH in {16, 32, 64}.  Shared memory: the Q, K, dO, V and O
+// tiles (128 x DH, TMA-swizzled with a one-row span) and a 32 KB region that
+// holds P (for dV = P^T dO), then scale * dS (for dK and dQ): dS waits in
+// registers until the dV product has consumed P.  At DH = 64 the P region
+// covers V and the 16 KB after it (96 KB per CTA: two CTAs per SM); at
+// DH = 16 / 32 it follows the five tiles (52 / 72 KB).  O comes in by TMA
+// with the other tiles (for Drow = dO . O).  The gradients leave through the
+// Q, K, dO tiles as staging, in the same layout, by TMA stores.
+template <int DH>
+__device__ __forceinline__ void stage_row(uint8_t* tile, int r, const float* v) {
+#pragma unroll
+  for (int u = 0; u < DH / 8; ++u)
+    *reinterpret_cast<uint4*>(tile + Geo<DH>::unit(r, u)) = pack8(v + 8 * u);
+}
+
+template <int DH> constexpr int bwd_smem_bytes() {
+  return (DH == 64 ? 6 * Geo<DH>::tile : 5 * Geo<DH>::tile + 32768) + 1024 + 64;
+}
+
+template <int NCH, int DH>
 __global__ void __launch_bounds__(128)
     attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mdO,
@@ -211,15 +226,17 @@ __global__ void __launch_bounds__(128)
                        const __grid_constant__ CUtensorMap mdV, const __grid_constant__ CUtensorMap mO,
                        const float* __restrict__ lse, int Tlen, int H, int L, float scale,
                        unsigned* status) {
+  using G = Geo<DH>;
+  constexpr uint32_t kT = G::tile;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sQ = smem;              // Q; then dQ staging
-  uint8_t* sK = smem + kTB;        // K; then dK staging
-  uint8_t* sdO = smem + 2 * kTB;   // dO; then dV staging
-  uint8_t* sV = smem + 3 * kTB;    // V, then (with the next 16 KB) P, then scale * dS
-  uint8_t* sP = sV;
-  uint8_t* sO = smem + 5 * kTB;    // O
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 6 * kTB);
+  uint8_t* sK = smem + kT;         // K; then dK staging
+  uint8_t* sdO = smem + 2 * kT;    // dO; then dV staging
+  uint8_t* sV = smem + 3 * kT;     // V
+  uint8_t* sO = smem + (DH == 64 ? 5 : 4) * kT;  // O
+  uint8_t* sP = DH == 64 ? sV : smem + 5 * kT;    // P, then scale * dS (32 KB)
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + (DH == 64 ? 6 * kT : 5 * kT + 32768));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -236,12 +253,12 @@ __global__ void __launch_bounds__(128)
   }
   pdl_enter();
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 5 * kTB);
-    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sdO, &mdO, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sO, &mO, &bar[0], h * kDh, t0, b);
+    tc::mbar_arrive_expect_tx(&bar[0], 5 * kT);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sO, &mO, &bar[0], h * DH, t0, b);
   }
   __syncwarp();
   if (warp == 0) {
@@ -260,13 +277,12 @@ __global__ void __launch_bounds__(128)
     if (ok) {
       constexpr uint32_t id128 = tc::idesc_bf16(128, 128, 0, 0);
 #pragma unroll
-      for (int kk = 0; kk < kDh / 16; ++kk)  // S = Q K^T -> TMEM columns 0..127
-        tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sQ) + kk * 32, 16, 1024),
-                     tc::sdesc(tc::smem_u32(sK) + kk * 32, 16, 1024), id128, kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < DH / 16; ++kk)  // S = Q K^T -> TMEM columns 0..127
+        tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 0, kk), id128, kk > 0 ? 1u : 0u);
 #pragma unroll
-      for (int kk = 0; kk < kDh / 16; ++kk)  // dP = dO V^T -> TMEM columns 128..255
-        tc::mma_bf16(tmem + 128, tc::sdesc(tc::smem_u32(sdO) + kk * 32, 16, 1024),
-                     tc::sdesc(tc::smem_u32(sV) + kk * 32, 16, 1024), id128, kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < DH / 16; ++kk)  // dP = dO V^T -> TMEM columns 128..255
+        tc::mma_bf16(tmem + 128, G::kmaj(sdO, 0, kk), G::kmaj(sV, 0, kk), id128,
+                     kk > 0 ? 1u : 0u);
     }
     tc::mma_commit(&bar[1]);
   }
@@ -279,9 +295,9 @@ __global__ void __launch_bounds__(128)
   float drow = 0.f;  // Drow = dO_r . O_r from the staged tiles
   if (row_ok) {
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const uint4 gv = *reinterpret_cast<const uint4*>(sdO + tc::sw128_offset(r, u));
-      const uint4 ov = *reinterpret_cast<const uint4*>(sO + tc::sw128_offset(r, u));
+    for (int u = 0; u < DH / 8; ++u) {
+      const uint4 gv = *reinterpret_cast<const uint4*>(sdO + G::unit(r, u));
+      const uint4 ov = *reinterpret_cast<const uint4*>(sO + G::unit(r, u));
       const bf16* gp = reinterpret_cast<const bf16*>(&gv);
       const bf16* op = reinterpret_cast<const bf16*>(&ov);
 #pragma unroll
@@ -343,12 +359,12 @@ __global__ void __launch_bounds__(128)
 
   if (tid == 0) {
     tc::fence_after_sync();
-    // dV = P^T dO -> columns 0..63 (A = P read MN-major: M = keys, K = queries)
-    constexpr uint32_t idMN = tc::idesc_bf16(128, kDh, 1, 1);
+    // dV = P^T dO -> columns 0.. (A = P read MN-major: M = keys, K = queries)
+    constexpr uint32_t idMN = tc::idesc_bf16(128, DH, 1, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
       tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sP) + kk * 2048, 16384, 1024),
-                   tc::sdesc(tc::smem_u32(sdO) + kk * 2048, 8192, 1024), idMN, kk > 0 ? 1u : 0u);
+                   G::mnmaj(sdO, 0, kk), idMN, kk > 0 ? 1u : 0u);
     tc::mma_commit(&bar[2]);
   }
   __syncwarp();
@@ -373,18 +389,17 @@ __global__ void __launch_bounds__(128)
   if (tid == 0) {
     tc::fence_after_sync();
     const uint32_t adS = tc::smem_u32(sP);
-    // dK = dS^T Q -> columns 64..127
-    constexpr uint32_t idMN = tc::idesc_bf16(128, kDh, 1, 1);
+    // dK = dS^T Q -> columns 64..
+    constexpr uint32_t idMN = tc::idesc_bf16(128, DH, 1, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
-      tc::mma_bf16(tmem + 64, tc::sdesc(adS + kk * 2048, 16384, 1024),
-                   tc::sdesc(tc::smem_u32(sQ) + kk * 2048, 8192, 1024), idMN, kk > 0 ? 1u : 0u);
-    // dQ = dS K -> columns 128..191 (A = dS K-major, B = K read MN-major)
-    constexpr uint32_t idKM = tc::idesc_bf16(128, kDh, 0, 1);
+      tc::mma_bf16(tmem + 64, tc::sdesc(adS + kk * 2048, 16384, 1024), G::mnmaj(sQ, 0, kk), idMN,
+                   kk > 0 ? 1u : 0u);
+    // dQ = dS K -> columns 128.. (A = dS K-major, B = K read MN-major)
+    constexpr uint32_t idKM = tc::idesc_bf16(128, DH, 0, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
-      tc::mma_bf16(tmem + 128, tc::sdesc(adS + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                   tc::sdesc(tc::smem_u32(sK) + kk * 2048, 8192, 1024), idKM, kk > 0 ? 1u : 0u);
+      tc::mma_bf16(tmem + 128, p_kmaj(sP, 0, kk), G::mnmaj(sK, 0, kk), idKM, kk > 0 ? 1u : 0u);
     tc::mma_commit(&bar[3]);
   }
   __syncwarp();
@@ -396,21 +411,18 @@ __global__ void __launch_bounds__(128)
     uint8_t* const dst[3] = {sdO, sK, sQ};  // dV, dK, dQ staging tiles
 #pragma unroll
     for (int q = 0; q < 3; ++q) {
-      uint32_t o[2][32];
-      tc::tmem_ld32_issue(trow + (uint32_t)(64 * q), o[0]);
-      tc::tmem_ld32_issue(trow + (uint32_t)(64 * q + 32), o[1]);
-      tc::tmem_wait();
-      stage_half(dst[q], r, 0, reinterpret_cast<const float*>(o[0]), 1.0f);
-      stage_half(dst[q], r, 1, reinterpret_cast<const float*>(o[1]), 1.0f);
+      float v[DH];
+      tmem_row<DH>(trow + (uint32_t)(64 * q), v);
+      stage_row<DH>(dst[q], r, v);
     }
   }
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
   if (tid == 0 && ok) {
-    tc::tma_store_3d(&mdQ, sQ, h * kDh, t0, b);
-    tc::tma_store_3d(&mdK, sK, h * kDh, t0, b);
-    tc::tma_store_3d(&mdV, sdO, h * kDh, t0, b);
+    tc::tma_store_3d(&mdQ, sQ, h * DH, t0, b);
+    tc::tma_store_3d(&mdK, sK, h * DH, t0, b);
+    tc::tma_store_3d(&mdV, sdO, h * DH, t0, b);
     tc::tma_store_commit();
     tc::tma_store_wait_read<0>();  // the staging is read; the writes finish with the grid
   }
@@ -424,15 +436,24 @@ bool attn_tc_supported(int dtype, int dh, int L) {
          tmap_encoder() != nullptr;
 }
 
-static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, int B) {
+bool attn_tc_bwd_supported(int dtype, int dh, int L) {
+  return dtype == 1 && (dh == 16 || dh == 32 || dh == 64) &&
+         (L == 16 || L == 32 || L == 64 || L == 128) && tmap_encoder() != nullptr;
+}
+
+// 128-token x DH boxes of one head, with the swizzle whose span is one row
+static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, int B,
+                     int dh = kDh) {
   const uint64_t dims[3] = {(uint64_t)D, (uint64_t)T, (uint64_t)B};
   const uint64_t st[2] = {(uint64_t)ld * 2, (uint64_t)ld * 2 * (uint64_t)T};
-  const uint32_t box[3] = {kDh, kTile, 1};
-  return make_tmap_bf16(m, base, 3, dims, st, box);
+  const uint32_t box[3] = {(uint32_t)dh, kTile, 1};
+  const CUtensorMapSwizzle sw = dh == 64   ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                           : CU_TENSOR_MAP_SWIZZLE_32B;
+  return make_tmap_bf16(m, base, 3, dims, st, box, sw);
 }
 
 static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
-static constexpr int kBwdSmem = 6 * kTB + 1024 + 64;
 
 static int chunks_for(int L) { return L <= 32 ? 1 : L / 32; }
 
@@ -461,33 +482,48 @@ cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
   }
 }
 
-template <int NCH>
+template <int NCH, int DH>
 static cudaError_t bwd_launch(const Launch& lc, const AttnBwdArgs& a, const CUtensorMap* m) {
   const AttnArgs& f = a.f;
   static std::atomic<unsigned long long> opted{0};
-  if (cudaError_t e = smem_opt_in(attn_bwd_tc_kernel<NCH>, kBwdSmem, &opted); e != cudaSuccess) return e;
+  auto kern = attn_bwd_tc_kernel<NCH, DH>;
+  constexpr int smem = bwd_smem_bytes<DH>();
+  if (cudaError_t e = smem_opt_in(kern, smem, &opted); e != cudaSuccess) return e;
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
-  cudaError_t e = launch_k(attn_bwd_tc_kernel<NCH>, grid, dim3(128), kBwdSmem, lc.stream, m[0],
-                           m[1], m[2], m[3], m[4], m[5], m[6], m[7], f.lse,
-                           f.T, f.H, f.L, 1.0f / sqrtf((float)f.dh), lc.status);
+  cudaError_t e = launch_k(kern, grid, dim3(128), smem, lc.stream, m[0], m[1], m[2], m[3], m[4],
+                           m[5], m[6], m[7], f.lse, f.T, f.H, f.L, 1.0f / sqrtf((float)f.dh),
+                           lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+template <int DH>
+static cudaError_t bwd_dh(const Launch& lc, const AttnBwdArgs& a) {
+  const AttnArgs& f = a.f;
+  const int D = f.H * DH;
+  CUtensorMap m[8];
+  if (!head_map(&m[0], f.Q, f.ld_qkv, D, f.T, f.B, DH) ||
+      !head_map(&m[1], f.K, f.ld_qkv, D, f.T, f.B, DH) ||
+      !head_map(&m[2], f.V, f.ld_qkv, D, f.T, f.B, DH) ||
+      !head_map(&m[3], a.dO, f.ld_o, D, f.T, f.B, DH) ||
+      !head_map(&m[4], a.dQ, a.ld_dqkv, D, f.T, f.B, DH) ||
+      !head_map(&m[5], a.dK, a.ld_dqkv, D, f.T, f.B, DH) ||
+      !head_map(&m[6], a.dV, a.ld_dqkv, D, f.T, f.B, DH) ||
+      !head_map(&m[7], f.O, f.ld_o, D, f.T, f.B, DH))
+    return cudaErrorInvalidValue;
+  switch (chunks_for(f.L)) {
+    case 1: return bwd_launch<1, DH>(lc, a, m);
+    case 2: return bwd_launch<2, DH>(lc, a, m);
+    default: return bwd_launch<4, DH>(lc, a, m);
+  }
 }
 
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
   const AttnArgs& f = a.f;
-  if (!attn_tc_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
-  const int D = f.H * kDh;
-  CUtensorMap m[8];
-  if (!head_map(&m[0], f.Q, f.ld_qkv, D, f.T, f.B) || !head_map(&m[1], f.K, f.ld_qkv, D, f.T, f.B) ||
-      !head_map(&m[2], f.V, f.ld_qkv, D, f.T, f.B) || !head_map(&m[3], a.dO, f.ld_o, D, f.T, f.B) ||
-      !head_map(&m[4], a.dQ, a.ld_dqkv, D, f.T, f.B) ||
-      !head_map(&m[5], a.dK, a.ld_dqkv, D, f.T, f.B) ||
-      !head_map(&m[6], a.dV, a.ld_dqkv, D, f.T, f.B) || !head_map(&m[7], f.O, f.ld_o, D, f.T, f.B))
-    return cudaErrorInvalidValue;
-  switch (chunks_for(f.L)) {
-    case 1: return bwd_launch<1>(lc, a, m);
-    case 2: return bwd_launch<2>(lc, a, m);
-    default: return bwd_launch<4>(lc, a, m);
+  if (!attn_tc_bwd_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
+  switch (f.dh) {
+    case 16: return bwd_dh<16>(lc, a);
+    case 32: return bwd_dh<32>(lc, a);
+    default: return bwd_dh<64>(lc, a);
   }
 }
 

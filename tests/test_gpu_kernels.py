@@ -111,6 +111,8 @@ ATTN_CASES = [
     (2, 130, 4, 16, 16, "bf16"),
     (1, 520, 2, 32, 256, "bf16"),
     (2, 150, 2, 32, 32, "bf16"),
+    (2, 256, 4, 32, 128, "bf16"),
+    (4, 1024, 8, 16, 64, "bf16"),     # the paper's layer shape, several CTA rounds
     (2, 100, 2, 32, 24, "fp32"),
     (1, 256, 4, 32, 32, "fp32"),
 ]
@@ -122,7 +124,7 @@ def _impl_ok(impl, dh, L, dtype):
     if dtype != "bf16":
         return False
     if impl == 1:
-        return dh == 64 and L in (16, 32, 64, 128)
+        return dh in (16, 32, 64) and L in (16, 32, 64, 128)
     return dh in (16, 32, 64) and ((L >= 16 and 128 % L == 0) or (L % 128 == 0 and L <= 1024))
 
 
