@@ -40,9 +40,8 @@ int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, cons
  * q, k, v: rows of token (b,t) start at q + (b*T+t)*ld, head h at column
  * h*D/H.  o [B*T, D] Concat(heads), lse [B,H,T] fp32 (written by the forward,
  * read by the backward).  Backward: dO [B*T, D]; drow [B,H,T] fp32 scratch;
- * dq, dk, dv with row stride ld_d.  impl: 0 SIMT, 1 single-tile tcgen05 (L
- * <= 128; head width 64 forward, 16/32/64 backward, with the key-walking
- * forward for 16/32), 2 key-tile-walking tcgen05 (head width 16/32/64, L
+ * dq, dk, dv with row stride ld_d.  impl: 0 SIMT, 1 single-tile tcgen05 (head
+ * width 16/32/64, L <= 128), 2 key-tile-walking tcgen05 (head width 16/32/64, L
  * dividing or a multiple of 128; its backward also writes drow).  Returns 0, or
  * -1 on error (bcmt_last_error()). */
 int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, const void* k,

@@ -48,20 +48,38 @@ __device__ __forceinline__ void stage_half(uint8_t* tile, int r, int half, const
 // otherwise); a warp reads only the chunks up to its own last row's key, the
 // rest of its P and dS rows are causal zeros.
 
+// Stores one DH-wide fp32 row as bf16 into row r of a 128 x DH swizzled tile
+// (the TMA store layout).
+template <int DH>
+__device__ __forceinline__ void stage_row(uint8_t* tile, int r, const float* v) {
+#pragma unroll
+  for (int u = 0; u < DH / 8; ++u)
+    *reinterpret_cast<uint4*>(tile + Geo<DH>::unit(r, u)) = pack8(v + 8 * u);
+}
+
 // ====================================================================== forward
-template <int NCH>
+// For head widths DH in {16, 32, 64}.  At DH = 64 the P tile (32 KB) covers
+// the Q and K tiles once S = Q K^T has consumed them; at DH = 16 / 32 it
+// follows the three tiles.  The output is staged in the Q tile.
+template <int DH> constexpr int fwd_smem_bytes() {
+  return (DH == 64 ? 3 * Geo<DH>::tile : 3 * Geo<DH>::tile + 32768) + 1024 + 64;
+}
+
+template <int NCH, int DH>
 __global__ void __launch_bounds__(128)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap mQ, const __grid_constant__ CUtensorMap mK,
                        const __grid_constant__ CUtensorMap mV, const __grid_constant__ CUtensorMap mO,
                        float* __restrict__ lse, int Tlen, int H, int L, float scale,
                        unsigned* status) {
+  using G = Geo<DH>;
+  constexpr uint32_t kT = G::tile;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* sQ = smem;             // Q; then P keys 0-63; then the output staging tile
-  uint8_t* sK = smem + kTB;       // K; then P keys 64-127
-  uint8_t* sV = smem + 2 * kTB;   // V
-  uint8_t* sP = sQ;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 3 * kTB);
+  uint8_t* sQ = smem;            // Q; then the output staging tile
+  uint8_t* sK = smem + kT;       // K
+  uint8_t* sV = smem + 2 * kT;   // V
+  uint8_t* sP = DH == 64 ? sQ : smem + 3 * kT;  // P (32 KB)
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + (DH == 64 ? 3 * kT : 3 * kT + 32768));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -78,10 +96,10 @@ __global__ void __launch_bounds__(128)
   }
   pdl_enter();
   if (tid == 0) {
-    tc::mbar_arrive_expect_tx(&bar[0], 3 * kTB);
-    tc::tma_load_3d(sQ, &mQ, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sK, &mK, &bar[0], h * kDh, t0, b);
-    tc::tma_load_3d(sV, &mV, &bar[0], h * kDh, t0, b);
+    tc::mbar_arrive_expect_tx(&bar[0], 3 * kT);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, t0, b);
   }
   __syncwarp();
   if (warp == 0) {
@@ -100,9 +118,8 @@ __global__ void __launch_bounds__(128)
     if (ok) {
       constexpr uint32_t idS = tc::idesc_bf16(128, 128, 0, 0);
 #pragma unroll
-      for (int kk = 0; kk < kDh / 16; ++kk)
-        tc::mma_bf16(tmem, tc::sdesc(tc::smem_u32(sQ) + kk * 32, 16, 1024),
-                     tc::sdesc(tc::smem_u32(sK) + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < DH / 16; ++kk)
+        tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 0, kk), idS, kk > 0 ? 1u : 0u);
     }
     tc::mma_commit(&bar[1]);
   }
@@ -163,12 +180,10 @@ __global__ void __launch_bounds__(128)
 
   if (tid == 0) {
     tc::fence_after_sync();
-    constexpr uint32_t idO = tc::idesc_bf16(128, kDh, 0, 1);
+    constexpr uint32_t idO = tc::idesc_bf16(128, DH, 0, 1);
 #pragma unroll
     for (int kk = 0; kk < kTile / 16; ++kk)
-      tc::mma_bf16(tmem,
-                   tc::sdesc(tc::smem_u32(sP) + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                   tc::sdesc(tc::smem_u32(sV) + kk * 2048, 8192, 1024), idO, kk > 0 ? 1u : 0u);
+      tc::mma_bf16(tmem, p_kmaj(sP, 0, kk), G::mnmaj(sV, 0, kk), idO, kk > 0 ? 1u : 0u);
     tc::mma_commit(&bar[2]);
   }
   __syncwarp();
@@ -178,19 +193,18 @@ __global__ void __launch_bounds__(128)
   // ---- epilogue: O = (P V) / sum, staged in the (now free) Q/P tile
   const float inv = 1.0f / sum;
   {
-    uint32_t o[2][32];
-    tc::tmem_ld32_issue(trow, o[0]);
-    tc::tmem_ld32_issue(trow + 32u, o[1]);
-    tc::tmem_wait();
-    stage_half(sQ, r, 0, reinterpret_cast<const float*>(o[0]), inv);
-    stage_half(sQ, r, 1, reinterpret_cast<const float*>(o[1]), inv);
+    float o[DH];
+    tmem_row<DH>(trow, o);
+#pragma unroll
+    for (int c = 0; c < DH; ++c) o[c] *= inv;
+    stage_row<DH>(sQ, r, o);
   }
   if (ok && t0 + r < Tlen) lse[((long)b * H + h) * Tlen + t0 + r] = mx * scale + logf(sum);
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
   if (tid == 0 && ok) {
-    tc::tma_store_3d(&mO, sQ, h * kDh, t0, b);
+    tc::tma_store_3d(&mO, sQ, h * DH, t0, b);
     tc::tma_store_commit();
     tc::tma_store_wait_read<0>();  // the staging is read; the writes finish with the grid
   }
@@ -207,13 +221,6 @@ __global__ void __launch_bounds__(128)
 // DH = 16 / 32 it follows the five tiles (52 / 72 KB).  O comes in by TMA
 // with the other tiles (for Drow = dO . O).  The gradients leave through the
 // Q, K, dO tiles as staging, in the same layout, by TMA stores.
-template <int DH>
-__device__ __forceinline__ void stage_row(uint8_t* tile, int r, const float* v) {
-#pragma unroll
-  for (int u = 0; u < DH / 8; ++u)
-    *reinterpret_cast<uint4*>(tile + Geo<DH>::unit(r, u)) = pack8(v + 8 * u);
-}
-
 template <int DH> constexpr int bwd_smem_bytes() {
   return (DH == 64 ? 6 * Geo<DH>::tile : 5 * Geo<DH>::tile + 32768) + 1024 + 64;
 }
@@ -432,11 +439,6 @@ __global__ void __launch_bounds__(128)
 
 // ========================================================================= host
 bool attn_tc_supported(int dtype, int dh, int L) {
-  return dtype == 1 && dh == kDh && (L == 16 || L == 32 || L == 64 || L == 128) &&
-         tmap_encoder() != nullptr;
-}
-
-bool attn_tc_bwd_supported(int dtype, int dh, int L) {
   return dtype == 1 && (dh == 16 || dh == 32 || dh == 64) &&
          (L == 16 || L == 32 || L == 64 || L == 128) && tmap_encoder() != nullptr;
 }
@@ -453,32 +455,43 @@ static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, in
   return make_tmap_bf16(m, base, 3, dims, st, box, sw);
 }
 
-static constexpr int kFwdSmem = 3 * kTB + 1024 + 64;
 
 static int chunks_for(int L) { return L <= 32 ? 1 : L / 32; }
 
-template <int NCH>
+template <int NCH, int DH>
 static cudaError_t fwd_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
   static std::atomic<unsigned long long> opted{0};
-  if (cudaError_t e = smem_opt_in(attn_fwd_tc_kernel<NCH>, kFwdSmem, &opted); e != cudaSuccess) return e;
+  auto kern = attn_fwd_tc_kernel<NCH, DH>;
+  constexpr int smem = fwd_smem_bytes<DH>();
+  if (cudaError_t e = smem_opt_in(kern, smem, &opted); e != cudaSuccess) return e;
   dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
-  cudaError_t e = launch_k(attn_fwd_tc_kernel<NCH>, grid, dim3(128), kFwdSmem, lc.stream, m[0],
-                           m[1], m[2], m[3], a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)a.dh),
-                           lc.status);
+  cudaError_t e = launch_k(kern, grid, dim3(128), smem, lc.stream, m[0], m[1], m[2], m[3], a.lse,
+                           a.T, a.H, a.L, 1.0f / sqrtf((float)a.dh), lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+template <int DH>
+static cudaError_t fwd_dh(const Launch& lc, const AttnArgs& a) {
+  const int D = a.H * DH;
+  CUtensorMap m[4];
+  if (!head_map(&m[0], a.Q, a.ld_qkv, D, a.T, a.B, DH) ||
+      !head_map(&m[1], a.K, a.ld_qkv, D, a.T, a.B, DH) ||
+      !head_map(&m[2], a.V, a.ld_qkv, D, a.T, a.B, DH) ||
+      !head_map(&m[3], a.O, a.ld_o, D, a.T, a.B, DH))
+    return cudaErrorInvalidValue;
+  switch (chunks_for(a.L)) {
+    case 1: return fwd_launch<1, DH>(lc, a, m);
+    case 2: return fwd_launch<2, DH>(lc, a, m);
+    default: return fwd_launch<4, DH>(lc, a, m);
+  }
 }
 
 cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a) {
   if (!attn_tc_supported(1, a.dh, a.L)) return cudaErrorNotSupported;
-  const int D = a.H * kDh;
-  CUtensorMap m[4];
-  if (!head_map(&m[0], a.Q, a.ld_qkv, D, a.T, a.B) || !head_map(&m[1], a.K, a.ld_qkv, D, a.T, a.B) ||
-      !head_map(&m[2], a.V, a.ld_qkv, D, a.T, a.B) || !head_map(&m[3], a.O, a.ld_o, D, a.T, a.B))
-    return cudaErrorInvalidValue;
-  switch (chunks_for(a.L)) {
-    case 1: return fwd_launch<1>(lc, a, m);
-    case 2: return fwd_launch<2>(lc, a, m);
-    default: return fwd_launch<4>(lc, a, m);
+  switch (a.dh) {
+    case 16: return fwd_dh<16>(lc, a);
+    case 32: return fwd_dh<32>(lc, a);
+    default: return fwd_dh<64>(lc, a);
   }
 }
 
@@ -519,7 +532,7 @@ static cudaError_t bwd_dh(const Launch& lc, const AttnBwdArgs& a) {
 
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a) {
   const AttnArgs& f = a.f;
-  if (!attn_tc_bwd_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
+  if (!attn_tc_supported(1, f.dh, f.L)) return cudaErrorNotSupported;
   switch (f.dh) {
     case 16: return bwd_dh<16>(lc, a);
     case 32: return bwd_dh<32>(lc, a);

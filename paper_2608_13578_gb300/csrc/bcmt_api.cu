@@ -426,13 +426,6 @@ int attn_kind(const Geometry& g) {
   if (attn_tc_supported(g.dtype, g.dh, g.L)) return 1;
   return attn_fl_supported(g.dtype, g.dh, g.L) ? 2 : 0;
 }
-// The backward may take the single-tile kernel after a key-walking forward
-// (one key tile per query tile: both write the same O and log-sum-exp).
-int attn_kind_bwd(const Geometry& g) {
-  if (!g_use_tc_attn) return 0;
-  if (attn_tc_bwd_supported(g.dtype, g.dh, g.L)) return 1;
-  return attn_fl_supported(g.dtype, g.dh, g.L) ? 2 : 0;
-}
 
 bcmt_status finish(const bcmt_params* p, cudaStream_t s) {
   cudaError_t e = cudaGetLastError();
@@ -782,10 +775,10 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     }
     AttnBwdArgs ab{{Qp, Kp, Vp, ld, w.hhat, D, w.lse, g.B, g.T, g.H, g.dh, g.L},
                    bw.dHhat, bw.Drow, dQ, dK, dV, ldd};
-    if (attn_kind_bwd(g) == 1) {
+    if (attn_kind(g) == 1) {
       pr.begin("attn_bwd_tc");
       e = attn_bwd_tc(lc, ab);
-    } else if (attn_kind_bwd(g) == 2) {
+    } else if (attn_kind(g) == 2) {
       pr.begin("attn_bwd_fl");
       e = attn_bwd_fl(lc, ab);
     } else {
@@ -1021,9 +1014,7 @@ int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, 
   AttnArgs aa{q, k, v, ld, o, g.D, lse, g.B, g.T, g.H, g.dh, g.L};
   cudaError_t e;
   if (!backward) {
-    // impl 1 with a head width the single-tile forward does not take: the
-    // key-walking forward, so that the single-tile backward can follow it
-    e = impl == 1 ? (attn_tc_supported(1, g.dh, g.L) ? attn_fwd_tc(lc, aa) : attn_fwd_fl(lc, aa))
+    e = impl == 1 ? attn_fwd_tc(lc, aa)
         : impl == 2 ? attn_fwd_fl(lc, aa)
                     : attn_fwd_simt(lc, g.dtype, aa);
   } else {

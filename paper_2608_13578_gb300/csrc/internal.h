@@ -112,9 +112,6 @@ cudaError_t attn_bwd_simt_noalloc(const Launch& lc, int dtype, const AttnBwdArgs
 cudaError_t attn_fwd_tc(const Launch& lc, const AttnArgs& a);
 cudaError_t attn_bwd_tc(const Launch& lc, const AttnBwdArgs& a);
 bool attn_tc_supported(int dtype, int dh, int L);
-// The single-tile backward also takes head widths 16 and 32 (after either
-// forward: both write the same O and log-sum-exp).
-bool attn_tc_bwd_supported(int dtype, int dh, int L);
 // tcgen05 attention that walks key tiles (head widths 16/32/64, L dividing or
 // a multiple of 128); the backward writes Drow itself (dQ kernel first).
 bool attn_fl_supported(int dtype, int dh, int L);
