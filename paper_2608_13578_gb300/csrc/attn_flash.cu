@@ -289,13 +289,14 @@ __global__ void __launch_bounds__(128)
   using G = Geo<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* sdS = smem;                      // 16 KB: scale * dS, one 64-key half
-  uint8_t* sQ = smem + 16384;
+  uint8_t* sdS = smem;                      // 2 x 16 KB: scale * dS of the two 64-key halves
+  uint8_t* sQ = smem + 32768;
   uint8_t* sdO = sQ + G::tile;
   uint8_t* sK = sdO + G::tile;
   uint8_t* sV = sK + G::tile;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);  // kv, s, q
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 3);
+  // K/V loaded; S/dP done; dQ product of half 0 / half 1 done
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(128)
   key_walk(t0, L, kstart, nkt);
 
   if (tid == 0) {
-    for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+    for (int i = 0; i < 4; ++i) tc::mbar_init(&bar[i], 1);
     tc::fence_mbar_init();
     tc::prefetch_tmap(&mQ);
     tc::prefetch_tmap(&mK);
@@ -353,29 +354,34 @@ __global__ void __launch_bounds__(128)
   const float nl2 = -lse2, ndr = -drow * scale;
   const int rbs = L < kTile ? (r / L) * L : 0;
   bool ok = true;
-  int ns = 0, nq = 0;  // commits to bar[1] and bar[2] so far
+  // S and dP of half hh of the loaded key tile into TMEM columns 0..127
+  auto issue_sdp = [&](int hh) {
+    if (ok) {
+      constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // S half -> columns 0..63
+        tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // dP half -> columns 64..127
+        tc::mma_bf16(tmem + 64, G::kmaj(sdO, 0, kk), G::kmaj(sV, 64 * hh, kk), id64,
+                     kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar[1]);
+  };
+  if (tid == 0) {
+    ok = tc::mbar_wait(&bar[0], 0, status) && ok;
+    tc::fence_after_sync();
+    issue_sdp(0);
+  }
+  __syncwarp();
+  int ns = 0;  // S/dP commits consumed so far
 
+  // Per key tile, the two 64-key halves overlap: S and dP of half 1 run under
+  // half 0's dS, and each half writes its own dS buffer (the one the dQ product
+  // of the same half of the previous tile read).
   for (int kt = 0; kt < nkt; ++kt) {
     const bool diag = kt == nkt - 1;
-    if (tid == 0) {
-      ok = tc::mbar_wait(&bar[0], kt & 1, status) && ok;
-      tc::fence_after_sync();
-    }
     for (int hh = 0; hh < 2; ++hh) {
-      if (tid == 0) {
-        if (ok) {
-          constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
-#pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk)  // S half -> columns 0..63
-            tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
-#pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk)  // dP half -> columns 64..127
-            tc::mma_bf16(tmem + 64, G::kmaj(sdO, 0, kk), G::kmaj(sV, 64 * hh, kk), id64,
-                         kk > 0 ? 1u : 0u);
-        }
-        tc::mma_commit(&bar[1]);
-      }
-      __syncwarp();
       ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
       ++ns;
       tc::fence_after_sync();
@@ -385,9 +391,15 @@ __global__ void __launch_bounds__(128)
       tc::tmem_ld32_issue(trow + 64u, rd[0]);
       tc::tmem_ld32_issue(trow + 96u, rd[1]);
       tc::tmem_wait();
-      // the previous dQ product must be done with the dS buffer it reads
-      if (nq > 0) {
-        ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+      tc::fence_before_sync();
+      __syncthreads();  // every thread has this half's S and dP: the columns are free
+      if (tid == 0 && hh == 0) {
+        tc::fence_after_sync();
+        issue_sdp(1);
+      }
+      uint8_t* sdSh = sdS + hh * 16384;
+      if (kt > 0) {  // the previous tile's dQ product of this half read sdSh
+        ok = tc::mbar_wait(&bar[2 + hh], (kt - 1) & 1, status) && ok;
         tc::fence_after_sync();
       }
       // dS = P (dP - Drow) scale; rows past the end see zero-filled Q and dO
@@ -411,7 +423,7 @@ __global__ void __launch_bounds__(128)
           }
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) put_unit(sdS, r, 4 * c + u, pack8(v + 8 * u));
+        for (int u = 0; u < 4; ++u) put_unit(sdSh, r, 4 * c + u, pack8(v + 8 * u));
       }
       tc::fence_proxy_async_smem();
       tc::fence_before_sync();
@@ -422,23 +434,26 @@ __global__ void __launch_bounds__(128)
           constexpr uint32_t idQ = tc::idesc_bf16(128, DH, 0, 1);
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)  // dQ += dS[:, 64hh..] K[64hh.., :]
-            tc::mma_bf16(tmem + 128, p_kmaj(sdS, 0, kk), G::mnmaj(sK, 64 * hh, kk), idQ,
+            tc::mma_bf16(tmem + 128, p_kmaj(sdSh, 0, kk), G::mnmaj(sK, 64 * hh, kk), idQ,
                          (kt > 0 || hh > 0 || kk > 0) ? 1u : 0u);
         }
-        tc::mma_commit(&bar[2]);
+        tc::mma_commit(&bar[2 + hh]);
       }
-      ++nq;
     }
-    // the next key tile may overwrite K and V once this tile's products are done
+    // the next key tile may overwrite K and V once this tile's products are
+    // done (the half-1 commit covers every earlier product); then its half 0
     if (tid == 0 && kt + 1 < nkt) {
-      ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+      ok = tc::mbar_wait(&bar[3], kt & 1, status) && ok;
       tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
       tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
       tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      ok = tc::mbar_wait(&bar[0], (kt + 1) & 1, status) && ok;
+      tc::fence_after_sync();
+      issue_sdp(0);
     }
     __syncwarp();
   }
-  ok = tc::mbar_wait(&bar[2], (nq - 1) & 1, status) && ok;
+  ok = tc::mbar_wait(&bar[3], (nkt - 1) & 1, status) && ok;
   tc::fence_after_sync();
   float q[DH];
   tmem_row<DH>(trow + 128u, q);
@@ -643,7 +658,7 @@ bool head_map_fl(CUtensorMap* m, const void* base, long ld, int D, int T, int B)
 
 // dynamic shared memory: 1 KB alignment slack + tiles + staging + barriers
 template <int DH> constexpr int fwd_smem() { return 1024 + 32768 + 4 * Geo<DH>::tile + 64; }
-template <int DH> constexpr int dq_smem() { return 1024 + 16384 + 4 * Geo<DH>::tile + 64; }
+template <int DH> constexpr int dq_smem() { return 1024 + 32768 + 4 * Geo<DH>::tile + 64; }
 template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
 }
