@@ -1,7 +1,8 @@
-// Intra-block causal attention on the tcgen05 tensor cores (Sec. 3.3) for the
-// shapes the single-tile kernels of attn_tc.cu do not take: head widths
-// DH in {16, 32, 64} and block sizes L that divide 128 or are multiples of 128
-// (up to 1024), bf16 operands.
+// Intra-block causal attention on the tcgen05 tensor cores (Sec. 3.3) that
+// walks key tiles: head widths DH in {16, 32, 64} and block sizes L that
+// divide 128 or are multiples of 128 (up to 1024), bf16 operands.  The layer
+// uses it for blocks longer than one 128-token tile (L >= 256); for L <= 128
+// it takes the single-tile kernels of attn_tc.cu.
 //
 // A CTA owns a 128-token tile of one head and walks the key tiles its rows
 // can see: for L >= 128 the tiles of its block from the block start up to the

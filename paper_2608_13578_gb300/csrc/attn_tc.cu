@@ -1,15 +1,16 @@
 // Intra-block causal attention on the tcgen05 tensor cores (Sec. 3.3), bf16
-// operands, head width 64, block size L in {16, 32, 64, 128}.
+// operands, head width DH in {16, 32, 64}, block size L in {16, 32, 64, 128}.
 //
 // One CTA per (128-token tile, head, batch); 128 % L == 0, so a tile holds
 // 128 / L whole blocks and its keys are its own 128 tokens.  The attention
 // pattern inside the tile is block-diagonal causal: query r sees keys
 // [blockstart(r), r].  TMA brings the Q, K, V head slices of the tile into
-// shared memory (128-byte swizzle; a 3-D tensor map per operand zero-fills
-// tokens past the end of the sequence), tcgen05.mma computes the scores into
-// TMEM, each thread owns one query row for the masked softmax (the whole row
-// fits in TMEM, so there is no online rescaling), writes P in bf16 back to
-// shared memory as the A operand of P V, and the normalised output leaves
+// shared memory (the swizzle whose span is one DH-wide row; a 3-D tensor map
+// per operand zero-fills tokens past the end of the sequence), tcgen05.mma
+// computes the scores into TMEM, each thread owns one query row for the
+// masked softmax (the whole row fits in TMEM, so there is no online
+// rescaling), writes P in bf16 back to shared memory as the A operand of
+// P V, and the normalised output leaves
 // through a TMA store.  The backward recomputes P from the saved log-sum-exp
 // and runs the five products S = Q K^T, dP = dO V^T, dV = P^T dO,
 // dQ = dS K, dK = dS^T Q on the tensor cores, reading the same shared tiles
@@ -25,22 +26,6 @@ using namespace attn;
 
 namespace {
 constexpr int kTile = 128;
-constexpr int kDh = 64;
-constexpr uint32_t kTB = kTile * kDh * 2;  // one 128 x 64 bf16 tile: 16 KB
-
-// Stores one 64-wide fp32 row (two 32-column halves) as bf16 into a
-// 128-row x 128-byte swizzled staging tile (the TMA store layout).
-__device__ __forceinline__ void stage_half(uint8_t* tile, int r, int half, const float* v, float mul) {
-#pragma unroll
-  for (int u = 0; u < 4; ++u) {
-    uint4 q;
-    q.x = pack2(v[8 * u + 0] * mul, v[8 * u + 1] * mul);
-    q.y = pack2(v[8 * u + 2] * mul, v[8 * u + 3] * mul);
-    q.z = pack2(v[8 * u + 4] * mul, v[8 * u + 5] * mul);
-    q.w = pack2(v[8 * u + 6] * mul, v[8 * u + 7] * mul);
-    *reinterpret_cast<uint4*>(tile + tc::sw128_offset(r, half * 4 + u)) = q;
-  }
-}
 }  // namespace
 
 // Both kernels are instantiated for NCH = the number of 32-key chunks of a
@@ -444,8 +429,7 @@ bool attn_tc_supported(int dtype, int dh, int L) {
 }
 
 // 128-token x DH boxes of one head, with the swizzle whose span is one row
-static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, int B,
-                     int dh = kDh) {
+static bool head_map(CUtensorMap* m, const void* base, long ld, int D, int T, int B, int dh) {
   const uint64_t dims[3] = {(uint64_t)D, (uint64_t)T, (uint64_t)B};
   const uint64_t st[2] = {(uint64_t)ld * 2, (uint64_t)ld * 2 * (uint64_t)T};
   const uint32_t box[3] = {(uint32_t)dh, kTile, 1};
