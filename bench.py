@@ -185,6 +185,8 @@ def kernel_model(w):
         "gemm_dw_g": g(D, D, n),
         "gemm_dw_o": g(D, D, n),
         "gemm_dw_qkv": g(D, 3 * D, n),
+        # one grouped CTA-pair launch when D is a multiple of 256: dX, dW_QKV, dW_g, dW_O
+        "gemm_dx_dw": ("tensor", 2 * 2.0 * n * D * 3 * D + 2 * 2.0 * n * D * D),
         # read Q, K, V; write Concat(heads) and the log-sum-exp
         "attn_fwd_tc": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),
         "attn_fwd_simt": ("hbm", 3 * n * D * es + n * D * es + n * H * 4),

@@ -35,6 +35,24 @@ int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, cons
                    long sam, long sak, const void* B, long sbk, long sbn, void* C, long ldc,
                    int splits, void* stream);
 
+/* Two or three products in one launch of the CTA-pair tcgen05 GEMM (bf16
+ * inputs), the grouping the backward pass uses for dX, dW_QKV and dW_g.
+ * Product 0: C0[M0,N0] = A0[M0,K0] B0[K0,N0] stored as bf16 into C0
+ * (row-major, leading dimension N0), with A0 row-major (leading dimension
+ * lda0) and B0 given as its transpose B0t[N0,K0] (leading dimension ldb0t):
+ * both operands K-major.  Products 1 and 2: the fp32 partial products of
+ * Ci[Mi,Ni] = Ai[Mi,Ki] Bi[Ki,Ni] over splits_i ranges of K (as
+ * bcmt_test_gemm), split z at part_i + z*Mi*Ni, with Ai given as its transpose
+ * Ait[Ki,Mi] (leading dimension lda_it) and Bi row-major (leading dimension
+ * ldb_i): both operands MN-major.  M2 = 0 leaves product 2 out.  N0, N1, N2
+ * multiples of 256, leading dimensions multiples of 8.  Returns the number of
+ * K-splits of product 1 written, or -1 on error (bcmt_last_error()). */
+int bcmt_test_gemm_group(int M0, int N0, int K0, const void* A0, long lda0, const void* B0t,
+                         long ldb0t, void* C0, int M1, int N1, int K1, const void* A1t, long lda1t,
+                         const void* B1, long ldb1, float* part1, int splits1, int M2, int N2,
+                         int K2, const void* A2t, long lda2t, const void* B2, long ldb2,
+                         float* part2, int splits2, void* stream);
+
 /* The intra-block causal attention of Sec. 3.3 alone, forward (backward = 0)
  * or backward (backward = 1), for the shape in *p (B, T, D, H, L, dtype).
  * q, k, v: rows of token (b,t) start at q + (b*T+t)*ld, head h at column

@@ -87,6 +87,10 @@ def _load():
                                                         ctypes.c_long, ctypes.c_long, _VP,
                                                         ctypes.c_long, ctypes.c_int, _VP]
     lib.bcmt_test_gemm.restype = ctypes.c_int
+    _gi = [ctypes.c_int] * 3 + [_VP, ctypes.c_long, _VP, ctypes.c_long, _VP, ctypes.c_int]
+    lib.bcmt_test_gemm_group.argtypes = ([ctypes.c_int] * 3 + [_VP, ctypes.c_long, _VP, ctypes.c_long,
+                                                               _VP] + _gi + _gi + [_VP])
+    lib.bcmt_test_gemm_group.restype = ctypes.c_int
     lib.bcmt_test_attn.argtypes = [ctypes.c_int, ctypes.c_int, _P, _VP, _VP, _VP, ctypes.c_long,
                                    _VP, _VP, _VP, _VP, _VP, _VP, _VP, ctypes.c_long, _VP]
     lib.bcmt_test_attn.restype = ctypes.c_int
@@ -100,7 +104,7 @@ EXPORTED = ("bcmt_workspace_size", "bcmt_scratch_size", "bcmt_forward", "bcmt_ba
             "bcmt_device_status", "bcmt_last_error", "bcmt_profile_read", "bcmt_profile_reset",
             "bcmt_attention_backward_noalloc",
             "bcmt_decode_state_size", "bcmt_decode_reset", "bcmt_decode_step",
-            "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_attn")
+            "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_gemm_group", "bcmt_test_attn")
 
 
 def _ptr(t) -> Optional[int]:
@@ -205,6 +209,18 @@ def bcmt_test_gemm(impl, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, C,
                    stream=None) -> int:
     r = LIB.bcmt_test_gemm(impl, dtype, dtype_out, M, N, K, _ptr(A), sam, sak, _ptr(B), sbk, sbn,
                            _ptr(C), ldc, splits, _stream(stream))
+    if r < 0:
+        raise BCMTError(BCMT_ERR_CUDA, bcmt_last_error())
+    return r
+
+
+def bcmt_test_gemm_group(M0, N0, K0, A0, lda0, B0t, ldb0t, C0, M1, N1, K1, A1t, lda1t, B1, ldb1,
+                         part1, splits1, M2=0, N2=0, K2=0, A2t=None, lda2t=0, B2=None, ldb2=0,
+                         part2=None, splits2=1, stream=None) -> int:
+    r = LIB.bcmt_test_gemm_group(M0, N0, K0, _ptr(A0), lda0, _ptr(B0t), ldb0t, _ptr(C0), M1, N1, K1,
+                                 _ptr(A1t), lda1t, _ptr(B1), ldb1, _ptr(part1), splits1, M2, N2,
+                                 K2, _ptr(A2t), lda2t, _ptr(B2), ldb2, _ptr(part2), splits2,
+                                 _stream(stream))
     if r < 0:
         raise BCMTError(BCMT_ERR_CUDA, bcmt_last_error())
     return r

@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <array>
 #include <memory>
 #include <mutex>
 #include <string>
@@ -291,6 +292,75 @@ int dw_splits(int dtype, int M, int N, long K, int max_pairs = 0) {
   return std::max(1, std::min(s, nkb / 8));
 }
 
+// The backward pass's last products -- dX = dQKV W_QKV^T and the K-split
+// weight gradients dW_QKV = X^T dQKV, dW_g = H^T dU (when the gate exists)
+// and dW_O = Hhat^T dH -- share one CTA-pair launch when they fit its
+// 256 x 256 tiles (bf16, D a multiple of 256).  The weight gradients then
+// leave the side streams, where they slowed the critical kernels beside them.
+bool tail_grouped(const Geometry& g) {
+  return g.from_x && dw_pair(g.dtype, g.D, 3 * g.D) && gemm_tc_available() && g.n >= 256;
+}
+// K splits of the weight gradients in that launch (in launch order: dW_QKV,
+// dW_g, dW_O; 0 = absent): the counts whose round-robin deal of dX's tiles,
+// then each gradient's items, over the SM pairs, followed by the reduction of
+// the partials, finishes first.  Unit: one 64-deep K slice of a 256 x 256
+// tile (8.4 MFLOP, about 0.45 us on a pair); each item costs its slices plus
+// 4 (pipeline fill and epilogue), and each split of an M x N product adds the
+// reduction's reading of M*N fp32 partials at about 3 MB per unit.  Up to 16
+// splits each; ties go to fewer splits.  Cached per shape: the search runs once.
+struct TailPlan {
+  int s[3] = {1, 0, 0};
+};
+TailPlan tail_plan(const Geometry& g) {
+  const int pairs = std::max(1, device_sms() / 2);
+  const long D = g.D, tiles0 = ((g.n + 255) / 256) * (D / 256);
+  const int nk0 = (int)((3 * D + 63) / 64), nkb = (int)((g.n + 63) / 64);
+  const long tiles[3] = {(D / 256) * (3 * D / 256), g.honly ? 0 : (D / 256) * (D / 256),
+                         (D / 256) * (D / 256)};
+  const double out_units[3] = {3.0 * D * D * 4.0 / 3.0e6, (double)D * D * 4.0 / 3.0e6,
+                               (double)D * D * 4.0 / 3.0e6};
+  static std::mutex mu;
+  static std::vector<std::pair<std::array<long, 4>, TailPlan>> cache;
+  const std::array<long, 4> key{pairs, (long)g.n, D, (long)g.honly};
+  std::lock_guard<std::mutex> lock(mu);
+  for (const auto& c : cache)
+    if (c.first == key) return c.second;
+  const int smax = std::min(16, std::max(1, nkb / 8));
+  TailPlan best, cur;
+  double best_t = -1.0;
+  std::vector<long> load((size_t)pairs);
+  for (int a = 1; a <= smax; ++a)
+    for (int b = tiles[1] ? 1 : 0; b <= (tiles[1] ? smax : 0); ++b)
+      for (int c = 1; c <= smax; ++c) {
+        cur.s[0] = a;
+        cur.s[1] = b;
+        cur.s[2] = c;
+        std::fill(load.begin(), load.end(), 0L);
+        long item = 0;
+        for (long t = 0; t < tiles0; ++t, ++item) load[(size_t)(item % pairs)] += nk0 + 4;
+        double red = 0.0;
+        for (int w = 0; w < 3; ++w) {
+          if (!tiles[w]) continue;
+          const int kps = (nkb + cur.s[w] - 1) / cur.s[w], se = (nkb + kps - 1) / kps;
+          for (long t = 0; t < tiles[w] * se; ++t, ++item) {  // split index slowest
+            const int z = (int)(t / tiles[w]);
+            load[(size_t)(item % pairs)] += std::min(nkb, (z + 1) * kps) - z * kps + 4;
+          }
+          red += se * out_units[w];
+        }
+        const double t_end = (double)*std::max_element(load.begin(), load.end()) + red;
+        if (best_t < 0 || t_end < best_t) {
+          best_t = t_end;
+          best = cur;
+        }
+      }
+  cache.emplace_back(key, best);
+  return best;
+}
+int dqkv_splits(const Geometry& g) {
+  return tail_grouped(g) ? tail_plan(g).s[0] : dw_splits(g.dtype, g.D, 3 * g.D, g.n);
+}
+
 struct FwdWs {
   char *qkv, *hhat, *hloc, *G, *Mb;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
@@ -331,7 +401,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
 
 struct BwdWs {
   char *dU, *dH, *dHhat, *dqkv, *dPb;
-  float *dP, *dM, *dS, *ds, *dwp_part, *da_part, *Drow, *part, *part_o;
+  float *dP, *dM, *dS, *ds, *dwp_part, *da_part, *Drow, *part, *part_o, *part_qkv;
   size_t bytes;
 };
 
@@ -362,13 +432,22 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
   w.dHhat = take((size_t)g.n * g.D * g.es);
   w.dqkv = g.from_x ? take((size_t)g.n * 3 * g.D * g.es) : nullptr;
   w.Drow = reinterpret_cast<float*>(take((size_t)g.B * g.H * g.T * 4));
-  size_t part = (size_t)dw_splits(g.dtype, g.D, g.D, g.n) * g.D * g.D * 4;
-  if (g.from_x)
-    part = std::max(part, (size_t)dw_splits(g.dtype, g.D, 3 * g.D, g.n) * g.D * 3 * g.D * 4);
+  const bool grouped = tail_grouped(g);
+  const TailPlan tp = grouped ? tail_plan(g) : TailPlan();
+  size_t part = (size_t)(grouped ? std::max(1, tp.s[1]) : dw_splits(g.dtype, g.D, g.D, g.n)) *
+                g.D * g.D * 4;
+  if (g.from_x && !grouped)
+    part = std::max(part, (size_t)dqkv_splits(g) * g.D * 3 * g.D * 4);
   w.part = reinterpret_cast<float*>(take(part));
-  // dW_O's K-split partials: its product runs on the critical stream while
-  // the side stream may still be reducing dW_g's partials
-  w.part_o = reinterpret_cast<float*>(take((size_t)dw_splits(g.dtype, g.D, g.D, g.n) * g.D * g.D * 4));
+  // dW_QKV's partials: on the side stream after dW_g they reuse dW_g's
+  // buffer; in the grouped launch, which also computes dW_g, they get their
+  // own
+  w.part_qkv = grouped ? reinterpret_cast<float*>(take((size_t)dqkv_splits(g) * g.D * 3 * g.D * 4))
+                       : w.part;
+  // dW_O's K-split partials: its product runs on the critical stream (or the
+  // second side stream) while the side stream may still be reducing dW_g's
+  w.part_o = reinterpret_cast<float*>(
+      take((size_t)(grouped ? tp.s[2] : dw_splits(g.dtype, g.D, g.D, g.n)) * g.D * g.D * 4));
   w.bytes = off;
   return w;
 }
@@ -682,11 +761,14 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
       if (e != cudaSuccess) return cuda_fail(e, "dW_m");
     }
     // (up to 32 GFLOP on a few SM pairs: it runs beside the pooling backward,
-    // which needs the rest, and has until the end of the backward)
-    e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
-                    bw.part, dw_g, nullptr, nullptr, nullptr,
-                    2.0 * D * D * (double)g.n <= 32e9 ? device_sms() / 8 : 0);
-    if (e != cudaSuccess) return cuda_fail(e, "dW_g");
+    // which needs the rest, and has until the end of the backward; with the
+    // grouped tail it joins dX and dW_QKV there instead)
+    if (!tail_grouped(g)) {
+      e = weight_grad(lcs, prs, "gemm_dw_g", g.dtype, g.dtype, D, D, g.n, w.hloc, D, bw.dU, D,
+                      bw.part, dw_g, nullptr, nullptr, nullptr,
+                      2.0 * D * D * (double)g.n <= 32e9 ? device_sms() / 8 : 0);
+      if (e != cudaSuccess) return cuda_fail(e, "dW_g");
+    }
     // main stream, meanwhile: dH = dY + dU W_g^T (the identity and gate paths)
     {
       EpiArgs ea;
@@ -736,7 +818,9 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     // few SM pairs and runs beside the tail of the step (dx, dW_QKV) without
     // holding up dW_QKV; a large one stays on the critical stream with its
     // reduction beside
-    if (2.0 * D * D * (double)g.n <= 8e9) {
+    if (tail_grouped(g)) {
+      // computed with dX at the end of the pass
+    } else if (2.0 * D * D * (double)g.n <= 8e9) {
       fork.point2();
       Launch lcs2{fork.side2(), sp};
       Prof prs2{profiling, fork.side2()};
@@ -789,7 +873,32 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     if (e != cudaSuccess) return cuda_fail(e, "attention backward");
   }
   // Sec. 3.3 reversed: dX = dQKV W_qkv^T, dW_qkv = X^T dQKV.
-  if (g.from_x) {
+  if (tail_grouped(g)) {
+    // dX and the weight gradients in one launch on the critical stream, then
+    // the ordered reductions of the gradients' partials in one more
+    const TailPlan tp = tail_plan(g);
+    const PairProduct pdx{n, D, 3 * D, bw.dqkv, 3 * D, 1, w_qkv, 1, 3 * D, dx_or_dq, D, 0, 1};
+    PairProduct pw[3];
+    SplitSum red[3];
+    int nw = 0;
+    pw[nw] = PairProduct{D, 3 * D, n, x_or_q, 1, D, bw.dqkv, 3 * D, 1, bw.part_qkv, 3 * D,
+                         (long)D * 3 * D, tp.s[0]};
+    red[nw++] = SplitSum{bw.part_qkv, effective_splits(n, tp.s[0]), (long)D * 3 * D, dw_qkv};
+    if (!g.honly) {
+      pw[nw] = PairProduct{D, D, n, w.hloc, 1, D, bw.dU, D, 1, bw.part, D, (long)D * D, tp.s[1]};
+      red[nw++] = SplitSum{bw.part, effective_splits(n, tp.s[1]), (long)D * D, dw_g};
+    }
+    pw[nw] = PairProduct{D, D, n, w.hhat, 1, D, dH, D, 1, bw.part_o, D, (long)D * D, tp.s[2]};
+    red[nw++] = SplitSum{bw.part_o, effective_splits(n, tp.s[2]), (long)D * D, dw_o};
+    pr.begin("gemm_dx_dw");
+    e = gemm_tc_pair_group(lc, pdx, pw, nw);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "dX and the weight gradients");
+    pr.begin("reduce_splits");
+    e = reduce_splits_n(lc, red, nw, g.dtype);
+    pr.end(nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "weight gradient reduction");
+  } else if (g.from_x) {
     EpiArgs ea;
     ea.out = dx_or_dq;
     ea.ldo = D;
@@ -1001,6 +1110,30 @@ int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, cons
     return -1;
   }
   return splits > 1 ? effective_splits(K, splits) : 1;
+}
+
+int bcmt_test_gemm_group(int M0, int N0, int K0, const void* A0, long lda0, const void* B0t,
+                         long ldb0t, void* C0, int M1, int N1, int K1, const void* A1t, long lda1t,
+                         const void* B1, long ldb1, float* part1, int splits1, int M2, int N2,
+                         int K2, const void* A2t, long lda2t, const void* B2, long ldb2,
+                         float* part2, int splits2, void* stream) {
+  unsigned* sp = status_ptr();
+  if (!sp) return -1;
+  if (!gemm_tc_available()) {
+    fail(BCMT_ERR_CUDA, "test gemm group: tcgen05 GEMM unavailable");
+    return -1;
+  }
+  Launch lc{static_cast<cudaStream_t>(stream), sp};
+  const PairProduct p0{M0, N0, K0, A0, lda0, 1, B0t, 1, ldb0t, C0, N0, 0, 1};
+  const PairProduct pw[2] = {
+      {M1, N1, K1, A1t, 1, lda1t, B1, ldb1, 1, part1, N1, (long)M1 * N1, splits1},
+      {M2, N2, K2, A2t, 1, lda2t, B2, ldb2, 1, part2, N2, (long)M2 * N2, splits2}};
+  cudaError_t e = gemm_tc_pair_group(lc, p0, pw, M2 > 0 ? 2 : 1);
+  if (e != cudaSuccess) {
+    fail(BCMT_ERR_CUDA, "test gemm group: %s", cudaGetErrorString(e));
+    return -1;
+  }
+  return effective_splits(K1, splits1);
 }
 
 int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, const void* k,

@@ -482,6 +482,14 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
 // the MMAs and its commits arrive on the stage and accumulator barriers of
 // both CTAs; each CTA's epilogue warps drain their own 128 accumulator rows
 // and report back to the even CTA.
+//
+// One launch may carry up to kTc2Max independent products (a group):
+// product 0 with operand layouts and epilogue Op0, the others with Op1 (each
+// with its own shape and tensor maps).  The products' tiles are numbered one
+// product after the other and the pairs take the combined list round-robin,
+// so products that would each leave SMs idle (dX and the K-split weight
+// gradients at the end of the backward pass) share one wave.  A single
+// product is a group of one.
 template <int BN, int STAGES, int ACC>
 struct Tc2Cfg {
   static constexpr int A_BYTES = kBM * kBK * 2;          // 16 KB
@@ -493,12 +501,150 @@ struct Tc2Cfg {
   static constexpr int TMEM_COLS = ACC * BN;
 };
 
-template <int BN, int STAGES, int ACC, bool A_MN, bool B_MN, class Epi>
+// Compile-time half of one product of a group: operand layouts and epilogue.
+template <bool A_MN_, bool B_MN_, class Epi_>
+struct Tc2Op {
+  static constexpr bool A_MN = A_MN_, B_MN = B_MN_;
+  using Epi = Epi_;
+};
+
+// Run-time half: shape, K slices per split and tile counts (tiles_m counts
+// 256-row pair tiles; n_tiles = tiles_m * tiles_n * splits).
+struct Tc2Shape {
+  int M, N, kps, nkb, tiles_m, tiles_n, n_tiles;
+};
+
+constexpr int kTc2Max = 4;
+// Kernel parameter block of a group: tensor maps (A, B, output) and shape of
+// each product, the epilogues, and the number of products.
+template <class Op0, class Op1>
+struct Tc2Params {
+  CUtensorMap map[kTc2Max][3];
+  Tc2Shape shape[kTc2Max];
+  typename Op0::Epi epi0;
+  typename Op1::Epi epi1[kTc2Max - 1];
+  int count;
+};
+
+// TMA producer, one tile (both CTAs): this CTA's rows of A and half of B.
+template <class Op, class Cfg, int BN, int STAGES>
+__device__ __forceinline__ bool tc2_produce(const CUtensorMap* mA, const CUtensorMap* mB,
+                                            const Tc2Shape& s, int tile, uint32_t rank,
+                                            uint8_t* smem, uint64_t* full, uint64_t* empty,
+                                            int& it, unsigned* status) {
+  const int m_blk = tile % s.tiles_m, rest = tile / s.tiles_m;
+  const int n_blk = rest % s.tiles_n, z = rest / s.tiles_n;
+  const int m0 = m_blk * 2 * kBM + (int)rank * kBM;
+  const int n0 = n_blk * BN + (int)rank * (BN / 2);
+  const int kb0 = z * s.kps;
+  const int nk = min(s.nkb, kb0 + s.kps) - kb0;
+  for (int i = 0; i < nk; ++i, ++it) {
+    const int st = it % STAGES;
+    if (it >= STAGES && !tc::mbar_wait(&empty[st], ((it / STAGES) - 1) & 1, status)) return false;
+    uint8_t* sa = smem + st * Cfg::STAGE_BYTES;
+    uint8_t* sb = sa + Cfg::A_BYTES;
+    const uint32_t fb = tc::mapa(tc::smem_u32(&full[st]), 0);
+    if (rank == 0) tc::mbar_arrive_expect_tx(&full[st], 2 * Cfg::STAGE_BYTES);
+    const int k0 = (kb0 + i) * kBK;
+    if (!Op::A_MN) {
+      tc::tma_load_2d_pair(sa, mA, fb, k0, m0);
+    } else {
+      tc::tma_load_2d_pair(sa, mA, fb, m0, k0);
+      tc::tma_load_2d_pair(sa + 8192, mA, fb, m0 + 64, k0);
+    }
+    if (!Op::B_MN) {
+      tc::tma_load_2d_pair(sb, mB, fb, k0, n0);
+    } else {
+#pragma unroll
+      for (int j = 0; j < BN / 128; ++j)
+        tc::tma_load_2d_pair(sb + j * 8192, mB, fb, n0 + 64 * j, k0);
+    }
+  }
+  return true;
+}
+
+// MMA issuer, one tile (even CTA): the j-th tile of this pair goes to
+// accumulator j % ACC once both CTAs' epilogues have drained its last use.
+template <class Op, class Cfg, int BN, int STAGES, int ACC>
+__device__ __forceinline__ bool tc2_mma(const Tc2Shape& s, int tile, int j, uint32_t tmem,
+                                        uint8_t* smem, uint64_t* full, uint64_t* empty,
+                                        uint64_t* tfull, uint64_t* tempty, int& it,
+                                        unsigned* status) {
+  constexpr uint32_t idesc = tc::idesc_bf16(2 * kBM, BN, Op::A_MN ? 1 : 0, Op::B_MN ? 1 : 0);
+  const int z = (tile / s.tiles_m) / s.tiles_n;
+  const int kb0 = z * s.kps, nk = min(s.nkb, kb0 + s.kps) - kb0;
+  const int acc = j % ACC, use = j / ACC;
+  if (use > 0 && !tc::mbar_wait_cluster(&tempty[acc], (use - 1) & 1, status)) return false;
+  tc::fence_after_sync();
+  const uint32_t d = tmem + (uint32_t)(acc * BN);
+  bool ok = true;
+  for (int i = 0; i < nk; ++i, ++it) {
+    const int st = it % STAGES;
+    if (!tc::mbar_wait_cluster(&full[st], (it / STAGES) & 1, status)) {
+      ok = false;
+      break;
+    }
+    tc::fence_after_sync();
+    const uint32_t sa = tc::smem_u32(smem + st * Cfg::STAGE_BYTES);
+    const uint32_t sb = sa + Cfg::A_BYTES;
+#pragma unroll
+    for (int kk = 0; kk < kBK / 16; ++kk) {
+      const uint64_t ad = Op::A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024)
+                                   : tc::sdesc(sa + kk * 32, 16, 1024);
+      const uint64_t bd = Op::B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024)
+                                   : tc::sdesc(sb + kk * 32, 16, 1024);
+      tc::mma_bf16_pair(d, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
+    }
+    tc::mma_commit_pair(&empty[st]);
+  }
+  tc::mma_commit_pair(&tfull[acc]);
+  return ok;
+}
+
+// Epilogue, one tile (warps 2..9 of both CTAs): this CTA's 128 accumulator
+// rows, warp w reading TMEM lane quarter w % 4 and half of the columns.
+template <class Op, int BN, int ACC>
+__device__ __forceinline__ bool tc2_epilogue(const typename Op::Epi& epi, const CUtensorMap* mC,
+                                             const Tc2Shape& s, int tile, int j, uint32_t rank,
+                                             int warp, int lane, uint32_t tmem, uint64_t* tfull,
+                                             uint32_t te0, uint8_t* sbuf, int& nout,
+                                             unsigned* status) {
+  using Epi = typename Op::Epi;
+  const int q = warp & 3;
+  const int c_beg = ((warp - 2) >> 2) * (BN / 2);
+  const int m_blk = tile % s.tiles_m, rest = tile / s.tiles_m;
+  const int n_blk = rest % s.tiles_n, z = rest / s.tiles_n;
+  const int acc = j % ACC, use = j / ACC;
+  const int row0 = m_blk * 2 * kBM + (int)rank * kBM + q * 32;
+  const int row = row0 + lane;
+  const int n0 = n_blk * BN;
+  const bool row_ok = row < s.M;
+  constexpr int NCH = BN / 64;
+  typename Epi::Pre pre[2];
+  if (row_ok && n0 + c_beg < s.N) epi.load(row, n0 + c_beg, pre[0]);
+  const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
+  tc::fence_after_sync();
+  const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll
+  for (int ci = 0; ci < NCH; ++ci) {
+    const int c = c_beg + ci * 32;
+    if (ci + 1 < NCH && row_ok && n0 + c + 32 < s.N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
+    float v[32];
+    tc::tmem_ld32(base + (uint32_t)c, v);
+    if (n0 + c < s.N)
+      epi_chunk(epi, mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1], ok && row_ok, ok);
+  }
+  tc::fence_before_sync();
+  __syncwarp();
+  if (lane == 0) tc::mbar_arrive_cluster(te0 + (uint32_t)(acc * 8));
+  return ok;
+}
+
+template <int BN, int STAGES, int ACC, class Op0, class Op1>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    gemm_tc2_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                    const __grid_constant__ CUtensorMap mC, int M, int N, int kps, int nkb,
-                    int tiles_m, int tiles_n, int n_tiles, Epi epi, unsigned* status) {
+    gemm_tc2_kernel(const __grid_constant__ Tc2Params<Op0, Op1> P, unsigned* status) {
   using Cfg = Tc2Cfg<BN, STAGES, ACC>;
+  constexpr bool kSame = std::is_same<Op0, Op1>::value;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -511,6 +657,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = tc::cluster_rank();
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  int total = 0;
+  for (int q = 0; q < P.count; ++q) total += P.shape[q].n_tiles;
+  // product of a combined item index; *tile becomes the tile within it
+  auto which = [&](int item, int* tile) {
+    int q = 0;
+    while (q + 1 < P.count && item >= P.shape[q].n_tiles) item -= P.shape[q++].n_tiles;
+    *tile = item;
+    return q;
+  };
 
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -522,8 +677,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       tc::mbar_init(&tempty[a], 16);  // 8 epilogue warps in each CTA
     }
     tc::fence_mbar_init();
-    tc::prefetch_tmap(&mA);
-    tc::prefetch_tmap(&mB);
+    for (int q = 0; q < P.count; ++q) {
+      tc::prefetch_tmap(&P.map[q][0]);
+      tc::prefetch_tmap(&P.map[q][1]);
+    }
   }
   if (warp == 1) {
     tc::tmem_alloc_pair(tslot, Cfg::TMEM_COLS);
@@ -538,112 +695,59 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---- TMA producer (both CTAs): this CTA's rows of A and half of B
       int it = 0;
-      bool ok = true;
-      for (int tile = pair; tile < n_tiles && ok; tile += npairs) {
-        const int m_blk = tile % tiles_m, rest = tile / tiles_m;
-        const int n_blk = rest % tiles_n, z = rest / tiles_n;
-        const int m0 = m_blk * 2 * kBM + (int)rank * kBM;
-        const int n0 = n_blk * BN + (int)rank * (BN / 2);
-        const int kb0 = z * kps;
-        const int nk = min(nkb, kb0 + kps) - kb0;
-        for (int i = 0; i < nk; ++i, ++it) {
-          const int s = it % STAGES;
-          if (it >= STAGES && !tc::mbar_wait(&empty[s], ((it / STAGES) - 1) & 1, status)) {
-            ok = false;
-            break;
-          }
-          uint8_t* sa = smem + s * Cfg::STAGE_BYTES;
-          uint8_t* sb = sa + Cfg::A_BYTES;
-          const uint32_t fb = tc::mapa(tc::smem_u32(&full[s]), 0);
-          if (rank == 0) tc::mbar_arrive_expect_tx(&full[s], 2 * Cfg::STAGE_BYTES);
-          const int k0 = (kb0 + i) * kBK;
-          if (!A_MN) {
-            tc::tma_load_2d_pair(sa, &mA, fb, k0, m0);
-          } else {
-            tc::tma_load_2d_pair(sa, &mA, fb, m0, k0);
-            tc::tma_load_2d_pair(sa + 8192, &mA, fb, m0 + 64, k0);
-          }
-          if (!B_MN) {
-            tc::tma_load_2d_pair(sb, &mB, fb, k0, n0);
-          } else {
-#pragma unroll
-            for (int j = 0; j < BN / 128; ++j)
-              tc::tma_load_2d_pair(sb + j * 8192, &mB, fb, n0 + 64 * j, k0);
-          }
-        }
+      for (int item = pair; item < total; item += npairs) {
+        int tile;
+        const int q = which(item, &tile);
+        bool ok;
+        if (kSame || q > 0)
+          ok = tc2_produce<Op1, Cfg, BN, STAGES>(&P.map[q][0], &P.map[q][1], P.shape[q], tile, rank,
+                                                 smem, full, empty, it, status);
+        else
+          ok = tc2_produce<Op0, Cfg, BN, STAGES>(&P.map[q][0], &P.map[q][1], P.shape[q], tile, rank,
+                                                 smem, full, empty, it, status);
+        if (!ok) break;
       }
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
-      // ---- MMA issuer (even CTA only)
-      constexpr uint32_t idesc = tc::idesc_bf16(2 * kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
       int it = 0, j = 0;
-      bool ok = true;
-      for (int tile = pair; tile < n_tiles && ok; tile += npairs, ++j) {
-        const int z = (tile / tiles_m) / tiles_n;
-        const int kb0 = z * kps, nk = min(nkb, kb0 + kps) - kb0;
-        const int acc = j % ACC, use = j / ACC;
-        if (use > 0 && !tc::mbar_wait_cluster(&tempty[acc], (use - 1) & 1, status)) break;
-        tc::fence_after_sync();
-        const uint32_t d = tmem + (uint32_t)(acc * BN);
-        for (int i = 0; i < nk; ++i, ++it) {
-          const int s = it % STAGES;
-          if (!tc::mbar_wait_cluster(&full[s], (it / STAGES) & 1, status)) {
-            ok = false;
-            break;
-          }
-          tc::fence_after_sync();
-          const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE_BYTES);
-          const uint32_t sb = sa + Cfg::A_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = A_MN ? tc::sdesc(sa + kk * 2048, 8192, 1024)
-                                     : tc::sdesc(sa + kk * 32, 16, 1024);
-            const uint64_t bd = B_MN ? tc::sdesc(sb + kk * 2048, 8192, 1024)
-                                     : tc::sdesc(sb + kk * 32, 16, 1024);
-            tc::mma_bf16_pair(d, ad, bd, idesc, (i | kk) != 0 ? 1u : 0u);
-          }
-          tc::mma_commit_pair(&empty[s]);
-        }
-        tc::mma_commit_pair(&tfull[acc]);
+      for (int item = pair; item < total; item += npairs, ++j) {
+        int tile;
+        const int q = which(item, &tile);
+        bool ok;
+        if (kSame || q > 0)
+          ok = tc2_mma<Op1, Cfg, BN, STAGES, ACC>(P.shape[q], tile, j, tmem, smem, full, empty,
+                                                  tfull, tempty, it, status);
+        else
+          ok = tc2_mma<Op0, Cfg, BN, STAGES, ACC>(P.shape[q], tile, j, tmem, smem, full, empty,
+                                                  tfull, tempty, it, status);
+        if (!ok) break;
       }
     }
   } else {
-    // ---- epilogue warps 2..9 (both CTAs): this CTA's 128 accumulator rows
-    const int q = warp & 3;
-    const int c_beg = ((warp - 2) >> 2) * (BN / 2);
     const uint32_t te0 = tc::mapa(tc::smem_u32(&tempty[0]), 0);
     uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
-    int j = 0, nout = 0;
-    for (int tile = pair; tile < n_tiles; tile += npairs, ++j) {
-      const int m_blk = tile % tiles_m, rest = tile / tiles_m;
-      const int n_blk = rest % tiles_n, z = rest / tiles_n;
-      const int acc = j % ACC, use = j / ACC;
-      const int row0 = m_blk * 2 * kBM + (int)rank * kBM + q * 32;
-      const int row = row0 + lane;
-      const int n0 = n_blk * BN;
-      const bool row_ok = row < M;
-      constexpr int NCH = BN / 64;
-      typename Epi::Pre pre[2];
-      if (row_ok && n0 + c_beg < N) epi.load(row, n0 + c_beg, pre[0]);
-      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
-      tc::fence_after_sync();
-      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-#pragma unroll
-      for (int ci = 0; ci < NCH; ++ci) {
-        const int c = c_beg + ci * 32;
-        if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
-        float v[32];
-        tc::tmem_ld32(base + (uint32_t)c, v);
-        if (n0 + c < N)
-          epi_chunk(epi, &mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1],
-                    ok && row_ok, ok);
+    int j = 0, nout = 0, prev = -1;
+    for (int item = pair; item < total; item += npairs, ++j) {
+      int tile;
+      const int q = which(item, &tile);
+      bool ok;
+      if constexpr (kSame) {
+        ok = tc2_epilogue<Op1, BN, ACC>(q == 0 ? P.epi0 : P.epi1[q - 1], &P.map[q][2], P.shape[q],
+                                        tile, j, rank, warp, lane, tmem, tfull, te0, sbuf, nout,
+                                        status);
+      } else {
+        // the ops may stage chunks of different sizes in the same buffer: the
+        // first tile after op 0's waits until op 0's staged chunks are read
+        if (q > 0 && prev == 0 && lane == 0) tc::tma_store_wait_read<0>();
+        ok = q > 0 ? tc2_epilogue<Op1, BN, ACC>(P.epi1[q - 1], &P.map[q][2], P.shape[q], tile, j,
+                                                rank, warp, lane, tmem, tfull, te0, sbuf, nout,
+                                                status)
+                   : tc2_epilogue<Op0, BN, ACC>(P.epi0, &P.map[q][2], P.shape[q], tile, j, rank,
+                                                warp, lane, tmem, tfull, te0, sbuf, nout, status);
       }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive_cluster(te0 + (uint32_t)(acc * 8));
+      prev = q;
       if (!ok) break;
     }
     if (lane == 0) tc::tma_store_wait_read<0>();  // staging read; the writes finish with the grid
@@ -655,44 +759,74 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (warp == 1) tc::tmem_dealloc_pair(tmem, Cfg::TMEM_COLS);
 }
 
-template <int BN, int STAGES, int ACC, bool A_MN, bool B_MN, class Epi>
-static cudaError_t tc2_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
-                              long sak, const void* B, long sbk, long sbn, const Epi& epi,
-                              int splits) {
-  using Cfg = Tc2Cfg<BN, STAGES, ACC>;
-  CUtensorMap mA, mB;
+// Operand tensor maps of one pair-kernel product (A: 128 x 64 boxes K-major,
+// or two 64 x 64 boxes MN-major; B: BN/2 x 64 K-major or 64 x 64 MN-major).
+template <int BN, bool A_MN, bool B_MN>
+static bool tc2_operand_maps(CUtensorMap* mA, CUtensorMap* mB, int M, int N, int K, const void* A,
+                             long sam, long sak, const void* B, long sbk, long sbn) {
   if (!A_MN) {
     uint64_t d[2] = {(uint64_t)K, (uint64_t)M}, st[1] = {(uint64_t)sam * 2};
     uint32_t box[2] = {64, 128};
-    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+    if (!make_tmap_bf16(mA, A, 2, d, st, box)) return false;
   } else {
     uint64_t d[2] = {(uint64_t)M, (uint64_t)K}, st[1] = {(uint64_t)sak * 2};
     uint32_t box[2] = {64, 64};
-    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+    if (!make_tmap_bf16(mA, A, 2, d, st, box)) return false;
   }
   if (!B_MN) {
     uint64_t d[2] = {(uint64_t)K, (uint64_t)N}, st[1] = {(uint64_t)sbn * 2};
     uint32_t box[2] = {64, (uint32_t)(BN / 2)};
-    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+    if (!make_tmap_bf16(mB, B, 2, d, st, box)) return false;
   } else {
     uint64_t d[2] = {(uint64_t)N, (uint64_t)K}, st[1] = {(uint64_t)sbk * 2};
     uint32_t box[2] = {64, 64};
-    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+    if (!make_tmap_bf16(mB, B, 2, d, st, box)) return false;
   }
-  const int nkb = (K + kBK - 1) / kBK;
-  const int kps = (nkb + splits - 1) / splits;
-  const int tiles_m = (M + 2 * kBM - 1) / (2 * kBM), tiles_n = (N + BN - 1) / BN;
-  const int n_tiles = tiles_m * tiles_n * splits;
-  auto kern = gemm_tc2_kernel<BN, STAGES, ACC, A_MN, B_MN, Epi>;
+  return true;
+}
+
+template <int BN>
+static Tc2Shape tc2_shape(int M, int N, int K, int splits) {
+  Tc2Shape s;
+  s.M = M;
+  s.N = N;
+  s.nkb = (K + kBK - 1) / kBK;
+  s.kps = (s.nkb + splits - 1) / splits;
+  s.tiles_m = (M + 2 * kBM - 1) / (2 * kBM);
+  s.tiles_n = (N + BN - 1) / BN;
+  s.n_tiles = s.tiles_m * s.tiles_n * splits;
+  return s;
+}
+
+template <int BN, int STAGES, int ACC, class Op0, class Op1>
+static cudaError_t tc2_run(const Launch& lc, const Tc2Params<Op0, Op1>& P) {
+  using Cfg = Tc2Cfg<BN, STAGES, ACC>;
+  auto kern = gemm_tc2_kernel<BN, STAGES, ACC, Op0, Op1>;
   static std::atomic<unsigned long long> opted{0};
   if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
-  CUtensorMap mC;
-  if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
-  const int pairs = n_tiles < sm_count() / 2 ? n_tiles : sm_count() / 2;
-  cudaError_t e = launch_k_cluster(kern, dim3(2 * pairs), dim3(kGemmThreads), Cfg::SMEM,
-                                   lc.stream, 2, mA, mB, mC, M, N, kps, nkb, tiles_m, tiles_n,
-                                   n_tiles, epi, lc.status);
+  int total = 0;
+  for (int q = 0; q < P.count; ++q) total += P.shape[q].n_tiles;
+  const int pairs = total < sm_count() / 2 ? total : sm_count() / 2;
+  cudaError_t e = launch_k_cluster(kern, dim3(2 * pairs), dim3(kGemmThreads), Cfg::SMEM, lc.stream,
+                                   2, P, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+template <int BN, int STAGES, int ACC, bool A_MN, bool B_MN, class Epi>
+static cudaError_t tc2_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                              long sak, const void* B, long sbk, long sbn, const Epi& epi,
+                              int splits) {
+  using Op = Tc2Op<A_MN, B_MN, Epi>;
+  Tc2Params<Op, Op> P;
+  memset(&P, 0, sizeof(P));
+  if (!tc2_operand_maps<BN, A_MN, B_MN>(&P.map[0][0], &P.map[0][1], M, N, K, A, sam, sak, B, sbk,
+                                        sbn))
+    return cudaErrorInvalidValue;
+  P.shape[0] = tc2_shape<BN>(M, N, K, splits);
+  if (!out_map(&P.map[0][2], epi, M, N, splits)) return cudaErrorInvalidValue;
+  P.epi0 = epi;
+  P.count = 1;
+  return tc2_run<BN, STAGES, ACC, Op, Op>(lc, P);
 }
 
 // Test path: the CTA-pair kernel with 256 x 256 tiles (plain and split-K stores).
@@ -722,6 +856,42 @@ cudaError_t gemm_tc_pair(const Launch& lc, int dtype_out, int M, int N, int K, c
   if (a_k && b_k) return go(F{}, F{});
   if (!a_k && !b_k) return go(T{}, T{});
   return go(T{}, F{});
+}
+
+cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const PairProduct* w,
+                               int nw) {
+  if (nw < 1 || nw > kTc2Max - 1) return cudaErrorInvalidValue;
+  auto valid = [](const PairProduct& q) { return q.N % 256 == 0 && q.M >= 1 && q.K >= 1; };
+  if (!valid(p0) || p0.sak != 1 || p0.sbk != 1) return valid(p0) ? cudaErrorNotSupported
+                                                                   : cudaErrorInvalidValue;
+  for (int i = 0; i < nw; ++i) {
+    if (!valid(w[i])) return cudaErrorInvalidValue;
+    if (w[i].sam != 1 || w[i].sbn != 1) return cudaErrorNotSupported;
+  }
+  constexpr int ST = 6, ACC = 2;
+  using Op0 = Tc2Op<false, false, EpiStoreF<bf16>>;
+  using Op1 = Tc2Op<true, true, EpiStoreF<float>>;
+  Tc2Params<Op0, Op1> P;
+  memset(&P, 0, sizeof(P));
+  P.epi0 = EpiStoreF<bf16>{(bf16*)p0.out, p0.ldo, 0};
+  if (!tc2_operand_maps<256, false, false>(&P.map[0][0], &P.map[0][1], p0.M, p0.N, p0.K, p0.A,
+                                           p0.sam, p0.sak, p0.B, p0.sbk, p0.sbn) ||
+      !out_map(&P.map[0][2], P.epi0, p0.M, p0.N, 1))
+    return cudaErrorInvalidValue;
+  P.shape[0] = tc2_shape<256>(p0.M, p0.N, p0.K, 1);
+  // the weight gradients: fp32 K-split partials, A and B MN-major
+  for (int i = 0; i < nw; ++i) {
+    const PairProduct& q = w[i];
+    const int sp = effective_splits(q.K, q.splits);
+    P.epi1[i] = EpiStoreF<float>{(float*)q.out, q.ldo, q.split_stride};
+    P.shape[i + 1] = tc2_shape<256>(q.M, q.N, q.K, sp);
+    if (!tc2_operand_maps<256, true, true>(&P.map[i + 1][0], &P.map[i + 1][1], q.M, q.N, q.K, q.A,
+                                           q.sam, q.sak, q.B, q.sbk, q.sbn) ||
+        !out_map(&P.map[i + 1][2], P.epi1[i], q.M, q.N, sp))
+      return cudaErrorInvalidValue;
+  }
+  P.count = 1 + nw;
+  return tc2_run<256, ST, ACC, Op0, Op1>(lc, P);
 }
 
 // Output tile widths: 128 x 256 tiles move 48 KB per 64-deep K slice for
@@ -834,36 +1004,69 @@ cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K
 }
 
 // ============================================================ split reduction
+// Up to kRedMax independent reductions (segments) in one launch: the first
+// count_0 / 4 threads reduce segment 0, the next count_1 / 4 segment 1, ...
+// Each thread sums its 4 elements over the splits in split order.
+constexpr int kRedMax = 3;
 template <class TO>
-__global__ void reduce_splits_kernel(const float* __restrict__ part, int splits, long count,
-                                     TO* __restrict__ out) {
+struct RedSegs {
+  const float* part[kRedMax];
+  TO* out[kRedMax];
+  long count[kRedMax];
+  int splits[kRedMax];
+  int n;
+};
+
+template <class TO>
+__global__ void reduce_splits_kernel(const __grid_constant__ RedSegs<TO> R) {
   pdl_enter();
-  const long i4 = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
-  if (i4 >= count) return;
+  long i4 = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  int q = 0;
+  while (q < R.n && i4 >= R.count[q]) i4 -= R.count[q++];
+  if (q >= R.n) return;
+  const float* part = R.part[q];
+  const long count = R.count[q];
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 4
-  for (int s = 0; s < splits; ++s) {
+  for (int s = 0; s < R.splits[q]; ++s) {
     float v[4];
     load4(part + (long)s * count + i4, v);
 #pragma unroll
     for (int e = 0; e < 4; ++e) acc[e] += v[e];
   }
-  store4(out + i4, acc);
+  store4(R.out[q] + i4, acc);
+}
+
+template <class TO>
+static cudaError_t reduce_typed(const Launch& lc, const SplitSum* segs, int n) {
+  RedSegs<TO> R;
+  memset(&R, 0, sizeof(R));
+  long n4 = 0;
+  for (int i = 0; i < n; ++i) {
+    R.part[i] = segs[i].part;
+    R.out[i] = static_cast<TO*>(segs[i].out);
+    R.count[i] = segs[i].count;
+    R.splits[i] = segs[i].splits;
+    n4 += segs[i].count / 4;
+  }
+  R.n = n;
+  const int threads = 256;
+  const unsigned blocks = (unsigned)((n4 + threads - 1) / threads);
+  launch_k(reduce_splits_kernel<TO>, dim3(blocks), dim3(threads), 0, lc.stream, R);
+  return cudaGetLastError();
+}
+
+cudaError_t reduce_splits_n(const Launch& lc, const SplitSum* segs, int n, int dtype_out) {
+  if (n < 1 || n > kRedMax) return cudaErrorInvalidValue;
+  for (int i = 0; i < n; ++i)
+    if (segs[i].count % 4 != 0) return cudaErrorInvalidValue;
+  return dtype_out == 0 ? reduce_typed<float>(lc, segs, n) : reduce_typed<bf16>(lc, segs, n);
 }
 
 cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long count,
                           int dtype_out, void* out) {
-  if (count % 4 != 0) return cudaErrorInvalidValue;
-  const long n4 = count / 4;
-  const int threads = 256;
-  const unsigned blocks = (unsigned)((n4 + threads - 1) / threads);
-  if (dtype_out == 0)
-    launch_k(reduce_splits_kernel<float>, dim3(blocks), dim3(threads), 0, lc.stream,
-part, splits, count, (float*)out);
-  else
-    launch_k(reduce_splits_kernel<bf16>, dim3(blocks), dim3(threads), 0, lc.stream,
-part, splits, count, (bf16*)out);
-  return cudaGetLastError();
+  const SplitSum seg{part, splits, count, out};
+  return reduce_splits_n(lc, &seg, 1, dtype_out);
 }
 
 }  // namespace bcmt

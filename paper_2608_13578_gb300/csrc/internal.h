@@ -67,6 +67,26 @@ extern int g_force_bn;
 cudaError_t gemm_tc_pair(const Launch& lc, int dtype_out, int M, int N, int K, const void* A,
                          long sam, long sak, const void* B, long sbk, long sbn, EpiKind epi,
                          const EpiArgs& ea, int splits);
+// One product of a grouped CTA-pair GEMM: C[M,N] = A[M,K] B[K,N] (bf16
+// inputs, element strides as for gemm), written to `out` with row stride ldo
+// and, for K-split partials, split_stride elements between splits.
+struct PairProduct {
+  int M, N, K;
+  const void* A;
+  long sam, sak;
+  const void* B;
+  long sbk, sbn;
+  void* out;
+  long ldo, split_stride;
+  int splits;
+};
+// Several products in one CTA-pair launch (256 x 256 tiles, N % 256 == 0 for
+// each): p0 stored as bf16 with A and B K-major (dX = dQKV W_QKV^T), then
+// w[0..nw-1] (1 <= nw <= 3) as fp32 K-split partials with A and B MN-major
+// (the weight gradients dW = X^T dY).  The pairs take p0's tiles, then each
+// w[i]'s in order, round-robin.  cudaErrorNotSupported for other layouts.
+cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const PairProduct* w,
+                               int nw);
 cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits);
@@ -76,6 +96,14 @@ bool gemm_tc_available();
 // order, stored in dtype_out.
 cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long count, int dtype_out,
                           void* out);
+// Up to three such reductions in one launch (the same dtype_out).
+struct SplitSum {
+  const float* part;
+  int splits;
+  long count;
+  void* out;
+};
+cudaError_t reduce_splits_n(const Launch& lc, const SplitSum* segs, int n, int dtype_out);
 
 // ------------------------------------------------------------ attention
 // Intra-block causal attention (Sec. 3.3).  Q, K, V rows of token (b,t) start

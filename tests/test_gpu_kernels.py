@@ -78,6 +78,57 @@ def test_gemm_split_k(C, impl):
     assert (got - ref).abs().max().item() / ref.abs().max().item() < 1e-5
 
 
+# Grouped CTA-pair launch (the backward's dX, K-split dW_QKV and dW_g): the
+# layer's own shapes at B*T = 1024, D = 512, then ragged rows, ragged K and
+# split counts that leave a short last range; the second case has no third
+# product.
+GROUP_SHAPES = [
+    # (M0, N0, K0), (M1, N1, K1, splits1), (M2, N2, K2, splits2) or None
+    ((1024, 512, 1536), (512, 1536, 1024, 7), (512, 512, 1024, 3)),
+    ((1000, 256, 768), (256, 768, 1000, 3), None),
+    ((300, 768, 320), (768, 512, 4096, 13), (256, 256, 4000, 5)),
+]
+
+
+def _eff_splits(K, s):
+    nkb = -(-K // 64)
+    kps = -(-nkb // max(1, min(s, nkb)))
+    return -(-nkb // kps)
+
+
+@pytest.mark.parametrize("p0,p1,p2", GROUP_SHAPES)
+def test_gemm_group(C, p0, p1, p2):
+    if not (C.bcmt_test_set_tensor_cores(True, True) & 1):
+        pytest.fail("tcgen05 GEMM unavailable on this GPU/build")
+    (M0, N0, K0), (M1, N1, K1, s1) = p0, p1
+    gen = torch.Generator().manual_seed(M0 + N1 + K1)
+    dt = torch.bfloat16
+    A0, lda0, _, A0l = _operand(M0, K0, True, dt, gen)       # K-major
+    B0t, _, ldb0t, B0l = _operand(K0, N0, False, dt, gen)    # stored [N0, K0]: K-major
+    A1t, _, lda1t, A1l = _operand(M1, K1, False, dt, gen)    # stored [K1, M1]: MN-major
+    B1, ldb1, _, B1l = _operand(K1, N1, True, dt, gen)       # stored [K1, N1]: MN-major
+    C0 = torch.full((M0, N0), float("nan"), dtype=dt, device="cuda")
+    part1 = torch.full((s1, M1, N1), float("nan"), dtype=torch.float32, device="cuda")
+    extra = {}
+    if p2 is not None:
+        M2, N2, K2, s2 = p2
+        A2t, _, lda2t, A2l = _operand(M2, K2, False, dt, gen)
+        B2, ldb2, _, B2l = _operand(K2, N2, True, dt, gen)
+        part2 = torch.full((s2, M2, N2), float("nan"), dtype=torch.float32, device="cuda")
+        extra = dict(M2=M2, N2=N2, K2=K2, A2t=A2t.cuda(), lda2t=lda2t, B2=B2.cuda(), ldb2=ldb2,
+                     part2=part2, splits2=s2)
+    n1 = C.bcmt_test_gemm_group(M0, N0, K0, A0.cuda(), lda0, B0t.cuda(), ldb0t, C0, M1, N1, K1,
+                                A1t.cuda(), lda1t, B1.cuda(), ldb1, part1, s1, **extra)
+    torch.cuda.synchronize()
+    assert n1 == _eff_splits(K1, s1)
+    rel = lambda got, ref: (got - ref).abs().max().item() / ref.abs().max().item()
+    assert rel(C0.double().cpu(), A0l.double() @ B0l.double()) < 8e-3
+    assert rel(part1[:n1].double().sum(0).cpu(), A1l.double() @ B1l.double()) < 1e-5
+    if p2 is not None:
+        n2 = _eff_splits(K2, s2)
+        assert rel(part2[:n2].double().sum(0).cpu(), A2l.double() @ B2l.double()) < 1e-5
+
+
 def test_gemm_fp32_simt_exact_enough(C):
     M, N, K = 130, 192, 300
     gen = torch.Generator().manual_seed(9)
