@@ -150,6 +150,24 @@ constexpr int kBM = 128, kBK = 64;
 constexpr int kEpiWarps = 8;
 constexpr int kOutStage = 4096;  // per epilogue warp: two 32x32 bf16 or one 32x32 fp32 chunk
 
+// Output tile of a persistent GEMM's tile index: K split z slowest; within a
+// split, bands of kBand m-blocks, and within a band m fastest, so that the
+// tiles running at one time share a few rows of A and columns of B in L2
+// instead of sweeping all of A for every column block.
+constexpr int kBand = 8;
+__device__ __forceinline__ void tile_mnz(int tile, int tiles_m, int tiles_n, int& m_blk,
+                                         int& n_blk, int& z) {
+  const int per_z = tiles_m * tiles_n;
+  z = tile / per_z;
+  const int t = tile - z * per_z;
+  const int band = t / (kBand * tiles_n);
+  const int m0 = band * kBand;
+  const int gm = min(kBand, tiles_m - m0);
+  const int r = t - band * kBand * tiles_n;
+  m_blk = m0 + r % gm;
+  n_blk = r / gm;
+}
+
 __device__ __forceinline__ uint4 pack8_bf16(const float* v) {
   uint4 q;
   __nv_bfloat162 t0 = __floats2bfloat162_rn(v[0], v[1]), t1 = __floats2bfloat162_rn(v[2], v[3]);
@@ -292,8 +310,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       int it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const int m_blk = tile % tiles_m, rest = tile / tiles_m;
-        const int n_blk = rest % tiles_n, z = rest / tiles_n;
+        int m_blk, n_blk, z;
+        tile_mnz(tile, tiles_m, tiles_n, m_blk, n_blk, z);
         const int m0 = m_blk * kBM, n0 = n_blk * BN, kb0 = z * kps;
         const int nk = min(nkb, kb0 + kps) - kb0;
         for (int i = 0; i < nk; ++i, ++it) {
@@ -368,8 +386,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
     int j = 0, nout = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++j) {
-      const int m_blk = tile % tiles_m, rest = tile / tiles_m;
-      const int n_blk = rest % tiles_n, z = rest / tiles_n;
+      int m_blk, n_blk, z;
+      tile_mnz(tile, tiles_m, tiles_n, m_blk, n_blk, z);
       const int acc = j & 1, use = j >> 1;
       const int row0 = m_blk * kBM + q * 32;
       const int row = row0 + lane;
@@ -532,8 +550,8 @@ __device__ __forceinline__ bool tc2_produce(const CUtensorMap* mA, const CUtenso
                                             const Tc2Shape& s, int tile, uint32_t rank,
                                             uint8_t* smem, uint64_t* full, uint64_t* empty,
                                             int& it, unsigned* status) {
-  const int m_blk = tile % s.tiles_m, rest = tile / s.tiles_m;
-  const int n_blk = rest % s.tiles_n, z = rest / s.tiles_n;
+  int m_blk, n_blk, z;
+  tile_mnz(tile, s.tiles_m, s.tiles_n, m_blk, n_blk, z);
   const int m0 = m_blk * 2 * kBM + (int)rank * kBM;
   const int n0 = n_blk * BN + (int)rank * (BN / 2);
   const int kb0 = z * s.kps;
@@ -612,8 +630,8 @@ __device__ __forceinline__ bool tc2_epilogue(const typename Op::Epi& epi, const 
   using Epi = typename Op::Epi;
   const int q = warp & 3;
   const int c_beg = ((warp - 2) >> 2) * (BN / 2);
-  const int m_blk = tile % s.tiles_m, rest = tile / s.tiles_m;
-  const int n_blk = rest % s.tiles_n, z = rest / s.tiles_n;
+  int m_blk, n_blk, z;
+  tile_mnz(tile, s.tiles_m, s.tiles_n, m_blk, n_blk, z);
   const int acc = j % ACC, use = j / ACC;
   const int row0 = m_blk * 2 * kBM + (int)rank * kBM + q * 32;
   const int row = row0 + lane;
