@@ -361,6 +361,15 @@ int dqkv_splits(const Geometry& g) {
   return tail_grouped(g) ? tail_plan(g).s[0] : dw_splits(g.dtype, g.D, 3 * g.D, g.n);
 }
 
+// K splits of the memory projections P = M W_m and dM = dP W_m^T ([B*Nb, D]
+// x [D, D]): a few hundred rows make one tile row, so splitting K spreads
+// the operand bytes over more SMs (each CTA of the unsplit product streams
+// all of M); the consumers sum the fp32 partials as they read them.  dM runs
+// beside dH = dY + dU W_g^T, which holds most SMs: two splits, so that its
+// CTAs fit in the SMs left over.
+int mem_splits(const Geometry& g) { return effective_splits(g.D, 4); }
+int dm_splits(const Geometry& g) { return effective_splits(g.D, 2); }
+
 struct FwdWs {
   char *qkv, *hhat, *hloc, *G, *Mb;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
@@ -389,7 +398,8 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     // M in the storage dtype: the A operand of the memory projection (and of dW_m)
     w.Mb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.M);
     w.Z = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
-    w.C = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    // the K-split partials of P = M W_m (the memory rows C, before the shift)
+    w.C = reinterpret_cast<float*>(take((size_t)mem_splits(g) * g.B * g.Nb * g.D * 4));
     w.G = take((size_t)g.n * g.D * g.es);
   } else {
     w.hloc = w.G = w.Mb = nullptr;
@@ -419,7 +429,7 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dH = take((size_t)g.n * g.D * g.es);
     w.dP = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.dPb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.dP);
-    w.dM = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
+    w.dM = reinterpret_cast<float*>(take((size_t)dm_splits(g) * g.B * g.Nb * g.D * 4));
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(
@@ -489,11 +499,12 @@ cudaError_t weight_grad(const Launch& lc, Prof& pr, const char* name, int dtype,
 
 cudaError_t run_gemm(const Launch& lc, Prof& pr, const char* name, int dtype, int dtype_out, int M,
                      int N, int K, const void* A, long sam, long sak, const void* B, long sbk,
-                     long sbn, EpiKind epi, const EpiArgs& ea) {
+                     long sbn, EpiKind epi, const EpiArgs& ea, int splits = 1) {
   pr.begin(name);
-  cudaError_t e = (dtype == 1 && g_use_tc_gemm)
-                      ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1)
-                      : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
+  cudaError_t e =
+      (dtype == 1 && g_use_tc_gemm)
+          ? gemm_tc(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits)
+          : gemm_simt(lc, dtype, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
   pr.end(nullptr);
   return e;
 }
@@ -652,23 +663,24 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
     pr.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.C,
-                        g.B, g.Nb, D);
+    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, g.B,
+                        g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "causal memory");
     {
+      // P = M W_m as K-split partials; the shift is applied by the readers
       EpiArgs ea;
       ea.out = w.C;
       ea.ldo = D;
-      ea.Nb = g.Nb;
+      ea.split_stride = (long)g.B * g.Nb * D;
       e = run_gemm(lc, pr, "gemm_wm", g.dtype, 0, g.B * g.Nb, D, D, w.Mb, D, 1, w_m, D, 1,
-                   EPI_SHIFT, ea);
+                   EPI_PARTIAL, ea, mem_splits(g));
       if (e != cudaSuccess) return cuda_fail(e, "memory projection");
     }
     // Sec. 3.7-3.8: Y = H + G * M_tokens once the gate is ready too
     fork.wait_mark(gate_done);
     pr.begin("inject");
-    e = inject(lc, g.dtype, w.hloc, w.G, w.C, y, g.B, g.T, D, g.L);
+    e = inject(lc, g.dtype, w.hloc, w.G, w.C, mem_splits(g), y, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "injection");
   }
@@ -730,7 +742,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
   if (!g.honly) {
     // Sec. 3.8 reversed: dU and the per-block memory gradient (shifted: dP).
     pr.begin("gate_bwd");
-    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, bw.dU, bw.dP, g.dtype == BCMT_BF16 ? bw.dPb : nullptr,
+    e = gate_bwd(lc, g.dtype, dy, w.G, w.C, mem_splits(g), bw.dU, bw.dP, g.dtype == BCMT_BF16 ? bw.dPb : nullptr,
                  g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "gate backward");
@@ -741,13 +753,14 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
       EpiArgs ea;
       ea.out = bw.dM;
       ea.ldo = D;
+      ea.split_stride = (long)g.B * g.Nb * D;
       e = run_gemm(lcs, prs, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
-                   EPI_STORE, ea);
+                   EPI_PARTIAL, ea, dm_splits(g));
       if (e != cudaSuccess) return cuda_fail(e, "dM");
     }
     prs.begin("memory_scan_bwd");
-    e = memory_scan_bwd(lcs, bw.dM, decay, w.Z, w.M, bw.dS, d_decay ? bw.da_part : nullptr, g.B,
-                        g.Nb, D);
+    e = memory_scan_bwd(lcs, bw.dM, dm_splits(g), decay, w.Z, w.M, bw.dS,
+                        d_decay ? bw.da_part : nullptr, g.B, g.Nb, D);
     prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "memory backward");
     const int scan_done = fork.mark();

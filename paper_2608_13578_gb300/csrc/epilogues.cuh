@@ -90,27 +90,6 @@ struct EpiStoreScoreF {
   }
 };
 
-// Sec. 3.5 shift: row m = b*Nb + i of M W_m becomes the memory row of block
-// i+1 of the same sequence; the last block's row is dropped.
-struct EpiShiftF {
-  using Pre = NoPre;
-  using OutT = float;
-  static constexpr bool kTma = false;  // rows move: stored directly
-  static constexpr long split_stride = 0;
-  float* out;
-  long ldo;
-  int Nb;
-  __device__ __forceinline__ void load(int, int, Pre&) const {}
-  __device__ __forceinline__ void apply(int row, int col, float* v, const Pre&, int z) const {
-    (*this)(row, col, v, 32, z);
-  }
-  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
-    if ((row % Nb) + 1 >= Nb) return;
-    float* p = out + (long)(row + 1) * ldo + col;
-    for (int j = 0; j < n; j += 4) store4(p + j, v + j);  // fp32: 16-byte stores
-  }
-};
-
 // Sec. 3.8 gate: G = sigmoid(H W_g) in the storage dtype.  The injection
 // Y = H + G * C_blk runs as its own pass once the memory rows C are ready, so
 // that this GEMM does not wait for the memory stage.

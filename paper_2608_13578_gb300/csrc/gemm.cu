@@ -124,9 +124,6 @@ static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int
                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo, (const bf16*)ea.w_p,
                                                   ea.spart, M},
                              1);
-    case EPI_SHIFT:
-      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                             EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
     case EPI_ADD:
       return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
                              EpiAddF<TI>{(const TI*)ea.add, (TI*)ea.out, ea.ldo}, 1);
@@ -947,9 +944,6 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
                                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
                                                                   (const bf16*)ea.w_p, ea.spart, M},
                                              1);
-      case EPI_SHIFT:
-        return tc_launch<BN, ST, A_MN, B_MN>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                                             EpiShiftF{(float*)ea.out, ea.ldo, ea.Nb}, 1);
       default:
         break;
     }

@@ -22,7 +22,6 @@ enum EpiKind {
   EPI_PARTIAL = 1,      // out(fp32)[z*split_stride + m*ldo + n] = acc of K-split z
   EPI_GATE = 2,         // out = G = sigmoid(acc) in the storage dtype        (Sec. 3.8)
   EPI_ADD = 3,          // out[m*ldo + n] = acc + add[m*ldo + n] (storage dtype)
-  EPI_SHIFT = 4,        // out(fp32)[m+1] = acc for row m = b*Nb + i with i+1 < Nb (Sec. 3.5 shift)
   EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
 };
 
@@ -35,8 +34,6 @@ struct EpiArgs {
   const void* w_p = nullptr;
   // EPI_ADD: the addend, same layout as out
   const void* add = nullptr;
-  // token geometry: row m = b*T + t, block blk(t) = t / L, Nb blocks, width D
-  int T = 1, L = 1, Nb = 1, D = 0;
   // EPI_GATE on the tensor cores: at most this many persistent CTAs (0: one
   // per SM), to leave SMs to a concurrent chain of small kernels
   int max_ctas = 0;
@@ -152,19 +149,24 @@ cudaError_t attn_bwd_fl(const Launch& lc, const AttnBwdArgs& a);
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
                         float* alpha, float* S, int B, int T, int D, int L);
 // Sec. 3.5: M = normalised decayed scan of S over blocks (fp32, plus a bf16
-// copy in Mb when non-null), Z its denominator [Nb, D], C[b, 0] = 0.  The
-// projection C[b, i+1] = M_i W_m is a GEMM with the EPI_SHIFT epilogue.
+// copy in Mb when non-null), Z its denominator [Nb, D].  The projection
+// P = M W_m is a K-split GEMM whose psplits fp32 partials [psplits][B*Nb][D]
+// the injection and the gate backward sum, with the shift C_0 = 0,
+// C_i = P_{i-1}, as they read them.
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D);
-// Backward of the gate and injection: dU = dY*C*G*(1-G); dP[b,i-1] = sum over
-// block i of dY*G (also in bf16 in dPb when non-null); dP[b,Nb-1] = 0.
-cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, void* dPb, int B, int T, int D, int L);
+                            void* Mb, float* Z, int B, int Nb, int D);
+// Backward of the gate and injection: dU = dY*C*G*(1-G) (C from the partials
+// Pm of P = M W_m); dP[b,i-1] = sum over block i of dY*G (also in bf16 in dPb
+// when non-null); dP[b,Nb-1] = 0.
+cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Pm,
+                     int psplits, void* dU, float* dP, void* dPb, int B, int T, int D, int L);
 // Backward of the memory scan: dS_j = sum_{i>=j} a^(i-j) dM_i / Z_i, given
-// dM = dP W_m^T; when da_part is non-null also the decay gradient of each
-// batch row, da_part [B, D] (M is the forward's fp32 memory, read only then).
-cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
-                            const float* M, float* dS, float* da_part, int B, int Nb, int D);
+// dM = dP W_m^T as msplits K-split fp32 partials [msplits][B*Nb][D]; when
+// da_part is non-null also the decay gradient of each batch row, da_part
+// [B, D] (M is the forward's fp32 memory, read only then).
+cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, const float* decay,
+                            const float* Z, const float* M, float* dS, float* da_part, int B,
+                            int Nb, int D);
 // Backward of the pooling, in chunks of 16 rows of a block (grid
 // summary_bwd_chunks(L) x Nb x B): g_t = H_t . dS_blk,
 // ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
@@ -174,9 +176,10 @@ int summary_bwd_chunks(int L);
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
                         const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
                         float* dwp_part, int B, int T, int D, int L);
-// Sec. 3.7-3.8 injection: Y = H + G * C[b, t / L].
-cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Cm,
-                   void* Y, int B, int T, int D, int L);
+// Sec. 3.7-3.8 injection: Y = H + G * C[b, t / L], C from the psplits
+// partials Pm of P = M W_m (shifted by one block, C_0 = 0).
+cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Pm,
+                   int psplits, void* Y, int B, int T, int D, int L);
 // Column sums of an fp32 [rows, cols] matrix in row order, stored in dtype_out.
 cudaError_t reduce_rows(const Launch& lc, const float* in, int rows, int cols, int dtype_out,
                         void* out);

@@ -6,6 +6,8 @@
 // before its first use, and reduces in a fixed order (deterministic).
 #include <algorithm>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -50,6 +52,47 @@ __device__ __forceinline__ void unraw(const Raw8<float>& r, float* v) {
   v[4] = r.hi.x; v[5] = r.hi.y; v[6] = r.hi.z; v[7] = r.hi.w;
 }
 __device__ __forceinline__ void unraw(const Raw8<bf16>& r, float* v) { unpack8(r.v, v); }
+
+// The memory projection P = M W_m arrives as PS K-split fp32 partials,
+// partial z of row r at Pm + z * pstride + r * D.  Sec. 3.5's shift makes the
+// memory row of block i of batch b C_i = P_{i-1} (row b*Nb + i - 1) and
+// C_0 = 0; N consecutive channels from c, all partials loaded first, then
+// summed in split order.
+template <int N, int PS>
+__device__ __forceinline__ void mem_row(const float* __restrict__ Pm, long pstride, int b, int i,
+                                        int Nb, int D, int c, float* v) {
+#pragma unroll
+  for (int e = 0; e < N; ++e) v[e] = 0.f;
+  if (i == 0) return;
+  const float* p = Pm + ((long)b * Nb + i - 1) * D + c;
+  float4 q[PS][N / 4];
+#pragma unroll
+  for (int z = 0; z < PS; ++z)
+#pragma unroll
+    for (int e = 0; e < N / 4; ++e) q[z][e] = *reinterpret_cast<const float4*>(p + z * pstride + 4 * e);
+#pragma unroll
+  for (int z = 0; z < PS; ++z)
+#pragma unroll
+    for (int e = 0; e < N / 4; ++e) {
+      v[4 * e] += q[z][e].x;
+      v[4 * e + 1] += q[z][e].y;
+      v[4 * e + 2] += q[z][e].z;
+      v[4 * e + 3] += q[z][e].w;
+    }
+}
+
+// Host: runs f(std::integral_constant<int, PS>) for the split count of the
+// memory projections (1 to 4).
+template <class F>
+cudaError_t with_splits(int psplits, F&& f) {
+  switch (psplits) {
+    case 1: return f(std::integral_constant<int, 1>());
+    case 2: return f(std::integral_constant<int, 2>());
+    case 3: return f(std::integral_constant<int, 3>());
+    case 4: return f(std::integral_constant<int, 4>());
+    default: return cudaErrorInvalidValue;
+  }
+}
 
 // Sec. 3.4: item (i, b, z): pooling scores of block i of batch b summed from
 // the npart partial dot products the W_O epilogue wrote, alpha = softmax over
@@ -130,11 +173,11 @@ __device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* _
 // the block's tokens dU = dY * C_i * G * (1 - G) (through G = sigmoid(U)),
 // and dC_i = sum_t dY_t * G_t (through Y = H + G * C_i) becomes dP[b, i-1]
 // (C_i = P_{i-1}); block 0 writes the zero row dP[b, Nb-1].
-template <class T>
+template <class T, int PS>
 __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __restrict__ G,
-                              const float* __restrict__ Cmem, T* __restrict__ dU,
-                              float* dP, bf16* dPb, int Tlen, int D, int L, int Nb, int x, int i,
-                              int b) {
+                              const float* __restrict__ Pm, long pstride,
+                              T* __restrict__ dU, float* dP, bf16* dPb, int Tlen, int D, int L,
+                              int Nb, int x, int i, int b) {
   float* part = sm;  // [8][132]
   const int rg = threadIdx.x >> 5, cq = threadIdx.x & 31;
   const int c = x * 128 + cq * 4;
@@ -142,7 +185,7 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   if (c < D) {
     float cm[4];
-    load4(Cmem + ((long)b * Nb + i) * D + c, cm);
+    mem_row<4, PS>(Pm, pstride, b, i, Nb, D, c, cm);
     // rows rg, rg+8, ... in batches of 4 (loads held packed): every load of
     // a batch is issued before its first store
     const long step = 8L * D;
@@ -199,10 +242,11 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
 // adjoint of Z, Q_i = -dM_i M_i / Z_i + a Q_{i+1}, and N_{i-1} = M_{i-1} Z_{i-1},
 //   d a = sum_{i>=1} (R_i N_{i-1} + Q_i Z_{i-1}) = sum_{i>=1} Z_{i-1} (R_i M_{i-1} + Q_i),
 // written per batch row (da_part[b, c]) and summed over b by the caller.
-__device__ void scan_bwd_item(const float* dM, const float* __restrict__ decay,
-                              const float* __restrict__ Z, const float* __restrict__ M,
-                              float* dS, float* __restrict__ da_part, int Nb, int D, int x,
-                              int b) {
+template <int PS>
+__device__ void scan_bwd_item(const float* dM, long mstride,
+                              const float* __restrict__ decay, const float* __restrict__ Z,
+                              const float* __restrict__ M, float* dS, float* __restrict__ da_part,
+                              int Nb, int D, int x, int b) {
   const int c = x * kThreads + threadIdx.x;
   if (c >= D) return;
   const float a = decay[c];
@@ -214,7 +258,12 @@ __device__ void scan_bwd_item(const float* dM, const float* __restrict__ decay,
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int i = i1 - 1 - u;
-      mv[u] = (i >= 0) ? __ldcg(dM + base + (long)i * D) : 0.f;
+      float dm[PS];  // dM from its K-split partials, loaded first, summed in split order
+#pragma unroll
+      for (int z = 0; z < PS; ++z) dm[z] = (i >= 0) ? __ldcg(dM + z * mstride + base + (long)i * D) : 0.f;
+      mv[u] = 0.f;
+#pragma unroll
+      for (int z = 0; z < PS; ++z) mv[u] += dm[z];
       zv[u] = (i >= 0) ? Z[(long)i * D + c] : 1.f;
       if (da_part) {
         mi[u] = (i >= 0) ? M[base + (long)i * D] : 0.f;
@@ -368,12 +417,11 @@ __global__ void __launch_bounds__(kThreads)
 //   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i,
 // the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j).
 // Writes M in fp32 and, when Mb is non-null, in bf16 (the A operand of the
-// tensor-core projection), Z (batch 0 only: it does not depend on b), and the
-// first block's memory row C[b, 0] = 0.
+// tensor-core projection), and Z (batch 0 only: it does not depend on b).
 __global__ void __launch_bounds__(kThreads)
     memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
-                           float* __restrict__ Cmem, int Nb, int D) {
+                           int Nb, int D) {
   pdl_enter();
   const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
   if (c >= D) return;
@@ -398,26 +446,28 @@ __global__ void __launch_bounds__(kThreads)
       }
     }
   }
-  Cmem[base] = 0.f;
 }
 
-template <class T>
+template <class T, int PS>
 __global__ void __launch_bounds__(kThreads)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
-                    const float* __restrict__ Cmem, T* __restrict__ dU, float* __restrict__ dP,
-                    bf16* __restrict__ dPb, int Tlen, int D, int L, int Nb) {
+                    const float* __restrict__ Pm, long pstride, T* __restrict__ dU,
+                    float* __restrict__ dP, bf16* __restrict__ dPb, int Tlen, int D, int L,
+                    int Nb) {
   pdl_enter();
   extern __shared__ __align__(16) float sm[];
-  gate_bwd_item<T>(sm, dY, G, Cmem, dU, dP, dPb, Tlen, D, L, Nb, blockIdx.x, blockIdx.y,
-                   blockIdx.z);
+  gate_bwd_item<T, PS>(sm, dY, G, Pm, pstride, dU, dP, dPb, Tlen, D, L, Nb, blockIdx.x,
+                   blockIdx.y, blockIdx.z);
 }
 
+template <int PS>
 __global__ void __launch_bounds__(kThreads)
-    memory_scan_bwd_kernel(const float* __restrict__ dM, const float* __restrict__ decay,
-                           const float* __restrict__ Z, const float* __restrict__ M,
-                           float* __restrict__ dS, float* __restrict__ da_part, int Nb, int D) {
+    memory_scan_bwd_kernel(const float* __restrict__ dM, long mstride,
+                           const float* __restrict__ decay, const float* __restrict__ Z,
+                           const float* __restrict__ M, float* __restrict__ dS,
+                           float* __restrict__ da_part, int Nb, int D) {
   pdl_enter();
-  scan_bwd_item(dM, decay, Z, M, dS, da_part, Nb, D, blockIdx.x, blockIdx.y);
+  scan_bwd_item<PS>(dM, mstride, decay, Z, M, dS, da_part, Nb, D, blockIdx.x, blockIdx.y);
 }
 
 template <class T>
@@ -440,45 +490,49 @@ __global__ void __launch_bounds__(kThreads, 2)
 }
 
 // Sec. 3.7-3.8: Y = H + G * C[b, t / L], the memory row of the token's block
-// broadcast by index.  Each thread takes two runs of 8 channels and issues
-// all their loads before its stores.
-template <class T>
-__global__ void __launch_bounds__(kThreads, 3)
-    inject_kernel(const T* __restrict__ Hm, const T* __restrict__ G, const float* __restrict__ Cm,
-                  T* __restrict__ Y, long n_rows, int Tlen, int D, int L, int Nb) {
+// broadcast by index.  Item (run, row group, block i, batch b): 8 channels of
+// kInjRows consecutive rows of one block, so the memory row (summed from the
+// projection's K-split partials, shifted by one block) is read once for all
+// of them; the rows' H and G loads are all issued before the first use.
+constexpr int kInjRows = 4;
+template <class T, int PS>
+__global__ void __launch_bounds__(kThreads, sizeof(T) == 2 ? 3 : 2)
+    inject_kernel(const T* __restrict__ Hm, const T* __restrict__ G, const float* __restrict__ Pm,
+                  long pstride, T* __restrict__ Y, int B, int Tlen, int D, int L, int Nb) {
   pdl_enter();
-  const int runs = D / 8;
-  const long total = n_rows * runs;
-  const long stride = (long)gridDim.x * kThreads;
-  for (long i0 = (long)blockIdx.x * kThreads + threadIdx.x; i0 < total; i0 += 2 * stride) {
-    Raw8<T> rh[2], rgt[2];
-    Raw8<float> rc[2];
-    long o[2];
-    bool live[2];
+  const int runs = D / 8, groups = (L + kInjRows - 1) / kInjRows;
+  const long total = (long)B * Nb * groups * runs;
+  for (long it = (long)blockIdx.x * kThreads + threadIdx.x; it < total;
+       it += (long)gridDim.x * kThreads) {
+    const int run = (int)(it % runs);
+    long rest = it / runs;
+    const int grp = (int)(rest % groups);
+    rest /= groups;
+    const int i = (int)(rest % Nb), b = (int)(rest / Nb);
+    const int t0 = i * L + grp * kInjRows;
+    const int nr = min(kInjRows, min((i + 1) * L, Tlen) - t0);
+    if (nr <= 0) continue;
+    const int cc = run * 8;
+    const long o0 = ((long)b * Tlen + t0) * D + cc;
+    Raw8<T> rh[kInjRows], rgt[kInjRows];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const long i = i0 + u * stride;
-      live[u] = i < total;
-      if (!live[u]) continue;
-      const long row = i / runs;
-      const int cc = (int)(i - row * runs) * 8;
-      const int b = (int)(row / Tlen), t = (int)(row - (long)b * Tlen);
-      o[u] = row * D + cc;
-      ld_raw(Hm + o[u], rh[u]);
-      ld_raw(G + o[u], rgt[u]);
-      ld_raw(Cm + ((long)b * Nb + t / L) * D + cc, rc[u]);
-    }
+    for (int r = 0; r < kInjRows; ++r)
+      if (r < nr) {
+        ld_raw(Hm + o0 + (long)r * D, rh[r]);
+        ld_raw(G + o0 + (long)r * D, rgt[r]);
+      }
+    float c[8];
+    mem_row<8, PS>(Pm, pstride, b, i, Nb, D, cc, c);
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      if (!live[u]) continue;
-      float h[8], g[8], c[8], y[8];
-      unraw(rh[u], h);
-      unraw(rgt[u], g);
-      unraw(rc[u], c);
+    for (int r = 0; r < kInjRows; ++r)
+      if (r < nr) {
+        float h[8], g[8], y[8];
+        unraw(rh[r], h);
+        unraw(rgt[r], g);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) y[e] = fmaf(g[e], c[e], h[e]);
-      store8(Y + o[u], y);
-    }
+        for (int e = 0; e < 8; ++e) y[e] = fmaf(g[e], c[e], h[e]);
+        store8(Y + o0 + (long)r * D, y);
+      }
   }
 }
 
@@ -506,32 +560,39 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 }
 
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, float* Cmem, int B, int Nb, int D) {
+                            void* Mb, float* Z, int B, int Nb, int D) {
   dim3 grid((D + kThreads - 1) / kThreads, B);
   cudaError_t e = launch_k(memory_scan_fwd_kernel, grid, dim3(kThreads), 0, lc.stream, S, decay,
-                           M, (bf16*)Mb, Z, Cmem, Nb, D);
+                           M, (bf16*)Mb, Z, Nb, D);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Cmem,
-                     void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
+cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Pm,
+                     int psplits, void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
+  const long pstride = (long)B * Nb * D;
   dim3 grid((D + 127) / 128, Nb, B);
-  cudaError_t e;
-  if (dtype == 0)
-    e = launch_k(gate_bwd_kernel<float>, grid, dim3(kThreads), kGateSmem, lc.stream,
-                 (const float*)dY, (const float*)G, Cmem, (float*)dU, dP, (bf16*)dPb, T, D, L, Nb);
-  else
-    e = launch_k(gate_bwd_kernel<bf16>, grid, dim3(kThreads), kGateSmem, lc.stream,
-                 (const bf16*)dY, (const bf16*)G, Cmem, (bf16*)dU, dP, (bf16*)dPb, T, D, L, Nb);
+  cudaError_t e = with_splits(psplits, [&](auto ps) {
+    constexpr int PS = decltype(ps)::value;
+    if (dtype == 0)
+      return launch_k(gate_bwd_kernel<float, PS>, grid, dim3(kThreads), kGateSmem, lc.stream,
+                      (const float*)dY, (const float*)G, Pm, pstride, (float*)dU, dP, (bf16*)dPb,
+                      T, D, L, Nb);
+    return launch_k(gate_bwd_kernel<bf16, PS>, grid, dim3(kThreads), kGateSmem, lc.stream,
+                    (const bf16*)dY, (const bf16*)G, Pm, pstride, (bf16*)dU, dP, (bf16*)dPb, T, D,
+                    L, Nb);
+  });
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, const float* decay, const float* Z,
-                            const float* M, float* dS, float* da_part, int B, int Nb, int D) {
+cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, const float* decay,
+                            const float* Z, const float* M, float* dS, float* da_part, int B,
+                            int Nb, int D) {
   dim3 grid((D + kThreads - 1) / kThreads, B);
-  cudaError_t e = launch_k(memory_scan_bwd_kernel, grid, dim3(kThreads), 0, lc.stream, dM, decay,
-                           Z, M, dS, da_part, Nb, D);
+  cudaError_t e = with_splits(msplits, [&](auto ms) {
+    return launch_k(memory_scan_bwd_kernel<decltype(ms)::value>, grid, dim3(kThreads), 0,
+                    lc.stream, dM, (long)B * Nb * D, decay, Z, M, dS, da_part, Nb, D);
+  });
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -553,20 +614,20 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Cm,
-                   void* Y, int B, int T, int D, int L) {
+cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Pm,
+                   int psplits, void* Y, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
-  const long n_rows = (long)B * T;
-  const long work = n_rows * (D / 8);
-  const int blocks = (int)std::max<long>(1, std::min<long>((work + 2 * kThreads - 1) / (2 * kThreads),
-                                                           1L << 16));
-  cudaError_t e;
-  if (dtype == 0)
-    e = launch_k(inject_kernel<float>, dim3(blocks), dim3(kThreads), 0, lc.stream,
-                 (const float*)Hm, (const float*)G, Cm, (float*)Y, n_rows, T, D, L, Nb);
-  else
-    e = launch_k(inject_kernel<bf16>, dim3(blocks), dim3(kThreads), 0, lc.stream,
-                 (const bf16*)Hm, (const bf16*)G, Cm, (bf16*)Y, n_rows, T, D, L, Nb);
+  const long pstride = (long)B * Nb * D;
+  const long items = (long)B * Nb * ((L + kInjRows - 1) / kInjRows) * (D / 8);
+  const int blocks = (int)std::max<long>(1, std::min<long>((items + kThreads - 1) / kThreads, 1L << 16));
+  cudaError_t e = with_splits(psplits, [&](auto ps) {
+    constexpr int PS = decltype(ps)::value;
+    if (dtype == 0)
+      return launch_k(inject_kernel<float, PS>, dim3(blocks), dim3(kThreads), 0, lc.stream,
+                      (const float*)Hm, (const float*)G, Pm, pstride, (float*)Y, B, T, D, L, Nb);
+    return launch_k(inject_kernel<bf16, PS>, dim3(blocks), dim3(kThreads), 0, lc.stream,
+                    (const bf16*)Hm, (const bf16*)G, Pm, pstride, (bf16*)Y, B, T, D, L, Nb);
+  });
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
