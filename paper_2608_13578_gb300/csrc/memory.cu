@@ -169,23 +169,27 @@ __device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* _
   __syncthreads();
 }
 
-// Sec. 3.8 reversed: item (x, i, b): 128 channels of block i of batch b.  For
-// the block's tokens dU = dY * C_i * G * (1 - G) (through G = sigmoid(U)),
+// Sec. 3.8 reversed: item (x, i, b): kGateCh channels of block i of batch b
+// (wide items: the whole backward gate fits in one wave of two CTAs per SM).
+// For the block's tokens dU = dY * C_i * G * (1 - G) (through G = sigmoid(U)),
 // and dC_i = sum_t dY_t * G_t (through Y = H + G * C_i) becomes dP[b, i-1]
 // (C_i = P_{i-1}); block 0 writes the zero row dP[b, Nb-1].
+constexpr int kGateCh = 256;
 template <class T, int PS>
 __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __restrict__ G,
                               const float* __restrict__ Pm, long pstride,
                               T* __restrict__ dU, float* dP, bf16* dPb, int Tlen, int D, int L,
                               int Nb, int x, int i, int b) {
-  float* part = sm;  // [8][132]
+  float* part = sm;  // [8][kGateCh + 4]
   const int rg = threadIdx.x >> 5, cq = threadIdx.x & 31;
-  const int c = x * 128 + cq * 4;
+  const int c = x * kGateCh + cq * 8;
   const int t0 = i * L, n = min(L, Tlen - t0);
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
   if (c < D) {
-    float cm[4];
-    mem_row<4, PS>(Pm, pstride, b, i, Nb, D, c, cm);
+    float cm[8];
+    mem_row<8, PS>(Pm, pstride, b, i, Nb, D, c, cm);
     // rows rg, rg+8, ... in batches of 4 (loads held packed): every load of
     // a batch is issued before its first store
     const long step = 8L * D;
@@ -195,7 +199,7 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
     T* dup = dU + o0;
 #pragma unroll 1
     for (int r0 = rg; r0 < n; r0 += 32, dyp += 4 * step, gp += 4 * step, dup += 4 * step) {
-      Raw4<T> rdy[4], rgt[4];
+      Raw8<T> rdy[4], rgt[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u)
         if (r0 + 8 * u < n) {
@@ -205,27 +209,27 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
 #pragma unroll
       for (int u = 0; u < 4; ++u)
         if (r0 + 8 * u < n) {
-          float dy[4], g[4], du[4];
+          float dy[8], g[8], du[8];
           unraw(rdy[u], dy);
           unraw(rgt[u], g);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
+          for (int e = 0; e < 8; ++e) {
             du[e] = dy[e] * cm[e] * g[e] * (1.0f - g[e]);
             acc[e] = fmaf(dy[e], g[e], acc[e]);
           }
-          store4(dup + u * step, du);
+          store8(dup + u * step, du);
         }
     }
   }
 #pragma unroll
-  for (int e = 0; e < 4; ++e) part[rg * 132 + cq * 4 + e] = acc[e];
+  for (int e = 0; e < 8; ++e) part[rg * (kGateCh + 4) + cq * 8 + e] = acc[e];
   __syncthreads();
-  if (threadIdx.x < 128) {
-    const int cc = x * 128 + threadIdx.x;
+  if (threadIdx.x < kGateCh) {
+    const int cc = x * kGateCh + threadIdx.x;
     if (cc < D) {
       float t = 0.f;
 #pragma unroll
-      for (int g = 0; g < 8; ++g) t += part[g * 132 + threadIdx.x];
+      for (int g = 0; g < 8; ++g) t += part[g * (kGateCh + 4) + threadIdx.x];
       const long o = (i > 0) ? ((long)b * Nb + i - 1) * D + cc : ((long)b * Nb + Nb - 1) * D + cc;
       dP[o] = (i > 0) ? t : 0.f;
       if (dPb) dPb[o] = __float2bfloat16_rn((i > 0) ? t : 0.f);
@@ -540,7 +544,7 @@ __global__ void __launch_bounds__(kThreads, sizeof(T) == 2 ? 3 : 2)
 namespace {
 // shared memory of the summary kernels: scores [kMaxL], two scalars, [8][260]
 constexpr size_t kSummarySmem = (size_t)(kMaxL + 4 + 8 * 260) * sizeof(float);
-constexpr size_t kGateSmem = (size_t)(8 * 132) * sizeof(float);
+constexpr size_t kGateSmem = (size_t)(8 * (kGateCh + 4)) * sizeof(float);
 }  // namespace
 
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
@@ -571,7 +575,7 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
                      int psplits, void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
   const long pstride = (long)B * Nb * D;
-  dim3 grid((D + 127) / 128, Nb, B);
+  dim3 grid((D + kGateCh - 1) / kGateCh, Nb, B);
   cudaError_t e = with_splits(psplits, [&](auto ps) {
     constexpr int PS = decltype(ps)::value;
     if (dtype == 0)
