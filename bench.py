@@ -373,7 +373,9 @@ def bench_ours(args):
     # from pinned host memory and its output and every gradient back out.  The
     # copies run on their own streams and overlap the previous/next step's
     # compute (double-buffered device inputs and outputs), as a training loop
-    # that streams its batches would.
+    # that streams its batches would; the compute of a step is the two C-ABI
+    # calls recorded once per buffer pair as a CUDA graph, as such a loop
+    # would record its step.
     x_h = t_cpu["x"].pin_memory()
     dy_h = t_cpu["dy"].pin_memory()
     outs_h = {"y": torch.empty_like(t_cpu["x"]).pin_memory()}
@@ -390,6 +392,24 @@ def bench_ours(args):
     ev_done = [torch.cuda.Event() for _ in range(2)]
     ev_out = [torch.cuda.Event() for _ in range(2)]
 
+    def e2e_compute(b):
+        gb = g_d[b]
+        C.bcmt_forward(p, x_d[b], None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
+                       t["w_g"], t["decay"], y_d[b], ws, None)
+        C.bcmt_backward(p, dy_d[b], x_d[b], None, None, t["w_qkv"], t["w_o"], t["w_p"],
+                        t["w_m"], t["w_g"], t["decay"], ws, sc, gb["dx"], None, None,
+                        gb["dw_qkv"], gb["dw_o"], gb["dw_p"], gb["dw_m"], gb["dw_g"], None)
+
+    e2e_graphs = []
+    for b in range(2):
+        e2e_compute(b)
+        torch.cuda.synchronize()
+        gr_b = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr_b):
+            e2e_compute(b)
+        e2e_graphs.append(gr_b)
+    torch.cuda.synchronize()
+
     def e2e_steps(k_steps):
         for i in range(k_steps):
             b = i % 2
@@ -403,11 +423,7 @@ def bench_ours(args):
             if i >= 2:
                 stream.wait_event(ev_out[b])  # step i-2's outputs are on the host
             gb = g_d[b]
-            C.bcmt_forward(p, x_d[b], None, None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
-                           t["w_g"], t["decay"], y_d[b], ws, stream)
-            C.bcmt_backward(p, dy_d[b], x_d[b], None, None, t["w_qkv"], t["w_o"], t["w_p"],
-                            t["w_m"], t["w_g"], t["decay"], ws, sc, gb["dx"], None, None,
-                            gb["dw_qkv"], gb["dw_o"], gb["dw_p"], gb["dw_m"], gb["dw_g"], stream)
+            e2e_graphs[b].replay()  # on `stream`, the current stream
             ev_done[b].record(stream)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_done[b])
