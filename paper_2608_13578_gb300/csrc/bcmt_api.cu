@@ -433,7 +433,7 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(
-        take((size_t)g.B * g.Nb * summary_bwd_chunks(g.L) * g.D * 4));
+        take((size_t)g.B * g.Nb * summary_bwd_chunks(g.L, g.D) * g.D * 4));
     w.da_part = reinterpret_cast<float*>(take((size_t)g.B * g.D * 4));
   } else {
     w.dU = w.dH = w.dPb = nullptr;
@@ -802,7 +802,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     fork.point();
     prs.begin("reduce_rows");
-    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb * summary_bwd_chunks(g.L), D, g.dtype, dw_p);
+    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb * summary_bwd_chunks(g.L, g.D), D, g.dtype, dw_p);
     prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "dW_p");
     if (d_decay) {  // fp32, summed over the batch rows in order

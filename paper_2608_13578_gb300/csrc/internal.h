@@ -167,12 +167,12 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, const float* decay,
                             const float* Z, const float* M, float* dS, float* da_part, int B,
                             int Nb, int D);
-// Backward of the pooling, in chunks of 16 rows of a block (grid
-// summary_bwd_chunks(L) x Nb x B): g_t = H_t . dS_blk,
+// Backward of the pooling, in chunks of 16 rows of a block (32 when D <= 256;
+// grid summary_bwd_chunks(L, D) x Nb x B): g_t = H_t . dS_blk,
 // ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
 // dwp_part[(b*Nb + i) * chunks + c] = sum over the chunk of ds_t H_t, and
 // dH_t += alpha_t dS_blk + ds_t w_p in place.
-int summary_bwd_chunks(int L);
+int summary_bwd_chunks(int L, int D);
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
                         const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
                         float* dwp_part, int B, int T, int D, int L);

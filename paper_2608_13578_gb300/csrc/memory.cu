@@ -292,27 +292,27 @@ __device__ void scan_bwd_item(const float* dM, long mstride,
   if (da_part) da_part[(long)b * D + c] = da;
 }
 
-// Sec. 3.4 reversed: item (c, i, b), rows 16c .. 16c+15 of block i of batch b.
+// Sec. 3.4 reversed: item (c, i, b), rows ROWS*c .. ROWS*c + ROWS-1 of block i of batch b.
 // With S_i = sum_t alpha_t H_t and alpha = softmax(s): g_t = H_t . dS_i and
 // ds_t = alpha_t (g_t - sum_u alpha_u g_u), where sum_u alpha_u g_u = S_i . dS_i
 // (the forward's block summary), so every row chunk of a block is independent.
 // The chunk's share of dW_p = sum_t ds_t H_t goes to dwp_part, and the same
 // pass completes the gradient of H in place: dH_t += alpha_t dS_i + ds_t w_p
 // (the pooling and score paths, added to dY + dU W_g^T already in dH).
-constexpr int kBwdRows = 16;
-constexpr int kBwdRowsPerWarp = kBwdRows / 8;
-template <class T>
+// ROWS rows per item: 16, or 32 at narrow widths (D <= 256), where a 16-row
+// item is too little work to cover its own latency.
+template <class T, int ROWS>
 __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
                                  const float* __restrict__ alpha, const float* __restrict__ Sb,
                                  const float* dS, const T* __restrict__ w_p, T* dH,
                                  float* __restrict__ ds_out, float* __restrict__ dwp_part,
                                  int Tlen, int D, int L, int Nb, int c, int i, int b) {
-  float* g = sm;                      // [kBwdRows]
-  float* red = sm + kBwdRows;         // [8]: per-warp partial sums of S_i . dS_i
-  float* part = sm + kBwdRows + 8;    // [8][260]
+  float* g = sm;                  // [ROWS]
+  float* red = sm + ROWS;         // [8]: per-warp partial sums of S_i . dS_i
+  float* part = sm + ROWS + 8;    // [8][260]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int blen = min(L, Tlen - i * L);
-  const int t0 = i * L + c * kBwdRows, n = min(kBwdRows, blen - c * kBwdRows);
+  const int t0 = i * L + c * ROWS, n = min(ROWS, blen - c * ROWS);
   const T* Hb = Hm + ((long)b * Tlen + t0) * D;
   const float* dSi = dS + ((long)b * Nb + i) * D;
   const float* Si = Sb + ((long)b * Nb + i) * D;
@@ -324,7 +324,7 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   if (lane == 0) red[warp] = cp;
   // g_t = H_t . dS_i: warp w takes rows w, w+8; all the loads of a
   // 256-channel chunk for its rows go out together
-  constexpr int RW = kBwdRowsPerWarp;
+  constexpr int RW = ROWS / 8;
   {
     float d[RW];
 #pragma unroll
@@ -363,7 +363,7 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   __syncthreads();
   const int rg = warp, co = lane;
   T* dHb = dH + ((long)b * Tlen + t0) * D;
-  const long prow = ((long)b * Nb + i) * ((L + kBwdRows - 1) / kBwdRows) + c;
+  const long prow = ((long)b * Nb + i) * ((L + ROWS - 1) / ROWS) + c;
   for (int c0 = 0; c0 < D; c0 += 256) {
     const int k = c0 + co * 8;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -474,23 +474,23 @@ __global__ void __launch_bounds__(kThreads)
   scan_bwd_item<PS>(dM, mstride, decay, Z, M, dS, da_part, Nb, D, blockIdx.x, blockIdx.y);
 }
 
-template <class T>
+template <class T, int ROWS>
 __global__ void __launch_bounds__(kThreads, 2)
     summary_bwd_kernel(const T* __restrict__ Hm, const float* __restrict__ alpha,
                        const float* __restrict__ Sb, const float* __restrict__ dS,
                        const T* __restrict__ w_p, T* dH, float* __restrict__ ds,
                        float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
   pdl_enter();
-  __shared__ __align__(16) float sm[kBwdRows + 8 + 8 * 260];
+  __shared__ __align__(16) float sm[ROWS + 8 + 8 * 260];
   // a ragged last block has fewer chunks than the grid's x extent: its empty
   // chunks contribute zero partials to dW_p
-  if ((int)blockIdx.x * kBwdRows >= min(L, Tlen - (int)blockIdx.y * L)) {
+  if ((int)blockIdx.x * ROWS >= min(L, Tlen - (int)blockIdx.y * L)) {
     const long prow = ((long)blockIdx.z * Nb + blockIdx.y) * gridDim.x + blockIdx.x;
     for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
     return;
   }
-  summary_bwd_item<T>(sm, Hm, alpha, Sb, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb, blockIdx.x,
-                      blockIdx.y, blockIdx.z);
+  summary_bwd_item<T, ROWS>(sm, Hm, alpha, Sb, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb,
+                            blockIdx.x, blockIdx.y, blockIdx.z);
 }
 
 // Sec. 3.7-3.8: Y = H + G * C[b, t / L], the memory row of the token's block
@@ -600,21 +600,30 @@ cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, cons
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-int summary_bwd_chunks(int L) { return (L + kBwdRows - 1) / kBwdRows; }
+static int summary_bwd_rows(int D) { return D <= 256 ? 32 : 16; }
+int summary_bwd_chunks(int L, int D) {
+  const int rows = summary_bwd_rows(D);
+  return (L + rows - 1) / rows;
+}
 
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
                         const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
                         float* dwp_part, int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
-  dim3 grid(summary_bwd_chunks(L), Nb, B);
-  cudaError_t e;
-  if (dtype == 0)
-    e = launch_k(summary_bwd_kernel<float>, grid, dim3(kThreads), 0, lc.stream, (const float*)Hm,
-                 alpha, Sb, dS, (const float*)w_p, (float*)dH, ds, dwp_part, T, D, L, Nb);
-  else
-    e = launch_k(summary_bwd_kernel<bf16>, grid, dim3(kThreads), 0, lc.stream, (const bf16*)Hm,
-                 alpha, Sb, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T, D, L, Nb);
+  dim3 grid(summary_bwd_chunks(L, D), Nb, B);
+  auto go = [&](auto rows) {
+    constexpr int R = decltype(rows)::value;
+    if (dtype == 0)
+      return launch_k(summary_bwd_kernel<float, R>, grid, dim3(kThreads), 0, lc.stream,
+                      (const float*)Hm, alpha, Sb, dS, (const float*)w_p, (float*)dH, ds,
+                      dwp_part, T, D, L, Nb);
+    return launch_k(summary_bwd_kernel<bf16, R>, grid, dim3(kThreads), 0, lc.stream,
+                    (const bf16*)Hm, alpha, Sb, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T,
+                    D, L, Nb);
+  };
+  cudaError_t e = summary_bwd_rows(D) == 32 ? go(std::integral_constant<int, 32>())
+                                            : go(std::integral_constant<int, 16>());
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
