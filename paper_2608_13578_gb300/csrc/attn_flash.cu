@@ -21,7 +21,8 @@
 //           S, dP (N = 64), dS = P (dP - Drow) scale, dQ += dS K (TMEM);
 //      dKV: per key tile, per query tile and 64-query half S^T = K Q^T,
 //           dP^T = V dO^T, dV += P^T dO, dK += dS^T Q (TMEM), with the query
-//           tile's log-sum-exp and Drow staged in shared memory.
+//           tile's log-sum-exp and Drow staged in shared memory; the second
+//           half's S^T and dP^T are issued ahead of the first half's dV/dK.
 #include "attn_common.cuh"
 #include "common.cuh"
 #include "internal.h"
@@ -542,20 +543,23 @@ __global__ void __launch_bounds__(128)
       tc::fence_after_sync();
     }
     __syncthreads();  // slse / sdr written
-    for (int hh = 0; hh < 2; ++hh) {
-      if (tid == 0) {
-        if (ok) {
-          constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
+    // S^T and dP^T of query half hh -> TMEM columns 0..127 (tid 0)
+    auto issue_scores = [&](int hh) {
+      if (ok) {
+        constexpr uint32_t id64 = tc::idesc_bf16(128, 64, 0, 0);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk)  // S^T half -> columns 0..63
-            tc::mma_bf16(tmem, G::kmaj(sK, 0, kk), G::kmaj(sQ, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < DH / 16; ++kk)  // S^T half -> columns 0..63
+          tc::mma_bf16(tmem, G::kmaj(sK, 0, kk), G::kmaj(sQ, 64 * hh, kk), id64, kk > 0 ? 1u : 0u);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk)  // dP^T half -> columns 64..127
-            tc::mma_bf16(tmem + 64, G::kmaj(sV, 0, kk), G::kmaj(sdO, 64 * hh, kk), id64,
-                         kk > 0 ? 1u : 0u);
-        }
-        tc::mma_commit(&bar[1]);
+        for (int kk = 0; kk < DH / 16; ++kk)  // dP^T half -> columns 64..127
+          tc::mma_bf16(tmem + 64, G::kmaj(sV, 0, kk), G::kmaj(sdO, 64 * hh, kk), id64,
+                       kk > 0 ? 1u : 0u);
       }
+      tc::mma_commit(&bar[1]);
+    };
+    for (int hh = 0; hh < 2; ++hh) {
+      // half 1's products were issued with half 0's dV/dK (below), ahead of them
+      if (tid == 0 && hh == 0) issue_scores(0);
       __syncwarp();
       ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
       ++ns;
@@ -603,6 +607,10 @@ __global__ void __launch_bounds__(128)
       __syncthreads();
       if (tid == 0) {
         tc::fence_after_sync();
+        // every thread has read this half's scores out of TMEM (the barrier
+        // above): the next half's products go first, under this half's dV/dK
+        // and the next elementwise pass
+        if (hh == 0) issue_scores(1);
         if (ok) {
           constexpr uint32_t idKV = tc::idesc_bf16(128, DH, 0, 1);
           const uint32_t acc0 = (qt > 0 || hh > 0) ? 1u : 0u;
