@@ -19,7 +19,9 @@ extern "C" {
 /* Selects the kernels bcmt_forward / bcmt_backward use from now on in this
  * process: gemm_on / attn_on = 1 for the tcgen05 tensor-core kernels (the
  * default), 0 for the SIMT kernels.  Returns a bit mask of what this GPU and
- * build support: bit 0 the tcgen05 GEMM, bit 1 the tcgen05 attention. */
+ * build support: bit 0 the tcgen05 GEMM, bit 1 the tcgen05 attention.  The
+ * sizes bcmt_workspace_size and bcmt_scratch_size report depend on this
+ * choice (the K-split layouts differ): query them after calling it. */
 int bcmt_test_set_tensor_cores(int gemm_on, int attn_on);
 
 /* C[M,N] = A[M,K] B[K,N] with fp32 accumulation, element (m,k) of A at
