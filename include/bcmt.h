@@ -33,9 +33,12 @@
  *  - Pointers must be 16-byte aligned.  Requirements on shapes: B, T >= 1;
  *    H >= 1 and D % H == 0; dh = D / H a multiple of 8 and <= 128; D a
  *    multiple of 64; 1 <= L <= 1024.  Any T is accepted: the last block may be
- *    ragged (Sec. 3.2).  bf16 shapes with dh == 64 and L a power of two in
- *    [16, 128] run the tcgen05 tensor-core attention; other valid shapes run a
- *    SIMT attention kernel.
+ *    ragged (Sec. 3.2).  bf16 shapes with dh in {16, 32, 64} run the tcgen05
+ *    tensor-core attention: L in {16, 32, 64, 128} on the single-tile kernels
+ *    (a 128-token tile holds whole blocks), L a multiple of 128 from 256 to
+ *    1024 on the key-tile-walking kernels (an online softmax over the block's
+ *    128-token key tiles).  fp32 shapes, other head widths and the remaining
+ *    block sizes run a SIMT attention kernel in fp32.
  *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls are
  *    asynchronous: they validate their arguments, enqueue kernels and return.
  *    On invalid arguments nothing is launched and an error code is returned;

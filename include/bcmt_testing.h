@@ -68,6 +68,16 @@ int bcmt_test_attn(int impl, int backward, const bcmt_params* p, const void* q, 
                    const void* v, long ld, void* o, float* lse, const void* dO, float* drow,
                    void* dq, void* dk, void* dv, long ld_d, void* stream);
 
+/* Failure detection without a fault: launches one single-thread CTA that
+ * waits on an mbarrier nothing ever arrives at, with the library's bounded
+ * wait cut to `cycles` SM clock cycles (1 <= cycles <= 2^31).  The wait
+ * expires, the kernel sets the timeout bit of the device status word and
+ * returns normally; bcmt_device_status() then reports BCMT_ERR_TIMEOUT (and
+ * clears the word).  The kernel issues no TMA copy or tcgen05 operation and
+ * holds no TMEM, so the context stays usable.  Returns 0, or -1 on a bad
+ * argument or launch error (bcmt_last_error()). */
+int bcmt_test_wait_expiry(long long cycles, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -94,6 +94,8 @@ def _load():
     lib.bcmt_test_attn.argtypes = [ctypes.c_int, ctypes.c_int, _P, _VP, _VP, _VP, ctypes.c_long,
                                    _VP, _VP, _VP, _VP, _VP, _VP, _VP, ctypes.c_long, _VP]
     lib.bcmt_test_attn.restype = ctypes.c_int
+    lib.bcmt_test_wait_expiry.argtypes = [ctypes.c_longlong, _VP]
+    lib.bcmt_test_wait_expiry.restype = ctypes.c_int
     return lib
 
 
@@ -104,7 +106,8 @@ EXPORTED = ("bcmt_workspace_size", "bcmt_scratch_size", "bcmt_forward", "bcmt_ba
             "bcmt_device_status", "bcmt_last_error", "bcmt_profile_read", "bcmt_profile_reset",
             "bcmt_attention_backward_noalloc",
             "bcmt_decode_state_size", "bcmt_decode_reset", "bcmt_decode_step",
-            "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_gemm_group", "bcmt_test_attn")
+            "bcmt_test_set_tensor_cores", "bcmt_test_gemm", "bcmt_test_gemm_group", "bcmt_test_attn",
+            "bcmt_test_wait_expiry")
 
 
 def _ptr(t) -> Optional[int]:
@@ -232,4 +235,11 @@ def bcmt_test_attn(impl, backward, p: bcmt_params, q, k, v, ld, o, lse, dO=None,
                            _ptr(lse), _ptr(dO), _ptr(drow), _ptr(dq), _ptr(dk), _ptr(dv), ld_d,
                            _stream(stream))
     if r != 0:
+        raise BCMTError(BCMT_ERR_CUDA, bcmt_last_error())
+
+
+def bcmt_test_wait_expiry(cycles: int, stream=None) -> None:
+    """Launches a wait that nothing ends, bounded by ``cycles`` SM clock
+    cycles; afterwards bcmt_device_status() reports BCMT_ERR_TIMEOUT."""
+    if LIB.bcmt_test_wait_expiry(cycles, _stream(stream)) != 0:
         raise BCMTError(BCMT_ERR_CUDA, bcmt_last_error())

@@ -16,6 +16,7 @@
 #include "../../include/bcmt_testing.h"
 #include "common.cuh"
 #include "internal.h"
+#include "tc.cuh"
 
 namespace bcmt {
 
@@ -53,18 +54,20 @@ unsigned* status_ptr() {
   return per_dev[dev];
 }
 
-// A second stream per device for the weight gradients of the backward pass,
-// which no later step of the pass reads: they run beside the dependent chain
-// (forked and joined with events, so the pair can also be captured into a
-// CUDA graph).  Streams and events are host-side objects: no device memory.
+// Side streams per device for work that runs beside the layer's critical
+// chain (the memory gradient and the small weight gradients of the backward
+// pass): forked from and joined back into the caller's stream with events,
+// so the branches can also be captured into a CUDA graph.  The critical chain
+// itself stays on the caller's stream, so that consecutive calls (forward,
+// then backward) chain by programmatic dependent launch; its launches carry
+// the device's highest stream priority as a launch attribute, the side
+// streams the lowest, so that when both have CTAs waiting the block scheduler
+// places the critical ones first.  Streams and events are host-side objects:
+// no device memory.
 constexpr int kSideEvents = 16;
-// Per device: the layer's critical path runs on `crit` (the highest stream
-// priority) and the work beside it (memory stage in the forward, weight
-// gradients in the backward) on `side` (the lowest), so that when both have
-// CTAs waiting the block scheduler places the critical ones first.  `side2`
-// (also lowest) takes work that must not hold up what is queued on `side`.
 struct SideStream {
-  cudaStream_t crit = nullptr, side = nullptr, side2 = nullptr;
+  cudaStream_t side = nullptr, side2 = nullptr;
+  int greatest = 0;  // the device's highest stream priority
   cudaEvent_t ev[kSideEvents] = {};
   std::mutex mu;  // one call at a time may use the streams' events
 };
@@ -80,10 +83,9 @@ SideStream* side_stream() {
     SideStream* ss = new SideStream();
     int least = 0, greatest = 0;
     bool ok = cudaDeviceGetStreamPriorityRange(&least, &greatest) == cudaSuccess &&
-              cudaStreamCreateWithPriority(&ss->crit, cudaStreamNonBlocking, greatest) ==
-                  cudaSuccess &&
               cudaStreamCreateWithPriority(&ss->side, cudaStreamNonBlocking, least) == cudaSuccess &&
               cudaStreamCreateWithPriority(&ss->side2, cudaStreamNonBlocking, least) == cudaSuccess;
+    ss->greatest = greatest;
     for (int i = 0; i < kSideEvents && ok; ++i)
       ok = cudaEventCreateWithFlags(&ss->ev[i], cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
@@ -95,31 +97,31 @@ SideStream* side_stream() {
   return per_dev[dev];
 }
 
-// Fork/join of one call: the critical stream starts after everything the
-// caller has enqueued, the side stream forks from it at point(), and on
-// destruction (every return path) both are joined back into the caller's
-// stream.  Plain event record/wait, so a CUDA graph capture of the caller's
-// stream captures all three.  Without a SideStream everything stays on the
-// caller's stream.
+// Fork/join of one call: the critical chain runs on the caller's stream at
+// the highest priority; the side streams fork from it at point() / point2(),
+// and on destruction (every return path) they are joined back into it.
+// Plain event record/wait, so a CUDA graph capture of the caller's stream
+// captures every branch.  Without a SideStream everything stays on the
+// caller's stream at its own priority.
 struct Fork {
   SideStream* ss;
   cudaStream_t user;
   int next = 0;
   bool forked = false, forked2 = false;
+  PriorityOverride saved;
   Fork(SideStream* s, cudaStream_t u) : ss(s), user(u) {
     if (!ss) return;
     ss->mu.lock();
-    cudaEventRecord(ss->ev[next], user);
-    cudaStreamWaitEvent(ss->crit, ss->ev[next], 0);
-    ++next;
+    saved = priority_override();
+    priority_override() = PriorityOverride{true, user, ss->greatest};
   }
-  cudaStream_t main() const { return ss ? ss->crit : user; }
+  cudaStream_t main() const { return user; }
   cudaStream_t side() const { return ss ? ss->side : user; }
   cudaStream_t side2() const { return ss ? ss->side2 : user; }
-  // the side stream waits for everything enqueued on the critical stream so far
+  // the side stream waits for everything enqueued on the critical chain so far
   bool point() {
     if (!ss || next >= kSideEvents - 3) return false;
-    cudaEventRecord(ss->ev[next], ss->crit);
+    cudaEventRecord(ss->ev[next], user);
     cudaStreamWaitEvent(ss->side, ss->ev[next], 0);
     ++next;
     forked = true;
@@ -128,34 +130,33 @@ struct Fork {
   // the same for the second side stream
   bool point2() {
     if (!ss || next >= kSideEvents - 3) return false;
-    cudaEventRecord(ss->ev[next], ss->crit);
+    cudaEventRecord(ss->ev[next], user);
     cudaStreamWaitEvent(ss->side2, ss->ev[next], 0);
     ++next;
     forked2 = true;
     return true;
   }
   // records what the side stream has been given so far; wait_mark(m) later
-  // makes the critical stream wait for exactly that
+  // makes the critical chain wait for exactly that
   int mark() {
     if (!ss || !forked || next >= kSideEvents - 3) return -1;
     cudaEventRecord(ss->ev[next], ss->side);
     return next++;
   }
   void wait_mark(int m) {
-    if (ss && m >= 0) cudaStreamWaitEvent(ss->crit, ss->ev[m], 0);
+    if (ss && m >= 0) cudaStreamWaitEvent(user, ss->ev[m], 0);
   }
   ~Fork() {
     if (!ss) return;
     if (forked2) {
       cudaEventRecord(ss->ev[kSideEvents - 3], ss->side2);
-      cudaStreamWaitEvent(ss->crit, ss->ev[kSideEvents - 3], 0);
+      cudaStreamWaitEvent(user, ss->ev[kSideEvents - 3], 0);
     }
     if (forked) {
       cudaEventRecord(ss->ev[kSideEvents - 2], ss->side);
-      cudaStreamWaitEvent(ss->crit, ss->ev[kSideEvents - 2], 0);
+      cudaStreamWaitEvent(user, ss->ev[kSideEvents - 2], 0);
     }
-    cudaEventRecord(ss->ev[kSideEvents - 1], ss->crit);
-    cudaStreamWaitEvent(user, ss->ev[kSideEvents - 1], 0);
+    priority_override() = saved;
     ss->mu.unlock();
   }
 };
@@ -301,57 +302,58 @@ bool tail_grouped(const Geometry& g) {
   return g.from_x && dw_pair(g.dtype, g.D, 3 * g.D) && gemm_tc_available() && g.n >= 256;
 }
 // K splits of the weight gradients in that launch (in launch order: dW_QKV,
-// dW_g, dW_O; 0 = absent): the counts whose round-robin deal of dX's tiles,
-// then each gradient's items, over the SM pairs, followed by the reduction of
-// the partials, finishes first.  Unit: one 64-deep K slice of a 256 x 256
-// tile (8.4 MFLOP, about 0.45 us on a pair); each item costs its slices plus
-// 4 (pipeline fill and epilogue), and each split of an M x N product adds the
-// reduction's reading of M*N fp32 partials at about 3 MB per unit.  Up to 16
-// splits each; ties go to fewer splits.  Cached per shape: the search runs once.
+// dW_g, dW_O; 0 = absent): the counts for which the launch, scheduled longest
+// item first onto the least loaded SM pair (gemm_tc_pair_group), followed by
+// the reduction of the partials, finishes first.  Unit: one 64-deep K slice
+// of a 256 x 256 tile (8.4 MFLOP, about 0.45 us on a pair); each item costs
+// its slices plus a fixed overhead for pipeline fill and epilogue, and each
+// split of an M x N product adds the reduction's reading of M*N fp32
+// partials at about 3 MB per unit.  Up to 16 splits each; ties go to fewer
+// splits.  Cached per shape: the search runs once.
 struct TailPlan {
   int s[3] = {1, 0, 0};
 };
 TailPlan tail_plan(const Geometry& g) {
   const int pairs = std::max(1, device_sms() / 2);
-  const long D = g.D, tiles0 = ((g.n + 255) / 256) * (D / 256);
-  const int nk0 = (int)((3 * D + 63) / 64), nkb = (int)((g.n + 63) / 64);
-  const long tiles[3] = {(D / 256) * (3 * D / 256), g.honly ? 0 : (D / 256) * (D / 256),
-                         (D / 256) * (D / 256)};
+  const int D = g.D, n = (int)g.n;
+  const int nkb = (int)((g.n + 63) / 64);
+  const bool gate = !g.honly;
   const double out_units[3] = {3.0 * D * D * 4.0 / 3.0e6, (double)D * D * 4.0 / 3.0e6,
                                (double)D * D * 4.0 / 3.0e6};
   static std::mutex mu;
   static std::vector<std::pair<std::array<long, 4>, TailPlan>> cache;
-  const std::array<long, 4> key{pairs, (long)g.n, D, (long)g.honly};
+  const std::array<long, 4> key{pairs, (long)g.n, (long)D, (long)g.honly};
   std::lock_guard<std::mutex> lock(mu);
   for (const auto& c : cache)
     if (c.first == key) return c.second;
   const int smax = std::min(16, std::max(1, nkb / 8));
-  TailPlan best, cur;
+  TailPlan best;
   double best_t = -1.0;
-  std::vector<long> load((size_t)pairs);
   for (int a = 1; a <= smax; ++a)
-    for (int b = tiles[1] ? 1 : 0; b <= (tiles[1] ? smax : 0); ++b)
+    for (int b = gate ? 1 : 0; b <= (gate ? smax : 0); ++b)
       for (int c = 1; c <= smax; ++c) {
-        cur.s[0] = a;
-        cur.s[1] = b;
-        cur.s[2] = c;
-        std::fill(load.begin(), load.end(), 0L);
-        long item = 0;
-        for (long t = 0; t < tiles0; ++t, ++item) load[(size_t)(item % pairs)] += nk0 + 4;
+        // the weight products in launch order (dW_QKV, dW_g when present, dW_O)
+        int Mw[3], Nw[3], Kw[3], sw[3], nw = 0;
+        const int sp[3] = {a, b, c};
+        const int Ns[3] = {3 * D, D, D};
         double red = 0.0;
         for (int w = 0; w < 3; ++w) {
-          if (!tiles[w]) continue;
-          const int kps = (nkb + cur.s[w] - 1) / cur.s[w], se = (nkb + kps - 1) / kps;
-          for (long t = 0; t < tiles[w] * se; ++t, ++item) {  // split index slowest
-            const int z = (int)(t / tiles[w]);
-            load[(size_t)(item % pairs)] += std::min(nkb, (z + 1) * kps) - z * kps + 4;
-          }
-          red += se * out_units[w];
+          if (w == 1 && !gate) continue;
+          Mw[nw] = D;
+          Nw[nw] = Ns[w];
+          Kw[nw] = n;
+          sw[nw] = sp[w];
+          red += effective_splits(n, sp[w]) * out_units[w];
+          ++nw;
         }
-        const double t_end = (double)*std::max_element(load.begin(), load.end()) + red;
+        const long ms = tc2_group_makespan(n, D, 3 * D, Mw, Nw, Kw, sw, nw, pairs);
+        if (ms < 0) continue;
+        const double t_end = (double)ms + red;
         if (best_t < 0 || t_end < best_t) {
           best_t = t_end;
-          best = cur;
+          best.s[0] = a;
+          best.s[1] = b;
+          best.s[2] = c;
         }
       }
   cache.emplace_back(key, best);
@@ -433,7 +435,7 @@ BwdWs bwd_layout(const Geometry& g, void* base) {
     w.dS = reinterpret_cast<float*>(take((size_t)g.B * g.Nb * g.D * 4));
     w.ds = reinterpret_cast<float*>(take((size_t)g.n * 4));
     w.dwp_part = reinterpret_cast<float*>(
-        take((size_t)g.B * g.Nb * summary_bwd_chunks(g.L, g.D) * g.D * 4));
+        take((size_t)g.B * g.Nb * summary_bwd_chunks(g.dtype, g.L, g.D) * g.D * 4));
     w.da_part = reinterpret_cast<float*>(take((size_t)g.B * g.D * 4));
   } else {
     w.dU = w.dH = w.dPb = nullptr;
@@ -522,6 +524,18 @@ bcmt_status finish(const bcmt_params* p, cudaStream_t s) {
   if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
   if (p->flags & BCMT_FLAG_CHECK) return bcmt_device_status(s);
   return BCMT_OK;
+}
+
+// A wait that cannot end, bounded by `cap` SM clock cycles: one thread
+// initialises an mbarrier for one arrival and waits for its first phase, which
+// nothing completes.  The bounded wait expires, ORs kStatusTimeout into the
+// status word and returns; the kernel holds no TMA copy, no tcgen05 operation
+// and no TMEM, so it leaves nothing behind.
+__global__ void wait_expiry_kernel(unsigned* status, long long cap) {
+  __shared__ __align__(8) uint64_t bar;
+  tc::mbar_init(&bar, 1);
+  tc::fence_mbar_init();
+  tc::mbar_wait(&bar, 0, status, cap);
 }
 
 }  // namespace
@@ -643,21 +657,20 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // side stream: Sec. 3.8 gate G = sigmoid(H W_g), independent of the memory
-    fork.point();
+    // Sec. 3.8 gate G = sigmoid(H W_g) on all SMs, then the memory chain: one
+    // stream of kernels chained by programmatic dependent launch.  (Beside the
+    // chain on half of the SMs the gate GEMM slowed the chain's kernels about
+    // twofold, and each join of two streams left a launch gap of several us.)
     {
       EpiArgs ea;
       ea.out = w.G;
       ea.ldo = D;
-      ea.max_ctas = device_sms() / 2;  // half the SMs stay with the memory chain
-      e = run_gemm(lcs, prs, "gemm_gate", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
+      e = run_gemm(lc, pr, "gemm_gate", g.dtype, g.dtype, n, D, D, w.hloc, D, 1, w_g, D, 1,
                    EPI_GATE, ea);
       if (e != cudaSuccess) return cuda_fail(e, "gate");
     }
-    const int gate_done = fork.mark();
-    // critical stream, meanwhile: Sec. 3.4 adaptive block summaries, Sec. 3.5
-    // exponential causal memory (scan), then its projection and one-block
-    // shift -> C (a chain of small kernels: the longer of the two paths)
+    // Sec. 3.4 adaptive block summaries, Sec. 3.5 exponential causal memory
+    // (scan), then its projection and one-block shift -> C
     pr.begin("summary_fwd");
     e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
     pr.end(nullptr);
@@ -677,8 +690,7 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
                    EPI_PARTIAL, ea, mem_splits(g));
       if (e != cudaSuccess) return cuda_fail(e, "memory projection");
     }
-    // Sec. 3.7-3.8: Y = H + G * M_tokens once the gate is ready too
-    fork.wait_mark(gate_done);
+    // Sec. 3.7-3.8: Y = H + G * M_tokens
     pr.begin("inject");
     e = inject(lc, g.dtype, w.hloc, w.G, w.C, mem_splits(g), y, g.B, g.T, D, g.L);
     pr.end(nullptr);
@@ -802,7 +814,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     fork.point();
     prs.begin("reduce_rows");
-    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb * summary_bwd_chunks(g.L, g.D), D, g.dtype, dw_p);
+    e = reduce_rows(lcs, bw.dwp_part, g.B * g.Nb * summary_bwd_chunks(g.dtype, g.L, g.D), D, g.dtype, dw_p);
     prs.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "dW_p");
     if (d_decay) {  // fp32, summed over the batch rows in order
@@ -1096,6 +1108,26 @@ int bcmt_test_set_tensor_cores(int gemm_on, int attn_on) {
   g_use_tc_gemm = gemm_on != 0;
   g_use_tc_attn = attn_on != 0;
   return (gemm_tc_available() ? 1 : 0) | (attn_tc_supported(1, 64, 64) ? 2 : 0);
+}
+
+int bcmt_test_wait_expiry(long long cycles, void* stream) {
+  if (cycles < 1 || cycles > tc::kWaitCycles) {
+    fail(BCMT_ERR_ARG, "cycles = %lld must be in [1, %lld]", cycles, tc::kWaitCycles);
+    return -1;
+  }
+  unsigned* sp = status_ptr();
+  if (!sp) {
+    fail(BCMT_ERR_CUDA, "device status word unavailable");
+    return -1;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  wait_expiry_kernel<<<1, 1, 0, s>>>(sp, cycles);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    fail(BCMT_ERR_CUDA, "wait expiry kernel: %s", cudaGetErrorString(e));
+    return -1;
+  }
+  return 0;
 }
 
 int bcmt_test_gemm(int impl, int dtype, int dtype_out, int M, int N, int K, const void* A, long sam,

@@ -33,8 +33,28 @@ __device__ __forceinline__ void pdl_enter() {
   pdl_wait();
 }
 
+// Host: while `on`, this thread's launches on `stream` carry `priority`
+// instead of the stream's own (the C-ABI calls raise their critical chain,
+// which runs on the caller's stream, above the work they put beside it).
+struct PriorityOverride {
+  bool on = false;
+  cudaStream_t stream = nullptr;
+  int priority = 0;
+};
+inline PriorityOverride& priority_override() {
+  static thread_local PriorityOverride p;
+  return p;
+}
+inline int launch_priority(cudaStream_t stream) {
+  const PriorityOverride& o = priority_override();
+  if (o.on && o.stream == stream) return o.priority;
+  int prio = 0;
+  if (cudaStreamGetPriority(stream, &prio) != cudaSuccess) prio = 0;
+  return prio;
+}
+
 // Host: launches `kernel` on `stream` with programmatic stream serialisation
-// and the stream's priority as the launch priority (so that the priority is
+// and launch_priority(stream) as the launch priority (so that the priority is
 // kept when the launch is captured into a CUDA graph).
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
@@ -44,8 +64,7 @@ inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, siz
   cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  int prio = 0;
-  if (cudaStreamGetPriority(stream, &prio) != cudaSuccess) prio = 0;
+  const int prio = launch_priority(stream);
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -81,8 +100,7 @@ inline cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 bl
   cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  int prio = 0;
-  if (cudaStreamGetPriority(stream, &prio) != cudaSuccess) prio = 0;
+  const int prio = launch_priority(stream);
   cudaLaunchAttribute attr[3];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;

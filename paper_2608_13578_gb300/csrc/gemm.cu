@@ -4,16 +4,19 @@
 //  * gemm_tc: bf16 inputs on the tcgen05 tensor cores.  One CTA computes a
 //    128 x BN output tile with the fp32 accumulator in TMEM.  Warp 0 (one lane)
 //    streams 64-deep K slices of A and B into a STAGES-deep shared-memory ring
-//    with TMA (128-byte swizzle); warp 1 (one lane) issues tcgen05.mma and
-//    releases each slot with tcgen05.commit; then all four warps read the
-//    accumulator back with tcgen05.ld (thread = output row) and run the fused
-//    epilogue.  Every mbarrier wait is bounded.
+//    with TMA (128-byte swizzle); warp 1 (one lane) issues tcgen05.mma into
+//    one of two TMEM accumulators and releases each slot with tcgen05.commit;
+//    warps 2-9 (two per TMEM lane quarter, each half of the tile's columns)
+//    read the other accumulator back with tcgen05.ld (thread = output row) and
+//    run the fused epilogue.  Every mbarrier wait is bounded.
 //  * gemm_simt: true-fp32 FMA, used for fp32 tensors (a TF32 tensor-core
 //    product cannot meet a 1e-4 absolute error bound).
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <type_traits>
+#include <vector>
 
 #include "common.cuh"
 #include "epilogues.cuh"
@@ -530,8 +533,13 @@ struct Tc2Shape {
 };
 
 constexpr int kTc2Max = 4;
+// A group's explicit schedule holds at most this many pairs and items.
+constexpr int kTc2SchedPairs = 128;
+constexpr int kTc2SchedItems = 512;
 // Kernel parameter block of a group: tensor maps (A, B, output) and shape of
-// each product, the epilogues, and the number of products.
+// each product, the epilogues, the number of products, and optionally the
+// items of each pair: pair p takes items list[start[p] .. start[p+1]) of the
+// combined numbering, in that order (npairs_sched == 0: round-robin).
 template <class Op0, class Op1>
 struct Tc2Params {
   CUtensorMap map[kTc2Max][3];
@@ -539,6 +547,9 @@ struct Tc2Params {
   typename Op0::Epi epi0;
   typename Op1::Epi epi1[kTc2Max - 1];
   int count;
+  int npairs_sched;
+  uint16_t start[kTc2SchedPairs + 1];
+  uint16_t list[kTc2SchedItems];
 };
 
 // TMA producer, one tile (both CTAs): this CTA's rows of A and half of B.
@@ -674,6 +685,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   int total = 0;
   for (int q = 0; q < P.count; ++q) total += P.shape[q].n_tiles;
+  // this pair's items: its list of the schedule, or every npairs-th item
+  const int nmine = P.npairs_sched ? (int)P.start[pair + 1] - (int)P.start[pair]
+                                   : (pair < total ? (total - 1 - pair) / npairs + 1 : 0);
+  auto item_at = [&](int r) {
+    return P.npairs_sched ? (int)P.list[P.start[pair] + r] : pair + r * npairs;
+  };
   // product of a combined item index; *tile becomes the tile within it
   auto which = [&](int item, int* tile) {
     int q = 0;
@@ -711,9 +728,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       int it = 0;
-      for (int item = pair; item < total; item += npairs) {
+      for (int r = 0; r < nmine; ++r) {
         int tile;
-        const int q = which(item, &tile);
+        const int q = which(item_at(r), &tile);
         bool ok;
         if (kSame || q > 0)
           ok = tc2_produce<Op1, Cfg, BN, STAGES>(&P.map[q][0], &P.map[q][1], P.shape[q], tile, rank,
@@ -726,10 +743,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
-      int it = 0, j = 0;
-      for (int item = pair; item < total; item += npairs, ++j) {
+      int it = 0;
+      for (int j = 0; j < nmine; ++j) {
         int tile;
-        const int q = which(item, &tile);
+        const int q = which(item_at(j), &tile);
         bool ok;
         if (kSame || q > 0)
           ok = tc2_mma<Op1, Cfg, BN, STAGES, ACC>(P.shape[q], tile, j, tmem, smem, full, empty,
@@ -743,19 +760,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else {
     const uint32_t te0 = tc::mapa(tc::smem_u32(&tempty[0]), 0);
     uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
-    int j = 0, nout = 0, prev = -1;
-    for (int item = pair; item < total; item += npairs, ++j) {
+    int nout = 0, prev = -1;
+    for (int j = 0; j < nmine; ++j) {
       int tile;
-      const int q = which(item, &tile);
+      const int q = which(item_at(j), &tile);
       bool ok;
       if constexpr (kSame) {
         ok = tc2_epilogue<Op1, BN, ACC>(q == 0 ? P.epi0 : P.epi1[q - 1], &P.map[q][2], P.shape[q],
                                         tile, j, rank, warp, lane, tmem, tfull, te0, sbuf, nout,
                                         status);
       } else {
-        // the ops may stage chunks of different sizes in the same buffer: the
-        // first tile after op 0's waits until op 0's staged chunks are read
-        if (q > 0 && prev == 0 && lane == 0) tc::tma_store_wait_read<0>();
+        // the ops stage chunks of different sizes in the same buffer: the
+        // first tile after a change of op waits until the other op's staged
+        // chunks are read
+        if (prev >= 0 && (q > 0) != (prev > 0) && lane == 0) tc::tma_store_wait_read<0>();
         ok = q > 0 ? tc2_epilogue<Op1, BN, ACC>(P.epi1[q - 1], &P.map[q][2], P.shape[q], tile, j,
                                                 rank, warp, lane, tmem, tfull, te0, sbuf, nout,
                                                 status)
@@ -821,7 +839,8 @@ static cudaError_t tc2_run(const Launch& lc, const Tc2Params<Op0, Op1>& P) {
   if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
   int total = 0;
   for (int q = 0; q < P.count; ++q) total += P.shape[q].n_tiles;
-  const int pairs = total < sm_count() / 2 ? total : sm_count() / 2;
+  const int pairs =
+      P.npairs_sched ? P.npairs_sched : (total < sm_count() / 2 ? total : sm_count() / 2);
   cudaError_t e = launch_k_cluster(kern, dim3(2 * pairs), dim3(kGemmThreads), Cfg::SMEM, lc.stream,
                                    2, P, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
@@ -873,6 +892,9 @@ cudaError_t gemm_tc_pair(const Launch& lc, int dtype_out, int M, int N, int K, c
   return go(T{}, F{});
 }
 
+bool tc2_group_schedule(const Tc2Shape* shape, int count, int max_pairs,
+                        std::vector<std::vector<int>>* lists, long* makespan);
+
 cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const PairProduct* w,
                                int nw) {
   if (nw < 1 || nw > kTc2Max - 1) return cudaErrorInvalidValue;
@@ -906,7 +928,81 @@ cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const Pa
       return cudaErrorInvalidValue;
   }
   P.count = 1 + nw;
+  // the pairs' item lists, longest first onto the least loaded pair
+  std::vector<std::vector<int>> lists;
+  if (tc2_group_schedule(P.shape, P.count, sm_count() / 2, &lists, nullptr)) {
+    P.npairs_sched = (int)lists.size();
+    int k = 0;
+    for (int p = 0; p < P.npairs_sched; ++p) {
+      P.start[p] = (uint16_t)k;
+      for (int item : lists[p]) P.list[k++] = (uint16_t)item;
+    }
+    P.start[P.npairs_sched] = (uint16_t)k;
+  }
   return tc2_run<256, ST, ACC, Op0, Op1>(lc, P);
+}
+
+// Cost of one item of a CTA-pair product in 64-deep K slices of a 256 x 256
+// tile, plus kTc2ItemOverhead for its share of pipeline fill and epilogue.
+constexpr int kTc2ItemOverhead = 4;
+static int tc2_item_cost(const Tc2Shape& s, int tile) {
+  const int z = tile / (s.tiles_m * s.tiles_n);
+  const int kb0 = z * s.kps;
+  return std::min(s.nkb, kb0 + s.kps) - kb0 + kTc2ItemOverhead;
+}
+
+// Longest processing time first: the group's items, by decreasing cost (ties
+// by item number), each onto the pair with the least load so far (ties to the
+// lower pair); every pair's list is then put in item order, so the products
+// follow each other in order within a pair.  Returns false when the group
+// has more items or pairs than a schedule holds (round-robin then); fills
+// *lists (one list per pair that has items) and *makespan (the largest
+// pair load) when non-null.
+bool tc2_group_schedule(const Tc2Shape* shape, int count, int max_pairs,
+                        std::vector<std::vector<int>>* lists, long* makespan) {
+  std::vector<std::pair<int, int>> items;  // (cost, item)
+  int item = 0;
+  for (int q = 0; q < count; ++q)
+    for (int t = 0; t < shape[q].n_tiles; ++t, ++item)
+      items.push_back({tc2_item_cost(shape[q], t), item});
+  const int total = item;
+  const int pairs = std::min(total, max_pairs);
+  if (total > kTc2SchedItems || pairs > kTc2SchedPairs || pairs < 1) return false;
+  std::stable_sort(items.begin(), items.end(),
+                   [](const std::pair<int, int>& a, const std::pair<int, int>& b) {
+                     return a.first > b.first;
+                   });
+  std::vector<long> load((size_t)pairs, 0);
+  std::vector<std::vector<int>> out((size_t)pairs);
+  for (const auto& it : items) {
+    const size_t p = (size_t)(std::min_element(load.begin(), load.end()) - load.begin());
+    load[p] += it.first;
+    out[p].push_back(it.second);
+  }
+  for (auto& l : out) std::sort(l.begin(), l.end());
+  if (makespan) *makespan = *std::max_element(load.begin(), load.end());
+  if (lists) *lists = std::move(out);
+  return true;
+}
+
+long tc2_group_makespan(int M0, int N0, int K0, const int* Mw, const int* Nw, const int* Kw,
+                        const int* splits, int nw, int max_pairs) {
+  Tc2Shape sh[kTc2Max];
+  if (nw < 0 || nw > kTc2Max - 1) return -1;
+  sh[0] = tc2_shape<256>(M0, N0, K0, 1);
+  for (int i = 0; i < nw; ++i)
+    sh[i + 1] = tc2_shape<256>(Mw[i], Nw[i], Kw[i], effective_splits(Kw[i], splits[i]));
+  long ms = -1;
+  if (tc2_group_schedule(sh, nw + 1, max_pairs, nullptr, &ms)) return ms;
+  // too many items for a schedule: the launch deals them round-robin
+  int total = 0;
+  for (int q = 0; q <= nw; ++q) total += sh[q].n_tiles;
+  const int pairs = std::max(1, std::min(total, max_pairs));
+  std::vector<long> load((size_t)pairs, 0);
+  int item = 0;
+  for (int q = 0; q <= nw; ++q)
+    for (int t = 0; t < sh[q].n_tiles; ++t, ++item) load[(size_t)(item % pairs)] += tc2_item_cost(sh[q], t);
+  return *std::max_element(load.begin(), load.end());
 }
 
 // Output tile widths: 128 x 256 tiles move 48 KB per 64-deep K slice for

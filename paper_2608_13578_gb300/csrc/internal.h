@@ -84,6 +84,13 @@ struct PairProduct {
 // w[i]'s in order, round-robin.  cudaErrorNotSupported for other layouts.
 cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const PairProduct* w,
                                int nw);
+// The largest pair load (in 64-deep slices of a 256 x 256 tile, plus a fixed
+// overhead per item) of such a group under the longest-first schedule the
+// launch uses: product 0 [M0, N0] over K0, weight products i [Mw, Nw] over Kw
+// split in splits[i] (round-robin, as the launch deals them, when the group
+// has too many items for a schedule).
+long tc2_group_makespan(int M0, int N0, int K0, const int* Mw, const int* Nw, const int* Kw,
+                        const int* splits, int nw, int max_pairs);
 cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits);
@@ -167,12 +174,12 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, const float* decay,
                             const float* Z, const float* M, float* dS, float* da_part, int B,
                             int Nb, int D);
-// Backward of the pooling, in chunks of 16 rows of a block (32 when D <= 256;
-// grid summary_bwd_chunks(L, D) x Nb x B): g_t = H_t . dS_blk,
+// Backward of the pooling, in chunks of a block's rows (grid
+// summary_bwd_chunks(dtype, L, D) x Nb x B): g_t = H_t . dS_blk,
 // ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
 // dwp_part[(b*Nb + i) * chunks + c] = sum over the chunk of ds_t H_t, and
 // dH_t += alpha_t dS_blk + ds_t w_p in place.
-int summary_bwd_chunks(int L, int D);
+int summary_bwd_chunks(int dtype, int L, int D);
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
                         const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
                         float* dwp_part, int B, int T, int D, int L);

@@ -94,20 +94,30 @@ cudaError_t with_splits(int psplits, F&& f) {
   }
 }
 
-// Sec. 3.4: item (i, b, z): pooling scores of block i of batch b summed from
-// the npart partial dot products the W_O epilogue wrote, alpha = softmax over
-// the block (stored by z == 0), S_i[256 z .. 256 z + 255] = sum_t alpha_t H_t.
+// Sec. 3.4 for block i of batch b, channels 256 z .. 256 z + 255: the pooling
+// scores s = H w_p summed from the npart partial dot products the W_O epilogue
+// wrote, alpha = softmax(s) over the block's tokens (stored by z == 0), and
+// S_i = sum_t alpha_t H_t.  The first 64 rows' H loads are issued before the
+// scores are known, so the block's H and score reads share one memory round
+// trip.  Returns S_i[256 z + threadIdx.x] (0 past D).
 template <class T>
-__device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* __restrict__ spart,
-                             int npart, long n_tok, float* __restrict__ alpha,
-                             float* S, int Tlen, int D, int L, int Nb, int i, int b,
-                             int z) {
+__device__ float pool_block(float* sm, const T* __restrict__ Hm, const float* __restrict__ spart,
+                            int npart, long n_tok, float* __restrict__ alpha, int Tlen, int D,
+                            int L, int i, int b, int z) {
   float* sc = sm;                 // [kMaxL]
   float* red = sm + kMaxL;        // [2]
   float* part = sm + kMaxL + 4;   // [8][260]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t0 = i * L, n = min(L, Tlen - t0);
   const long row0 = (long)b * Tlen + t0;
+  // 8 row groups (warps) x 32 threads of 8 channels
+  const int c = z * 256 + lane * 8;
+  const bool cin = c < D;
+  const T* Hc = Hm + row0 * D + c;
+  Raw8<T> h0[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (cin && warp + 8 * u < n) ld_raw(Hc + (long)(warp + 8 * u) * D, h0[u]);
   for (int r = threadIdx.x; r < n; r += kThreads) {
     float s = 0.f;
 #pragma unroll 16
@@ -135,38 +145,41 @@ __device__ void summary_item(float* sm, const T* __restrict__ Hm, const float* _
     sc[r] = a;
   }
   __syncthreads();
-  // 8 row groups x 32 threads of 8 channels, then a fixed-order sum of the groups
-  const int rg = warp, co = lane;
-  const int c = z * 256 + co * 8;
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  if (c < D) {
-    // the thread's rows rg, rg+8, ... four at a time, all loads first
-    const T* Hc = Hm + row0 * D + c;
-    for (int r = rg; r < n; r += 32) {
-      float h[4][8];
+  if (cin) {
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (r + 8 * u < n) load8(Hc + (long)(r + 8 * u) * D, h[u]);
+    for (int u = 0; u < 8; ++u)
+      if (warp + 8 * u < n) {
+        float h[8];
+        unraw(h0[u], h);
+        const float a = sc[warp + 8 * u];
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (r + 8 * u < n) {
-          const float a = sc[r + 8 * u];
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[e], acc[e]);
+      }
+    // blocks longer than 64 tokens: further batches of 64 rows, loads first
+    for (int r0 = 64; r0 < n; r0 += 64) {
+      Raw8<T> hb[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[u][e], acc[e]);
+      for (int u = 0; u < 8; ++u)
+        if (r0 + warp + 8 * u < n) ld_raw(Hc + (long)(r0 + warp + 8 * u) * D, hb[u]);
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (r0 + warp + 8 * u < n) {
+          float h[8];
+          unraw(hb[u], h);
+          const float a = sc[r0 + warp + 8 * u];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[e] = fmaf(a, h[e], acc[e]);
         }
     }
   }
 #pragma unroll
-  for (int e = 0; e < 8; ++e) part[rg * 260 + co * 8 + e] = acc[e];
+  for (int e = 0; e < 8; ++e) part[warp * 260 + lane * 8 + e] = acc[e];
   __syncthreads();
-  const int cc = z * 256 + threadIdx.x;
-  if (cc < D) {
-    float t = 0.f;
+  float t = 0.f;
 #pragma unroll
-    for (int g = 0; g < 8; ++g) t += part[g * 260 + threadIdx.x];
-    S[((long)b * Nb + i) * D + cc] = t;
-  }
-  __syncthreads();
+  for (int g = 0; g < 8; ++g) t += part[g * 260 + threadIdx.x];
+  return t;
 }
 
 // Sec. 3.8 reversed: item (x, i, b): kGateCh channels of block i of batch b
@@ -180,34 +193,61 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
                               const float* __restrict__ Pm, long pstride,
                               T* __restrict__ dU, float* dP, bf16* dPb, int Tlen, int D, int L,
                               int Nb, int x, int i, int b) {
-  float* part = sm;  // [8][kGateCh + 4]
+  float* part = sm;                      // [8][kGateCh + 4]
+  float* crow = sm + 8 * (kGateCh + 4);  // [kGateCh]: the block's memory row C_i
   const int rg = threadIdx.x >> 5, cq = threadIdx.x & 31;
   const int c = x * kGateCh + cq * 8;
+  const bool cin = c < D;
   const int t0 = i * L, n = min(L, Tlen - t0);
+  // rows rg, rg+8, ... in batches of 8 (64 rows of the block, loads held
+  // packed): every load of a batch is issued before its first store
+  const long step = 8L * D;
+  const long o0 = ((long)b * Tlen + t0 + rg) * D + c;
+  const T* dyp = dY + o0;
+  const T* gp = G + o0;
+  T* dup = dU + o0;
+  Raw8<T> rdy[8], rgt[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (cin && rg + 8 * u < n) {
+      ld_raw(dyp + u * step, rdy[u]);
+      ld_raw(gp + u * step, rgt[u]);
+    }
+  // meanwhile the memory row, one channel per thread, its K-split partials
+  // summed in split order (C_0 = 0, C_i = P_{i-1})
+  {
+    const int cc = x * kGateCh + threadIdx.x;
+    float v = 0.f;
+    if (i > 0 && cc < D) {
+      const float* p = Pm + ((long)b * Nb + i - 1) * D + cc;
+      float q[PS];
+#pragma unroll
+      for (int z = 0; z < PS; ++z) q[z] = p[z * pstride];
+#pragma unroll
+      for (int z = 0; z < PS; ++z) v += q[z];
+    }
+    crow[threadIdx.x] = v;
+  }
+  __syncthreads();
   float acc[8];
 #pragma unroll
   for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-  if (c < D) {
+  if (cin) {
     float cm[8];
-    mem_row<8, PS>(Pm, pstride, b, i, Nb, D, c, cm);
-    // rows rg, rg+8, ... in batches of 4 (loads held packed): every load of
-    // a batch is issued before its first store
-    const long step = 8L * D;
-    const long o0 = ((long)b * Tlen + t0 + rg) * D + c;
-    const T* dyp = dY + o0;
-    const T* gp = G + o0;
-    T* dup = dU + o0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) cm[e] = crow[cq * 8 + e];
 #pragma unroll 1
-    for (int r0 = rg; r0 < n; r0 += 32, dyp += 4 * step, gp += 4 * step, dup += 4 * step) {
-      Raw8<T> rdy[4], rgt[4];
+    for (int r0 = rg; r0 < n; r0 += 64, dyp += 8 * step, gp += 8 * step, dup += 8 * step) {
+      if (r0 != rg) {  // blocks longer than 64 tokens: the next batch
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (r0 + 8 * u < n) {
-          ld_raw(dyp + u * step, rdy[u]);
-          ld_raw(gp + u * step, rgt[u]);
-        }
+        for (int u = 0; u < 8; ++u)
+          if (r0 + 8 * u < n) {
+            ld_raw(dyp + u * step, rdy[u]);
+            ld_raw(gp + u * step, rgt[u]);
+          }
+      }
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+      for (int u = 0; u < 8; ++u)
         if (r0 + 8 * u < n) {
           float dy[8], g[8], du[8];
           unraw(rdy[u], dy);
@@ -251,12 +291,12 @@ __device__ void scan_bwd_item(const float* dM, long mstride,
                               const float* __restrict__ decay, const float* __restrict__ Z,
                               const float* __restrict__ M, float* dS, float* __restrict__ da_part,
                               int Nb, int D, int x, int b) {
-  const int c = x * kThreads + threadIdx.x;
+  const int c = x * blockDim.x + threadIdx.x;
   if (c >= D) return;
   const float a = decay[c];
   const long base = (long)b * Nb * D + c;
   float R = 0.f, Qz = 0.f, da = 0.f;
-  constexpr int U = 8;
+  constexpr int U = 16;
   for (int i1 = Nb; i1 > 0; i1 -= U) {
     float mv[U], zv[U], mi[U], mp[U], zp[U];
 #pragma unroll
@@ -405,7 +445,130 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   }
 }
 
+// The same pooling backward for bf16 at D <= 1024, item (c, i, b) = rows
+// ROWS*c .. ROWS*c + ROWS-1 of block i of batch b with ROWS = 8*RW: warp w owns
+// rows w, w+8, ..., lane l the channels 256 j + 8 l .. +7 (j < KC).  Every
+// thread issues the loads of its rows of H and dH first; meanwhile the CTA
+// stages dS_i and w_p in shared memory and forms S_i . dS_i.  The H rows stay
+// in registers from the dot products g_t = H_t . dS_i to the update, so the
+// item costs one memory round trip.  RW * KC <= 8 keeps the held rows within
+// the registers of two CTAs per SM.
+template <int RW, int KC>
+__global__ void __launch_bounds__(kThreads, 2)
+    summary_bwd_reg_kernel(const bf16* __restrict__ Hm, const float* __restrict__ alpha,
+                           const float* __restrict__ Sb, const float* dS,
+                           const bf16* __restrict__ w_p, bf16* dH, float* __restrict__ ds_out,
+                           float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
+  pdl_enter();
+  constexpr int ROWS = 8 * RW;
+  constexpr int PW = KC * 256 + 4;  // row-group stride of the dW_p partials
+  __shared__ __align__(16) float dss[KC * 256];
+  __shared__ __align__(16) float wps[KC * 256];
+  __shared__ __align__(16) float part[8 * PW];
+  __shared__ float red[8];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x, i = blockIdx.y, b = blockIdx.z;
+  const int blen = min(L, Tlen - i * L);
+  const int t0 = i * L + c * ROWS, n = min(ROWS, blen - c * ROWS);
+  const long prow = ((long)b * Nb + i) * gridDim.x + c;
+  if (n <= 0) {  // a ragged last block's empty chunk: zero partials of dW_p
+    for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
+    return;
+  }
+  const long rowbase = (long)b * Tlen + t0;
+  const bf16* Hb = Hm + rowbase * D;
+  bf16* dHb = dH + rowbase * D;
+  uint4 h[RW][KC], d[RW][KC];
+#pragma unroll
+  for (int u = 0; u < RW; ++u)
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      const int k = 256 * j + 8 * lane;
+      if (warp + 8 * u < n && k < D) {
+        const long o = (long)(warp + 8 * u) * D + k;
+        load8_raw(Hb + o, h[u][j]);
+        load8_raw(dHb + o, d[u][j]);
+      }
+    }
+  float a[RW];
+#pragma unroll
+  for (int u = 0; u < RW; ++u) a[u] = (warp + 8 * u < n) ? alpha[rowbase + warp + 8 * u] : 0.f;
+  // dS_i and w_p to shared memory; sum_u alpha_u g_u = S_i . dS_i
+  const float* dSi = dS + ((long)b * Nb + i) * D;
+  const float* Si = Sb + ((long)b * Nb + i) * D;
+  float cp = 0.f;
+  for (int k = 4 * threadIdx.x; k < D; k += 4 * kThreads) {
+    const float4 dv = __ldcg(reinterpret_cast<const float4*>(dSi + k));
+    const float4 sv = *reinterpret_cast<const float4*>(Si + k);
+    float w[4];
+    load4(w_p + k, w);
+    *reinterpret_cast<float4*>(dss + k) = dv;
+    *reinterpret_cast<float4*>(wps + k) = make_float4(w[0], w[1], w[2], w[3]);
+    cp = fmaf(sv.x, dv.x, cp);
+    cp = fmaf(sv.y, dv.y, cp);
+    cp = fmaf(sv.z, dv.z, cp);
+    cp = fmaf(sv.w, dv.w, cp);
+  }
+  cp = warp_sum(cp);
+  if (lane == 0) red[warp] = cp;
+  __syncthreads();
+  float cd = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) cd += red[w];
+  // g_t = H_t . dS_i and ds_t = alpha_t (g_t - S_i . dS_i) per row of the warp
+  float dsr[RW];
+#pragma unroll
+  for (int u = 0; u < RW; ++u) {
+    float g = 0.f;
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      const int k = 256 * j + 8 * lane;
+      if (warp + 8 * u < n && k < D) {
+        float hv[8];
+        unpack8(h[u][j], hv);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) g = fmaf(hv[e], dss[k + e], g);
+      }
+    }
+    g = warp_sum(g);
+    dsr[u] = a[u] * (g - cd);
+    if (lane == 0 && warp + 8 * u < n) ds_out[rowbase + warp + 8 * u] = dsr[u];
+  }
+  // dH_t += alpha_t dS_i + ds_t w_p; the chunk's dW_p partial sum_t ds_t H_t
+#pragma unroll
+  for (int j = 0; j < KC; ++j) {
+    const int k = 256 * j + 8 * lane;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (k < D) {
+#pragma unroll
+      for (int u = 0; u < RW; ++u)
+        if (warp + 8 * u < n) {
+          float hv[8], dv[8];
+          unpack8(h[u][j], hv);
+          unpack8(d[u][j], dv);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            acc[e] = fmaf(dsr[u], hv[e], acc[e]);
+            dv[e] += a[u] * dss[k + e] + dsr[u] * wps[k + e];
+          }
+          store8(dHb + (long)(warp + 8 * u) * D + k, dv);
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part[warp * PW + 256 * j + 8 * lane + e] = acc[e];
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < D; k += kThreads) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += part[w * PW + k];
+    dwp_part[prow * D + k] = t;
+  }
+}
+
 // ======================================================== kernels (one per stage)
+// Sec. 3.4: item (block i, batch b, chunk z) pools its block (pool_block)
+// and stores S_i[256 z .. 256 z + 255].
 template <class T>
 __global__ void __launch_bounds__(kThreads)
     summary_fwd_kernel(const T* __restrict__ Hm, const float* __restrict__ spart, int npart,
@@ -413,32 +576,37 @@ __global__ void __launch_bounds__(kThreads)
                        int D, int L, int Nb) {
   pdl_enter();
   extern __shared__ __align__(16) float sm[];
-  summary_item<T>(sm, Hm, spart, npart, n_tok, alpha, S, Tlen, D, L, Nb, blockIdx.x, blockIdx.y,
-                  blockIdx.z);
+  const int i = blockIdx.x, b = blockIdx.y, z = blockIdx.z;
+  const float Si = pool_block<T>(sm, Hm, spart, npart, n_tok, alpha, Tlen, D, L, i, b, z);
+  const int c = z * 256 + threadIdx.x;
+  if (c < D) S[((long)b * Nb + i) * D + c] = Si;
 }
 
 // Sec. 3.5: one thread per (batch b, channel c): the decayed scan
 //   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i,
-// the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j).
+// the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j),
+// over blocks in batches of kScanU whose loads all go out before the first
+// step.  kScanThreads threads per CTA spread the B * D chains over many SMs.
 // Writes M in fp32 and, when Mb is non-null, in bf16 (the A operand of the
 // tensor-core projection), and Z (batch 0 only: it does not depend on b).
-__global__ void __launch_bounds__(kThreads)
+constexpr int kScanThreads = 64;
+constexpr int kScanU = 16;
+__global__ void __launch_bounds__(kScanThreads)
     memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
                            int Nb, int D) {
   pdl_enter();
-  const int c = blockIdx.x * blockDim.x + threadIdx.x, b = blockIdx.y;
+  const int c = blockIdx.x * kScanThreads + threadIdx.x, b = blockIdx.y;
   if (c >= D) return;
   const float a = decay[c];
   const long base = (long)b * Nb * D + c;
   float Nn = 0.f, Zz = 0.f;
-  constexpr int U = 16;
-  for (int i0 = 0; i0 < Nb; i0 += U) {
-    float sv[U];
+  for (int i0 = 0; i0 < Nb; i0 += kScanU) {
+    float sv[kScanU];
 #pragma unroll
-    for (int u = 0; u < U; ++u) sv[u] = (i0 + u < Nb) ? S[base + (long)(i0 + u) * D] : 0.f;
+    for (int u = 0; u < kScanU; ++u) sv[u] = (i0 + u < Nb) ? S[base + (long)(i0 + u) * D] : 0.f;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
+    for (int u = 0; u < kScanU; ++u) {
       const int i = i0 + u;
       if (i < Nb) {
         Nn = fmaf(a, Nn, sv[u]);
@@ -453,7 +621,7 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 template <class T, int PS>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 2)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
                     const float* __restrict__ Pm, long pstride, T* __restrict__ dU,
                     float* __restrict__ dP, bf16* __restrict__ dPb, int Tlen, int D, int L,
@@ -465,7 +633,7 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 template <int PS>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kScanThreads)
     memory_scan_bwd_kernel(const float* __restrict__ dM, long mstride,
                            const float* __restrict__ decay, const float* __restrict__ Z,
                            const float* __restrict__ M, float* __restrict__ dS,
@@ -497,13 +665,18 @@ __global__ void __launch_bounds__(kThreads, 2)
 // broadcast by index.  Item (run, row group, block i, batch b): 8 channels of
 // kInjRows consecutive rows of one block, so the memory row (summed from the
 // projection's K-split partials, shifted by one block) is read once for all
-// of them; the rows' H and G loads are all issued before the first use.
-constexpr int kInjRows = 4;
+// of them; the rows' H and G loads are all issued before the first use.  The
+// host sizes the grid so that every item's thread is resident at once (one
+// wave): a second, partial wave would add a whole memory round trip.
+// kInjRows rows per item in bf16 (4 in fp32, whose rows take twice the registers).
+constexpr int kInjRows = 8;
+__host__ __device__ constexpr int inj_rows(int elem_bytes) { return elem_bytes == 2 ? kInjRows : kInjRows / 2; }
 template <class T, int PS>
-__global__ void __launch_bounds__(kThreads, sizeof(T) == 2 ? 3 : 2)
+__global__ void __launch_bounds__(kThreads, 2)
     inject_kernel(const T* __restrict__ Hm, const T* __restrict__ G, const float* __restrict__ Pm,
                   long pstride, T* __restrict__ Y, int B, int Tlen, int D, int L, int Nb) {
   pdl_enter();
+  constexpr int kInjRows = inj_rows(sizeof(T));
   const int runs = D / 8, groups = (L + kInjRows - 1) / kInjRows;
   const long total = (long)B * Nb * groups * runs;
   for (long it = (long)blockIdx.x * kThreads + threadIdx.x; it < total;
@@ -544,7 +717,7 @@ __global__ void __launch_bounds__(kThreads, sizeof(T) == 2 ? 3 : 2)
 namespace {
 // shared memory of the summary kernels: scores [kMaxL], two scalars, [8][260]
 constexpr size_t kSummarySmem = (size_t)(kMaxL + 4 + 8 * 260) * sizeof(float);
-constexpr size_t kGateSmem = (size_t)(8 * (kGateCh + 4)) * sizeof(float);
+constexpr size_t kGateSmem = (size_t)(8 * (kGateCh + 4) + kGateCh) * sizeof(float);
 }  // namespace
 
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
@@ -565,9 +738,9 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
                             void* Mb, float* Z, int B, int Nb, int D) {
-  dim3 grid((D + kThreads - 1) / kThreads, B);
-  cudaError_t e = launch_k(memory_scan_fwd_kernel, grid, dim3(kThreads), 0, lc.stream, S, decay,
-                           M, (bf16*)Mb, Z, Nb, D);
+  dim3 grid((D + kScanThreads - 1) / kScanThreads, B);
+  cudaError_t e = launch_k(memory_scan_fwd_kernel, grid, dim3(kScanThreads), 0, lc.stream, S,
+                           decay, M, (bf16*)Mb, Z, Nb, D);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -592,17 +765,29 @@ cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G,
 cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, const float* decay,
                             const float* Z, const float* M, float* dS, float* da_part, int B,
                             int Nb, int D) {
-  dim3 grid((D + kThreads - 1) / kThreads, B);
+  dim3 grid((D + kScanThreads - 1) / kScanThreads, B);
   cudaError_t e = with_splits(msplits, [&](auto ms) {
-    return launch_k(memory_scan_bwd_kernel<decltype(ms)::value>, grid, dim3(kThreads), 0,
+    return launch_k(memory_scan_bwd_kernel<decltype(ms)::value>, grid, dim3(kScanThreads), 0,
                     lc.stream, dM, (long)B * Nb * D, decay, Z, M, dS, da_part, Nb, D);
   });
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-static int summary_bwd_rows(int D) { return D <= 256 ? 32 : 16; }
-int summary_bwd_chunks(int L, int D) {
-  const int rows = summary_bwd_rows(D);
+// Rows per pooling-backward item: the register-held kernel (bf16, D <= 1024)
+// takes 8 * RW rows with RW * ceil(D / 256) <= 8; the general kernel takes 16
+// rows, or 32 when D <= 256.
+static int summary_bwd_reg_rw(int dtype, int D) {
+  if (dtype != 1 || D > 1024) return 0;
+  const int kc = (D + 255) / 256;
+  return kc == 1 ? 8 : kc == 2 ? 4 : 2;
+}
+static int summary_bwd_rows(int dtype, int D) {
+  const int rw = summary_bwd_reg_rw(dtype, D);
+  if (rw) return 8 * rw;
+  return D <= 256 ? 32 : 16;
+}
+int summary_bwd_chunks(int dtype, int L, int D) {
+  const int rows = summary_bwd_rows(dtype, D);
   return (L + rows - 1) / rows;
 }
 
@@ -611,7 +796,21 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
                         float* dwp_part, int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
-  dim3 grid(summary_bwd_chunks(L, D), Nb, B);
+  dim3 grid(summary_bwd_chunks(dtype, L, D), Nb, B);
+  const int rw = summary_bwd_reg_rw(dtype, D);
+  cudaError_t e;
+  if (rw) {
+    const bf16 *H = (const bf16*)Hm, *wp = (const bf16*)w_p;
+    bf16* dh = (bf16*)dH;
+    const int kc = (D + 255) / 256;
+#define BCMT_SBWD(RW_, KC_)                                                                   \
+  launch_k(summary_bwd_reg_kernel<RW_, KC_>, grid, dim3(kThreads), 0, lc.stream, H, alpha, Sb, \
+           dS, wp, dh, ds, dwp_part, T, D, L, Nb)
+    e = kc == 1 ? BCMT_SBWD(8, 1) : kc == 2 ? BCMT_SBWD(4, 2) : kc == 3 ? BCMT_SBWD(2, 3)
+                                                                  : BCMT_SBWD(2, 4);
+#undef BCMT_SBWD
+    return e != cudaSuccess ? e : cudaGetLastError();
+  }
   auto go = [&](auto rows) {
     constexpr int R = decltype(rows)::value;
     if (dtype == 0)
@@ -622,17 +821,38 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
                     (const bf16*)Hm, alpha, Sb, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T,
                     D, L, Nb);
   };
-  cudaError_t e = summary_bwd_rows(D) == 32 ? go(std::integral_constant<int, 32>())
-                                            : go(std::integral_constant<int, 16>());
+  e = summary_bwd_rows(dtype, D) == 32 ? go(std::integral_constant<int, 32>())
+                                       : go(std::integral_constant<int, 16>());
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Resident CTAs of `kern` (kThreads threads, no dynamic shared memory) on
+// the whole device, looked up once per kernel.
+template <class K>
+static long resident_ctas(K kern) {
+  static long n = 0;
+  if (!n) {
+    int dev = 0, sms = 0, per_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0) != cudaSuccess ||
+        sms < 1 || per_sm < 1)
+      return 148;
+    n = (long)sms * per_sm;
+  }
+  return n;
 }
 
 cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Pm,
                    int psplits, void* Y, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
   const long pstride = (long)B * Nb * D;
-  const long items = (long)B * Nb * ((L + kInjRows - 1) / kInjRows) * (D / 8);
-  const int blocks = (int)std::max<long>(1, std::min<long>((items + kThreads - 1) / kThreads, 1L << 16));
+  const int rows = inj_rows(dtype == 0 ? 4 : 2);
+  const long items = (long)B * Nb * ((L + rows - 1) / rows) * (D / 8);
+  const long want = (items + kThreads - 1) / kThreads;
+  const long cap = dtype == 0 ? resident_ctas(inject_kernel<float, 4>)
+                              : resident_ctas(inject_kernel<bf16, 4>);
+  const int blocks = (int)std::max<long>(1, std::min<long>(want, cap));
   cudaError_t e = with_splits(psplits, [&](auto ps) {
     constexpr int PS = decltype(ps)::value;
     if (dtype == 0)

@@ -57,14 +57,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
   return done != 0;
 }
 // Waits until the phase with the given parity has completed.  Gives up after
-// kWaitCycles, sets kStatusTimeout in *status and returns false.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status) {
+// `cap` SM clock cycles (kWaitCycles unless a caller passes a shorter bound),
+// sets kStatusTimeout in *status and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status,
+                                          long long cap = kWaitCycles) {
   const uint32_t addr = smem_u32(bar);
   if (mbar_try_wait(addr, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(addr, parity)) return true;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > cap) {
       atomicOr(status, kStatusTimeout);
       return false;
     }

@@ -57,22 +57,15 @@ VARIANTS = [
 ]
 
 
-def _check(w: Workload, backward=True, batch=None):
+def _check(w: Workload, backward=True):
     t = make_inputs(w)
     y, g = gpu_run(w, to_device(t), backward)
-    fw, gr = oracle_run(w, t, backward, batch=batch)
-    if batch is not None:
-        y = y[batch]
+    fw, gr = oracle_run(w, t, backward)
     assert_close("Y", y, fw["Y"], w.dtype)
     if backward:
         names = GRAD_NAMES_X if w.input_is_x else GRAD_NAMES_QKV
         for n in names:
             got = g[n]
-            if batch is not None:
-                if n in ("dx", "dq", "dk", "dv"):
-                    got = got[batch]
-                else:
-                    continue
             if w.honly and n in ("dw_p", "dw_m", "dw_g", "d_decay"):
                 assert torch.count_nonzero(got).item() == 0
                 continue
@@ -142,10 +135,20 @@ def test_block_size_sweep(cuda_ok, L):
 
 @pytest.mark.parametrize("T", [2048, 4096, 8192, 16384])
 def test_sequence_scaling(cuda_ok, T):
-    w = WORKLOADS[f"seqscale_bf16_b4_t{T}_l128_d1024_h16"]
-    # Full comparison at the shortest length; batch element 0 of Y and dX at the
-    # longer ones (the mixer is independent across the batch).
-    _check(w, backward=True, batch=None if T == 2048 else slice(0, 1))
+    """The sequence-length sweep at its full size (B = 4, D = 1024, L = 128),
+    every output and gradient against the oracle: the weight gradients reduce
+    over K = B*T up to 65536 tokens with their own split counts, and the
+    reverse scan of Sec. 3.5 runs N_b up to 128 dependent steps."""
+    _check(WORKLOADS[f"seqscale_bf16_b4_t{T}_l128_d1024_h16"], backward=True)
+
+
+@pytest.mark.parametrize("L", [256, 512])
+def test_sequence_scaling_key_walk(cuda_ok, L):
+    """The sequence sweep's shape at T = 4096 with blocks of 256 and 512
+    tokens, which take the key-tile-walking attention kernels (several key
+    tiles per block), every gradient against the oracle."""
+    w = WORKLOADS["seqscale_bf16_b4_t4096_l128_d1024_h16"]
+    _check(w.replace(name=f"seqscale_bf16_b4_t4096_l{L}_d1024_h16", L=L), backward=True)
 
 
 @pytest.mark.parametrize("L", [64, 128, 256, 512])
