@@ -196,10 +196,10 @@ def kernel_model(w):
         "attn_bwd_simt": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es),
         # two kernels (dQ, then dK/dV); the row dot products Drow are written and re-read
         "attn_bwd_fl": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es + 2 * n * H * 4),
-        # Sec. 3.4 summaries and Sec. 3.5 scan in one launch: read H and the score
-        # partials; write alpha, S, M (fp32 and the bf16 operand copy) and Z
-        "memory_fwd": ("hbm", n * D * es + n * 4 * npart + n * 4 + B * Nb * D * (4 + 4 + 2)
-                       + Nb * D * 4),
+        # Sec. 3.4 summaries: read H and the score partials, write alpha and S
+        "summary_fwd": ("hbm", n * D * es + n * 4 * npart + n * 4 + B * Nb * D * 4),
+        # Sec. 3.5 scan: read S, write M (fp32 and the bf16 operand copy) and Z
+        "memory_scan_fwd": ("hbm", B * Nb * D * (4 + 4 + 2) + Nb * D * 4),
         "gemm_wm": g(B * Nb, D, D),
         # Sec. 3.8 reversed: read dY, G and C; write dU and dP (fp32 + bf16)
         "gate_bwd": ("hbm", 3 * n * D * es + B * Nb * D * (4 + 4 + 2)),
