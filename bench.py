@@ -177,6 +177,11 @@ def kernel_model(w):
         "gemm_qkv": g(n, 3 * D, D),
         "gemm_wo": g(n, D, D),
         "gemm_gate": g(n, D, D),
+        # H and the gate pre-activation in one product: Concat [W_O | W_O W_g]
+        "gemm_wo_gate": g(n, 2 * D, D),
+        "gemm_wog": g(D, D, D),
+        # the Q/K/V projection with the weight product W_O W_g in the same launch
+        "gemm_qkv_wog": ("tensor", 2.0 * n * 3 * D * D + 2.0 * D * D * D),
         # Sec. 3.8 injection: read H, G and C; write Y
         "inject": ("hbm", 3 * n * D * es + B * Nb * D * 4),
         "gemm_dh": g(n, D, D),

@@ -372,8 +372,16 @@ int dqkv_splits(const Geometry& g) {
 int mem_splits(const Geometry& g) { return effective_splits(g.D, 4); }
 int dm_splits(const Geometry& g) { return effective_splits(g.D, 2); }
 
+// The forward's output projection and gate share one product,
+// Concat [W_O | W_O W_g] (bf16 tensor-core path): H W_g = Concat (W_O W_g).
+// The weight product W_O W_g rides in the Q/K/V projection's launch when that
+// runs on the single-CTA kernel, else it is a launch of its own before it.
+bool fused_gate(const Geometry& g) {
+  return !g.honly && g.dtype == BCMT_BF16 && g_use_tc_gemm && gemm_tc_available();
+}
+
 struct FwdWs {
-  char *qkv, *hhat, *hloc, *G, *Mb;
+  char *qkv, *hhat, *hloc, *G, *Mb, *wog;
   float *lse, *alpha, *S, *M, *Z, *C, *spart;
   size_t bytes;
 };
@@ -403,7 +411,10 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     // the K-split partials of P = M W_m (the memory rows C, before the shift)
     w.C = reinterpret_cast<float*>(take((size_t)mem_splits(g) * g.B * g.Nb * g.D * 4));
     w.G = take((size_t)g.n * g.D * g.es);
+    // W_O W_g [D, D]: the B operand of the gate columns of the fused projection
+    w.wog = fused_gate(g) ? take((size_t)g.D * g.D * g.es) : nullptr;
   } else {
+    w.wog = nullptr;
     w.hloc = w.G = w.Mb = nullptr;
     w.alpha = w.S = w.M = w.Z = w.C = w.spart = nullptr;
   }
@@ -612,16 +623,38 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   FwdWs w = fwd_layout(g, workspace);
   const int D = g.D, n = (int)g.n;
   cudaError_t e;
+  const bool fuse = fused_gate(g);
+  // the weight product W_O W_g of the fused output projection
+  const GemmProd wog{D, D, D, w_o, D, 1, w_g, D, 1, w.wog, D};
+  bool wog_done = false;
 
-  // Sec. 3.3: Q, K, V projections.
+  // Sec. 3.3: Q, K, V projections (with W_O W_g in the same launch when it fits).
   const void *Qp = q, *Kp = k, *Vp = v;
   long ld = D;
   if (g.from_x) {
-    EpiArgs ea;
-    ea.out = w.qkv;
-    ea.ldo = 3 * D;
-    e = run_gemm(lc, pr, "gemm_qkv", g.dtype, g.dtype, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1,
-                 EPI_STORE, ea);
+    e = cudaErrorNotSupported;
+    if (fuse) {
+      pr.begin("gemm_qkv_wog");
+      e = gemm_tc_two(lc, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1, w.qkv, 3 * D, wog);
+      pr.end(nullptr);
+      wog_done = e == cudaSuccess;
+    }
+    if (e == cudaErrorNotSupported) {
+      if (fuse) {
+        EpiArgs ea;
+        ea.out = w.wog;
+        ea.ldo = D;
+        e = run_gemm(lc, pr, "gemm_wog", g.dtype, g.dtype, D, D, D, w_o, D, 1, w_g, D, 1,
+                     EPI_STORE, ea);
+        if (e != cudaSuccess) return cuda_fail(e, "W_O W_g");
+        wog_done = true;
+      }
+      EpiArgs ea;
+      ea.out = w.qkv;
+      ea.ldo = 3 * D;
+      e = run_gemm(lc, pr, "gemm_qkv", g.dtype, g.dtype, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1,
+                   EPI_STORE, ea);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "QKV projection");
     Qp = w.qkv;
     Kp = w.qkv + (size_t)D * g.es;
@@ -646,7 +679,30 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   // epilogue also forms partial pooling scores H w_p over each run of columns
   // it stores (32 columns per tcgen05 TMEM load, 4 per SIMT thread).
   const int npart = D / ((g.dtype == BCMT_BF16 && g_use_tc_gemm) ? 32 : 4);
-  {
+  if (fuse) {
+    // H and the gate G = sigmoid(H W_g) (Sec. 3.8) in one product over all
+    // SMs, [H | U] = Concat [W_O | W_O W_g]
+    if (!wog_done) {
+      EpiArgs ea;
+      ea.out = w.wog;
+      ea.ldo = D;
+      e = run_gemm(lc, pr, "gemm_wog", g.dtype, g.dtype, D, D, D, w_o, D, 1, w_g, D, 1,
+                   EPI_STORE, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "W_O W_g");
+    }
+    EpiArgs ea;
+    ea.out = w.hloc;
+    ea.ldo = D;
+    ea.w_p = w_p;
+    ea.spart = w.spart;
+    ea.out2 = w.G;
+    ea.ldo2 = D;
+    ea.n_split = D;
+    ea.b2 = w.wog;
+    e = run_gemm(lc, pr, "gemm_wo_gate", g.dtype, g.dtype, n, 2 * D, D, w.hhat, D, 1, w_o, D, 1,
+                 EPI_HGATE, ea);
+    if (e != cudaSuccess) return cuda_fail(e, "output projection and gate");
+  } else {
     EpiArgs ea;
     ea.out = g.honly ? y : w.hloc;
     ea.ldo = D;
@@ -657,11 +713,11 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     if (e != cudaSuccess) return cuda_fail(e, "output projection");
   }
   if (!g.honly) {
-    // Sec. 3.8 gate G = sigmoid(H W_g) on all SMs, then the memory chain: one
-    // stream of kernels chained by programmatic dependent launch.  (Beside the
-    // chain on half of the SMs the gate GEMM slowed the chain's kernels about
-    // twofold, and each join of two streams left a launch gap of several us.)
-    {
+    // Sec. 3.8 gate G = sigmoid(H W_g) (unless fused above), then the memory
+    // chain: one stream of kernels chained by programmatic dependent launch.
+    // (Beside the chain on half of the SMs the gate GEMM slowed the chain's
+    // kernels about twofold, and each join of two streams left a launch gap.)
+    if (!fuse) {
       EpiArgs ea;
       ea.out = w.G;
       ea.ldo = D;

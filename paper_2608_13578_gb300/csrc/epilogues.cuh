@@ -23,6 +23,7 @@ struct EpiStoreF {
   using Pre = NoPre;
   using OutT = TO;
   static constexpr bool kTma = true;
+  static constexpr bool kDual = false;
   TO* out;
   long ldo;
   long split_stride;
@@ -52,6 +53,7 @@ struct EpiStoreScoreF {
   };
   using OutT = TO;
   static constexpr bool kTma = true;
+  static constexpr bool kDual = false;
   static constexpr long split_stride = 0;
   TO* out;
   long ldo;
@@ -98,6 +100,7 @@ struct EpiGateF {
   using Pre = NoPre;
   using OutT = T;
   static constexpr bool kTma = true;
+  static constexpr bool kDual = false;
   static constexpr long split_stride = 0;
   T* out;
   long ldo;
@@ -118,6 +121,57 @@ struct EpiGateF {
   }
 };
 
+// Sec. 3.3, 3.4 and 3.8 in one product: Concat(heads) [W_O | W_O W_g] gives
+// H (columns [0, n_split)) and the gate's pre-activation U = H W_g (columns
+// [n_split, N)), because H W_g = Concat (W_O W_g).  The first part is stored
+// as H together with the pooling-score partials (as EpiStoreScoreF), the
+// second as G = sigmoid(U) through the second output (out2, row stride ldo2,
+// its own tensor map: the GEMM stores column col of the second part at
+// col - n_split).  tcgen05 path only; every tile lies in one part.
+template <class TO>
+struct EpiHGateF {
+  struct Pre {
+    uint4 w[4];
+  };
+  using OutT = TO;
+  static constexpr bool kTma = true;
+  static constexpr bool kDual = true;
+  static constexpr long split_stride = 0;
+  TO* out;
+  long ldo;
+  const TO* w_p;
+  float* spart;
+  long n_rows;
+  TO* out2;
+  long ldo2;
+  int n_split;
+  __device__ __forceinline__ void load(int, int col, Pre& pre) const {
+    if (col >= n_split) return;
+    const bf16* wp = reinterpret_cast<const bf16*>(w_p) + col;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) load8_raw(wp + 8 * j, pre.w[j]);
+  }
+  __device__ __forceinline__ void apply(int row, int col, float* v, const Pre& pre, int) const {
+    if (col >= n_split) {
+#pragma unroll
+      for (int e = 0; e < 32; ++e) v[e] = sigmoid_bf16out(v[e]);
+      return;
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float w[8];
+      unpack8(pre.w[q], w);
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        s = fmaf(__bfloat162float(__float2bfloat16_rn(v[8 * q + e])), w[e], s);
+    }
+    spart[(long)(col / 32) * n_rows + row] = s;
+  }
+  // the SIMT GEMM does not take this epilogue (fp32 runs W_O and W_g apart)
+  __device__ __forceinline__ void operator()(int, int, const float*, int, int) const {}
+};
+
 // out = acc + add, same row-major layout (e.g. dU W_g^T + dY: the identity
 // path of Y = H + ... joins the gate path's gradient).
 template <class T>
@@ -128,6 +182,7 @@ struct EpiAddF {
   };
   using OutT = T;
   static constexpr bool kTma = true;
+  static constexpr bool kDual = false;
   static constexpr long split_stride = 0;
   const T* add;
   T* out;

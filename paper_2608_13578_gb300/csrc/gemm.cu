@@ -187,11 +187,14 @@ __device__ __forceinline__ uint4 pack8_bf16(const float* v) {
 // buffers.  Other epilogues store from registers.
 // apply: this thread's row is valid; store: lane 0 issues the chunk's store
 // (rows past M are clipped by the tensor map).  Called by the whole warp.
+// col: the chunk's column in the product; scol: its column in the output
+// tensor map mC (col, or col - n_split in the second output of a dual
+// epilogue).
 template <class Epi>
 __device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC, uint8_t* sbuf,
-                                          int& nout, int lane, int row, int row0, int col, int z,
-                                          float* v, const typename Epi::Pre& pre, bool apply,
-                                          bool store) {
+                                          int& nout, int lane, int row, int row0, int col,
+                                          int scol, int z, float* v,
+                                          const typename Epi::Pre& pre, bool apply, bool store) {
   if constexpr (Epi::kTma) {
     using OT = typename Epi::OutT;
     if (apply) epi.apply(row, col, v, pre, z);
@@ -218,7 +221,7 @@ __device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC,
     tc::fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0 && store) {
-      tc::tma_store_3d(mC, buf, col, row0, z);
+      tc::tma_store_3d(mC, buf, scol, row0, z);
       tc::tma_store_commit();
     }
     ++nout;
@@ -227,6 +230,7 @@ __device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC,
     (void)sbuf;
     (void)nout;
     (void)row0;
+    (void)scol;
     (void)store;
     if (apply) epi.apply(row, col, v, pre, z);
   }
@@ -264,11 +268,67 @@ int sm_count() {
 // half of the tile's columns), so a tile's epilogue overlaps the next tile's
 // main loop.
 constexpr int kGemmThreads = 320;
+
+// The rest of a launch's description, beside product 0 (the kernel's own
+// arguments):
+//  * mB2, mC2: for a dual epilogue (Epi::kDual), the B operand and the output
+//    of the columns from epi.n_split on (their own tensors, columns counted
+//    from n_split);
+//  * a second product with the same operand layouts and a plain store
+//    epilogue (has1): its n_tiles1 tiles follow product 0's in the round-robin
+//    order, so a small product fills the idle slots of a large one's last wave.
+struct TcAux {
+  CUtensorMap mB2, mC2;
+  CUtensorMap mA1, mB1, mC1;
+  int M1, N1, kps1, nkb1, tiles_m1, tiles_n1, n_tiles1;
+  int has1;
+};
+
+// Where one tile of a launch reads and writes: its product's tensor maps,
+// shape and K range, and its origin.
+struct TcTile {
+  const CUtensorMap *a, *b, *c;
+  int M, N, m0, n0, nb0, nc0, z, kb0, nk;
+};
+template <int BN, class Epi>
+__device__ __forceinline__ TcTile tc_tile(int tile, const CUtensorMap& mA, const CUtensorMap& mB,
+                                          const CUtensorMap& mC, const TcAux& aux, int M, int N,
+                                          int kps, int nkb, int tiles_m, int tiles_n, int n_tiles,
+                                          const Epi& epi) {
+  TcTile t;
+  const bool p1 = tile >= n_tiles;
+  const int tl = p1 ? tile - n_tiles : tile;
+  const int tm = p1 ? aux.tiles_m1 : tiles_m, tn = p1 ? aux.tiles_n1 : tiles_n;
+  const int ks = p1 ? aux.kps1 : kps, nb = p1 ? aux.nkb1 : nkb;
+  int m_blk, n_blk;
+  tile_mnz(tl, tm, tn, m_blk, n_blk, t.z);
+  t.a = p1 ? &aux.mA1 : &mA;
+  t.b = p1 ? &aux.mB1 : &mB;
+  t.c = p1 ? &aux.mC1 : &mC;
+  t.M = p1 ? aux.M1 : M;
+  t.N = p1 ? aux.N1 : N;
+  t.m0 = m_blk * kBM;
+  t.n0 = n_blk * BN;
+  t.nb0 = t.nc0 = t.n0;
+  if constexpr (Epi::kDual) {
+    if (!p1 && t.n0 >= epi.n_split) {
+      t.b = &aux.mB2;
+      t.c = &aux.mC2;
+      t.nb0 = t.nc0 = t.n0 - epi.n_split;
+    }
+  }
+  t.kb0 = t.z * ks;
+  t.nk = min(nb, t.kb0 + ks) - t.kb0;
+  return t;
+}
+
 template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   const __grid_constant__ CUtensorMap mC, int M, int N, int kps, int nkb,
-                   int tiles_m, int tiles_n, int n_tiles, Epi epi, unsigned* status) {
+                   const __grid_constant__ CUtensorMap mC, const __grid_constant__ TcAux aux,
+                   int M, int N, int kps, int nkb, int tiles_m, int tiles_n, int n_tiles, Epi epi,
+                   unsigned* status) {
+  const int total = n_tiles + (aux.has1 ? aux.n_tiles1 : 0);
   using Cfg = TcCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -293,6 +353,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tc::fence_mbar_init();
     tc::prefetch_tmap(&mA);
     tc::prefetch_tmap(&mB);
+    if (Epi::kDual) tc::prefetch_tmap(&aux.mB2);
+    if (aux.has1) {
+      tc::prefetch_tmap(&aux.mA1);
+      tc::prefetch_tmap(&aux.mB1);
+    }
   }
   if (warp == 1) {
     tc::tmem_alloc(tslot, Cfg::TMEM_COLS);
@@ -309,11 +374,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // ---- TMA producer
       int it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        int m_blk, n_blk, z;
-        tile_mnz(tile, tiles_m, tiles_n, m_blk, n_blk, z);
-        const int m0 = m_blk * kBM, n0 = n_blk * BN, kb0 = z * kps;
-        const int nk = min(nkb, kb0 + kps) - kb0;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        const TcTile t = tc_tile<BN>(tile, mA, mB, mC, aux, M, N, kps, nkb, tiles_m, tiles_n,
+                                     n_tiles, epi);
+        const int m0 = t.m0, n0 = t.nb0, kb0 = t.kb0, nk = t.nk;
         for (int i = 0; i < nk; ++i, ++it) {
           const int s = it % STAGES;
           if (it >= STAGES && !tc::mbar_wait(&empty[s], ((it / STAGES) - 1) & 1, status)) {
@@ -325,17 +389,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tc::mbar_arrive_expect_tx(&full[s], Cfg::STAGE_BYTES);
           const int k0 = (kb0 + i) * kBK;
           if (!A_MN) {
-            tc::tma_load_2d(sa, &mA, &full[s], k0, m0);
+            tc::tma_load_2d(sa, t.a, &full[s], k0, m0);
           } else {
-            tc::tma_load_2d(sa, &mA, &full[s], m0, k0);
-            tc::tma_load_2d(sa + 8192, &mA, &full[s], m0 + 64, k0);
+            tc::tma_load_2d(sa, t.a, &full[s], m0, k0);
+            tc::tma_load_2d(sa + 8192, t.a, &full[s], m0 + 64, k0);
           }
           if (!B_MN) {
-            tc::tma_load_2d(sb, &mB, &full[s], k0, n0);
+            tc::tma_load_2d(sb, t.b, &full[s], k0, n0);
           } else {
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j)
-              tc::tma_load_2d(sb + j * 8192, &mB, &full[s], n0 + 64 * j, k0);
+              tc::tma_load_2d(sb + j * 8192, t.b, &full[s], n0 + 64 * j, k0);
           }
         }
       }
@@ -349,9 +413,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       constexpr uint32_t idesc = tc::idesc_bf16(kBM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
       int it = 0, j = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++j) {
-        const int z = (tile / tiles_m) / tiles_n;
-        const int kb0 = z * kps, nk = min(nkb, kb0 + kps) - kb0;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++j) {
+        const TcTile t = tc_tile<BN>(tile, mA, mB, mC, aux, M, N, kps, nkb, tiles_m, tiles_n,
+                                     n_tiles, epi);
+        const int nk = t.nk;
         const int acc = j & 1, use = j >> 1;
         if (use > 0 && !tc::mbar_wait(&tempty[acc], (use - 1) & 1, status)) break;
         tc::fence_after_sync();
@@ -385,14 +450,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int c_beg = ((warp - 2) >> 2) * (BN / 2);
     uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
     int j = 0, nout = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++j) {
-      int m_blk, n_blk, z;
-      tile_mnz(tile, tiles_m, tiles_n, m_blk, n_blk, z);
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++j) {
+      const TcTile t = tc_tile<BN>(tile, mA, mB, mC, aux, M, N, kps, nkb, tiles_m, tiles_n,
+                                   n_tiles, epi);
+      const int z = t.z, N = t.N;
       const int acc = j & 1, use = j >> 1;
-      const int row0 = m_blk * kBM + q * 32;
+      const int row0 = t.m0 + q * 32;
       const int row = row0 + lane;
-      const int n0 = n_blk * BN;
-      const bool row_ok = row < M;
+      const int n0 = t.n0;
+      const bool row_ok = row < t.M;
+      // the output map and column of this tile (a dual epilogue's second part
+      // and a second product have their own)
+      const int soff = t.n0 - t.nc0;
+      const CUtensorMap* mo = t.c;
       // The epilogue's own inputs do not depend on the accumulator: fetch the
       // first chunk's before waiting for it, and each next chunk's one ahead.
       constexpr int NCH = BN / 64;  // 32-column chunks per epilogue warp
@@ -408,8 +478,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         float v[32];
         tc::tmem_ld32(base + (uint32_t)c, v);
         if (n0 + c < N)
-          epi_chunk(epi, &mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1],
-                    ok && row_ok, ok);
+          epi_chunk(epi, mo, sbuf, nout, lane, row, row0, n0 + c, n0 + c - soff, z, v,
+                    pre[ci & 1], ok && row_ok, ok);
       }
       tc::fence_before_sync();
       __syncwarp();
@@ -431,6 +501,24 @@ bool gemm_tc_available() { return g_tc_ok && tmap_encoder() != nullptr; }
 
 // Tensor map of an epilogue's output for its TMA stores: [splits][M][N] with
 // row stride ldo, 32 x 32 boxes (64-byte swizzle for bf16, 128-byte for fp32).
+// The second output of a dual epilogue: [M][N - n_split], row stride ldo2.
+template <class Epi>
+static bool out_map2(CUtensorMap* m, const Epi& epi, int M, int N) {
+  memset(m, 0, sizeof(*m));
+  if constexpr (!Epi::kDual) {
+    return true;
+  } else {
+    using OT = typename Epi::OutT;
+    const uint64_t es = sizeof(OT);
+    const uint64_t d[3] = {(uint64_t)(N - epi.n_split), (uint64_t)M, 1};
+    const uint64_t st[2] = {(uint64_t)epi.ldo2 * es, (uint64_t)epi.ldo2 * es * (uint64_t)M};
+    const uint32_t box[3] = {32, 32, 1};
+    return make_tmap(m, es == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                     epi.out2, 3, d, st, box,
+                     es == 2 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
+  }
+}
+
 template <class Epi>
 static bool out_map(CUtensorMap* m, const Epi& epi, int M, int N, int splits) {
   memset(m, 0, sizeof(*m));
@@ -449,30 +537,48 @@ static bool out_map(CUtensorMap* m, const Epi& epi, int M, int N, int splits) {
   }
 }
 
-template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
-static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
-                             long sak, const void* B, long sbk, long sbn, const Epi& epi,
-                             int splits, int max_ctas = 0) {
-  using Cfg = TcCfg<BN, STAGES>;
-  CUtensorMap mA, mB;
+// Operand tensor maps of the single-CTA kernel: A as 128 x 64 boxes (K-major)
+// or 64 x 64 boxes (MN-major), B as BN x 64 (K-major) or 64 x 64 (MN-major).
+template <bool A_MN>
+static bool tc_a_map(CUtensorMap* m, const void* A, int M, int K, long sam, long sak) {
   if (!A_MN) {
     uint64_t d[2] = {(uint64_t)K, (uint64_t)M}, st[1] = {(uint64_t)sam * 2};
     uint32_t box[2] = {64, 128};
-    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
-  } else {
-    uint64_t d[2] = {(uint64_t)M, (uint64_t)K}, st[1] = {(uint64_t)sak * 2};
-    uint32_t box[2] = {64, 64};
-    if (!make_tmap_bf16(&mA, A, 2, d, st, box)) return cudaErrorInvalidValue;
+    return make_tmap_bf16(m, A, 2, d, st, box);
   }
+  uint64_t d[2] = {(uint64_t)M, (uint64_t)K}, st[1] = {(uint64_t)sak * 2};
+  uint32_t box[2] = {64, 64};
+  return make_tmap_bf16(m, A, 2, d, st, box);
+}
+template <int BN, bool B_MN>
+static bool tc_b_map(CUtensorMap* m, const void* B, int N, int K, long sbk, long sbn) {
   if (!B_MN) {
     uint64_t d[2] = {(uint64_t)K, (uint64_t)N}, st[1] = {(uint64_t)sbn * 2};
     uint32_t box[2] = {64, (uint32_t)BN};
-    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
-  } else {
-    uint64_t d[2] = {(uint64_t)N, (uint64_t)K}, st[1] = {(uint64_t)sbk * 2};
-    uint32_t box[2] = {64, 64};
-    if (!make_tmap_bf16(&mB, B, 2, d, st, box)) return cudaErrorInvalidValue;
+    return make_tmap_bf16(m, B, 2, d, st, box);
   }
+  uint64_t d[2] = {(uint64_t)N, (uint64_t)K}, st[1] = {(uint64_t)sbk * 2};
+  uint32_t box[2] = {64, 64};
+  return make_tmap_bf16(m, B, 2, d, st, box);
+}
+
+// One launch of the single-CTA kernel: product 0 (M, N, K, A, B, epi), for a
+// dual epilogue the B operand b2 of its columns from epi.n_split on, and
+// optionally a second product p1 stored as bf16 after product 0's tiles
+// (plain-store epilogues only).
+template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
+static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                             long sak, const void* B, long sbk, long sbn, const Epi& epi,
+                             int splits, int max_ctas = 0, const void* b2 = nullptr,
+                             const GemmProd* p1 = nullptr) {
+  using Cfg = TcCfg<BN, STAGES>;
+  CUtensorMap mA, mB, mC;
+  TcAux aux;
+  memset(&aux, 0, sizeof(aux));
+  int nb = N;  // B columns of the first map
+  if constexpr (Epi::kDual) nb = epi.n_split;
+  if (!tc_a_map<A_MN>(&mA, A, M, K, sam, sak) || !tc_b_map<BN, B_MN>(&mB, B, nb, K, sbk, sbn))
+    return cudaErrorInvalidValue;
   const int nkb = (K + kBK - 1) / kBK;
   const int kps = (nkb + splits - 1) / splits;
   const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
@@ -480,12 +586,37 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi>;
   static std::atomic<unsigned long long> opted{0};
   if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
-  CUtensorMap mC;
-  if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
-  int grid = n_tiles < sm_count() ? n_tiles : sm_count();
+  if constexpr (Epi::kDual) {
+    // every tile lies on one side of n_split
+    if (epi.n_split % BN != 0 || epi.n_split <= 0 || epi.n_split >= N || !b2)
+      return cudaErrorInvalidValue;
+    if (!out_map(&mC, epi, M, epi.n_split, 1) || !out_map2(&aux.mC2, epi, M, N) ||
+        !tc_b_map<BN, B_MN>(&aux.mB2, b2, N - epi.n_split, K, sbk, sbn))
+      return cudaErrorInvalidValue;
+  } else {
+    if (!out_map(&mC, epi, M, N, splits)) return cudaErrorInvalidValue;
+  }
+  if (p1) {
+    if (Epi::kDual || splits != 1) return cudaErrorInvalidValue;
+    const EpiStoreF<bf16> e1{(bf16*)p1->out, p1->ldo, 0};
+    if (!tc_a_map<A_MN>(&aux.mA1, p1->A, p1->M, p1->K, p1->sam, p1->sak) ||
+        !tc_b_map<BN, B_MN>(&aux.mB1, p1->B, p1->N, p1->K, p1->sbk, p1->sbn) ||
+        !out_map(&aux.mC1, e1, p1->M, p1->N, 1))
+      return cudaErrorInvalidValue;
+    aux.has1 = 1;
+    aux.M1 = p1->M;
+    aux.N1 = p1->N;
+    aux.nkb1 = (p1->K + kBK - 1) / kBK;
+    aux.kps1 = aux.nkb1;
+    aux.tiles_m1 = (p1->M + kBM - 1) / kBM;
+    aux.tiles_n1 = (p1->N + BN - 1) / BN;
+    aux.n_tiles1 = aux.tiles_m1 * aux.tiles_n1;
+  }
+  const int total = n_tiles + (aux.has1 ? aux.n_tiles1 : 0);
+  int grid = total < sm_count() ? total : sm_count();
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   cudaError_t e = launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream, mA, mB, mC,
-                           M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, lc.status);
+                           aux, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -658,7 +789,8 @@ __device__ __forceinline__ bool tc2_epilogue(const typename Op::Epi& epi, const 
     float v[32];
     tc::tmem_ld32(base + (uint32_t)c, v);
     if (n0 + c < s.N)
-      epi_chunk(epi, mC, sbuf, nout, lane, row, row0, n0 + c, z, v, pre[ci & 1], ok && row_ok, ok);
+      epi_chunk(epi, mC, sbuf, nout, lane, row, row0, n0 + c, n0 + c, z, v, pre[ci & 1],
+                ok && row_ok, ok);
   }
   tc::fence_before_sync();
   __syncwarp();
@@ -1040,6 +1172,12 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
                                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo,
                                                                   (const bf16*)ea.w_p, ea.spart, M},
                                              1);
+      case EPI_HGATE:
+        return tc_launch<BN, ST, A_MN, B_MN>(
+            lc, M, N, K, A, sam, sak, B, sbk, sbn,
+            EpiHGateF<bf16>{(bf16*)ea.out, ea.ldo, (const bf16*)ea.w_p, ea.spart, M,
+                            (bf16*)ea.out2, ea.ldo2, ea.n_split},
+            1, 0, ea.b2);
       default:
         break;
     }
@@ -1069,6 +1207,13 @@ static cudaError_t tc_pick(const Launch& lc, int dtype_out, int M, int N, int K,
   const long tm = (M + kBM - 1) / kBM;
   const long tiles256 = tm * ((N + 255) / 256) * splits;
   const long tiles128 = tm * ((N + 127) / 128) * splits;
+  if (epi == EPI_HGATE) {  // the tile width must divide the first output's width
+    if (N % 256 == 0 && ea.n_split % 256 == 0 && tiles256 * 4 >= (long)sm_count() * 3)
+      return tc_epi<256, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
+    if (ea.n_split % 128 == 0)
+      return tc_epi<128, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
+    return tc_epi<64, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
+  }
   if (N % 256 == 0 && tiles256 * 4 >= (long)sm_count() * 3)
     return tc_epi<256, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea,
                                    splits);
@@ -1080,14 +1225,18 @@ static cudaError_t tc_pick(const Launch& lc, int dtype_out, int M, int N, int K,
   return tc_epi<128, A_MN, B_MN>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
 }
 
+// Long K or wide N: the CTA-pair kernel's 256 x 256 tiles need 2/3 of the
+// operand bytes per flop of a single CTA's 128 x 256 tile (measured faster
+// from K = 1024, or K = 768 with N >= 1024; no slower at K = 512).
+static bool store_on_pair(int M, int N, int K) {
+  return N % 256 == 0 && M >= 512 && (K >= 1024 || (K >= 768 && N >= 1024));
+}
+
 cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits) {
   if (N % 64 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
-  // long K or wide N: the CTA-pair kernel's 256 x 256 tiles need 2/3 of the
-  // operand bytes per flop of a single CTA's 128 x 256 tile (measured faster
-  // from K = 1024, or K = 768 with N >= 1024; no slower at K = 512)
-  if (epi == EPI_STORE && N % 256 == 0 && M >= 512 && (K >= 1024 || (K >= 768 && N >= 1024)))
+  if (epi == EPI_STORE && store_on_pair(M, N, K))
     return gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
   splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
   const bool a_k = (sak == 1), a_m = (sam == 1) && !a_k;
@@ -1097,6 +1246,28 @@ cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const 
   if (a_m && b_n) return tc_pick<true, true>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
   if (a_m && b_k) return tc_pick<true, false>(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, splits);
   return cudaErrorNotSupported;
+}
+
+cudaError_t gemm_tc_two(const Launch& lc, int M, int N, int K, const void* A, long sam, long sak,
+                        const void* B, long sbk, long sbn, void* out, long ldo,
+                        const GemmProd& p1) {
+  if (!gemm_tc_available()) return cudaErrorNotSupported;
+  if (N % 64 != 0 || M < 1 || K < 1 || p1.N % 64 != 0 || p1.M < 1 || p1.K < 1)
+    return cudaErrorInvalidValue;
+  // product 0 on the CTA-pair kernel, or other operand layouts: not here
+  if (store_on_pair(M, N, K) || sak != 1 || sbn != 1 || p1.sak != 1 || p1.sbn != 1)
+    return cudaErrorNotSupported;
+  const EpiStoreF<bf16> epi{(bf16*)out, ldo, 0};
+  const long tm = (M + kBM - 1) / kBM;
+  // product 0 picks the tile width, as in tc_pick
+  if (N % 256 == 0 && tm * (N / 256) * 4 >= (long)sm_count() * 3)
+    return tc_launch<256, 4, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0,
+                                          nullptr, &p1);
+  if (tm * ((N + 127) / 128) * 4 < (long)sm_count())
+    return tc_launch<64, 8, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0, nullptr,
+                                         &p1);
+  return tc_launch<128, 6, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0, nullptr,
+                                        &p1);
 }
 
 cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K, const void* A,

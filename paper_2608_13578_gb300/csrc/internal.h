@@ -23,6 +23,10 @@ enum EpiKind {
   EPI_GATE = 2,         // out = G = sigmoid(acc) in the storage dtype        (Sec. 3.8)
   EPI_ADD = 3,          // out[m*ldo + n] = acc + add[m*ldo + n] (storage dtype)
   EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
+  // columns [0, n_split): EPI_STORE_SCORE into out; columns [n_split, N):
+  // sigmoid(acc) into out2 (row stride ldo2) -- H and the gate G in one product
+  // (tcgen05 path, bf16; n_split a multiple of 64)
+  EPI_HGATE = 6,
 };
 
 struct EpiArgs {
@@ -34,9 +38,27 @@ struct EpiArgs {
   const void* w_p = nullptr;
   // EPI_ADD: the addend, same layout as out
   const void* add = nullptr;
+  // EPI_HGATE: the second output and the first column that goes to it, and
+  // the B operand of those columns (same strides as B, columns from 0)
+  void* out2 = nullptr;
+  long ldo2 = 0;
+  int n_split = 0;
+  const void* b2 = nullptr;
   // EPI_GATE on the tensor cores: at most this many persistent CTAs (0: one
   // per SM), to leave SMs to a concurrent chain of small kernels
   int max_ctas = 0;
+};
+
+// A second product of a single-CTA tcgen05 launch: out[M, N] (bf16, row
+// stride ldo) = A[M, K] B[K, N] with element strides as for gemm.
+struct GemmProd {
+  int M, N, K;
+  const void* A;
+  long sam, sak;
+  const void* B;
+  long sbk, sbn;
+  void* out;
+  long ldo;
 };
 
 // Number of non-empty K-splits when K (in 64-deep slices) is cut into
@@ -95,6 +117,13 @@ cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const 
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits);
 bool gemm_tc_available();
+// Two bf16 products in one single-CTA tcgen05 launch, both with A K-major and
+// B MN-major and plain bf16 stores: out[M, N] = A B (row stride ldo), then
+// p1's tiles in the idle slots of its last wave.  cudaErrorNotSupported when
+// product 0 belongs on the CTA-pair kernel or the layouts differ.
+cudaError_t gemm_tc_two(const Launch& lc, int M, int N, int K, const void* A, long sam, long sak,
+                        const void* B, long sbk, long sbn, void* out, long ldo,
+                        const GemmProd& p1);
 
 // Sum of `splits` fp32 partial buffers of `count` elements each, in split
 // order, stored in dtype_out.
