@@ -185,6 +185,8 @@ def kernel_model(w):
         # Sec. 3.8 injection: read H, G and C; write Y
         "inject": ("hbm", 3 * n * D * es + B * Nb * D * 4),
         "gemm_dh": g(n, D, D),
+        # dM^T = W_m dP^T with the reverse scan of Sec. 3.5 in its epilogue
+        "gemm_dm_scan": g(D, B * Nb, D),
         "gemm_dhhat": g(n, D, D),
         "gemm_dx": g(n, D, 3 * D),
         "gemm_dw_g": g(D, D, n),

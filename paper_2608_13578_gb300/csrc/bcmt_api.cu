@@ -382,7 +382,7 @@ bool fused_gate(const Geometry& g) {
 
 struct FwdWs {
   char *qkv, *hhat, *hloc, *G, *Mb, *wog;
-  float *lse, *alpha, *S, *M, *Z, *C, *spart;
+  float *lse, *alpha, *S, *M, *Z, *Zinv, *C, *spart;
   size_t bytes;
 };
 
@@ -408,6 +408,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
     // M in the storage dtype: the A operand of the memory projection (and of dW_m)
     w.Mb = g.dtype == BCMT_BF16 ? take((size_t)g.B * g.Nb * g.D * 2) : reinterpret_cast<char*>(w.M);
     w.Z = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
+    w.Zinv = reinterpret_cast<float*>(take((size_t)g.Nb * g.D * 4));
     // the K-split partials of P = M W_m (the memory rows C, before the shift)
     w.C = reinterpret_cast<float*>(take((size_t)mem_splits(g) * g.B * g.Nb * g.D * 4));
     w.G = take((size_t)g.n * g.D * g.es);
@@ -416,7 +417,7 @@ FwdWs fwd_layout(const Geometry& g, void* base) {
   } else {
     w.wog = nullptr;
     w.hloc = w.G = w.Mb = nullptr;
-    w.alpha = w.S = w.M = w.Z = w.C = w.spart = nullptr;
+    w.alpha = w.S = w.M = w.Z = w.Zinv = w.C = w.spart = nullptr;
   }
   w.bytes = off;
   return w;
@@ -732,8 +733,8 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
     pr.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, g.B,
-                        g.Nb, D);
+    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.Zinv,
+                        g.B, g.Nb, D);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "causal memory");
     {
@@ -815,22 +816,40 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "gate backward");
     // side stream: Sec. 3.5 reversed, dM = dP W_m^T and the reverse decayed
-    // scan -> dS (and the decay gradient's batch rows)
+    // scan -> dS (and the decay gradient's batch rows).  On the bf16 tensor
+    // cores without a decay gradient, when Nb divides 32, one launch computes
+    // dM transposed (dM^T = W_m dP^T: a row per channel) and its epilogue runs
+    // each channel's scan in registers; otherwise dM as K-split partials and
+    // the scan kernel.
     fork.point();
-    {
+    const bool scan_in_gemm = !d_decay && g.dtype == BCMT_BF16 && g_use_tc_gemm &&
+                              gemm_tc_available() && g.Nb <= 32 && 32 % g.Nb == 0;
+    if (scan_in_gemm) {
       EpiArgs ea;
-      ea.out = bw.dM;
+      ea.out = bw.dS;
       ea.ldo = D;
-      ea.split_stride = (long)g.B * g.Nb * D;
-      e = run_gemm(lcs, prs, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
-                   EPI_PARTIAL, ea, dm_splits(g));
-      if (e != cudaSuccess) return cuda_fail(e, "dM");
+      ea.scan_zinv = w.Zinv;
+      ea.scan_decay = decay;
+      ea.scan_nb = g.Nb;
+      e = run_gemm(lcs, prs, "gemm_dm_scan", g.dtype, 0, D, g.B * g.Nb, D, w_m, D, 1, bw.dPb, 1,
+                   D, EPI_REVSCAN, ea);
+      if (e != cudaSuccess) return cuda_fail(e, "dM and its reverse scan");
+    } else {
+      {
+        EpiArgs ea;
+        ea.out = bw.dM;
+        ea.ldo = D;
+        ea.split_stride = (long)g.B * g.Nb * D;
+        e = run_gemm(lcs, prs, "gemm_dm", g.dtype, 0, g.B * g.Nb, D, D, bw.dPb, D, 1, w_m, 1, D,
+                     EPI_PARTIAL, ea, dm_splits(g));
+        if (e != cudaSuccess) return cuda_fail(e, "dM");
+      }
+      prs.begin("memory_scan_bwd");
+      e = memory_scan_bwd(lcs, bw.dM, dm_splits(g), decay, w.Z, w.M, bw.dS,
+                          d_decay ? bw.da_part : nullptr, g.B, g.Nb, D);
+      prs.end(nullptr);
+      if (e != cudaSuccess) return cuda_fail(e, "memory backward");
     }
-    prs.begin("memory_scan_bwd");
-    e = memory_scan_bwd(lcs, bw.dM, dm_splits(g), decay, w.Z, w.M, bw.dS,
-                        d_decay ? bw.da_part : nullptr, g.B, g.Nb, D);
-    prs.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "memory backward");
     const int scan_done = fork.mark();
     // side stream, then: dW_m = M^T dP and dW_g = H^T dU
     {
@@ -864,8 +883,8 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     // and dH += alpha dS + ds w_p
     fork.wait_mark(scan_done);
     pr.begin("summary_bwd");
-    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, w.S, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part, g.B,
-                    g.T, D, g.L);
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, w.S, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part,
+                    g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");
     fork.point();

@@ -24,6 +24,7 @@ struct EpiStoreF {
   using OutT = TO;
   static constexpr bool kTma = true;
   static constexpr bool kDual = false;
+  static constexpr bool kWarpWide = false;
   TO* out;
   long ldo;
   long split_stride;
@@ -54,6 +55,7 @@ struct EpiStoreScoreF {
   using OutT = TO;
   static constexpr bool kTma = true;
   static constexpr bool kDual = false;
+  static constexpr bool kWarpWide = false;
   static constexpr long split_stride = 0;
   TO* out;
   long ldo;
@@ -101,6 +103,7 @@ struct EpiGateF {
   using OutT = T;
   static constexpr bool kTma = true;
   static constexpr bool kDual = false;
+  static constexpr bool kWarpWide = false;
   static constexpr long split_stride = 0;
   T* out;
   long ldo;
@@ -136,6 +139,7 @@ struct EpiHGateF {
   using OutT = TO;
   static constexpr bool kTma = true;
   static constexpr bool kDual = true;
+  static constexpr bool kWarpWide = false;
   static constexpr long split_stride = 0;
   TO* out;
   long ldo;
@@ -172,6 +176,53 @@ struct EpiHGateF {
   __device__ __forceinline__ void operator()(int, int, const float*, int, int) const {}
 };
 
+// Sec. 3.5 reversed inside the memory-gradient product, computed transposed:
+// dM^T = W_m dP^T, so that an output row is one channel c and its columns
+// are the blocks (b, i) in order (column b*Nb + i).  The epilogue turns each
+// batch's run of Nb columns into the summary gradients
+//   dS_i = sum_{j>=i} a^(j-i) dM_j / Z_j,  i.e. R_i = dM_i / Z_i + a R_{i+1},
+// the backward of M_i = N_i / Z_i, N_i = a N_{i-1} + S_i, with a the channel's
+// decay: a thread's 32 columns hold 32 / Nb whole batches (Nb divides 32), so
+// the recurrence runs in its registers, block Nb-1 down to 0.  It stores dS
+// [B*Nb, ldo] row-major itself (lanes are consecutive channels: coalesced).
+// Zinv [Nb, ldo] holds 1 / Z_i (written by the forward's scan).
+struct EpiRevScanT {
+  using Pre = NoPre;
+  using OutT = float;
+  static constexpr bool kTma = false;
+  static constexpr bool kDual = false;
+  static constexpr bool kWarpWide = false;
+  static constexpr long split_stride = 0;
+  float* out;           // dS [ncols, ldo]
+  long ldo;             // D
+  const float* Zinv;    // [Nb, ldo]
+  const float* decay;   // [ldo]
+  int Nb;
+  int ncols;            // B * Nb
+  __device__ __forceinline__ void load(int, int, Pre&) const {}
+  __device__ __forceinline__ void apply(int row, int col, float* v, const Pre&, int) const {
+    // Nb divides 32 (a power of two) and col is a multiple of 32, so column
+    // col + e is block (e & (Nb - 1)) of its batch; all loads go out first
+    const int msk = Nb - 1;
+    float zi[32];
+#pragma unroll
+    for (int e = 0; e < 32; ++e) zi[e] = Zinv[(long)(e & msk) * ldo + row];
+    const float a = decay[row];
+    float R = 0.f;
+#pragma unroll
+    for (int e = 31; e >= 0; --e) {
+      if ((e & msk) == msk) R = 0.f;  // a batch's last block starts its run
+      R = fmaf(a, R, v[e] * zi[e]);
+      v[e] = R;
+    }
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      if (col + e < ncols) out[(long)(col + e) * ldo + row] = v[e];
+  }
+  // the SIMT GEMM does not take this epilogue
+  __device__ __forceinline__ void operator()(int, int, const float*, int, int) const {}
+};
+
 // out = acc + add, same row-major layout (e.g. dU W_g^T + dY: the identity
 // path of Y = H + ... joins the gate path's gradient).
 template <class T>
@@ -183,6 +234,7 @@ struct EpiAddF {
   using OutT = T;
   static constexpr bool kTma = true;
   static constexpr bool kDual = false;
+  static constexpr bool kWarpWide = false;
   static constexpr long split_stride = 0;
   const T* add;
   T* out;

@@ -197,7 +197,8 @@ __device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC,
                                           const typename Epi::Pre& pre, bool apply, bool store) {
   if constexpr (Epi::kTma) {
     using OT = typename Epi::OutT;
-    if (apply) epi.apply(row, col, v, pre, z);
+    // a warp-wide epilogue (lane shuffles) runs on every lane of a valid tile
+    if (Epi::kWarpWide ? store : apply) epi.apply(row, col, v, pre, z);
     constexpr bool kBf = sizeof(OT) == 2;
     uint8_t* buf = sbuf + (kBf ? (nout & 1) * 2048 : 0);
     if (lane == 0) {
@@ -275,8 +276,9 @@ constexpr int kGemmThreads = 320;
 //    of the columns from epi.n_split on (their own tensors, columns counted
 //    from n_split);
 //  * a second product with the same operand layouts and a plain store
-//    epilogue (has1): its n_tiles1 tiles follow product 0's in the round-robin
-//    order, so a small product fills the idle slots of a large one's last wave.
+//    epilogue of its own (has1, the kernel's Epi1): its n_tiles1 tiles follow
+//    product 0's in the round-robin order, so a small product fills the idle
+//    slots of a large one's last wave.
 struct TcAux {
   CUtensorMap mB2, mC2;
   CUtensorMap mA1, mB1, mC1;
@@ -289,6 +291,7 @@ struct TcAux {
 struct TcTile {
   const CUtensorMap *a, *b, *c;
   int M, N, m0, n0, nb0, nc0, z, kb0, nk;
+  bool p1;  // a tile of the second product
 };
 template <int BN, class Epi>
 __device__ __forceinline__ TcTile tc_tile(int tile, const CUtensorMap& mA, const CUtensorMap& mB,
@@ -302,6 +305,7 @@ __device__ __forceinline__ TcTile tc_tile(int tile, const CUtensorMap& mA, const
   const int ks = p1 ? aux.kps1 : kps, nb = p1 ? aux.nkb1 : nkb;
   int m_blk, n_blk;
   tile_mnz(tl, tm, tn, m_blk, n_blk, t.z);
+  t.p1 = p1;
   t.a = p1 ? &aux.mA1 : &mA;
   t.b = p1 ? &aux.mB1 : &mB;
   t.c = p1 ? &aux.mC1 : &mC;
@@ -322,12 +326,49 @@ __device__ __forceinline__ TcTile tc_tile(int tile, const CUtensorMap& mA, const
   return t;
 }
 
-template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
+// One tile's epilogue (warps 2..9): warp w reads TMEM lanes 32*(w%4) .. +31
+// and the columns of half (w-2)/4 of the tile, transforms and stores them.
+template <int BN, class Epi>
+__device__ __forceinline__ bool tc_epilogue(const Epi& epi, const TcTile& t, int warp, int lane,
+                                            uint32_t tmem, int acc, int use, uint64_t* tfull,
+                                            uint8_t* sbuf, int& nout, unsigned* status) {
+  const int q = warp & 3;
+  const int c_beg = ((warp - 2) >> 2) * (BN / 2);
+  const int z = t.z, N = t.N;
+  const int row0 = t.m0 + q * 32;
+  const int row = row0 + lane;
+  const int n0 = t.n0;
+  const bool row_ok = row < t.M;
+  // the output map and column of this tile (a dual epilogue's second part
+  // and a second product have their own)
+  const int soff = t.n0 - t.nc0;
+  // The epilogue's own inputs do not depend on the accumulator: fetch the
+  // first chunk's before waiting for it, and each next chunk's one ahead.
+  constexpr int NCH = BN / 64;  // 32-column chunks per epilogue warp
+  typename Epi::Pre pre[2];
+  if (row_ok && n0 + c_beg < N) epi.load(row, n0 + c_beg, pre[0]);
+  const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
+  tc::fence_after_sync();
+  const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll
+  for (int ci = 0; ci < NCH; ++ci) {
+    const int c = c_beg + ci * 32;
+    if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
+    float v[32];
+    tc::tmem_ld32(base + (uint32_t)c, v);
+    if (n0 + c < N)
+      epi_chunk(epi, t.c, sbuf, nout, lane, row, row0, n0 + c, n0 + c - soff, z, v, pre[ci & 1],
+                ok && row_ok, ok);
+  }
+  return ok;
+}
+
+template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi, class Epi1 = EpiStoreF<bf16>>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mC, const __grid_constant__ TcAux aux,
                    int M, int N, int kps, int nkb, int tiles_m, int tiles_n, int n_tiles, Epi epi,
-                   unsigned* status) {
+                   Epi1 epi1, unsigned* status) {
   const int total = n_tiles + (aux.has1 ? aux.n_tiles1 : 0);
   using Cfg = TcCfg<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
@@ -444,43 +485,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
   } else {
-    // ---- epilogue warps 2..9: warp w reads TMEM lanes 32*(w%4) .. +31 and
-    // the columns of half (w-2)/4 of the tile
-    const int q = warp & 3;
-    const int c_beg = ((warp - 2) >> 2) * (BN / 2);
+    // ---- epilogue warps 2..9 (tc_epilogue), the second product's tiles
+    // through its own epilogue
     uint8_t* sbuf = smem + Cfg::OUT_OFF + (warp - 2) * kOutStage;
     int j = 0, nout = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++j) {
       const TcTile t = tc_tile<BN>(tile, mA, mB, mC, aux, M, N, kps, nkb, tiles_m, tiles_n,
                                    n_tiles, epi);
-      const int z = t.z, N = t.N;
       const int acc = j & 1, use = j >> 1;
-      const int row0 = t.m0 + q * 32;
-      const int row = row0 + lane;
-      const int n0 = t.n0;
-      const bool row_ok = row < t.M;
-      // the output map and column of this tile (a dual epilogue's second part
-      // and a second product have their own)
-      const int soff = t.n0 - t.nc0;
-      const CUtensorMap* mo = t.c;
-      // The epilogue's own inputs do not depend on the accumulator: fetch the
-      // first chunk's before waiting for it, and each next chunk's one ahead.
-      constexpr int NCH = BN / 64;  // 32-column chunks per epilogue warp
-      typename Epi::Pre pre[2];
-      if (row_ok && n0 + c_beg < N) epi.load(row, n0 + c_beg, pre[0]);
-      const bool ok = tc::mbar_wait(&tfull[acc], use & 1, status);
-      tc::fence_after_sync();
-      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-#pragma unroll
-      for (int ci = 0; ci < NCH; ++ci) {
-        const int c = c_beg + ci * 32;
-        if (ci + 1 < NCH && row_ok && n0 + c + 32 < N) epi.load(row, n0 + c + 32, pre[(ci + 1) & 1]);
-        float v[32];
-        tc::tmem_ld32(base + (uint32_t)c, v);
-        if (n0 + c < N)
-          epi_chunk(epi, mo, sbuf, nout, lane, row, row0, n0 + c, n0 + c - soff, z, v,
-                    pre[ci & 1], ok && row_ok, ok);
-      }
+      const bool ok = t.p1 ? tc_epilogue<BN>(epi1, t, warp, lane, tmem, acc, use, tfull, sbuf,
+                                             nout, status)
+                           : tc_epilogue<BN>(epi, t, warp, lane, tmem, acc, use, tfull, sbuf,
+                                             nout, status);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&tempty[acc]);
@@ -566,11 +582,11 @@ static bool tc_b_map(CUtensorMap* m, const void* B, int N, int K, long sbk, long
 // dual epilogue the B operand b2 of its columns from epi.n_split on, and
 // optionally a second product p1 stored as bf16 after product 0's tiles
 // (plain-store epilogues only).
-template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi>
+template <int BN, int STAGES, bool A_MN, bool B_MN, class Epi, class Epi1 = EpiStoreF<bf16>>
 static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* A, long sam,
                              long sak, const void* B, long sbk, long sbn, const Epi& epi,
                              int splits, int max_ctas = 0, const void* b2 = nullptr,
-                             const GemmProd* p1 = nullptr) {
+                             const GemmProd* p1 = nullptr, const Epi1& epi1 = Epi1{}) {
   using Cfg = TcCfg<BN, STAGES>;
   CUtensorMap mA, mB, mC;
   TcAux aux;
@@ -583,7 +599,7 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   const int kps = (nkb + splits - 1) / splits;
   const int tiles_m = (M + kBM - 1) / kBM, tiles_n = (N + BN - 1) / BN;
   const int n_tiles = tiles_m * tiles_n * splits;
-  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi>;
+  auto kern = gemm_tc_kernel<BN, STAGES, A_MN, B_MN, Epi, Epi1>;
   static std::atomic<unsigned long long> opted{0};
   if (cudaError_t e = smem_opt_in(kern, Cfg::SMEM, &opted); e != cudaSuccess) return e;
   if constexpr (Epi::kDual) {
@@ -598,10 +614,9 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   }
   if (p1) {
     if (Epi::kDual || splits != 1) return cudaErrorInvalidValue;
-    const EpiStoreF<bf16> e1{(bf16*)p1->out, p1->ldo, 0};
     if (!tc_a_map<A_MN>(&aux.mA1, p1->A, p1->M, p1->K, p1->sam, p1->sak) ||
         !tc_b_map<BN, B_MN>(&aux.mB1, p1->B, p1->N, p1->K, p1->sbk, p1->sbn) ||
-        !out_map(&aux.mC1, e1, p1->M, p1->N, 1))
+        !out_map(&aux.mC1, epi1, p1->M, p1->N, 1))
       return cudaErrorInvalidValue;
     aux.has1 = 1;
     aux.M1 = p1->M;
@@ -616,7 +631,7 @@ static cudaError_t tc_launch(const Launch& lc, int M, int N, int K, const void* 
   int grid = total < sm_count() ? total : sm_count();
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   cudaError_t e = launch_k(kern, dim3(grid), dim3(kGemmThreads), Cfg::SMEM, lc.stream, mA, mB, mC,
-                           aux, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, lc.status);
+                           aux, M, N, kps, nkb, tiles_m, tiles_n, n_tiles, epi, epi1, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -1187,6 +1202,10 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,
           EpiAddF<bf16>{(const bf16*)ea.add, (bf16*)ea.out, ea.ldo}, 1);
+    if (epi == EPI_REVSCAN)
+      return tc_launch<BN, ST, A_MN, B_MN>(
+          lc, M, N, K, A, sam, sak, B, sbk, sbn,
+          EpiRevScanT{(float*)ea.out, ea.ldo, ea.scan_zinv, ea.scan_decay, ea.scan_nb, N}, 1);
   }
   return cudaErrorNotSupported;
 }
@@ -1235,7 +1254,10 @@ static bool store_on_pair(int M, int N, int K) {
 cudaError_t gemm_tc(const Launch& lc, int dtype_out, int M, int N, int K, const void* A, long sam,
                     long sak, const void* B, long sbk, long sbn, EpiKind epi, const EpiArgs& ea,
                     int splits) {
-  if (N % 64 != 0 || M < 1 || K < 1) return cudaErrorInvalidValue;
+  if (M < 1 || K < 1) return cudaErrorInvalidValue;
+  // the scan epilogue takes any column count (B*Nb); the others multiples of 64
+  if (N % 64 != 0 && epi != EPI_REVSCAN) return cudaErrorInvalidValue;
+  if (epi == EPI_REVSCAN && (ea.scan_nb < 1 || 32 % ea.scan_nb != 0)) return cudaErrorInvalidValue;
   if (epi == EPI_STORE && store_on_pair(M, N, K))
     return gemm_tc_pair(lc, dtype_out, M, N, K, A, sam, sak, B, sbk, sbn, epi, ea, 1);
   splits = (epi == EPI_PARTIAL) ? effective_splits(K, splits) : 1;
@@ -1258,16 +1280,17 @@ cudaError_t gemm_tc_two(const Launch& lc, int M, int N, int K, const void* A, lo
   if (store_on_pair(M, N, K) || sak != 1 || sbn != 1 || p1.sak != 1 || p1.sbn != 1)
     return cudaErrorNotSupported;
   const EpiStoreF<bf16> epi{(bf16*)out, ldo, 0};
+  const EpiStoreF<bf16> epi1{(bf16*)p1.out, p1.ldo, 0};
   const long tm = (M + kBM - 1) / kBM;
   // product 0 picks the tile width, as in tc_pick
   if (N % 256 == 0 && tm * (N / 256) * 4 >= (long)sm_count() * 3)
     return tc_launch<256, 4, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0,
-                                          nullptr, &p1);
+                                          nullptr, &p1, epi1);
   if (tm * ((N + 127) / 128) * 4 < (long)sm_count())
     return tc_launch<64, 8, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0, nullptr,
-                                         &p1);
+                                         &p1, epi1);
   return tc_launch<128, 6, false, true>(lc, M, N, K, A, sam, sak, B, sbk, sbn, epi, 1, 0, nullptr,
-                                        &p1);
+                                        &p1, epi1);
 }
 
 cudaError_t gemm(const Launch& lc, int dtype, int dtype_out, int M, int N, int K, const void* A,

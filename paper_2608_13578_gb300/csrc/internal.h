@@ -23,6 +23,10 @@ enum EpiKind {
   EPI_GATE = 2,         // out = G = sigmoid(acc) in the storage dtype        (Sec. 3.8)
   EPI_ADD = 3,          // out[m*ldo + n] = acc + add[m*ldo + n] (storage dtype)
   EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
+  // the memory-gradient product dM^T = W_m dP^T [D, B*Nb] turned into its
+  // reverse decayed scan dS [B*Nb, D] (fp32, row stride ldo) by the epilogue:
+  // scan_nb divides 32, scan_zinv [scan_nb, D] = 1 / Z, scan_decay [D]
+  EPI_REVSCAN = 7,
   // columns [0, n_split): EPI_STORE_SCORE into out; columns [n_split, N):
   // sigmoid(acc) into out2 (row stride ldo2) -- H and the gate G in one product
   // (tcgen05 path, bf16; n_split a multiple of 64)
@@ -44,6 +48,10 @@ struct EpiArgs {
   long ldo2 = 0;
   int n_split = 0;
   const void* b2 = nullptr;
+  // EPI_REVSCAN
+  const float* scan_zinv = nullptr;
+  const float* scan_decay = nullptr;
+  int scan_nb = 0;
   // EPI_GATE on the tensor cores: at most this many persistent CTAs (0: one
   // per SM), to leave SMs to a concurrent chain of small kernels
   int max_ctas = 0;
@@ -185,12 +193,12 @@ cudaError_t attn_bwd_fl(const Launch& lc, const AttnBwdArgs& a);
 cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float* spart, int npart,
                         float* alpha, float* S, int B, int T, int D, int L);
 // Sec. 3.5: M = normalised decayed scan of S over blocks (fp32, plus a bf16
-// copy in Mb when non-null), Z its denominator [Nb, D].  The projection
+// copy in Mb when non-null), Z its denominator [Nb, D] and Zinv = 1 / Z.  The projection
 // P = M W_m is a K-split GEMM whose psplits fp32 partials [psplits][B*Nb][D]
 // the injection and the gate backward sum, with the shift C_0 = 0,
 // C_i = P_{i-1}, as they read them.
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, int B, int Nb, int D);
+                            void* Mb, float* Z, float* Zinv, int B, int Nb, int D);
 // Backward of the gate and injection: dU = dY*C*G*(1-G) (C from the partials
 // Pm of P = M W_m); dP[b,i-1] = sum over block i of dY*G (also in bf16 in dPb
 // when non-null); dP[b,Nb-1] = 0.

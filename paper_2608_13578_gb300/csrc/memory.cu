@@ -588,13 +588,14 @@ __global__ void __launch_bounds__(kThreads)
 // over blocks in batches of kScanU whose loads all go out before the first
 // step.  kScanThreads threads per CTA spread the B * D chains over many SMs.
 // Writes M in fp32 and, when Mb is non-null, in bf16 (the A operand of the
-// tensor-core projection), and Z (batch 0 only: it does not depend on b).
+// tensor-core projection), and Z and 1 / Z (batch 0 only: they do not depend
+// on b).
 constexpr int kScanThreads = 64;
 constexpr int kScanU = 16;
 __global__ void __launch_bounds__(kScanThreads)
     memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
-                           int Nb, int D) {
+                           float* __restrict__ Zinv, int Nb, int D) {
   pdl_enter();
   const int c = blockIdx.x * kScanThreads + threadIdx.x, b = blockIdx.y;
   if (c >= D) return;
@@ -614,7 +615,10 @@ __global__ void __launch_bounds__(kScanThreads)
         const float m = Nn / Zz;
         M[base + (long)i * D] = m;
         if (Mb) Mb[base + (long)i * D] = __float2bfloat16_rn(m);
-        if (b == 0) Z[(long)i * D + c] = Zz;
+        if (b == 0) {
+          Z[(long)i * D + c] = Zz;
+          Zinv[(long)i * D + c] = 1.0f / Zz;
+        }
       }
     }
   }
@@ -737,10 +741,10 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 }
 
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
-                            void* Mb, float* Z, int B, int Nb, int D) {
+                            void* Mb, float* Z, float* Zinv, int B, int Nb, int D) {
   dim3 grid((D + kScanThreads - 1) / kScanThreads, B);
   cudaError_t e = launch_k(memory_scan_fwd_kernel, grid, dim3(kScanThreads), 0, lc.stream, S,
-                           decay, M, (bf16*)Mb, Z, Nb, D);
+                           decay, M, (bf16*)Mb, Z, Zinv, Nb, D);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 

@@ -54,11 +54,14 @@ def oracle_run(w: Workload, t_cpu: dict, backward: bool = True, batch=None):
     return fw, gr
 
 
-def gpu_run(w: Workload, t_dev: dict, backward: bool = True):
+def gpu_run(w: Workload, t_dev: dict, backward: bool = True, decay_grad: bool = False):
+    """Forward (and backward) through the C ABI.  Without decay_grad the
+    backward runs as in training with the paper's fixed decay (the benchmark's
+    launch sequence); with it the decay gradient d_decay is returned too."""
     from paper_2608_13578_gb300 import layer
     p = layer.params_for(w.B, w.T, w.D, w.H, w.L, w.dtype, w.input_is_x, w.honly,
                          flags=layer.C.BCMT_FLAG_CHECK)
     y, ws = layer.forward(p, t_dev)
-    g = layer.backward(p, t_dev, ws, t_dev["dy"], decay_grad=True) if backward else None
+    g = layer.backward(p, t_dev, ws, t_dev["dy"], decay_grad=decay_grad) if backward else None
     torch.cuda.synchronize()
     return y, g

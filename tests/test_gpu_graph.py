@@ -21,11 +21,12 @@ def _run(C, p, t, ws, sc, y, g, stream=None):
                    t["w_g"], t["decay"], y, ws, stream)
     C.bcmt_backward(p, t["dy"], t["x"], None, None, t["w_qkv"], t["w_o"], t["w_p"], t["w_m"],
                     t["w_g"], t["decay"], ws, sc, g["dx"], None, None, g["dw_qkv"], g["dw_o"],
-                    g["dw_p"], g["dw_m"], g["dw_g"], stream, g["d_decay"])
+                    g["dw_p"], g["dw_m"], g["dw_g"], stream, g.get("d_decay"))
 
 
+@pytest.mark.parametrize("decay_grad", [False, True], ids=["fixed_decay", "decay_grad"])
 @pytest.mark.parametrize("L", [64, 256])
-def test_graph_replay_matches_direct_calls(cuda_ok, L):
+def test_graph_replay_matches_direct_calls(cuda_ok, L, decay_grad):
     from paper_2608_13578_gb300 import bcmt as C
     from paper_2608_13578_gb300 import layer
     w = Workload("graph", 2, 512, 256, 4, L, "bf16", True, (0.5, 0.99), 41)
@@ -34,8 +35,9 @@ def test_graph_replay_matches_direct_calls(cuda_ok, L):
     ws = torch.empty(C.bcmt_workspace_size(p), dtype=torch.uint8, device="cuda")
     sc = torch.empty(C.bcmt_scratch_size(p), dtype=torch.uint8, device="cuda")
     y = torch.empty_like(t["x"])
-    g = {"dx": torch.empty_like(t["x"]), "dw_qkv": torch.empty_like(t["w_qkv"]),
-         "d_decay": torch.empty_like(t["decay"])}
+    g = {"dx": torch.empty_like(t["x"]), "dw_qkv": torch.empty_like(t["w_qkv"])}
+    if decay_grad:
+        g["d_decay"] = torch.empty_like(t["decay"])
     for n in ("w_o", "w_p", "w_m", "w_g"):
         g["d" + n] = torch.empty_like(t[n])
     s = torch.cuda.Stream()

@@ -57,14 +57,17 @@ VARIANTS = [
 ]
 
 
-def _check(w: Workload, backward=True):
+def _check(w: Workload, backward=True, decay_grad=False):
     t = make_inputs(w)
-    y, g = gpu_run(w, to_device(t), backward)
+    y, g = gpu_run(w, to_device(t), backward, decay_grad)
     fw, gr = oracle_run(w, t, backward)
     assert_close("Y", y, fw["Y"], w.dtype)
     if backward:
         names = GRAD_NAMES_X if w.input_is_x else GRAD_NAMES_QKV
         for n in names:
+            if n == "d_decay" and not decay_grad:
+                assert n not in g
+                continue
             got = g[n]
             if w.honly and n in ("dw_p", "dw_m", "dw_g", "d_decay"):
                 assert torch.count_nonzero(got).item() == 0
@@ -72,9 +75,20 @@ def _check(w: Workload, backward=True):
             assert_close(n, got, gr[n], w.dtype)
 
 
-@pytest.mark.parametrize("w", SMALL + VARIANTS, ids=lambda w: w.name + ("_qkv" if not w.input_is_x else "") + ("_honly" if w.honly else ""))
+def _wid(w):
+    return w.name + ("_qkv" if not w.input_is_x else "") + ("_honly" if w.honly else "")
+
+
+@pytest.mark.parametrize("w", SMALL + VARIANTS, ids=_wid)
 def test_layer_small(cuda_ok, w):
     _check(w)
+
+
+@pytest.mark.parametrize("w", SMALL + VARIANTS, ids=_wid)
+def test_layer_small_decay_grad(cuda_ok, w):
+    """The same layers with the learned-decay gradient requested (the memory
+    gradient then takes the separate reverse-scan kernel)."""
+    _check(w, decay_grad=True)
 
 
 def test_tensor_core_and_simt_paths_agree(cuda_ok):
@@ -90,7 +104,7 @@ def test_tensor_core_and_simt_paths_agree(cuda_ok):
     y1, g1 = gpu_run(w, t)
     scale = y0.float().abs().max().item()
     assert (y0.float() - y1.float()).abs().max().item() / scale < 2e-2
-    for n in GRAD_NAMES_X:
+    for n in g0:
         s = g0[n].float().abs().max().item()
         assert (g0[n].float() - g1[n].float()).abs().max().item() / s < 2e-2, n
 
@@ -101,7 +115,7 @@ def test_deterministic(cuda_ok):
     y0, g0 = gpu_run(w, t)
     y1, g1 = gpu_run(w, t)
     assert torch.equal(y0, y1)
-    for n in GRAD_NAMES_X:
+    for n in g0:
         assert torch.equal(g0[n], g1[n]), n
 
 
@@ -122,10 +136,11 @@ def test_causality_bitwise(cuda_ok):
 
 
 # ------------------------------------------------- the named workloads, full size
+@pytest.mark.parametrize("decay_grad", [False, True], ids=["fixed_decay", "decay_grad"])
 @pytest.mark.parametrize("name", ["fwd_fp32_b1_t256_l32_d128_h4", "fwdbwd_bf16_b8_t1024_l64_d512_h8"])
-def test_workload_full(cuda_ok, name):
+def test_workload_full(cuda_ok, name, decay_grad):
     w = WORKLOADS[name]
-    _check(w, backward=True)
+    _check(w, backward=True, decay_grad=decay_grad)
 
 
 @pytest.mark.parametrize("L", [32, 64, 128, 256])
@@ -139,7 +154,8 @@ def test_sequence_scaling(cuda_ok, T):
     every output and gradient against the oracle: the weight gradients reduce
     over K = B*T up to 65536 tokens with their own split counts, and the
     reverse scan of Sec. 3.5 runs N_b up to 128 dependent steps."""
-    _check(WORKLOADS[f"seqscale_bf16_b4_t{T}_l128_d1024_h16"], backward=True)
+    _check(WORKLOADS[f"seqscale_bf16_b4_t{T}_l128_d1024_h16"], backward=True,
+           decay_grad=T == 16384)
 
 
 @pytest.mark.parametrize("L", [256, 512])
