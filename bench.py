@@ -205,6 +205,10 @@ def kernel_model(w):
         "attn_bwd_fl": ("hbm", 5 * n * D * es + n * H * 4 + 3 * n * D * es + 2 * n * H * 4),
         # Sec. 3.4 summaries: read H and the score partials, write alpha and S
         "summary_fwd": ("hbm", n * D * es + n * 4 * npart + n * 4 + B * Nb * D * 4),
+        # Sec. 3.5 scan with the projection P = M W_m (warp-level mma): read S and
+        # W_m, write P, M (fp32 and bf16), Z and 1/Z
+        "memory_proj_fwd": ("hbm", B * Nb * D * 4 + D * D * es + B * Nb * D * (4 + 4 + 2)
+                            + 2 * Nb * D * 4),
         # Sec. 3.5 scan: read S, write M (fp32 and the bf16 operand copy) and Z
         "memory_scan_fwd": ("hbm", B * Nb * D * (4 + 4 + 2) + Nb * D * 4),
         "gemm_wm": g(B * Nb, D, D),
@@ -213,9 +217,9 @@ def kernel_model(w):
         "gemm_dm": g(B * Nb, D, D),
         # reverse scan: read dM and Z, write dS
         "memory_scan_bwd": ("hbm", 2 * B * Nb * D * 4 + Nb * D * 4),
-        # pooling backward: read H, alpha and dS; write ds and the dW_p partials;
-        # complete dH in place (read and write)
-        "summary_bwd": ("hbm", 3 * n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
+        # pooling backward: read H, dY, alpha and dS; write ds and the dW_p
+        # partials; complete dH in place (read and write)
+        "summary_bwd": ("hbm", 4 * n * D * es + 2 * n * 4 + 2 * B * Nb * D * 4),
         "gemm_dwm": g(D, D, B * Nb),
         "reduce_rows": ("hbm", B * Nb * D * 4 + D * es),
     }

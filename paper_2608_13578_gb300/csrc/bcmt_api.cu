@@ -369,7 +369,15 @@ int dqkv_splits(const Geometry& g) {
 // all of M); the consumers sum the fp32 partials as they read them.  dM runs
 // beside dH = dY + dU W_g^T, which holds most SMs: two splits, so that its
 // CTAs fit in the SMs left over.
-int mem_splits(const Geometry& g) { return effective_splits(g.D, 4); }
+// The forward memory scan and its D x D projection in one launch
+// (memory_proj_fwd, warp-level mma) when the shape is small enough; else the
+// scan kernel and the tcgen05 projection.
+bool mem_fused(const Geometry& g) {
+  return !g.honly && g_use_tc_gemm && memory_proj_fits(g.dtype, g.B, g.Nb, g.D);
+}
+// fp32 partials of P = M W_m that the memory row's readers sum (one when the
+// fused kernel computes P whole)
+int mem_splits(const Geometry& g) { return mem_fused(g) ? 1 : effective_splits(g.D, 4); }
 int dm_splits(const Geometry& g) { return effective_splits(g.D, 2); }
 
 // The forward's output projection and gate share one product,
@@ -732,12 +740,19 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
     e = summary_fwd(lc, g.dtype, w.hloc, w.spart, npart, w.alpha, w.S, g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "block summaries");
-    pr.begin("memory_scan_fwd");
-    e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z, w.Zinv,
-                        g.B, g.Nb, D);
-    pr.end(nullptr);
-    if (e != cudaSuccess) return cuda_fail(e, "causal memory");
-    {
+    if (mem_fused(g)) {
+      // the scan and P = M W_m in one launch (P whole; the shift is applied
+      // by the readers)
+      pr.begin("memory_proj_fwd");
+      e = memory_proj_fwd(lc, w.S, decay, w_m, w.C, w.M, w.Mb, w.Z, w.Zinv, g.B, g.Nb, D);
+      pr.end(nullptr);
+      if (e != cudaSuccess) return cuda_fail(e, "causal memory and its projection");
+    } else {
+      pr.begin("memory_scan_fwd");
+      e = memory_scan_fwd(lc, w.S, decay, w.M, g.dtype == BCMT_BF16 ? w.Mb : nullptr, w.Z,
+                          w.Zinv, g.B, g.Nb, D);
+      pr.end(nullptr);
+      if (e != cudaSuccess) return cuda_fail(e, "causal memory");
       // P = M W_m as K-split partials; the shift is applied by the readers
       EpiArgs ea;
       ea.out = w.C;
@@ -869,13 +884,15 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
                       2.0 * D * D * (double)g.n <= 32e9 ? device_sms() / 8 : 0);
       if (e != cudaSuccess) return cuda_fail(e, "dW_g");
     }
-    // main stream, meanwhile: dH = dY + dU W_g^T (the identity and gate paths)
+    // main stream, meanwhile: dH = dU W_g^T (the gate path; the identity
+    // path's dY is added by the pooling backward)
     {
+      // (the identity path's dY is added by the pooling backward, which
+      // reads and writes every row of dH anyway)
       EpiArgs ea;
       ea.out = bw.dH;
       ea.ldo = D;
-      ea.add = dy;
-      e = run_gemm(lc, pr, "gemm_dh", g.dtype, g.dtype, n, D, D, bw.dU, D, 1, w_g, 1, D, EPI_ADD,
+      e = run_gemm(lc, pr, "gemm_dh", g.dtype, g.dtype, n, D, D, bw.dU, D, 1, w_g, 1, D, EPI_STORE,
                    ea);
       if (e != cudaSuccess) return cuda_fail(e, "dH");
     }
@@ -883,7 +900,7 @@ bcmt_status bcmt_backward(const bcmt_params* p, const void* dy, const void* x_or
     // and dH += alpha dS + ds w_p
     fork.wait_mark(scan_done);
     pr.begin("summary_bwd");
-    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, w.S, bw.dS, w_p, bw.dH, bw.ds, bw.dwp_part,
+    e = summary_bwd(lc, g.dtype, w.hloc, w.alpha, w.S, bw.dS, w_p, dy, bw.dH, bw.ds, bw.dwp_part,
                     g.B, g.T, D, g.L);
     pr.end(nullptr);
     if (e != cudaSuccess) return cuda_fail(e, "summary backward");

@@ -223,47 +223,4 @@ struct EpiRevScanT {
   __device__ __forceinline__ void operator()(int, int, const float*, int, int) const {}
 };
 
-// out = acc + add, same row-major layout (e.g. dU W_g^T + dY: the identity
-// path of Y = H + ... joins the gate path's gradient).
-template <class T>
-struct EpiAddF {
-  // tcgen05 path (bf16 only): the addend as raw bf16 pairs
-  struct Pre {
-    uint4 a[4];
-  };
-  using OutT = T;
-  static constexpr bool kTma = true;
-  static constexpr bool kDual = false;
-  static constexpr bool kWarpWide = false;
-  static constexpr long split_stride = 0;
-  const T* add;
-  T* out;
-  long ldo;
-  __device__ __forceinline__ void load(int row, int col, Pre& pre) const {
-    const bf16* a = reinterpret_cast<const bf16*>(add) + (long)row * ldo + col;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) load8_raw(a + 8 * j, pre.a[j]);
-  }
-  __device__ __forceinline__ void apply(int, int, float* v, const Pre& pre, int) const {
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      float a[8];
-      unpack8(pre.a[q], a);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) v[8 * q + e] += a[e];
-    }
-  }
-  __device__ __forceinline__ void operator()(int row, int col, const float* v, int n, int) const {
-    const long o = (long)row * ldo + col;
-    float a[32];
-    for (int j = 0; j < n; j += 4) load4(add + o + j, a + j);
-    for (int j = 0; j < n; ++j) a[j] += v[j];
-    if (n % 8 == 0) {
-      for (int j = 0; j < n; j += 8) store8(out + o + j, a + j);
-    } else {
-      for (int j = 0; j < n; j += 4) store4(out + o + j, a + j);
-    }
-  }
-};
-
 }  // namespace bcmt

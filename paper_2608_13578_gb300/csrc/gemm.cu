@@ -127,9 +127,6 @@ static cudaError_t simt_typed(const Launch& lc, int dtype_out, int M, int N, int
                              EpiStoreScoreF<bf16>{(bf16*)ea.out, ea.ldo, (const bf16*)ea.w_p,
                                                   ea.spart, M},
                              1);
-    case EPI_ADD:
-      return simt_launch<TI>(lc, M, N, K, A, sam, sak, B, sbk, sbn,
-                             EpiAddF<TI>{(const TI*)ea.add, (TI*)ea.out, ea.ldo}, 1);
   }
   return cudaErrorInvalidValue;
 }
@@ -208,6 +205,7 @@ __device__ __forceinline__ void epi_chunk(const Epi& epi, const CUtensorMap* mC,
         tc::tma_store_wait_read<0>();
     }
     __syncwarp();
+
     if (kBf) {
 #pragma unroll
       for (int u = 0; u < 4; ++u)
@@ -1198,10 +1196,6 @@ static cudaError_t tc_epi(const Launch& lc, int dtype_out, int M, int N, int K, 
     }
   }
   if constexpr (!A_MN && !B_MN) {
-    if (epi == EPI_ADD)
-      return tc_launch<BN, ST, A_MN, B_MN>(
-          lc, M, N, K, A, sam, sak, B, sbk, sbn,
-          EpiAddF<bf16>{(const bf16*)ea.add, (bf16*)ea.out, ea.ldo}, 1);
     if (epi == EPI_REVSCAN)
       return tc_launch<BN, ST, A_MN, B_MN>(
           lc, M, N, K, A, sam, sak, B, sbk, sbn,

@@ -21,7 +21,6 @@ enum EpiKind {
   EPI_STORE = 0,        // out[m*ldo + n] = acc                       (out dtype = dtype_out)
   EPI_PARTIAL = 1,      // out(fp32)[z*split_stride + m*ldo + n] = acc of K-split z
   EPI_GATE = 2,         // out = G = sigmoid(acc) in the storage dtype        (Sec. 3.8)
-  EPI_ADD = 3,          // out[m*ldo + n] = acc + add[m*ldo + n] (storage dtype)
   EPI_STORE_SCORE = 5,  // EPI_STORE, plus spart[col/n][m] = sum over the n columns of acc * w_p
   // the memory-gradient product dM^T = W_m dP^T [D, B*Nb] turned into its
   // reverse decayed scan dS [B*Nb, D] (fp32, row stride ldo) by the epilogue:
@@ -40,8 +39,6 @@ struct EpiArgs {
   // EPI_STORE_SCORE: partial pooling scores, [D / n, M] fp32, and w_p
   float* spart = nullptr;
   const void* w_p = nullptr;
-  // EPI_ADD: the addend, same layout as out
-  const void* add = nullptr;
   // EPI_HGATE: the second output and the first column that goes to it, and
   // the B operand of those columns (same strides as B, columns from 0)
   void* out2 = nullptr;
@@ -199,6 +196,14 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 // C_i = P_{i-1}, as they read them.
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
                             void* Mb, float* Z, float* Zinv, int B, int Nb, int D);
+// Sec. 3.5 and the projection P = M W_m in one launch (bf16; P unshifted, one
+// split [B*Nb, D]; also M, Mb, Z, Zinv), for shapes memory_proj_fits accepts
+// (a batch's memory rows and a weight chunk in one CTA's shared memory, a
+// small projection).
+bool memory_proj_fits(int dtype, int B, int Nb, int D);
+cudaError_t memory_proj_fwd(const Launch& lc, const float* S, const float* decay, const void* Wm,
+                            float* P, float* M, void* Mb, float* Z, float* Zinv, int B, int Nb,
+                            int D);
 // Backward of the gate and injection: dU = dY*C*G*(1-G) (C from the partials
 // Pm of P = M W_m); dP[b,i-1] = sum over block i of dY*G (also in bf16 in dPb
 // when non-null); dP[b,Nb-1] = 0.
@@ -215,11 +220,12 @@ cudaError_t memory_scan_bwd(const Launch& lc, const float* dM, int msplits, cons
 // summary_bwd_chunks(dtype, L, D) x Nb x B): g_t = H_t . dS_blk,
 // ds_t = alpha_t (g_t - S_blk . dS_blk) (Sb: the forward's summaries),
 // dwp_part[(b*Nb + i) * chunks + c] = sum over the chunk of ds_t H_t, and
-// dH_t += alpha_t dS_blk + ds_t w_p in place.
+// dH_t += dY_t + alpha_t dS_blk + ds_t w_p in place (dH holds dU W_g^T: the
+// identity path's dY joins here).
 int summary_bwd_chunks(int dtype, int L, int D);
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
-                        float* dwp_part, int B, int T, int D, int L);
+                        const float* Sb, const float* dS, const void* w_p, const void* dY,
+                        void* dH, float* ds, float* dwp_part, int B, int T, int D, int L);
 // Sec. 3.7-3.8 injection: Y = H + G * C[b, t / L], C from the psplits
 // partials Pm of P = M W_m (shifted by one block, C_0 = 0).
 cudaError_t inject(const Launch& lc, int dtype, const void* Hm, const void* G, const float* Pm,

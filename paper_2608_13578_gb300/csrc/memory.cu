@@ -5,6 +5,7 @@
 // Every kernel reads rows with 16-byte vector loads, issues a batch's loads
 // before its first use, and reduces in a fixed order (deterministic).
 #include <algorithm>
+#include <atomic>
 
 #include <type_traits>
 
@@ -17,6 +18,21 @@ namespace {
 constexpr int kMaxL = 1024;
 constexpr int kThreads = 256;
 }  // namespace
+
+// 16-byte global -> shared copies that hold no registers while in flight
+// (cp.async, cached in L2 only); a thread waits for its own copies.
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(smem_dst)),
+               "l"(gmem_src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
 
 // ======================================================== work items (device)
 // Four or eight consecutive values of a row, held as loaded: bf16 stays packed
@@ -344,7 +360,8 @@ __device__ void scan_bwd_item(const float* dM, long mstride,
 template <class T, int ROWS>
 __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
                                  const float* __restrict__ alpha, const float* __restrict__ Sb,
-                                 const float* dS, const T* __restrict__ w_p, T* dH,
+                                 const float* dS, const T* __restrict__ w_p,
+                                 const T* __restrict__ dY, T* dH,
                                  float* __restrict__ ds_out, float* __restrict__ dwp_part,
                                  int Tlen, int D, int L, int Nb, int c, int i, int b) {
   float* g = sm;                  // [ROWS]
@@ -403,6 +420,7 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
   __syncthreads();
   const int rg = warp, co = lane;
   T* dHb = dH + ((long)b * Tlen + t0) * D;
+  const T* dYb = dY + ((long)b * Tlen + t0) * D;
   const long prow = ((long)b * Nb + i) * ((L + ROWS - 1) / ROWS) + c;
   for (int c0 = 0; c0 < D; c0 += 256) {
     const int k = c0 + co * 8;
@@ -412,12 +430,13 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
       load8_cg(dSi + k, sv);
       load8(w_p + k, wp);
       // rows rg, rg+8: all their loads before the first store
-      float h[RW][8], d[RW][8];
+      float h[RW][8], d[RW][8], yv[RW][8];
 #pragma unroll
       for (int u = 0; u < RW; ++u)
         if (rg + 8 * u < n) {
           load8(Hb + (long)(rg + 8 * u) * D + k, h[u]);
           load8(dHb + (long)(rg + 8 * u) * D + k, d[u]);
+          load8(dYb + (long)(rg + 8 * u) * D + k, yv[u]);
         }
 #pragma unroll
       for (int u = 0; u < RW; ++u)
@@ -426,7 +445,7 @@ __device__ void summary_bwd_item(float* sm, const T* __restrict__ Hm,
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             acc[e] = fmaf(w, h[u][e], acc[e]);
-            d[u][e] += a * sv[e] + w * wp[e];
+            d[u][e] += yv[u][e] + a * sv[e] + w * wp[e];
           }
           store8(dHb + (long)(rg + 8 * u) * D + k, d[u]);
         }
@@ -457,8 +476,9 @@ template <int RW, int KC>
 __global__ void __launch_bounds__(kThreads, 2)
     summary_bwd_reg_kernel(const bf16* __restrict__ Hm, const float* __restrict__ alpha,
                            const float* __restrict__ Sb, const float* dS,
-                           const bf16* __restrict__ w_p, bf16* dH, float* __restrict__ ds_out,
-                           float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
+                           const bf16* __restrict__ w_p, const bf16* __restrict__ dY, bf16* dH,
+                           float* __restrict__ ds_out, float* __restrict__ dwp_part, int Tlen,
+                           int D, int L, int Nb) {
   pdl_enter();
   constexpr int ROWS = 8 * RW;
   constexpr int PW = KC * 256 + 4;  // row-group stride of the dW_p partials
@@ -478,6 +498,11 @@ __global__ void __launch_bounds__(kThreads, 2)
   const long rowbase = (long)b * Tlen + t0;
   const bf16* Hb = Hm + rowbase * D;
   bf16* dHb = dH + rowbase * D;
+  const bf16* dYb = dY + rowbase * D;
+  // dY goes straight to shared memory (cp.async: no registers held while it
+  // is in flight), each thread's own pieces, read back by the same thread
+  extern __shared__ __align__(16) uint8_t ys_raw[];  // [8 RW rows][KC * 256] bf16
+  bf16* ys = reinterpret_cast<bf16*>(ys_raw);
   uint4 h[RW][KC], d[RW][KC];
 #pragma unroll
   for (int u = 0; u < RW; ++u)
@@ -486,10 +511,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       const int k = 256 * j + 8 * lane;
       if (warp + 8 * u < n && k < D) {
         const long o = (long)(warp + 8 * u) * D + k;
+        cp_async16(ys + ((warp + 8 * u) * KC + j) * 256 + 8 * lane, dYb + o);
         load8_raw(Hb + o, h[u][j]);
         load8_raw(dHb + o, d[u][j]);
       }
     }
+  cp_async_commit();
   float a[RW];
 #pragma unroll
   for (int u = 0; u < RW; ++u) a[u] = (warp + 8 * u < n) ? alpha[rowbase + warp + 8 * u] : 0.f;
@@ -534,26 +561,31 @@ __global__ void __launch_bounds__(kThreads, 2)
     dsr[u] = a[u] * (g - cd);
     if (lane == 0 && warp + 8 * u < n) ds_out[rowbase + warp + 8 * u] = dsr[u];
   }
-  // dH_t += alpha_t dS_i + ds_t w_p; the chunk's dW_p partial sum_t ds_t H_t
+  // dH_t = dY_t + (dU W_g^T)_t + alpha_t dS_i + ds_t w_p (the identity, gate
+  // and pooling paths); the chunk's dW_p partial sum_t ds_t H_t
 #pragma unroll
   for (int j = 0; j < KC; ++j) {
     const int k = 256 * j + 8 * lane;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (j == 0) cp_async_wait_all();  // this thread's dY pieces have landed
     if (k < D) {
 #pragma unroll
       for (int u = 0; u < RW; ++u)
         if (warp + 8 * u < n) {
-          float hv[8], dv[8];
+          float hv[8], dv[8], yv[8];
           unpack8(h[u][j], hv);
           unpack8(d[u][j], dv);
+          unpack8(*reinterpret_cast<const uint4*>(ys + ((warp + 8 * u) * KC + j) * 256 + 8 * lane),
+                  yv);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             acc[e] = fmaf(dsr[u], hv[e], acc[e]);
-            dv[e] += a[u] * dss[k + e] + dsr[u] * wps[k + e];
+            dv[e] += yv[e] + a[u] * dss[k + e] + dsr[u] * wps[k + e];
           }
           store8(dHb + (long)(warp + 8 * u) * D + k, dv);
         }
     }
+
 #pragma unroll
     for (int e = 0; e < 8; ++e) part[warp * PW + 256 * j + 8 * lane + e] = acc[e];
   }
@@ -624,6 +656,204 @@ __global__ void __launch_bounds__(kScanThreads)
   }
 }
 
+// ------------------------------------------------ warp-level bf16 products
+// The memory's D x D projections at small shapes are [B*Nb, D] x [D, D]: a
+// few tens of MFLOP, far too little for the tcgen05 GEMM's launch and ring
+// fill.  Here one CTA per (column chunk, batch) multiplies the batch's Nb
+// memory rows by a 32-column chunk of the weight with mma.sync m16n8k16
+// (bf16 operands from shared memory through ldmatrix, fp32 accumulators):
+// warp w takes columns 8 (w % 4) .. +7 and half w / 4 of the K range, and the
+// two halves are added through shared memory.  Operand rows are padded by 8
+// elements so that the 8 rows an ldmatrix reads fall in distinct banks.
+// Copies rows of 16-byte pieces from global to shared memory, all threads of
+// the CTA, up to eight loads of a thread in flight before their stores.
+// copy_rows16<P>: `rows` rows of P pieces (src row stride lds elements, dst ldd).
+// copy_rows16v: `rows` rows of `pieces` pieces, rows past `rows` up to `rows_pad`
+// zero-filled.
+template <int NT = kThreads>
+__device__ __forceinline__ void copy_rows16v(bf16* dst, int ldd, const bf16* src, long lds,
+                                             int rows, int pieces, int rows_pad) {
+  const int total = rows_pad * pieces;
+  for (int o0 = threadIdx.x; o0 < total; o0 += 8 * NT) {
+    uint4 v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int o = o0 + j * NT;
+      const int r = o / pieces, c = o % pieces;
+      v[j] = make_uint4(0u, 0u, 0u, 0u);
+      if (o < total && r < rows) v[j] = *reinterpret_cast<const uint4*>(src + r * lds + 8 * c);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int o = o0 + j * NT;
+      if (o < total)
+        *reinterpret_cast<uint4*>(dst + (long)(o / pieces) * ldd + 8 * (o % pieces)) = v[j];
+    }
+  }
+}
+template <int P, int NT = kThreads>
+__device__ __forceinline__ void copy_rows16(bf16* dst, int ldd, const bf16* src, long lds,
+                                            int rows) {
+  copy_rows16v<NT>(dst, ldd, src, lds, rows, P, rows);
+}
+
+constexpr int kProjNC = 32;   // output columns per CTA
+constexpr int kProjPad = 8;   // bf16 elements of padding per shared-memory row
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r[0]), "=r"(r[1])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r[0]), "=r"(r[1])
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, const uint32_t* b) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+// One warp's 16 x 8 product over K range [k0, k1) (multiples of 16): A rows
+// r0 .. r0+15 of a row-major [.., lda] bf16 tile (K contiguous); B either
+// [K][ldb] with N contiguous (kBT = false: ldmatrix .trans) or [N][ldb] with
+// K contiguous (kBT = true), columns n0 .. n0+7.  acc: the mma C fragment.
+template <bool kBT>
+__device__ __forceinline__ void warp_mma_16x8(const bf16* A, int lda, int r0, const bf16* Bm,
+                                              int ldb, int n0, int k0, int k1, float* acc) {
+  const int lane = threadIdx.x & 31;
+  const int mi = lane >> 3, rr = lane & 7;
+  const uint32_t a_base = (uint32_t)__cvta_generic_to_shared(
+      A + (long)(r0 + rr + 8 * (mi & 1)) * lda + 8 * (mi >> 1));
+  // lanes 0-7 address B's k rows k .. k+7, lanes 8-15 rows k+8 .. k+15
+  // (kBT: n rows n0 .. n0+7 at k and k+8)
+  const int bl = lane & 15;
+  const uint32_t b_base = kBT ? (uint32_t)__cvta_generic_to_shared(
+                                    Bm + (long)(n0 + (bl & 7)) * ldb + 8 * (bl >> 3))
+                              : (uint32_t)__cvta_generic_to_shared(Bm + (long)bl * ldb + n0);
+  for (int k = k0; k < k1; k += 16) {
+    uint32_t a[4], b[2];
+    ldsm_x4(a_base + (uint32_t)(k * 2), a);
+    if (kBT)
+      ldsm_x2(b_base + (uint32_t)(k * 2), b);
+    else
+      ldsm_x2_t(b_base + (uint32_t)((long)k * ldb * 2), b);
+    mma_bf16_16816(acc, a, b);
+  }
+}
+
+// Sec. 3.5 and the memory projection in one launch (bf16), for shapes whose
+// memory fits one CTA's shared memory: item (x, b) = output columns
+// kProjNC*x .. kProjNC*x + kProjNC-1 of batch b, kProjThreads threads.  The
+// weight chunk W_m[:, x] is fetched before the wait for the previous kernel
+// (it is an input, not a product of the step).  The CTA runs the decayed scan
+// of every channel over the batch's Nb blocks (thread t: channels t,
+// t + kProjThreads; N_i = a N_{i-1} + S_i, Z_i = a Z_{i-1} + 1,
+// M_i = N_i * (1 / Z_i)) into shared memory as bf16 (the operand the
+// tensor-core path uses too), then P_i[c] = sum_k M_i[k] W_m[k][c] on the
+// tensor cores: warp w takes columns 8 (w % 4) .. +7 and K quarter w / 4, the
+// quarters added in order.  x == 0 also stores M (fp32 and bf16) and, for
+// batch 0, Z and 1/Z.  P is stored unshifted [B*Nb, D]: its readers take
+// C_i = P_{i-1}, C_0 = 0.
+constexpr int kProjThreads = 512;
+constexpr int kProjKQ = kProjThreads / 32 / 4;  // K ranges per column group
+__global__ void __launch_bounds__(kProjThreads)
+    memory_proj_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
+                           const bf16* __restrict__ Wm, float* __restrict__ P,
+                           float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
+                           float* __restrict__ Zinv, int Nb, int D) {
+  extern __shared__ __align__(16) uint8_t smb[];
+  const int Nr = (Nb + 15) & ~15;            // rows padded to the mma's 16
+  const int lda = D + kProjPad, ldw = kProjNC + kProjPad;
+  bf16* Ws = reinterpret_cast<bf16*>(smb);                         // [D][ldw]
+  bf16* Ms = Ws + (long)D * ldw;                                   // [Nr][lda]
+  float* red = reinterpret_cast<float*>(Ms + (long)Nr * lda);      // [KQ-1][4][16][8]
+  const int x = blockIdx.x, b = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the weight chunk: D rows of kProjNC columns (16 bytes per load, a batch
+  // of loads in flight before their shared-memory stores)
+  copy_rows16<kProjNC / 8, kProjThreads>(Ws, ldw, Wm + x * kProjNC, D, D);
+  pdl_enter();
+#pragma unroll 1
+  for (int k = threadIdx.x; k < D; k += kProjThreads) {
+    const float a = decay[k];
+    float Nn = 0.f, Zz = 0.f;
+#pragma unroll 1
+    for (int i0 = 0; i0 < Nr; i0 += 16) {
+      float sv[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        sv[u] = (i0 + u < Nb) ? S[((long)b * Nb + i0 + u) * D + k] : 0.f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int i = i0 + u;
+        bf16 mb = __float2bfloat16_rn(0.f);
+        if (i < Nb) {
+          Nn = fmaf(a, Nn, sv[u]);
+          Zz = fmaf(a, Zz, 1.0f);
+          const float zi = __frcp_rn(Zz);
+          const float m = Nn * zi;
+          mb = __float2bfloat16_rn(m);
+          if (x == 0) {
+            const long o = ((long)b * Nb + i) * D + k;
+            M[o] = m;
+            Mb[o] = mb;
+            if (b == 0) {
+              Z[(long)i * D + k] = Zz;
+              Zinv[(long)i * D + k] = zi;
+            }
+          }
+        }
+        Ms[(long)i * lda + k] = mb;
+      }
+    }
+  }
+  __syncthreads();
+  // warp w: columns 8 (w & 3) .. +7, K range w >> 2 of kProjKQ
+  const int n0 = 8 * (warp & 3), kq = warp >> 2, kr = D / kProjKQ;
+  const int fr = lane >> 2, fc = 2 * (lane & 3);
+  for (int r0 = 0; r0 < Nr; r0 += 16) {
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    warp_mma_16x8<false>(Ms, lda, r0, Ws, ldw, n0, kq * kr, (kq + 1) * kr, acc);
+    // C fragment: rows r0 + lane/4 (+8), columns n0 + 2 (lane % 4) (+1)
+    if (kq > 0) {
+      float* rw = red + (((kq - 1) * 4 + (warp & 3)) * 16) * 8;
+      rw[fr * 8 + fc] = acc[0];
+      rw[fr * 8 + fc + 1] = acc[1];
+      rw[(fr + 8) * 8 + fc] = acc[2];
+      rw[(fr + 8) * 8 + fc + 1] = acc[3];
+    }
+    __syncthreads();
+    if (kq == 0) {
+#pragma unroll
+      for (int q = 1; q < kProjKQ; ++q) {
+        const float* rw = red + (((q - 1) * 4 + (warp & 3)) * 16) * 8;
+        acc[0] += rw[fr * 8 + fc];
+        acc[1] += rw[fr * 8 + fc + 1];
+        acc[2] += rw[(fr + 8) * 8 + fc];
+        acc[3] += rw[(fr + 8) * 8 + fc + 1];
+      }
+      const long base = ((long)b * Nb + r0) * D + x * kProjNC + n0 + fc;
+      if (r0 + fr < Nb) {
+        P[base + (long)fr * D] = acc[0];
+        P[base + (long)fr * D + 1] = acc[1];
+      }
+      if (r0 + fr + 8 < Nb) {
+        P[base + (long)(fr + 8) * D] = acc[2];
+        P[base + (long)(fr + 8) * D + 1] = acc[3];
+      }
+    }
+    __syncthreads();
+  }
+}
+
 template <class T, int PS>
 __global__ void __launch_bounds__(kThreads, 2)
     gate_bwd_kernel(const T* __restrict__ dY, const T* __restrict__ G,
@@ -650,8 +880,9 @@ template <class T, int ROWS>
 __global__ void __launch_bounds__(kThreads, 2)
     summary_bwd_kernel(const T* __restrict__ Hm, const float* __restrict__ alpha,
                        const float* __restrict__ Sb, const float* __restrict__ dS,
-                       const T* __restrict__ w_p, T* dH, float* __restrict__ ds,
-                       float* __restrict__ dwp_part, int Tlen, int D, int L, int Nb) {
+                       const T* __restrict__ w_p, const T* __restrict__ dY, T* dH,
+                       float* __restrict__ ds, float* __restrict__ dwp_part, int Tlen, int D,
+                       int L, int Nb) {
   pdl_enter();
   __shared__ __align__(16) float sm[ROWS + 8 + 8 * 260];
   // a ragged last block has fewer chunks than the grid's x extent: its empty
@@ -661,7 +892,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
     return;
   }
-  summary_bwd_item<T, ROWS>(sm, Hm, alpha, Sb, dS, w_p, dH, ds, dwp_part, Tlen, D, L, Nb,
+  summary_bwd_item<T, ROWS>(sm, Hm, alpha, Sb, dS, w_p, dY, dH, ds, dwp_part, Tlen, D, L, Nb,
                             blockIdx.x, blockIdx.y, blockIdx.z);
 }
 
@@ -748,6 +979,37 @@ cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// The one-CTA-per-(column chunk, batch) memory kernel holds a batch's memory
+// rows and a weight chunk in shared memory and runs the D x D projection with
+// warp-level bf16 mma: taken for bf16 when that fits and the projection is
+// small (B*Nb*D*D <= 2^28 multiply-adds), where the tcgen05 GEMM's launch and
+// ring fill would dominate.
+constexpr int kProjSmemMax = 200 * 1024;
+static size_t proj_fwd_smem(int Nb, int D) {
+  const size_t Nr = (size_t)((Nb + 15) & ~15);
+  return ((size_t)D * (kProjNC + kProjPad) + Nr * (D + kProjPad)) * 2 +
+         (size_t)(kProjKQ - 1) * 4 * 16 * 8 * 4;
+}
+bool memory_proj_fits(int dtype, int B, int Nb, int D) {
+  return dtype == 1 && D % 64 == 0 && D % (16 * kProjKQ) == 0 &&
+         proj_fwd_smem(Nb, D) <= (size_t)kProjSmemMax &&
+         (double)B * Nb * D * D <= (double)(1 << 28);
+}
+
+cudaError_t memory_proj_fwd(const Launch& lc, const float* S, const float* decay, const void* Wm,
+                            float* P, float* M, void* Mb, float* Z, float* Zinv, int B, int Nb,
+                            int D) {
+  if (!memory_proj_fits(1, B, Nb, D) || !Mb) return cudaErrorInvalidValue;
+  // the limit is raised once per kernel and device, to the largest size any
+  // accepted shape needs
+  static std::atomic<unsigned long long> opted{0};
+  cudaError_t e = smem_opt_in(memory_proj_fwd_kernel, kProjSmemMax, &opted);
+  if (e != cudaSuccess) return e;
+  e = launch_k(memory_proj_fwd_kernel, dim3(D / kProjNC, B), dim3(kProjThreads), proj_fwd_smem(Nb, D),
+               lc.stream, S, decay, (const bf16*)Wm, P, M, (bf16*)Mb, Z, Zinv, Nb, D);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 cudaError_t gate_bwd(const Launch& lc, int dtype, const void* dY, const void* G, const float* Pm,
                      int psplits, void* dU, float* dP, void* dPb, int B, int T, int D, int L) {
   const int Nb = (T + L - 1) / L;
@@ -796,8 +1058,8 @@ int summary_bwd_chunks(int dtype, int L, int D) {
 }
 
 cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float* alpha,
-                        const float* Sb, const float* dS, const void* w_p, void* dH, float* ds,
-                        float* dwp_part, int B, int T, int D, int L) {
+                        const float* Sb, const float* dS, const void* w_p, const void* dY,
+                        void* dH, float* ds, float* dwp_part, int B, int T, int D, int L) {
   if (L > kMaxL) return cudaErrorInvalidValue;
   const int Nb = (T + L - 1) / L;
   dim3 grid(summary_bwd_chunks(dtype, L, D), Nb, B);
@@ -807,23 +1069,33 @@ cudaError_t summary_bwd(const Launch& lc, int dtype, const void* Hm, const float
     const bf16 *H = (const bf16*)Hm, *wp = (const bf16*)w_p;
     bf16* dh = (bf16*)dH;
     const int kc = (D + 255) / 256;
-#define BCMT_SBWD(RW_, KC_)                                                                   \
-  launch_k(summary_bwd_reg_kernel<RW_, KC_>, grid, dim3(kThreads), 0, lc.stream, H, alpha, Sb, \
-           dS, wp, dh, ds, dwp_part, T, D, L, Nb)
-    e = kc == 1 ? BCMT_SBWD(8, 1) : kc == 2 ? BCMT_SBWD(4, 2) : kc == 3 ? BCMT_SBWD(2, 3)
-                                                                  : BCMT_SBWD(2, 4);
-#undef BCMT_SBWD
+    auto go = [&](auto rw, auto kcc) -> cudaError_t {
+      constexpr int RW_ = decltype(rw)::value, KC_ = decltype(kcc)::value;
+      // the dY staging buffer (dynamic shared memory beside the static arrays)
+      constexpr int ys_bytes = 8 * RW_ * KC_ * 256 * 2;
+      static std::atomic<unsigned long long> opted{0};
+      cudaError_t r = smem_opt_in(summary_bwd_reg_kernel<RW_, KC_>, ys_bytes, &opted);
+      if (r != cudaSuccess) return r;
+      return launch_k(summary_bwd_reg_kernel<RW_, KC_>, grid, dim3(kThreads), ys_bytes, lc.stream,
+                      H, alpha, Sb, dS, wp, (const bf16*)dY, dh, ds, dwp_part, T, D, L, Nb);
+    };
+    using I1 = std::integral_constant<int, 1>;
+    using I2 = std::integral_constant<int, 2>;
+    using I3 = std::integral_constant<int, 3>;
+    using I4 = std::integral_constant<int, 4>;
+    using I8 = std::integral_constant<int, 8>;
+    e = kc == 1 ? go(I8(), I1()) : kc == 2 ? go(I4(), I2()) : kc == 3 ? go(I2(), I3()) : go(I2(), I4());
     return e != cudaSuccess ? e : cudaGetLastError();
   }
   auto go = [&](auto rows) {
     constexpr int R = decltype(rows)::value;
     if (dtype == 0)
       return launch_k(summary_bwd_kernel<float, R>, grid, dim3(kThreads), 0, lc.stream,
-                      (const float*)Hm, alpha, Sb, dS, (const float*)w_p, (float*)dH, ds,
-                      dwp_part, T, D, L, Nb);
+                      (const float*)Hm, alpha, Sb, dS, (const float*)w_p, (const float*)dY,
+                      (float*)dH, ds, dwp_part, T, D, L, Nb);
     return launch_k(summary_bwd_kernel<bf16, R>, grid, dim3(kThreads), 0, lc.stream,
-                    (const bf16*)Hm, alpha, Sb, dS, (const bf16*)w_p, (bf16*)dH, ds, dwp_part, T,
-                    D, L, Nb);
+                    (const bf16*)Hm, alpha, Sb, dS, (const bf16*)w_p, (const bf16*)dY, (bf16*)dH,
+                    ds, dwp_part, T, D, L, Nb);
   };
   e = summary_bwd_rows(dtype, D) == 32 ? go(std::integral_constant<int, 32>())
                                        : go(std::integral_constant<int, 16>());
