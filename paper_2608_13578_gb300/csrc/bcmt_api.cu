@@ -643,8 +643,12 @@ bcmt_status bcmt_forward(const bcmt_params* p, const void* x, const void* q, con
   if (g.from_x) {
     e = cudaErrorNotSupported;
     if (fuse) {
+      // on CTA pairs (256 x 256 tiles: 2/3 of a single CTA's operand bytes
+      // per flop) when both widths allow, else the single-CTA kernel
       pr.begin("gemm_qkv_wog");
-      e = gemm_tc_two(lc, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1, w.qkv, 3 * D, wog);
+      e = gemm_tc_pair_two(lc, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1, w.qkv, 3 * D, wog);
+      if (e == cudaErrorNotSupported)
+        e = gemm_tc_two(lc, n, 3 * D, D, x, D, 1, w_qkv, 3 * D, 1, w.qkv, 3 * D, wog);
       pr.end(nullptr);
       wog_done = e == cudaSuccess;
     }

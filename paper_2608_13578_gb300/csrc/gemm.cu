@@ -1087,6 +1087,46 @@ cudaError_t gemm_tc_pair_group(const Launch& lc, const PairProduct& p0, const Pa
   return tc2_run<256, ST, ACC, Op0, Op1>(lc, P);
 }
 
+// Two bf16 products with A K-major, B MN-major and plain bf16 stores in one
+// CTA-pair launch (256 x 256 tiles, both N multiples of 256): product 0
+// out[M, N] = A B, then p1; the items are scheduled longest first onto the
+// least loaded pair (equal lengths: an even deal).
+cudaError_t gemm_tc_pair_two(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                             long sak, const void* B, long sbk, long sbn, void* out, long ldo,
+                             const GemmProd& p1) {
+  if (!gemm_tc_available()) return cudaErrorNotSupported;
+  if (N % 256 != 0 || p1.N % 256 != 0 || sak != 1 || sbn != 1 || p1.sak != 1 || p1.sbn != 1)
+    return cudaErrorNotSupported;
+  if (M < 1 || K < 1 || p1.M < 1 || p1.K < 1) return cudaErrorInvalidValue;
+  constexpr int ST = 6, ACC = 2;
+  using Op = Tc2Op<false, true, EpiStoreF<bf16>>;
+  Tc2Params<Op, Op> P;
+  memset(&P, 0, sizeof(P));
+  P.epi0 = EpiStoreF<bf16>{(bf16*)out, ldo, 0};
+  P.epi1[0] = EpiStoreF<bf16>{(bf16*)p1.out, p1.ldo, 0};
+  if (!tc2_operand_maps<256, false, true>(&P.map[0][0], &P.map[0][1], M, N, K, A, sam, sak, B,
+                                          sbk, sbn) ||
+      !out_map(&P.map[0][2], P.epi0, M, N, 1) ||
+      !tc2_operand_maps<256, false, true>(&P.map[1][0], &P.map[1][1], p1.M, p1.N, p1.K, p1.A,
+                                          p1.sam, p1.sak, p1.B, p1.sbk, p1.sbn) ||
+      !out_map(&P.map[1][2], P.epi1[0], p1.M, p1.N, 1))
+    return cudaErrorInvalidValue;
+  P.shape[0] = tc2_shape<256>(M, N, K, 1);
+  P.shape[1] = tc2_shape<256>(p1.M, p1.N, p1.K, 1);
+  P.count = 2;
+  std::vector<std::vector<int>> lists;
+  if (tc2_group_schedule(P.shape, P.count, sm_count() / 2, &lists, nullptr)) {
+    P.npairs_sched = (int)lists.size();
+    int k = 0;
+    for (int q = 0; q < P.npairs_sched; ++q) {
+      P.start[q] = (uint16_t)k;
+      for (int item : lists[q]) P.list[k++] = (uint16_t)item;
+    }
+    P.start[P.npairs_sched] = (uint16_t)k;
+  }
+  return tc2_run<256, ST, ACC, Op, Op>(lc, P);
+}
+
 // Cost of one item of a CTA-pair product in 64-deep K slices of a 256 x 256
 // tile, plus kTc2ItemOverhead for its share of pipeline fill and epilogue.
 constexpr int kTc2ItemOverhead = 4;

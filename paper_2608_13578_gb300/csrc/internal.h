@@ -130,6 +130,11 @@ cudaError_t gemm_tc_two(const Launch& lc, int M, int N, int K, const void* A, lo
                         const void* B, long sbk, long sbn, void* out, long ldo,
                         const GemmProd& p1);
 
+// The same two products in one CTA-pair launch (both N multiples of 256).
+cudaError_t gemm_tc_pair_two(const Launch& lc, int M, int N, int K, const void* A, long sam,
+                             long sak, const void* B, long sbk, long sbn, void* out, long ldo,
+                             const GemmProd& p1);
+
 // Sum of `splits` fp32 partial buffers of `count` elements each, in split
 // order, stored in dtype_out.
 cudaError_t reduce_splits(const Launch& lc, const float* part, int splits, long count, int dtype_out,

@@ -981,9 +981,10 @@ cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay
 
 // The one-CTA-per-(column chunk, batch) memory kernel holds a batch's memory
 // rows and a weight chunk in shared memory and runs the D x D projection with
-// warp-level bf16 mma: taken for bf16 when that fits and the projection is
-// small (B*Nb*D*D <= 2^28 multiply-adds), where the tcgen05 GEMM's launch and
-// ring fill would dominate.
+// warp-level bf16 mma: taken for bf16 when that fits, Nb <= 16 (one row group
+// of the mma) and the projection is small (B*Nb*D*D <= 2^28 multiply-adds),
+// where the tcgen05 GEMM's launch and ring fill would dominate (measured: at
+// Nb = 32, D = 1024 the scan kernel and tcgen05 projection were faster).
 constexpr int kProjSmemMax = 200 * 1024;
 static size_t proj_fwd_smem(int Nb, int D) {
   const size_t Nr = (size_t)((Nb + 15) & ~15);
@@ -991,7 +992,7 @@ static size_t proj_fwd_smem(int Nb, int D) {
          (size_t)(kProjKQ - 1) * 4 * 16 * 8 * 4;
 }
 bool memory_proj_fits(int dtype, int B, int Nb, int D) {
-  return dtype == 1 && D % 64 == 0 && D % (16 * kProjKQ) == 0 &&
+  return dtype == 1 && D % 64 == 0 && D % (16 * kProjKQ) == 0 && Nb <= 16 &&
          proj_fwd_smem(Nb, D) <= (size_t)kProjSmemMax &&
          (double)B * Nb * D * D <= (double)(1 << 28);
 }
