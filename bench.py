@@ -387,17 +387,45 @@ def bench_ours(args):
     # that streams its batches would; the compute of a step is the two C-ABI
     # calls recorded once per buffer pair as a CUDA graph, as such a loop
     # would record its step.
-    x_h = t_cpu["x"].pin_memory()
-    dy_h = t_cpu["dy"].pin_memory()
-    outs_h = {"y": torch.empty_like(t_cpu["x"]).pin_memory()}
-    for n, g_ in grads.items():
-        outs_h[n] = torch.empty(g_.shape, dtype=g_.dtype).pin_memory()
-    x_d = [torch.empty_like(t["x"]) for _ in range(2)]
-    dy_d = [torch.empty_like(t["dy"]) for _ in range(2)]
-    y_d = [torch.empty_like(t["x"]) for _ in range(2)]
-    g_d = [{n: torch.empty_like(g_) for n, g_ in grads.items()} for _ in range(2)]
-    h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
-    d2h = sum(v.numel() * v.element_size() for v in outs_h.values())
+    # the step's inputs (x, dY) and its outputs (Y and every gradient) each
+    # live in one contiguous buffer, host and device side, so that a step moves
+    # one copy in and one copy out; the C ABI gets views into them
+    def packed(specs, pin, device=None):
+        """One flat buffer holding tensors of the given (name, shape, dtype),
+        each at a 256-byte aligned offset; returns (flat, {name: view})."""
+        offs, total = [], 0
+        for _, shape, dtype in specs:
+            nbytes = int(torch.Size(shape).numel()) * torch.empty((), dtype=dtype).element_size()
+            offs.append(total)
+            total += (nbytes + 255) // 256 * 256
+        flat = torch.empty(total, dtype=torch.uint8, device=device)
+        if pin:
+            flat = flat.pin_memory()
+        views = {}
+        for (name, shape, dtype), off in zip(specs, offs):
+            nbytes = int(torch.Size(shape).numel()) * torch.empty((), dtype=dtype).element_size()
+            views[name] = flat[off:off + nbytes].view(dtype).view(shape)
+        return flat, views
+
+    in_specs = [("x", t_cpu["x"].shape, t_cpu["x"].dtype), ("dy", t_cpu["dy"].shape, t_cpu["dy"].dtype)]
+    out_specs = [("y", t_cpu["x"].shape, t_cpu["x"].dtype)] + \
+        [(n, g_.shape, g_.dtype) for n, g_ in grads.items()]
+    in_h, in_hv = packed(in_specs, pin=True)
+    in_hv["x"].copy_(t_cpu["x"])
+    in_hv["dy"].copy_(t_cpu["dy"])
+    out_h, _ = packed(out_specs, pin=True)
+    in_d, out_d = [], []
+    for _ in range(2):
+        in_d.append(packed(in_specs, pin=False, device=dev))
+        out_d.append(packed(out_specs, pin=False, device=dev))
+    x_d = [v["x"] for _, v in in_d]
+    dy_d = [v["dy"] for _, v in in_d]
+    y_d = [v["y"] for _, v in out_d]
+    g_d = [{n: v[n] for n in grads} for _, v in out_d]
+    h2d = sum(int(torch.Size(sh).numel()) * torch.empty((), dtype=dt).element_size()
+              for _, sh, dt in in_specs)
+    d2h = sum(int(torch.Size(sh).numel()) * torch.empty((), dtype=dt).element_size()
+              for _, sh, dt in out_specs)
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
     ev_in = [torch.cuda.Event() for _ in range(2)]
     ev_done = [torch.cuda.Event() for _ in range(2)]
@@ -427,8 +455,7 @@ def bench_ours(args):
             with torch.cuda.stream(s_in):
                 if i >= 2:
                     s_in.wait_event(ev_done[b])  # step i-2 has read buffer b
-                x_d[b].copy_(x_h, non_blocking=True)
-                dy_d[b].copy_(dy_h, non_blocking=True)
+                in_d[b][0].copy_(in_h, non_blocking=True)
                 ev_in[b].record(s_in)
             stream.wait_event(ev_in[b])
             if i >= 2:
@@ -438,9 +465,7 @@ def bench_ours(args):
             ev_done[b].record(stream)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_done[b])
-                outs_h["y"].copy_(y_d[b], non_blocking=True)
-                for n, g_ in gb.items():
-                    outs_h[n].copy_(g_, non_blocking=True)
+                out_h.copy_(out_d[b][0], non_blocking=True)
                 ev_out[b].record(s_out)
 
     e2e_steps(3)
