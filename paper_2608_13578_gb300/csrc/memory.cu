@@ -753,15 +753,16 @@ __device__ __forceinline__ void warp_mma_16x8(const bf16* A, int lda, int r0, co
 // memory fits one CTA's shared memory: item (x, b) = output columns
 // kProjNC*x .. kProjNC*x + kProjNC-1 of batch b, kProjThreads threads.  The
 // weight chunk W_m[:, x] is fetched before the wait for the previous kernel
-// (it is an input, not a product of the step).  The CTA runs the decayed scan
-// of every channel over the batch's Nb blocks (thread t: channels t,
+// (it is an input, not a product of the step).  After the wait the CTA
+// copies the batch's summaries S [Nb, D] to shared memory and runs the
+// decayed scan of every channel over the Nb blocks (thread t: channels t,
 // t + kProjThreads; N_i = a N_{i-1} + S_i, Z_i = a Z_{i-1} + 1,
 // M_i = N_i * (1 / Z_i)) into shared memory as bf16 (the operand the
 // tensor-core path uses too), then P_i[c] = sum_k M_i[k] W_m[k][c] on the
 // tensor cores: warp w takes columns 8 (w % 4) .. +7 and K quarter w / 4, the
-// quarters added in order.  x == 0 also stores M (fp32 and bf16) and, for
-// batch 0, Z and 1/Z.  P is stored unshifted [B*Nb, D]: its readers take
-// C_i = P_{i-1}, C_0 = 0.
+// quarters added in order.  CTA x also stores M (fp32 and bf16) of its own
+// kProjNC channels and, for batch 0, their Z and 1/Z.  P is stored unshifted
+// [B*Nb, D]: its readers take C_i = P_{i-1}, C_0 = 0.
 constexpr int kProjThreads = 512;
 constexpr int kProjKQ = kProjThreads / 32 / 4;  // K ranges per column group
 __global__ void __launch_bounds__(kProjThreads)
@@ -775,45 +776,48 @@ __global__ void __launch_bounds__(kProjThreads)
   bf16* Ws = reinterpret_cast<bf16*>(smb);                         // [D][ldw]
   bf16* Ms = Ws + (long)D * ldw;                                   // [Nr][lda]
   float* red = reinterpret_cast<float*>(Ms + (long)Nr * lda);      // [KQ-1][4][16][8]
+  float* Ss = red + (kProjKQ - 1) * 4 * 16 * 8;                    // [Nb][D]
   const int x = blockIdx.x, b = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // the weight chunk: D rows of kProjNC columns (16 bytes per load, a batch
   // of loads in flight before their shared-memory stores)
   copy_rows16<kProjNC / 8, kProjThreads>(Ws, ldw, Wm + x * kProjNC, D, D);
   pdl_enter();
+  // the batch's summaries to shared memory in 16-byte pieces (all in flight
+  // at once, no registers held)
+  {
+    const float* Sb = S + (long)b * Nb * D;
+    for (int o = 4 * threadIdx.x; o < Nb * D; o += 4 * kProjThreads) cp_async16(Ss + o, Sb + o);
+    cp_async_commit();
+    cp_async_wait_all();
+    __syncthreads();
+  }
+  // the scan, one channel per thread (a rolled loop: little code to fetch);
+  // CTA x stores M, Mb (and for b == 0, Z and 1/Z) of its own 32 channels
 #pragma unroll 1
   for (int k = threadIdx.x; k < D; k += kProjThreads) {
     const float a = decay[k];
+    const bool mine = k / kProjNC == x;
     float Nn = 0.f, Zz = 0.f;
 #pragma unroll 1
-    for (int i0 = 0; i0 < Nr; i0 += 16) {
-      float sv[16];
-#pragma unroll
-      for (int u = 0; u < 16; ++u)
-        sv[u] = (i0 + u < Nb) ? S[((long)b * Nb + i0 + u) * D + k] : 0.f;
-#pragma unroll
-      for (int u = 0; u < 16; ++u) {
-        const int i = i0 + u;
-        bf16 mb = __float2bfloat16_rn(0.f);
-        if (i < Nb) {
-          Nn = fmaf(a, Nn, sv[u]);
-          Zz = fmaf(a, Zz, 1.0f);
-          const float zi = __frcp_rn(Zz);
-          const float m = Nn * zi;
-          mb = __float2bfloat16_rn(m);
-          if (x == 0) {
-            const long o = ((long)b * Nb + i) * D + k;
-            M[o] = m;
-            Mb[o] = mb;
-            if (b == 0) {
-              Z[(long)i * D + k] = Zz;
-              Zinv[(long)i * D + k] = zi;
-            }
-          }
+    for (int i = 0; i < Nb; ++i) {
+      Nn = fmaf(a, Nn, Ss[i * D + k]);
+      Zz = fmaf(a, Zz, 1.0f);
+      const float zi = __frcp_rn(Zz);
+      const float m = Nn * zi;
+      const bf16 mb = __float2bfloat16_rn(m);
+      if (mine) {
+        const long o = ((long)b * Nb + i) * D + k;
+        M[o] = m;
+        Mb[o] = mb;
+        if (b == 0) {
+          Z[(long)i * D + k] = Zz;
+          Zinv[(long)i * D + k] = zi;
         }
-        Ms[(long)i * lda + k] = mb;
       }
+      Ms[(long)i * lda + k] = mb;
     }
+    for (int i = Nb; i < Nr; ++i) Ms[(long)i * lda + k] = __float2bfloat16_rn(0.f);
   }
   __syncthreads();
   // warp w: columns 8 (w & 3) .. +7, K range w >> 2 of kProjKQ
@@ -989,7 +993,7 @@ constexpr int kProjSmemMax = 200 * 1024;
 static size_t proj_fwd_smem(int Nb, int D) {
   const size_t Nr = (size_t)((Nb + 15) & ~15);
   return ((size_t)D * (kProjNC + kProjPad) + Nr * (D + kProjPad)) * 2 +
-         (size_t)(kProjKQ - 1) * 4 * 16 * 8 * 4;
+         (size_t)(kProjKQ - 1) * 4 * 16 * 8 * 4 + (size_t)Nb * D * 4;
 }
 bool memory_proj_fits(int dtype, int B, int Nb, int D) {
   return dtype == 1 && D % 64 == 0 && D % (16 * kProjKQ) == 0 && Nb <= 16 &&
