@@ -35,6 +35,13 @@ using namespace attn;
 namespace {
 constexpr int kTile = 128;
 
+// max(a, b, c) in one instruction (three-input max.f32, sm_100 and later)
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 // First key of the key-tile walk of the query tile at t0, and the tile count.
 __device__ __forceinline__ void key_walk(int t0, int L, int& kstart, int& nkt) {
   kstart = L >= kTile ? (t0 / L) * L : t0;
@@ -175,32 +182,53 @@ __global__ void __launch_bounds__(128, NCH <= 2 ? 3 : 2)
 
     // ---- online softmax (P to shared memory; the previous P V has completed).
     // Tiles left of the diagonal need no mask: their max, exponentials and
-    // sum run with independent partial accumulators.
+    // sum run with independent partial accumulators.  For L <= 128 (one
+    // tile) the masked branch below serves.
     float m_new, psum;
-    if (!ONE && !diag) {
+    if (!ONE && diag) {
+      // the diagonal tile of a walk (L > 128: no block offset, wbs = rbs = 0)
+      // goes through the unmasked code below with its hidden scores set to
+      // -inf (exp2 gives 0): one softmax body keeps the kernel's code small
+      // (with a masked copy of it, instruction fetch was the top stall)
+#pragma unroll
+      for (int ci = 0; ci < NCH; ++ci)
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (ci >= nld || ci * 32 + j > r) sr[ci][j] = __float_as_uint(-INFINITY);
+    }
+    if (!ONE) {
+      // three-input max, and the exponent arguments and the partial sums as
+      // packed fp32 pairs: about a third fewer instructions per score
       float mx[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
 #pragma unroll
       for (int ci = 0; ci < NCH; ++ci)
 #pragma unroll
-        for (int j = 0; j < 32; ++j) mx[j & 7] = fmaxf(mx[j & 7], __uint_as_float(sr[ci][j]));
-      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        for (int j = 0; j < 32; j += 2)
+          mx[(j >> 1) & 7] = max3f(mx[(j >> 1) & 7], __uint_as_float(sr[ci][j]),
+                                   __uint_as_float(sr[ci][j + 1]));
+      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                             fmaxf(mx[6], mx[7]));
       m_new = fmaxf(m, mt * sl2);
-      const float nm = -m_new;
-      float ps[4] = {0.f, 0.f, 0.f, 0.f};
+      const float2 sl2x2 = make_float2(sl2, sl2), nm2 = make_float2(-m_new, -m_new);
+      float2 ps[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
       for (int u = 0; u < 4 * NCH; ++u) {
         float v[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          v[e] = ex2(fmaf(__uint_as_float(sr[u >> 2][(u & 3) * 8 + e]), sl2, nm));
-          ps[e & 3] += v[e];
+        for (int e = 0; e < 8; e += 2) {
+          const float2 a = __ffma2_rn(
+              make_float2(__uint_as_float(sr[u >> 2][(u & 3) * 8 + e]),
+                          __uint_as_float(sr[u >> 2][(u & 3) * 8 + e + 1])),
+              sl2x2, nm2);
+          v[e] = ex2(a.x);
+          v[e + 1] = ex2(a.y);
+          ps[(e >> 1) & 1] = __fadd2_rn(ps[(e >> 1) & 1], make_float2(v[e], v[e + 1]));
         }
         put_unit(sP, r, u, pack8(v));
       }
-      psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
+      psum = (ps[0].x + ps[0].y) + (ps[1].x + ps[1].y);
     } else {
       float mt = -INFINITY;
 #pragma unroll
