@@ -799,7 +799,7 @@ __global__ void __launch_bounds__(kProjThreads)
     const float a = decay[k];
     const bool mine = k / kProjNC == x;
     float Nn = 0.f, Zz = 0.f;
-#pragma unroll 1
+#pragma unroll 4
     for (int i = 0; i < Nb; ++i) {
       Nn = fmaf(a, Nn, Ss[i * D + k]);
       Zz = fmaf(a, Zz, 1.0f);
