@@ -307,6 +307,218 @@ __global__ void __launch_bounds__(128, NCH <= 2 ? 3 : 2)
   if (warp == 0) tc::tmem_dealloc(tmem, kCols);
 }
 
+// The forward at L > 128 for head widths up to 32, with each 128-key tile
+// taken as two 64-key halves in turn: S of a half (N = 64) and O need at most
+// 96 TMEM columns and P one 16 KB half, so a CTA allocates 128 columns and
+// three or four CTAs share an SM (twice the warps of the kernel above, whose
+// per-score chains are latency-bound).  Per half: S = Q K_h^T, online softmax
+// of its 64 scores (the diagonal tile's hidden keys set to -inf first), P_h in
+// bf16 to shared memory, P_h V_h into TMEM, folded into O in registers.  The
+// next half's S is issued as soon as every thread has read this half's scores
+// and runs under its softmax; K is double-buffered across tiles (K of tile
+// kt+2 streams in once tile kt's second half has its scores) and V is
+// reloaded once tile kt's second P V has completed.
+template <int DH>
+__global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
+    attn_fwd_fl_half_kernel(const __grid_constant__ CUtensorMap mQ,
+                            const __grid_constant__ CUtensorMap mK,
+                            const __grid_constant__ CUtensorMap mV, bf16* __restrict__ O,
+                            long ld_o, float* __restrict__ lse, int Tlen, int H, int L,
+                            float scale, unsigned* status) {
+  static_assert(DH <= 32, "two 64-key halves and O fit 128 TMEM columns for DH <= 32 (and 64)");
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sP = smem;                       // 16 KB: P of one half [128 queries x 64 keys]
+  uint8_t* sQ = smem + 16384;
+  uint8_t* sK0 = sQ + G::tile;              // K, two buffers
+  uint8_t* sV = sK0 + 2 * G::tile;
+  // barriers: K buffer 0/1 loaded (buffer 0 also counts Q), V loaded, S ready, P V done
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);
+  uint64_t* bar_k = bar;
+  uint64_t* bar_v = bar + 2;
+  uint64_t* bar_s = bar + 3;
+  uint64_t* bar_o = bar + 4;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 5);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  int kstart, nkt;
+  key_walk(t0, L, kstart, nkt);
+
+  if (tid == 0) {
+    for (int i = 0; i < 5; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar_k[0], 2 * G::tile);
+    tc::tma_load_3d(sQ, &mQ, &bar_k[0], h * DH, t0, b);
+    tc::tma_load_3d(sK0, &mK, &bar_k[0], h * DH, kstart, b);
+    tc::mbar_arrive_expect_tx(bar_v, G::tile);
+    tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart, b);
+    if (nkt > 1) {
+      tc::mbar_arrive_expect_tx(&bar_k[1], G::tile);
+      tc::tma_load_3d(sK0 + G::tile, &mK, &bar_k[1], h * DH, kstart + kTile, b);
+    }
+  }
+  __syncwarp();
+  constexpr uint32_t kCols = 128, kOcol = 64;  // S half at 0..63, O at 64..
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, kCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  constexpr uint32_t idS = tc::idesc_bf16(128, 64, 0, 0);
+  constexpr uint32_t idO = tc::idesc_bf16(128, DH, 0, 1);
+  // S of half hh of the key tile in K buffer kb
+  auto issue_s = [&](int kb, int hh) {
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk)
+      tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK0 + kb * G::tile, 64 * hh, kk), idS,
+                   kk > 0 ? 1u : 0u);
+    tc::mma_commit(bar_s);
+  };
+
+  if (tid == 0) {
+    const bool okk = tc::mbar_wait(&bar_k[0], 0, status);
+    tc::fence_after_sync();
+    if (okk) issue_s(0, 0);
+    else tc::mma_commit(bar_s);
+  }
+  __syncwarp();
+
+  const int r = warp * 32 + lane;
+  const float sl2 = scale * kLog2e;
+  float m = -INFINITY, l = 0.f;
+  float oacc[DH];
+#pragma unroll
+  for (int c = 0; c < DH; ++c) oacc[c] = 0.f;
+  bool ok = true;
+  int ns = 0, no = 0;  // S and P V commits consumed
+
+  for (int kt = 0; kt < nkt; ++kt) {
+    const bool diag = kt == nkt - 1;
+    const int kb = kt & 1;
+    for (int hh = 0; hh < 2; ++hh) {
+      ok = tc::mbar_wait(bar_s, ns & 1, status) && ok;
+      ++ns;
+      tc::fence_after_sync();
+      uint32_t sr[2][32];
+      tc::tmem_ld32_issue(trow, sr[0]);
+      tc::tmem_ld32_issue(trow + 32u, sr[1]);
+      tc::tmem_wait();
+      tc::fence_before_sync();
+      __syncthreads();  // every thread has this half's scores: the S columns are free
+      if (tid == 0) {
+        tc::fence_after_sync();
+        if (hh == 0) {  // the tile's second half
+          if (ok) issue_s(kb, 1);
+          else tc::mma_commit(bar_s);
+        } else if (kt + 1 < nkt) {  // the next tile's first half
+          const int nb = (kt + 1) & 1;
+          const bool okk = tc::mbar_wait(&bar_k[nb], ((kt + 1) >> 1) & 1, status);
+          tc::fence_after_sync();
+          if (okk && ok) issue_s(nb, 0);
+          else tc::mma_commit(bar_s);
+        }
+        // K buffer kb: both halves' scores are read (tile kt done with it)
+        if (hh == 1 && kt + 2 < nkt) {
+          tc::mbar_arrive_expect_tx(&bar_k[kb], G::tile);
+          tc::tma_load_3d(sK0 + kb * G::tile, &mK, &bar_k[kb], h * DH, kstart + (kt + 2) * kTile, b);
+        }
+      }
+      if (diag) {  // keys past the query row (L > 128: no block offset in the tile)
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (64 * hh + 32 * c + j > r) sr[c][j] = __float_as_uint(-INFINITY);
+      }
+      // online softmax of the half's 64 scores (P to shared memory; the
+      // previous P V has completed)
+      float mx[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int j = 0; j < 32; j += 2)
+          mx[(j >> 1) & 7] = max3f(mx[(j >> 1) & 7], __uint_as_float(sr[c][j]),
+                                   __uint_as_float(sr[c][j + 1]));
+      const float mt = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                             fmaxf(mx[6], mx[7]));
+      const float m_new = fmaxf(m, mt * sl2);
+      const float2 sl2x2 = make_float2(sl2, sl2), nm2 = make_float2(-m_new, -m_new);
+      float2 ps[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+          const float2 a = __ffma2_rn(make_float2(__uint_as_float(sr[u >> 2][(u & 3) * 8 + e]),
+                                                  __uint_as_float(sr[u >> 2][(u & 3) * 8 + e + 1])),
+                                      sl2x2, nm2);
+          v[e] = ex2(a.x);
+          v[e + 1] = ex2(a.y);
+          ps[(e >> 1) & 1] = __fadd2_rn(ps[(e >> 1) & 1], make_float2(v[e], v[e + 1]));
+        }
+        put_unit(sP, r, u, pack8(v));
+      }
+      const float psum = (ps[0].x + ps[0].y) + (ps[1].x + ps[1].y);
+      const float alpha = ex2(m - m_new);  // 0 on the first half (m = -inf)
+      l = l * alpha + psum;
+      m = m_new;
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+
+      if (tid == 0) {
+        tc::fence_after_sync();
+        const bool okv = tc::mbar_wait(bar_v, kt & 1, status);
+        tc::fence_after_sync();
+        if (okv && ok) {
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // O_h = P_h V[64 hh .., :]
+            tc::mma_bf16(tmem + kOcol, p_kmaj(sP, 0, kk), G::mnmaj(sV, 64 * hh, kk), idO,
+                         kk > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(bar_o);
+      }
+      __syncwarp();
+      ok = tc::mbar_wait(bar_o, no & 1, status) && ok;
+      ++no;
+      tc::fence_after_sync();
+      // V is free after the tile's second P V: fetch the next tile's V while
+      // this product is folded in
+      if (tid == 0 && hh == 1 && kt + 1 < nkt) {
+        tc::mbar_arrive_expect_tx(bar_v, G::tile);
+        tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart + (kt + 1) * kTile, b);
+      }
+      float o[DH];
+      tmem_row<DH>(trow + kOcol, o);
+#pragma unroll
+      for (int c = 0; c < DH; ++c) oacc[c] = fmaf(oacc[c], alpha, o[c]);
+    }
+  }
+
+  const int t = t0 + r;
+  if (ok && t < Tlen) {
+    store_row<DH>(O + ((long)b * Tlen + t) * ld_o + h * DH, oacc, 1.0f / l);
+    lse[((long)b * H + h) * Tlen + t] = m * kLn2 + logf(l);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
+}
+
 // ================================================================ backward: dQ
 template <int DH>
 __global__ void __launch_bounds__(128)
@@ -700,6 +912,20 @@ template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
 }
 
+template <int DH> constexpr int fwd_half_smem() { return 1024 + 16384 + 4 * Geo<DH>::tile + 64; }
+
+template <int DH>
+cudaError_t fwd_fl_half_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
+  static std::atomic<unsigned long long> opted{0};
+  auto kern = attn_fwd_fl_half_kernel<DH>;
+  cudaError_t e = smem_opt_in(kern, fwd_half_smem<DH>(), &opted);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.T + kTile - 1) / kTile, a.H, a.B);
+  e = launch_k(kern, grid, dim3(128), fwd_half_smem<DH>(), lc.stream, m[0], m[1], m[2],
+               (bf16*)a.O, a.ld_o, a.lse, a.T, a.H, a.L, 1.0f / sqrtf((float)DH), lc.status);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 template <int DH, int NCH, bool ONE>
 cudaError_t fwd_fl_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
   static std::atomic<unsigned long long> opted{0};
@@ -720,7 +946,10 @@ cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
       !head_map_fl<DH>(&m[1], a.K, a.ld_qkv, D, a.T, a.B) ||
       !head_map_fl<DH>(&m[2], a.V, a.ld_qkv, D, a.T, a.B))
     return cudaErrorInvalidValue;
-  if (a.L > kTile) return fwd_fl_launch<DH, 4, false>(lc, a, m);
+  if (a.L > kTile) {
+    if constexpr (DH <= 32) return fwd_fl_half_launch<DH>(lc, a, m);
+    return fwd_fl_launch<DH, 4, false>(lc, a, m);
+  }
   if (a.L <= 32) return fwd_fl_launch<DH, 1, true>(lc, a, m);
   if (a.L == 64) return fwd_fl_launch<DH, 2, true>(lc, a, m);
   return fwd_fl_launch<DH, 4, true>(lc, a, m);
