@@ -705,6 +705,196 @@ __global__ void __launch_bounds__(128)
   if (warp == 0) tc::tmem_dealloc(tmem, 256);
 }
 
+// The dQ kernel for head widths up to 32 with each key tile taken as four
+// 32-key quarters in turn: S and dP of a quarter (N = 32 each) and the dQ
+// accumulator need at most 96 TMEM columns, so a CTA allocates 128 and three
+// or four CTAs share an SM (the kernel above, at 256 columns, runs two, and
+// its per-half chains wait on barriers and TMEM).  Quarter q's scale * dS goes
+// to columns 32 (q % 2) .. of the 64-key half buffer q / 2, which the dQ
+// product of the same quarter of the previous tile read (bar[2 + q] tracks
+// it); S and dP of the next quarter are issued as soon as every thread has
+// read this quarter's and run under its elementwise pass.
+template <int DH>
+__global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
+    attn_bwd_dq_fl_q_kernel(const __grid_constant__ CUtensorMap mQ,
+                            const __grid_constant__ CUtensorMap mK,
+                            const __grid_constant__ CUtensorMap mV,
+                            const __grid_constant__ CUtensorMap mdO, const bf16* __restrict__ O,
+                            const bf16* __restrict__ dO, long ld_o, const float* __restrict__ lse,
+                            float* __restrict__ Drow, bf16* __restrict__ dQ, long ld_d, int Tlen,
+                            int H, int L, float scale, unsigned* status) {
+  static_assert(DH <= 32, "S, dP quarters and dQ fit 128 TMEM columns for DH <= 64; smem for <= 32");
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sdS = smem;                      // 2 x 16 KB: scale * dS, quarters 0-1 / 2-3
+  uint8_t* sQ = smem + 32768;
+  uint8_t* sdO = sQ + G::tile;
+  uint8_t* sK = sdO + G::tile;
+  uint8_t* sV = sK + G::tile;
+  // K/V loaded; S/dP of a quarter done; dQ product of quarter 0..3 done
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 6);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  int kstart, nkt;
+  key_walk(t0, L, kstart, nkt);
+
+  if (tid == 0) {
+    for (int i = 0; i < 6; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+    tc::prefetch_tmap(&mdO);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * G::tile);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, t0, b);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart, b);
+  }
+  __syncwarp();
+  constexpr uint32_t kCols = 128, kQcol = 64;  // S quarter 0..31, dP quarter 32..63, dQ 64..
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, kCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  // Drow_t = dO_t . O_t and the row's log-sum-exp (global rows)
+  const int r = warp * 32 + lane;
+  const int t = t0 + r;
+  const bool row_ok = t < Tlen;
+  float drow = 0.f, lse2 = 0.f;
+  if (row_ok) {
+    const bf16* orow = O + ((long)b * Tlen + t) * ld_o + h * DH;
+    const bf16* grow = dO + ((long)b * Tlen + t) * ld_o + h * DH;
+#pragma unroll
+    for (int u = 0; u < DH / 8; ++u) {
+      float ov[8], gv[8];
+      load8(orow + 8 * u, ov);
+      load8(grow + 8 * u, gv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) drow = fmaf(ov[e], gv[e], drow);
+    }
+    const long li = ((long)b * H + h) * Tlen + t;
+    Drow[li] = drow;
+    lse2 = lse[li] * kLog2e;
+  }
+  const float sl2 = scale * kLog2e;
+  const float nl2 = -lse2, ndr = -drow * scale;
+  const int rbs = L < kTile ? (r / L) * L : 0;
+  bool ok = true;
+  // S and dP of quarter q of the loaded key tile into TMEM columns 0..63
+  auto issue_sdp = [&](int q) {
+    if (ok) {
+      constexpr uint32_t id32 = tc::idesc_bf16(128, 32, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // S quarter -> columns 0..31
+        tc::mma_bf16(tmem, G::kmaj(sQ, 0, kk), G::kmaj(sK, 32 * q, kk), id32, kk > 0 ? 1u : 0u);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // dP quarter -> columns 32..63
+        tc::mma_bf16(tmem + 32, G::kmaj(sdO, 0, kk), G::kmaj(sV, 32 * q, kk), id32,
+                     kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar[1]);
+  };
+  if (tid == 0) {
+    ok = tc::mbar_wait(&bar[0], 0, status) && ok;
+    tc::fence_after_sync();
+    issue_sdp(0);
+  }
+  __syncwarp();
+  int ns = 0;  // S/dP commits consumed so far
+
+  for (int kt = 0; kt < nkt; ++kt) {
+    const bool diag = kt == nkt - 1;
+    for (int q = 0; q < 4; ++q) {
+      ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
+      ++ns;
+      tc::fence_after_sync();
+      uint32_t rs[32], rd[32];
+      tc::tmem_ld32_issue(trow, rs);
+      tc::tmem_ld32_issue(trow + 32u, rd);
+      tc::tmem_wait();
+      tc::fence_before_sync();
+      __syncthreads();  // every thread has this quarter's S and dP: the columns are free
+      if (tid == 0 && q < 3) {
+        tc::fence_after_sync();
+        issue_sdp(q + 1);
+      }
+      uint8_t* sdSq = sdS + (q >> 1) * 16384;
+      if (kt > 0) {  // the previous tile's dQ product of this quarter read its columns
+        ok = tc::mbar_wait(&bar[2 + q], (kt - 1) & 1, status) && ok;
+        tc::fence_after_sync();
+      }
+      // dS = P (dP - Drow) scale; rows past the end see zero-filled Q and dO
+      // (P finite, dP = Drow = 0), so only the diagonal tile needs a mask
+      float v[32];
+      if (!diag) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          v[j] = ex2(fmaf(__uint_as_float(rs[j]), sl2, nl2)) *
+                 fmaf(__uint_as_float(rd[j]), scale, ndr);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int kk = 32 * q + j;  // key column within the tile
+          const bool valid = row_ok && kk >= rbs && kk <= r;
+          v[j] = valid ? ex2(fmaf(__uint_as_float(rs[j]), sl2, nl2)) *
+                             fmaf(__uint_as_float(rd[j]), scale, ndr)
+                       : 0.f;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) put_unit(sdSq, r, 4 * (q & 1) + u, pack8(v + 8 * u));
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid == 0) {
+        tc::fence_after_sync();
+        if (ok) {
+          constexpr uint32_t idQ = tc::idesc_bf16(128, DH, 0, 1);
+#pragma unroll
+          for (int kk = 0; kk < 2; ++kk)  // dQ += dS[:, 32q..] K[32q.., :]
+            tc::mma_bf16(tmem + kQcol, p_kmaj(sdSq, 0, 2 * (q & 1) + kk),
+                         G::mnmaj(sK, 32 * q, kk), idQ, (kt > 0 || q > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[2 + q]);
+      }
+    }
+    // the next key tile may overwrite K and V once this tile's products are
+    // done (the last quarter's commit covers every earlier product); then its
+    // first quarter
+    if (tid == 0 && kt + 1 < nkt) {
+      ok = tc::mbar_wait(&bar[5], kt & 1, status) && ok;
+      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
+      tc::tma_load_3d(sK, &mK, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      tc::tma_load_3d(sV, &mV, &bar[0], h * DH, kstart + (kt + 1) * kTile, b);
+      ok = tc::mbar_wait(&bar[0], (kt + 1) & 1, status) && ok;
+      tc::fence_after_sync();
+      issue_sdp(0);
+    }
+    __syncwarp();
+  }
+  ok = tc::mbar_wait(&bar[5], (nkt - 1) & 1, status) && ok;
+  tc::fence_after_sync();
+  float qv[DH];
+  tmem_row<DH>(trow + kQcol, qv);
+  if (ok && row_ok) store_row<DH>(dQ + ((long)b * Tlen + t) * ld_d + h * DH, qv, 1.0f);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
+}
+
 // =============================================================== backward: dKV
 template <int DH>
 __global__ void __launch_bounds__(128)
@@ -966,12 +1156,14 @@ cudaError_t bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
       !head_map_fl<DH>(&mdo, a.dO, f.ld_o, D, f.T, f.B))
     return cudaErrorInvalidValue;
   static std::atomic<unsigned long long> opted_q{0}, opted_kv{0};
-  cudaError_t e = smem_opt_in(attn_bwd_dq_fl_kernel<DH>, dq_smem<DH>(), &opted_q);
+  // head widths up to 32: the dQ kernel that walks 32-key quarters
+  auto dq_kern = DH <= 32 ? attn_bwd_dq_fl_q_kernel<DH <= 32 ? DH : 32> : attn_bwd_dq_fl_kernel<DH>;
+  cudaError_t e = smem_opt_in(dq_kern, dq_smem<DH>(), &opted_q);
   if (e == cudaSuccess) e = smem_opt_in(attn_bwd_dkv_fl_kernel<DH>, dkv_smem<DH>(), &opted_kv);
   if (e != cudaSuccess) return e;
   const float scale = 1.0f / sqrtf((float)DH);
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
-  e = launch_k(attn_bwd_dq_fl_kernel<DH>, grid, dim3(128), dq_smem<DH>(), lc.stream, mq, mk, mv,
+  e = launch_k(dq_kern, grid, dim3(128), dq_smem<DH>(), lc.stream, mq, mk, mv,
                mdo, (const bf16*)f.O, (const bf16*)a.dO, f.ld_o, (const float*)f.lse, a.Drow,
                (bf16*)a.dQ, a.ld_dqkv, f.T, f.H, f.L, scale, lc.status);
   if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
