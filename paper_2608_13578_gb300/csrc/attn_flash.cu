@@ -1077,6 +1077,192 @@ __global__ void __launch_bounds__(128)
   if (warp == 0) tc::tmem_dealloc(tmem, 256);
 }
 
+// The dK/dV kernel for head widths up to 32 with each query tile taken as
+// four 32-query quarters in turn: S^T and dP^T of a quarter (N = 32 each), dV
+// and dK need at most 128 TMEM columns, so three or four CTAs share an SM.
+// Quarter n (counted over the walk) writes P^T and scale * dS^T to columns
+// 32 (n % 2) .. of the 16 KB P^T / dS^T buffers, which quarter n - 2's dV/dK
+// products read (bar[2 + n % 2] tracks them).
+template <int DH>
+__global__ void __launch_bounds__(128, 3)
+    attn_bwd_dkv_fl_q_kernel(const __grid_constant__ CUtensorMap mQ,
+                             const __grid_constant__ CUtensorMap mK,
+                             const __grid_constant__ CUtensorMap mV,
+                             const __grid_constant__ CUtensorMap mdO,
+                             const float* __restrict__ lse, const float* __restrict__ Drow,
+                             bf16* __restrict__ dK, bf16* __restrict__ dV, long ld_d, int Tlen,
+                             int H, int L, float scale, unsigned* status) {
+  static_assert(DH <= 32, "S^T, dP^T quarters, dV and dK fit 128 TMEM columns for DH <= 32");
+  using G = Geo<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sPt = smem;                      // 16 KB: P^T, two 32-query quarters
+  uint8_t* sdSt = smem + 16384;             // 16 KB: scale * dS^T, the same quarters
+  uint8_t* sK = smem + 32768;
+  uint8_t* sV = sK + G::tile;
+  uint8_t* sQ = sV + G::tile;
+  uint8_t* sdO = sQ + G::tile;
+  float* slse = reinterpret_cast<float*>(sdO + G::tile);  // [128] -lse * log2(e)
+  float* sdr = slse + kTile;                               // [128] -Drow * scale
+  // tiles loaded; S^T/dP^T of a quarter done; dV/dK of even / odd quarters done
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sdr + kTile);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 4);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int k0 = blockIdx.x * kTile, h = blockIdx.y, b = blockIdx.z;
+  const int qend = min(L >= kTile ? (k0 / L + 1) * L : k0 + kTile, Tlen);
+  const int nqt = (qend - k0 + kTile - 1) / kTile;
+
+  if (tid == 0) {
+    for (int i = 0; i < 4; ++i) tc::mbar_init(&bar[i], 1);
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&mQ);
+    tc::prefetch_tmap(&mK);
+    tc::prefetch_tmap(&mV);
+    tc::prefetch_tmap(&mdO);
+  }
+  pdl_enter();
+  if (tid == 0) {
+    tc::mbar_arrive_expect_tx(&bar[0], 4 * G::tile);
+    tc::tma_load_3d(sK, &mK, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sV, &mV, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, k0, b);
+    tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, k0, b);
+  }
+  __syncwarp();
+  constexpr uint32_t kCols = 128, kVcol = 64, kKcol = 64 + DH;
+  if (warp == 0) {
+    tc::tmem_alloc(tslot, kCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+  const int r = warp * 32 + lane;  // key row
+  const int key = k0 + r;
+  const float sl2 = scale * kLog2e;
+  const int kbe = L < kTile ? (r / L) * L + L : kTile;
+  bool ok = true;
+  int ns = 0, nq = 0;
+  // S^T and dP^T of query quarter q -> TMEM columns 0..63 (tid 0)
+  auto issue_scores = [&](int q) {
+    if (ok) {
+      constexpr uint32_t id32 = tc::idesc_bf16(128, 32, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // S^T quarter -> columns 0..31
+        tc::mma_bf16(tmem, G::kmaj(sK, 0, kk), G::kmaj(sQ, 32 * q, kk), id32, kk > 0 ? 1u : 0u);
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)  // dP^T quarter -> columns 32..63
+        tc::mma_bf16(tmem + 32, G::kmaj(sV, 0, kk), G::kmaj(sdO, 32 * q, kk), id32,
+                     kk > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar[1]);
+  };
+
+  for (int qt = 0; qt < nqt; ++qt) {
+    const int q0 = k0 + qt * kTile;
+    const bool diag = qt == 0;
+    {
+      const int tq = q0 + tid;
+      const long li = ((long)b * H + h) * Tlen + tq;
+      slse[tid] = tq < Tlen ? -lse[li] * kLog2e : 0.f;
+      sdr[tid] = tq < Tlen ? -Drow[li] * scale : 0.f;
+    }
+    if (tid == 0) {
+      ok = tc::mbar_wait(&bar[0], qt & 1, status) && ok;
+      tc::fence_after_sync();
+    }
+    __syncthreads();  // slse / sdr written
+    for (int q = 0; q < 4; ++q) {
+      if (tid == 0 && q == 0) issue_scores(0);
+      __syncwarp();
+      ok = tc::mbar_wait(&bar[1], ns & 1, status) && ok;
+      ++ns;
+      tc::fence_after_sync();
+      uint32_t rs[32], rd[32];
+      tc::tmem_ld32_issue(trow, rs);
+      tc::tmem_ld32_issue(trow + 32u, rd);
+      tc::tmem_wait();
+      const int qb = nq & 1;  // the column half of the P^T / dS^T buffers
+      if (nq >= 2) {  // quarter nq - 2's dV/dK products are done with these columns
+        ok = tc::mbar_wait(&bar[2 + qb], ((nq - 2) >> 1) & 1, status) && ok;
+        tc::fence_after_sync();
+      }
+      // P^T and dS^T = P^T (dP^T - Drow) scale.  Query columns past the end
+      // see zero-filled Q and dO (no contribution), so only the diagonal tile
+      // needs a mask.
+      float pv[32], dv[32];
+      {
+        const float4* nl4 = reinterpret_cast<const float4*>(slse + 32 * q);
+        const float4* nd4 = reinterpret_cast<const float4*>(sdr + 32 * q);
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          const float4 a = nl4[j4], d = nd4[j4];
+          const float na[4] = {a.x, a.y, a.z, a.w}, nd[4] = {d.x, d.y, d.z, d.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int j = 4 * j4 + e;
+            const int jq = 32 * q + j;  // query column within the tile
+            const bool valid = !diag || (q0 + jq < Tlen && jq >= r && jq < kbe);
+            const float p = valid ? ex2(fmaf(__uint_as_float(rs[j]), sl2, na[e])) : 0.f;
+            pv[j] = p;
+            dv[j] = p * fmaf(__uint_as_float(rd[j]), scale, nd[e]);
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        put_unit(sPt, r, 4 * qb + u, pack8(pv + 8 * u));
+        put_unit(sdSt, r, 4 * qb + u, pack8(dv + 8 * u));
+      }
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid == 0) {
+        tc::fence_after_sync();
+        // every thread has read this quarter's scores out of TMEM (the barrier
+        // above): the next quarter's products go first, under this quarter's
+        // dV/dK and the next elementwise pass
+        if (q < 3) issue_scores(q + 1);
+        if (ok) {
+          constexpr uint32_t idKV = tc::idesc_bf16(128, DH, 0, 1);
+          const uint32_t acc0 = (qt > 0 || q > 0) ? 1u : 0u;
+#pragma unroll
+          for (int kk = 0; kk < 2; ++kk)  // dV += P^T[:, 32q..] dO[32q.., :]
+            tc::mma_bf16(tmem + kVcol, p_kmaj(sPt, 0, 2 * qb + kk), G::mnmaj(sdO, 32 * q, kk), idKV,
+                         (acc0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < 2; ++kk)  // dK += dS^T[:, 32q..] Q[32q.., :]
+            tc::mma_bf16(tmem + kKcol, p_kmaj(sdSt, 0, 2 * qb + kk), G::mnmaj(sQ, 32 * q, kk), idKV,
+                         (acc0 || kk > 0) ? 1u : 0u);
+        }
+        tc::mma_commit(&bar[2 + qb]);
+      }
+      ++nq;
+    }
+    if (tid == 0 && qt + 1 < nqt) {  // every product of the tile is done with Q / dO
+      ok = tc::mbar_wait(&bar[2 + ((nq - 1) & 1)], ((nq - 1) >> 1) & 1, status) && ok;
+      tc::mbar_arrive_expect_tx(&bar[0], 2 * G::tile);
+      tc::tma_load_3d(sQ, &mQ, &bar[0], h * DH, q0 + kTile, b);
+      tc::tma_load_3d(sdO, &mdO, &bar[0], h * DH, q0 + kTile, b);
+    }
+    __syncthreads();  // slse / sdr are rewritten next
+  }
+  ok = tc::mbar_wait(&bar[2 + ((nq - 1) & 1)], ((nq - 1) >> 1) & 1, status) && ok;
+  tc::fence_after_sync();
+  float v[DH];
+  tmem_row<DH>(trow + kVcol, v);
+  if (ok && key < Tlen) store_row<DH>(dV + ((long)b * Tlen + key) * ld_d + h * DH, v, 1.0f);
+  tmem_row<DH>(trow + kKcol, v);
+  if (ok && key < Tlen) store_row<DH>(dK + ((long)b * Tlen + key) * ld_d + h * DH, v, 1.0f);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
+}
+
 // ========================================================================= host
 bool attn_fl_supported(int dtype, int dh, int L) {
   const bool l_ok = (L >= 16 && kTile % L == 0) || (L % kTile == 0 && L <= 1024);
@@ -1159,7 +1345,9 @@ cudaError_t bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
   // head widths up to 32: the dQ kernel that walks 32-key quarters
   auto dq_kern = DH <= 32 ? attn_bwd_dq_fl_q_kernel<DH <= 32 ? DH : 32> : attn_bwd_dq_fl_kernel<DH>;
   cudaError_t e = smem_opt_in(dq_kern, dq_smem<DH>(), &opted_q);
-  if (e == cudaSuccess) e = smem_opt_in(attn_bwd_dkv_fl_kernel<DH>, dkv_smem<DH>(), &opted_kv);
+  auto dkv_kern =
+      DH <= 32 ? attn_bwd_dkv_fl_q_kernel<DH <= 32 ? DH : 32> : attn_bwd_dkv_fl_kernel<DH>;
+  if (e == cudaSuccess) e = smem_opt_in(dkv_kern, dkv_smem<DH>(), &opted_kv);
   if (e != cudaSuccess) return e;
   const float scale = 1.0f / sqrtf((float)DH);
   dim3 grid((f.T + kTile - 1) / kTile, f.H, f.B);
@@ -1167,7 +1355,7 @@ cudaError_t bwd_fl(const Launch& lc, const AttnBwdArgs& a) {
                mdo, (const bf16*)f.O, (const bf16*)a.dO, f.ld_o, (const float*)f.lse, a.Drow,
                (bf16*)a.dQ, a.ld_dqkv, f.T, f.H, f.L, scale, lc.status);
   if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
-  e = launch_k(attn_bwd_dkv_fl_kernel<DH>, grid, dim3(128), dkv_smem<DH>(), lc.stream, mq, mk, mv,
+  e = launch_k(dkv_kern, grid, dim3(128), dkv_smem<DH>(), lc.stream, mq, mk, mv,
                mdo, (const float*)f.lse, (const float*)a.Drow, (bf16*)a.dK, (bf16*)a.dV,
                a.ld_dqkv, f.T, f.H, f.L, scale, lc.status);
   return e != cudaSuccess ? e : cudaGetLastError();
