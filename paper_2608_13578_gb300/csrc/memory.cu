@@ -614,47 +614,135 @@ __global__ void __launch_bounds__(kThreads)
   if (c < D) S[((long)b * Nb + i) * D + c] = Si;
 }
 
-// Sec. 3.5: one thread per (batch b, channel c): the decayed scan
-//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i,
-// the recurrence form of M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j),
-// over blocks in batches of kScanU whose loads all go out before the first
-// step.  kScanThreads threads per CTA spread the B * D chains over many SMs.
-// Writes M in fp32 and, when Mb is non-null, in bf16 (the A operand of the
-// tensor-core projection), and Z and 1 / Z (batch 0 only: they do not depend
-// on b).
-constexpr int kScanThreads = 64;
-constexpr int kScanU = 16;
-__global__ void __launch_bounds__(kScanThreads)
+// Sec. 3.5 as a parallel scan over blocks: item (x, b) = channels
+// 32x .. 32x+31 of batch b, 256 threads (8 warps).  The decayed sums
+//   N_i = a N_{i-1} + S_i,  Z_i = a Z_{i-1} + 1,  M_i = N_i / Z_i
+// (M_i = sum_{j<=i} a^(i-j) S_j / sum_{j<=i} a^(i-j)) compose associatively:
+// a run of k blocks acts on the sums before it as (N, Z) -> (A N + n, A Z + z)
+// with A = a^k and (n, z) the run's own sums from zero, and two runs combine
+// as (A1, n1, z1) then (A2, n2, z2) = (A1 A2, A2 n1 + n2, A2 z1 + z2).  The
+// blocks go in windows of up to kPsWin rows: the window's S rows come into
+// shared memory with coalesced 16-byte loads; warp w takes channels w, w+8,
+// w+16, w+24 in turn, lane l a run of ceil(rows / 32) consecutive blocks: the
+// lane scans its run from zero, a warp-shuffle inclusive scan of the runs'
+// (A, n, z) gives each lane the sums entering its run (with the previous
+// windows' carry), and the lane walks its run again to form N, Z and M in
+// shared memory; the window's M (fp32 and, when Mb is non-null, bf16) and,
+// for batch 0, Z and 1 / Z leave as coalesced rows.
+constexpr int kPsCh = 32;      // channels per CTA
+constexpr int kPsThreads = 256;
+constexpr int kPsWin = 256;    // blocks per shared-memory window
+constexpr int kPsLd = kPsCh + 1;
+__global__ void __launch_bounds__(kPsThreads)
     memory_scan_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            float* __restrict__ M, bf16* __restrict__ Mb, float* __restrict__ Z,
                            float* __restrict__ Zinv, int Nb, int D) {
+  extern __shared__ __align__(16) float ps_sm[];
+  const int win = min(Nb, kPsWin);
+  float* Ss = ps_sm;                 // [win][kPsLd]: S, then M
+  float* Zs = ps_sm + win * kPsLd;   // [win][kPsLd]: Z (batch 0)
+  const int x = blockIdx.x, b = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c0 = x * kPsCh;
   pdl_enter();
-  const int c = blockIdx.x * kScanThreads + threadIdx.x, b = blockIdx.y;
-  if (c >= D) return;
-  const float a = decay[c];
-  const long base = (long)b * Nb * D + c;
-  float Nn = 0.f, Zz = 0.f;
-  for (int i0 = 0; i0 < Nb; i0 += kScanU) {
-    float sv[kScanU];
+  // the carry of the earlier windows, per channel this warp scans
+  float cn[kPsCh / 8], cz[kPsCh / 8];
 #pragma unroll
-    for (int u = 0; u < kScanU; ++u) sv[u] = (i0 + u < Nb) ? S[base + (long)(i0 + u) * D] : 0.f;
+  for (int q = 0; q < kPsCh / 8; ++q) cn[q] = cz[q] = 0.f;
+  float av[kPsCh / 8];
 #pragma unroll
-    for (int u = 0; u < kScanU; ++u) {
-      const int i = i0 + u;
-      if (i < Nb) {
-        Nn = fmaf(a, Nn, sv[u]);
-        Zz = fmaf(a, Zz, 1.0f);
-        const float m = Nn / Zz;
-        M[base + (long)i * D] = m;
-        if (Mb) Mb[base + (long)i * D] = __float2bfloat16_rn(m);
-        if (b == 0) {
-          Z[(long)i * D + c] = Zz;
-          Zinv[(long)i * D + c] = 1.0f / Zz;
+  for (int q = 0; q < kPsCh / 8; ++q) av[q] = decay[c0 + warp + 8 * q];
+  for (int w0 = 0; w0 < Nb; w0 += kPsWin) {
+    const int rows = min(kPsWin, Nb - w0);
+    // S rows w0 .. w0+rows-1 of the chunk: 8 threads per row, 16 bytes each
+    for (int o = threadIdx.x; o < rows * (kPsCh / 4); o += kPsThreads) {
+      const int rr = o / (kPsCh / 4), p4 = o % (kPsCh / 4);
+      const float4 v =
+          *reinterpret_cast<const float4*>(S + ((long)b * Nb + w0 + rr) * D + c0 + 4 * p4);
+      float* d = Ss + rr * kPsLd + 4 * p4;
+      d[0] = v.x;
+      d[1] = v.y;
+      d[2] = v.z;
+      d[3] = v.w;
+    }
+    __syncthreads();
+    const int seg = (rows + 31) / 32;
+    const int i0 = lane * seg, i1 = min(i0 + seg, rows);
+#pragma unroll
+    for (int q = 0; q < kPsCh / 8; ++q) {
+      const int c = warp + 8 * q;
+      const float a = av[q];
+      // the lane's run from zero, and a^(run length)
+      float n = 0.f, z = 0.f, A = 1.f;
+      for (int i = i0; i < i1; ++i) {
+        n = fmaf(a, n, Ss[i * kPsLd + c]);
+        z = fmaf(a, z, 1.0f);
+        A *= a;
+      }
+      // inclusive scan of the runs across the warp
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const float Ap = __shfl_up_sync(0xffffffffu, A, off);
+        const float np = __shfl_up_sync(0xffffffffu, n, off);
+        const float zp = __shfl_up_sync(0xffffffffu, z, off);
+        if (lane >= off) {
+          n = fmaf(A, np, n);
+          z = fmaf(A, zp, z);
+          A *= Ap;
         }
       }
+      // the sums entering this lane's run: the earlier lanes (exclusive
+      // prefix) applied to the earlier windows' carry
+      float Ae = __shfl_up_sync(0xffffffffu, A, 1);
+      float ne = __shfl_up_sync(0xffffffffu, n, 1);
+      float ze = __shfl_up_sync(0xffffffffu, z, 1);
+      if (lane == 0) {
+        Ae = 1.f;
+        ne = ze = 0.f;
+      }
+      float N = fmaf(Ae, cn[q], ne), Zz = fmaf(Ae, cz[q], ze);
+      // the carry out of this window (lane 31's inclusive sums)
+      const float At = __shfl_sync(0xffffffffu, A, 31);
+      const float nt = __shfl_sync(0xffffffffu, n, 31);
+      const float zt = __shfl_sync(0xffffffffu, z, 31);
+      cn[q] = fmaf(At, cn[q], nt);
+      cz[q] = fmaf(At, cz[q], zt);
+      for (int i = i0; i < i1; ++i) {
+        N = fmaf(a, N, Ss[i * kPsLd + c]);
+        Zz = fmaf(a, Zz, 1.0f);
+        Ss[i * kPsLd + c] = N / Zz;
+        Zs[i * kPsLd + c] = Zz;
+      }
     }
+    __syncthreads();
+    // the window's rows of M (and Mb; Z, 1/Z for batch 0)
+    for (int o = threadIdx.x; o < rows * (kPsCh / 4); o += kPsThreads) {
+      const int rr = o / (kPsCh / 4), p4 = o % (kPsCh / 4);
+      const float* s = Ss + rr * kPsLd + 4 * p4;
+      const long g = ((long)b * Nb + w0 + rr) * D + c0 + 4 * p4;
+      *reinterpret_cast<float4*>(M + g) = make_float4(s[0], s[1], s[2], s[3]);
+      if (Mb) {
+        __nv_bfloat162 lo = __floats2bfloat162_rn(s[0], s[1]), hi = __floats2bfloat162_rn(s[2], s[3]);
+        uint2 u;
+        u.x = *reinterpret_cast<uint32_t*>(&lo);
+        u.y = *reinterpret_cast<uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(Mb + g) = u;
+      }
+      if (b == 0) {
+        const float* zz = Zs + rr * kPsLd + 4 * p4;
+        const long gz = (long)(w0 + rr) * D + c0 + 4 * p4;
+        *reinterpret_cast<float4*>(Z + gz) = make_float4(zz[0], zz[1], zz[2], zz[3]);
+        *reinterpret_cast<float4*>(Zinv + gz) =
+            make_float4(1.0f / zz[0], 1.0f / zz[1], 1.0f / zz[2], 1.0f / zz[3]);
+      }
+    }
+    __syncthreads();  // the window's shared memory is reused
   }
 }
+
+// The reverse scan (memory_scan_bwd_kernel): kScanThreads threads per CTA
+// spread the B * D chains over many SMs.
+constexpr int kScanThreads = 64;
 
 // ------------------------------------------------ warp-level bf16 products
 // The memory's D x D projections at small shapes are [B*Nb, D] x [D, D]: a
@@ -977,9 +1065,15 @@ cudaError_t summary_fwd(const Launch& lc, int dtype, const void* Hm, const float
 
 cudaError_t memory_scan_fwd(const Launch& lc, const float* S, const float* decay, float* M,
                             void* Mb, float* Z, float* Zinv, int B, int Nb, int D) {
-  dim3 grid((D + kScanThreads - 1) / kScanThreads, B);
-  cudaError_t e = launch_k(memory_scan_fwd_kernel, grid, dim3(kScanThreads), 0, lc.stream, S,
-                           decay, M, (bf16*)Mb, Z, Zinv, Nb, D);
+  if (D % kPsCh != 0) return cudaErrorInvalidValue;
+  const size_t smem = (size_t)2 * std::min(Nb, kPsWin) * kPsLd * sizeof(float);
+  static std::atomic<unsigned long long> opted{0};
+  cudaError_t e = smem_opt_in(memory_scan_fwd_kernel, (int)((size_t)2 * kPsWin * kPsLd * sizeof(float)),
+                              &opted);
+  if (e != cudaSuccess) return e;
+  dim3 grid(D / kPsCh, B);
+  e = launch_k(memory_scan_fwd_kernel, grid, dim3(kPsThreads), smem, lc.stream, S, decay, M,
+               (bf16*)Mb, Z, Zinv, Nb, D);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
