@@ -223,12 +223,16 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
   const T* gp = G + o0;
   T* dup = dU + o0;
   Raw8<T> rdy[8], rgt[8];
+  // dY is an input of the call, complete before the layer's first kernel
+  // started: its loads go out before the wait for the previous kernel (the
+  // caller's pdl_enter is here)
 #pragma unroll
   for (int u = 0; u < 8; ++u)
-    if (cin && rg + 8 * u < n) {
-      ld_raw(dyp + u * step, rdy[u]);
-      ld_raw(gp + u * step, rgt[u]);
-    }
+    if (cin && rg + 8 * u < n) ld_raw(dyp + u * step, rdy[u]);
+  pdl_enter();
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (cin && rg + 8 * u < n) ld_raw(gp + u * step, rgt[u]);
   // meanwhile the memory row, one channel per thread, its K-split partials
   // summed in split order (C_0 = 0, C_i = P_{i-1})
   {
@@ -479,7 +483,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                            const bf16* __restrict__ w_p, const bf16* __restrict__ dY, bf16* dH,
                            float* __restrict__ ds_out, float* __restrict__ dwp_part, int Tlen,
                            int D, int L, int Nb) {
-  pdl_enter();
   constexpr int ROWS = 8 * RW;
   constexpr int PW = KC * 256 + 4;  // row-group stride of the dW_p partials
   __shared__ __align__(16) float dss[KC * 256];
@@ -491,18 +494,31 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int blen = min(L, Tlen - i * L);
   const int t0 = i * L + c * ROWS, n = min(ROWS, blen - c * ROWS);
   const long prow = ((long)b * Nb + i) * gridDim.x + c;
-  if (n <= 0) {  // a ragged last block's empty chunk: zero partials of dW_p
-    for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
-    return;
-  }
   const long rowbase = (long)b * Tlen + t0;
   const bf16* Hb = Hm + rowbase * D;
   bf16* dHb = dH + rowbase * D;
   const bf16* dYb = dY + rowbase * D;
   // dY goes straight to shared memory (cp.async: no registers held while it
-  // is in flight), each thread's own pieces, read back by the same thread
+  // is in flight), each thread's own pieces, read back by the same thread.
+  // dY is an input of the call, complete before the layer's first kernel
+  // started, so its copies go out before the wait for the previous kernel.
   extern __shared__ __align__(16) uint8_t ys_raw[];  // [8 RW rows][KC * 256] bf16
   bf16* ys = reinterpret_cast<bf16*>(ys_raw);
+#pragma unroll
+  for (int u = 0; u < RW; ++u)
+#pragma unroll
+    for (int j = 0; j < KC; ++j) {
+      const int k = 256 * j + 8 * lane;
+      if (warp + 8 * u < n && k < D)
+        cp_async16(ys + ((warp + 8 * u) * KC + j) * 256 + 8 * lane,
+                   dYb + (long)(warp + 8 * u) * D + k);
+    }
+  cp_async_commit();
+  pdl_enter();
+  if (n <= 0) {  // a ragged last block's empty chunk: zero partials of dW_p
+    for (int k = threadIdx.x; k < D; k += kThreads) dwp_part[prow * D + k] = 0.f;
+    return;
+  }
   uint4 h[RW][KC], d[RW][KC];
 #pragma unroll
   for (int u = 0; u < RW; ++u)
@@ -511,12 +527,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       const int k = 256 * j + 8 * lane;
       if (warp + 8 * u < n && k < D) {
         const long o = (long)(warp + 8 * u) * D + k;
-        cp_async16(ys + ((warp + 8 * u) * KC + j) * 256 + 8 * lane, dYb + o);
         load8_raw(Hb + o, h[u][j]);
         load8_raw(dHb + o, d[u][j]);
       }
     }
-  cp_async_commit();
   float a[RW];
 #pragma unroll
   for (int u = 0; u < RW; ++u) a[u] = (warp + 8 * u < n) ? alpha[rowbase + warp + 8 * u] : 0.f;
@@ -853,6 +867,7 @@ __device__ __forceinline__ void warp_mma_16x8(const bf16* A, int lda, int r0, co
 // [B*Nb, D]: its readers take C_i = P_{i-1}, C_0 = 0.
 constexpr int kProjThreads = 512;
 constexpr int kProjKQ = kProjThreads / 32 / 4;  // K ranges per column group
+constexpr int kProjMaxCh = 4;                   // channels per thread (D <= 2048)
 __global__ void __launch_bounds__(kProjThreads)
     memory_proj_fwd_kernel(const float* __restrict__ S, const float* __restrict__ decay,
                            const bf16* __restrict__ Wm, float* __restrict__ P,
@@ -870,6 +885,13 @@ __global__ void __launch_bounds__(kProjThreads)
   // the weight chunk: D rows of kProjNC columns (16 bytes per load, a batch
   // of loads in flight before their shared-memory stores)
   copy_rows16<kProjNC / 8, kProjThreads>(Ws, ldw, Wm + x * kProjNC, D, D);
+  // the decay of this thread's channels (an input too)
+  float apre[kProjMaxCh];
+#pragma unroll
+  for (int q = 0; q < kProjMaxCh; ++q) {
+    const int k = threadIdx.x + q * kProjThreads;
+    apre[q] = k < D ? decay[k] : 0.f;
+  }
   pdl_enter();
   // the batch's summaries to shared memory in 16-byte pieces (all in flight
   // at once, no registers held)
@@ -882,9 +904,11 @@ __global__ void __launch_bounds__(kProjThreads)
   }
   // the scan, one channel per thread (a rolled loop: little code to fetch);
   // CTA x stores M, Mb (and for b == 0, Z and 1/Z) of its own 32 channels
-#pragma unroll 1
-  for (int k = threadIdx.x; k < D; k += kProjThreads) {
-    const float a = decay[k];
+#pragma unroll
+  for (int q = 0; q < kProjMaxCh; ++q) {
+    const int k = threadIdx.x + q * kProjThreads;
+    if (k >= D) break;
+    const float a = apre[q];
     const bool mine = k / kProjNC == x;
     float Nn = 0.f, Zz = 0.f;
 #pragma unroll 4
@@ -952,7 +976,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const float* __restrict__ Pm, long pstride, T* __restrict__ dU,
                     float* __restrict__ dP, bf16* __restrict__ dPb, int Tlen, int D, int L,
                     int Nb) {
-  pdl_enter();
   extern __shared__ __align__(16) float sm[];
   gate_bwd_item<T, PS>(sm, dY, G, Pm, pstride, dU, dP, dPb, Tlen, D, L, Nb, blockIdx.x,
                    blockIdx.y, blockIdx.z);
@@ -1091,6 +1114,7 @@ static size_t proj_fwd_smem(int Nb, int D) {
 }
 bool memory_proj_fits(int dtype, int B, int Nb, int D) {
   return dtype == 1 && D % 64 == 0 && D % (16 * kProjKQ) == 0 && Nb <= 16 &&
+         D <= kProjMaxCh * kProjThreads &&
          proj_fwd_smem(Nb, D) <= (size_t)kProjSmemMax &&
          (double)B * Nb * D * D <= (double)(1 << 28);
 }
