@@ -325,14 +325,18 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
                             const __grid_constant__ CUtensorMap mV, bf16* __restrict__ O,
                             long ld_o, float* __restrict__ lse, int Tlen, int H, int L,
                             float scale, unsigned* status) {
-  static_assert(DH <= 32, "two 64-key halves and O fit 128 TMEM columns for DH <= 32 (and 64)");
+  static_assert(DH <= 64, "a 64-key S half and O fit 128 TMEM columns for DH <= 64");
+  // K double-buffered across tiles up to width 32; at 64 one K buffer keeps
+  // the CTA at 66 KB of shared memory (three per SM), and the next tile's K
+  // is loaded once this tile's second half has its scores
+  constexpr int NKB = DH <= 32 ? 2 : 1;
   using G = Geo<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sP = smem;                       // 16 KB: P of one half [128 queries x 64 keys]
   uint8_t* sQ = smem + 16384;
-  uint8_t* sK0 = sQ + G::tile;              // K, two buffers
-  uint8_t* sV = sK0 + 2 * G::tile;
+  uint8_t* sK0 = sQ + G::tile;              // K, NKB buffers
+  uint8_t* sV = sK0 + NKB * G::tile;
   // barriers: K buffer 0/1 loaded (buffer 0 also counts Q), V loaded, S ready, P V done
   uint64_t* bar = reinterpret_cast<uint64_t*>(sV + G::tile);
   uint64_t* bar_k = bar;
@@ -360,9 +364,9 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
     tc::tma_load_3d(sK0, &mK, &bar_k[0], h * DH, kstart, b);
     tc::mbar_arrive_expect_tx(bar_v, G::tile);
     tc::tma_load_3d(sV, &mV, bar_v, h * DH, kstart, b);
-    if (nkt > 1) {
-      tc::mbar_arrive_expect_tx(&bar_k[1], G::tile);
-      tc::tma_load_3d(sK0 + G::tile, &mK, &bar_k[1], h * DH, kstart + kTile, b);
+    if (NKB == 2 && nkt > 1) {
+      tc::mbar_arrive_expect_tx(&bar_k[NKB - 1], G::tile);
+      tc::tma_load_3d(sK0 + (NKB - 1) * G::tile, &mK, &bar_k[NKB - 1], h * DH, kstart + kTile, b);
     }
   }
   __syncwarp();
@@ -406,7 +410,16 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
 
   for (int kt = 0; kt < nkt; ++kt) {
     const bool diag = kt == nkt - 1;
-    const int kb = kt & 1;
+    const int kb = NKB == 2 ? (kt & 1) : 0;
+    if constexpr (NKB == 1) {
+      if (kt > 0 && tid == 0) {  // this tile's K (loaded during the last tile)
+        const bool okk = tc::mbar_wait(&bar_k[0], kt & 1, status);
+        tc::fence_after_sync();
+        if (okk && ok) issue_s(0, 0);
+        else tc::mma_commit(bar_s);
+      }
+      __syncwarp();
+    }
     for (int hh = 0; hh < 2; ++hh) {
       ok = tc::mbar_wait(bar_s, ns & 1, status) && ok;
       ++ns;
@@ -422,7 +435,7 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
         if (hh == 0) {  // the tile's second half
           if (ok) issue_s(kb, 1);
           else tc::mma_commit(bar_s);
-        } else if (kt + 1 < nkt) {  // the next tile's first half
+        } else if (NKB == 2 && kt + 1 < nkt) {  // the next tile's first half (K prefetched)
           const int nb = (kt + 1) & 1;
           const bool okk = tc::mbar_wait(&bar_k[nb], ((kt + 1) >> 1) & 1, status);
           tc::fence_after_sync();
@@ -430,9 +443,10 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
           else tc::mma_commit(bar_s);
         }
         // K buffer kb: both halves' scores are read (tile kt done with it)
-        if (hh == 1 && kt + 2 < nkt) {
+        if (hh == 1 && kt + NKB < nkt) {
           tc::mbar_arrive_expect_tx(&bar_k[kb], G::tile);
-          tc::tma_load_3d(sK0 + kb * G::tile, &mK, &bar_k[kb], h * DH, kstart + (kt + 2) * kTile, b);
+          tc::tma_load_3d(sK0 + kb * G::tile, &mK, &bar_k[kb], h * DH,
+                          kstart + (kt + NKB) * kTile, b);
         }
       }
       if (diag) {  // keys past the query row (L > 128: no block offset in the tile)
@@ -1288,7 +1302,9 @@ template <int DH> constexpr int dkv_smem() {
   return 1024 + 32768 + 4 * Geo<DH>::tile + 2 * kTile * 4 + 64;
 }
 
-template <int DH> constexpr int fwd_half_smem() { return 1024 + 16384 + 4 * Geo<DH>::tile + 64; }
+template <int DH> constexpr int fwd_half_smem() {
+  return 1024 + 16384 + (DH <= 32 ? 4 : 3) * Geo<DH>::tile + 64;
+}
 
 template <int DH>
 cudaError_t fwd_fl_half_launch(const Launch& lc, const AttnArgs& a, const CUtensorMap* m) {
@@ -1322,10 +1338,7 @@ cudaError_t fwd_fl(const Launch& lc, const AttnArgs& a) {
       !head_map_fl<DH>(&m[1], a.K, a.ld_qkv, D, a.T, a.B) ||
       !head_map_fl<DH>(&m[2], a.V, a.ld_qkv, D, a.T, a.B))
     return cudaErrorInvalidValue;
-  if (a.L > kTile) {
-    if constexpr (DH <= 32) return fwd_fl_half_launch<DH>(lc, a, m);
-    return fwd_fl_launch<DH, 4, false>(lc, a, m);
-  }
+  if (a.L > kTile) return fwd_fl_half_launch<DH>(lc, a, m);
   if (a.L <= 32) return fwd_fl_launch<DH, 1, true>(lc, a, m);
   if (a.L == 64) return fwd_fl_launch<DH, 2, true>(lc, a, m);
   return fwd_fl_launch<DH, 4, true>(lc, a, m);
