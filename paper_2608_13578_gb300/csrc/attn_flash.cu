@@ -307,17 +307,19 @@ __global__ void __launch_bounds__(128, NCH <= 2 ? 3 : 2)
   if (warp == 0) tc::tmem_dealloc(tmem, kCols);
 }
 
-// The forward at L > 128 for head widths up to 32, with each 128-key tile
-// taken as two 64-key halves in turn: S of a half (N = 64) and O need at most
-// 96 TMEM columns and P one 16 KB half, so a CTA allocates 128 columns and
-// three or four CTAs share an SM (twice the warps of the kernel above, whose
-// per-score chains are latency-bound).  Per half: S = Q K_h^T, online softmax
-// of its 64 scores (the diagonal tile's hidden keys set to -inf first), P_h in
-// bf16 to shared memory, P_h V_h into TMEM, folded into O in registers.  The
-// next half's S is issued as soon as every thread has read this half's scores
-// and runs under its softmax; K is double-buffered across tiles (K of tile
-// kt+2 streams in once tile kt's second half has its scores) and V is
-// reloaded once tile kt's second P V has completed.
+// The forward at L > 128, with each 128-key tile taken as two 64-key halves
+// in turn: S of a half (N = 64) and O need at most 128 TMEM columns and P one
+// 16 KB half, so a CTA allocates 128 columns and three or four CTAs share an
+// SM (more warps than the kernel above, whose per-score chains are
+// latency-bound).  Per half: S = Q K_h^T, online softmax of its 64 scores (the
+// diagonal tile's hidden keys set to -inf first), P_h in bf16 to shared
+// memory, P_h V_h into TMEM, folded into O in registers.  The next half's S is
+// issued as soon as every thread has read this half's scores and runs under
+// its softmax.  Up to width 32, K is double-buffered across tiles (K of tile
+// kt+2 streams in once tile kt's second half has its scores); at width 64 one
+// K buffer (66 KB per CTA: three per SM) takes tile kt+1's K at that point
+// and its first S waits for it.  V is reloaded once tile kt's second P V has
+// completed.
 template <int DH>
 __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
     attn_fwd_fl_half_kernel(const __grid_constant__ CUtensorMap mQ,
@@ -326,10 +328,7 @@ __global__ void __launch_bounds__(128, DH <= 16 ? 4 : 3)
                             long ld_o, float* __restrict__ lse, int Tlen, int H, int L,
                             float scale, unsigned* status) {
   static_assert(DH <= 64, "a 64-key S half and O fit 128 TMEM columns for DH <= 64");
-  // K double-buffered across tiles up to width 32; at 64 one K buffer keeps
-  // the CTA at 66 KB of shared memory (three per SM), and the next tile's K
-  // is loaded once this tile's second half has its scores
-  constexpr int NKB = DH <= 32 ? 2 : 1;
+  constexpr int NKB = DH <= 32 ? 2 : 1;  // K buffers
   using G = Geo<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
