@@ -15,7 +15,9 @@
 //  * forward: per key tile S = Q K^T (N = 128), online softmax with the
 //    thread owning one query row (running max and sum in registers), P in
 //    bf16 to shared memory, P V into TMEM, O rescaled and accumulated in
-//    registers; O and the log-sum-exp are stored at the end.
+//    registers; O and the log-sum-exp are stored at the end.  At L > 128
+//    the layer runs the half-tile form (64-key halves, 128 TMEM columns per
+//    CTA, more CTAs per SM).
 //  * backward, two kernels (no atomics, fixed summation order):
 //      dQ:  per query tile, Drow = dO . O, then per key tile and 64-key half
 //           S, dP (N = 64), dS = P (dP - Drow) scale, dQ += dS K (TMEM);
@@ -23,6 +25,8 @@
 //           dP^T = V dO^T, dV += P^T dO, dK += dS^T Q (TMEM), with the query
 //           tile's log-sum-exp and Drow staged in shared memory; the second
 //           half's S^T and dP^T are issued ahead of the first half's dV/dK.
+//    For head widths up to 32 both walk 32-key / 32-query quarters instead
+//    (128 TMEM columns per CTA: three or four CTAs per SM).
 #include "attn_common.cuh"
 #include "common.cuh"
 #include "internal.h"
