@@ -215,23 +215,25 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
   const int c = x * kGateCh + cq * 8;
   const bool cin = c < D;
   const int t0 = i * L, n = min(L, Tlen - t0);
-  // rows rg, rg+8, ... in batches of 8 (64 rows of the block, loads held
-  // packed): every load of a batch is issued before its first store
+  // rows rg, rg+8, ... in batches of RB (64 rows of the block in bf16, 32 in
+  // fp32, whose rows take twice the registers; loads held packed): every
+  // load of a batch is issued before its first store
+  constexpr int RB = sizeof(T) == 2 ? 8 : 4;
   const long step = 8L * D;
   const long o0 = ((long)b * Tlen + t0 + rg) * D + c;
   const T* dyp = dY + o0;
   const T* gp = G + o0;
   T* dup = dU + o0;
-  Raw8<T> rdy[8], rgt[8];
+  Raw8<T> rdy[RB], rgt[RB];
   // dY is an input of the call, complete before the layer's first kernel
   // started: its loads go out before the wait for the previous kernel (the
   // caller's pdl_enter is here)
 #pragma unroll
-  for (int u = 0; u < 8; ++u)
+  for (int u = 0; u < RB; ++u)
     if (cin && rg + 8 * u < n) ld_raw(dyp + u * step, rdy[u]);
   pdl_enter();
 #pragma unroll
-  for (int u = 0; u < 8; ++u)
+  for (int u = 0; u < RB; ++u)
     if (cin && rg + 8 * u < n) ld_raw(gp + u * step, rgt[u]);
   // meanwhile the memory row, one channel per thread, its K-split partials
   // summed in split order (C_0 = 0, C_i = P_{i-1})
@@ -257,17 +259,17 @@ __device__ void gate_bwd_item(float* sm, const T* __restrict__ dY, const T* __re
 #pragma unroll
     for (int e = 0; e < 8; ++e) cm[e] = crow[cq * 8 + e];
 #pragma unroll 1
-    for (int r0 = rg; r0 < n; r0 += 64, dyp += 8 * step, gp += 8 * step, dup += 8 * step) {
-      if (r0 != rg) {  // blocks longer than 64 tokens: the next batch
+    for (int r0 = rg; r0 < n; r0 += 8 * RB, dyp += RB * step, gp += RB * step, dup += RB * step) {
+      if (r0 != rg) {  // the block's next batch of rows
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
+        for (int u = 0; u < RB; ++u)
           if (r0 + 8 * u < n) {
             ld_raw(dyp + u * step, rdy[u]);
             ld_raw(gp + u * step, rgt[u]);
           }
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
+      for (int u = 0; u < RB; ++u)
         if (r0 + 8 * u < n) {
           float dy[8], g[8], du[8];
           unraw(rdy[u], dy);
