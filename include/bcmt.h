@@ -64,7 +64,7 @@ typedef enum {
   BCMT_ERR_ALIGN = 3,       /* a pointer is not 16-byte aligned                    */
   BCMT_ERR_CUDA = 4,        /* a CUDA runtime call or kernel launch failed         */
   BCMT_ERR_TIMEOUT = 5,     /* a bounded device-side wait expired                  */
-  BCMT_ERR_UNSUPPORTED = 6  /* valid for the method, not implemented by this build */
+  BCMT_ERR_UNSUPPORTED = 6  /* valid for the method, not implemented by the library */
 } bcmt_status;
 
 typedef enum { BCMT_F32 = 0, BCMT_BF16 = 1 } bcmt_dtype;
